@@ -1,0 +1,397 @@
+"""Benchmark: the attribution join (enclose + match + aggregate) on the
+20M-kernel synthetic trace, one pass per step, on N GPUs (one independent
+trace per rank: weak scaling, no collective on the data path).
+
+Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle on a
+bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "M kernel records attributed/sec (1 GB300) and % of HBM roofline"
+UNIT = "M kernels/s"
+NOMINAL_HBM_GBS = 8000.0
+L2_BYTES = 129 * 2**20
+
+# Algorithmic bytes per unit (the minimum each step must move):
+#   per kernel: stream 1 + start 8 + dur 8 + name 4 read, range 4 + ncu_idx 4 written
+#   per range: stream 1 + start 8 + end 8 + depth 1 + op 4 read
+#   per ncu row: name 4 + 20 counters x 4 read;  per op: 3 x 8 + 20 x 8 written
+PATH_BYTES = dict(kernel=29, range=22, ncu=84, op=184)
+
+# Per-launch algorithmic bytes of the kernels that can dominate a step.
+KERNEL_BYTES = {
+    "agg_owned": lambda K, R, M, O: 96 * K + 12 * R + 184 * O,
+    "enclose": lambda K, R, M, O: 14 * K + 20 * R,
+    "match_identity": lambda K, R, M, O: 13 * K,
+    "agg_check_kernels": lambda K, R, M, O: 20 * K,
+    "check_kernel_order": lambda K, R, M, O: 9 * K,
+    "check_ranges": lambda K, R, M, O: 18 * R,
+    "level_gather": lambda K, R, M, O: 44 * R,
+    "validate_levels": lambda K, R, M, O: 22 * R,
+    "agg_check_ranges": lambda K, R, M, O: 12 * R,
+    "window_table": lambda K, R, M, O: 0,
+}
+
+WORKLOADS = {
+    "large": "16 streams, 20,000,000 kernels, ~5,000,000 NVTX ranges depth <= 8, 5,000 names Zipf 1.1, "
+             "20 fp32 counters per ncu row U[0,100], 5% of kernels uncovered (seed 3)",
+    "adversarial": "64 streams, 50,000,000 kernels, 85% of runtime outside ranges, depth up to 32, "
+                   "50,000 names Zipf 1.5 (seed 4)",
+    "dedup": "48 layers in 3 classes on 4 streams, 400,000 kernels, 25,000 ncu rows (seed 2)",
+    "gpt2": "GPT-2-small-shaped: 12 layers x 40 kernels x 50 iterations on 2 streams (seed 1)",
+    "tiny": "1 stream, 2,000 kernels, ~300 ranges (seed 0)",
+}
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+# ---------------------------------------------------------------- rank plumbing
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def combine_ranks(elapsed_s: float, units: int, world: int, reduce_max, reduce_sum):
+    """Max elapsed over ranks and the units all ranks processed."""
+    t = reduce_max(elapsed_s) if world > 1 else elapsed_s
+    u = reduce_sum(units) if world > 1 else units
+    return t, u
+
+
+def run_timed(step, steps: int, warmup: int, sync, barrier, start_clock=None, stop_clock=None):
+    """W untimed steps, then exactly K steps between barrier + sync pairs.
+    Returns seconds of the timed region (device-timed by `sync` pairs)."""
+    for _ in range(warmup):
+        step()
+    sync()
+    barrier()
+    sync()
+    if start_clock:
+        start_clock()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        step()
+    sync()
+    barrier()
+    sync()
+    t1 = time.perf_counter()
+    if stop_clock:
+        stop_clock()
+    return t1 - t0
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled every 100 ms."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device: int):
+        self.device = device
+        self.proc = None
+        self.path = None
+        self.windows = []
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.device), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+
+    def mark(self, begin: bool):
+        if begin:
+            self.windows.append([time.time(), None])
+        else:
+            self.windows[-1][1] = time.time()
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.proc or not self.path:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = [r.split(", ") for r in open(self.path).read().strip().splitlines() if r.strip()]
+        os.unlink(self.path)
+        sm = [float(r[1]) for r in rows if len(r) >= 9 and r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if len(r) >= 9 and r[2].replace(".", "").isdigit()]
+        power = [float(r[3]) for r in rows if len(r) >= 9 and r[3].replace(".", "").isdigit()]
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        reasons = sorted({n for r in rows if len(r) >= 9 for n, v in zip(names, r[5:9]) if v.strip() == "Active"})
+        loaded = sorted(sm)[len(sm) // 2:] if sm else []
+        return {"sm_mhz": statistics.median(loaded) if loaded else None, "sm_max_mhz": max(mx) if mx else None,
+                "samples": len(sm), "power_w_max": max(power) if power else None, "reasons": reasons,
+                "window": "warm-up + timed region + 1 s soak of the same step"}
+
+
+# ---------------------------------------------------------------- CPU baseline (the oracle)
+def oracle_sample_config(config_name: str, n_kernels: int):
+    import tracegen
+    cfg = tracegen.config(config_name)
+    if cfg.get("shape", 0) == 0:
+        cfg["n_kernels"] = n_kernels
+    return cfg
+
+
+def time_oracle(config_name: str, n_kernels: int = 1_000_000, reps: int = 1):
+    """The CPU oracle (indexed mode, single thread) on a bounded sample of the
+    workload: the same generator parameters with fewer kernels."""
+    import oracle
+    import tracegen
+    t = tracegen.generate(oracle_sample_config(config_name, n_kernels))
+    best = None
+    for _ in range(reps):
+        t0 = time.perf_counter()
+        res = oracle.run(t, enclose_mode="indexed")
+        dt = time.perf_counter() - t0
+        assert res["aggregate_status"] == 0
+        best = dt if best is None else min(best, dt)
+    return t.K, best
+
+
+# ---------------------------------------------------------------- main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", default="large", choices=sorted(WORKLOADS))
+    ap.add_argument("--shuffle", action="store_true", help="permute kernel and range arrays (general paths)")
+    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--oracle-kernels", type=int, default=1_000_000)
+    args = ap.parse_args()
+    world, rank, local = dist_env()
+    if args.warmup < 3:
+        args.warmup = 3
+
+    if args.impl == "reference":
+        if rank != 0:
+            return
+        n, _ = time_oracle(args.config, args.oracle_kernels, reps=1)       # warm caches
+        times = []
+        for _ in range(args.warmup):
+            time_oracle(args.config, args.oracle_kernels)
+        for _ in range(args.steps):
+            times.append(time_oracle(args.config, args.oracle_kernels)[1])
+        tot = sum(times)
+        value = n * len(times) / tot / 1e6
+        line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+                "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / len(times),
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+                "data": "synthetic", "config": {"workload": f"{args.config}: {WORKLOADS[args.config]}",
+                                                "sample_kernels": n},
+                "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                                 "sample": f"{n} kernels drawn with the {args.config} generator parameters; "
+                                           f"indexed oracle (enclose + match + aggregate), single thread"},
+                "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return
+
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    import paper_2609_11938_gb300 as opa
+    import tracegen
+
+    if world > 1:
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = local
+    opa.build()
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    def rmax(x):
+        t = torch.tensor([float(x)], device=f"cuda:{dev}")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def rsum(x):
+        t = torch.tensor([float(x)], device=f"cuda:{dev}", dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.SUM)
+        return int(t.item())
+
+    cfg = tracegen.config(args.config)
+    cfg["seed"] = cfg["seed"] + 1000 * rank          # each rank attributes its own trace
+    trace = tracegen.generate(cfg, shuffle=args.shuffle)
+    K, R, M, O = trace.K, trace.R, trace.M, trace.n_ops
+    use_dedup = bool(cfg.get("dedup")) and trace.k_layer is not None
+    tr = opa.to_device(trace, dev)
+    torch.cuda.synchronize(dev)
+    stream = torch.cuda.Stream(dev)
+    ctx = opa.Context(dev, stream=stream)
+    rk = torch.empty(K, dtype=torch.int32, device=f"cuda:{dev}")
+    nop = torch.empty(K, dtype=torch.uint8, device=f"cuda:{dev}")
+    idx = torch.empty(K, dtype=torch.int32, device=f"cuda:{dev}")
+    kind = torch.empty(K, dtype=torch.uint8, device=f"cuda:{dev}")
+    ops = ctx.alloc_ops(O)
+    in_bytes = sum(x.numel() * x.element_size() for x in (tr.k_stream, tr.k_start, tr.k_dur, tr.k_name,
+                                                           tr.r_stream, tr.r_start, tr.r_end, tr.r_depth, tr.r_op,
+                                                           tr.ncu_name, tr.counters))
+    flush = None
+    if in_bytes < 2 * L2_BYTES:
+        flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=f"cuda:{dev}")
+
+    def step():
+        if flush is not None:
+            with torch.cuda.stream(stream):
+                flush.fill_(1.0)
+        ctx.enclose(tr, rk, nop)
+        ctx.match(tr, dedup=use_dedup, out_idx=idx, out_kind=kind)
+        ctx.aggregate(tr, rk, idx, ops)
+
+    def sync():
+        stream.synchronize()
+
+    clocks = ClockSampler(dev)
+    clocks.start()
+    for _ in range(args.warmup):
+        step()
+    sync()
+    ctx.set_timing(True)
+    ctx.timing_reset()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier(); sync()
+    ev0.record(stream)
+    wall0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    ev1.record(stream)
+    sync(); barrier(); sync()
+    wall = time.perf_counter() - wall0
+    elapsed = ev0.elapsed_time(ev1) / 1e3
+    launches = ctx.launch_count()
+    report = ctx.timing_report()
+    ctx.set_timing(False)
+    # keep the GPU busy with the same step for ~1 s so the clock sampler sees it
+    soak_end = time.perf_counter() + 1.0
+    while time.perf_counter() < soak_end:
+        step()
+    sync()
+    clocks.stop()
+    t_max, units = combine_ranks(max(elapsed, 1e-9), K * args.steps, world, rmax, rsum)
+
+    # ---- end to end through the C ABI with host buffers (pinned), per step:
+    # H2D of every input array, the three calls, D2H of every output
+    host = {name: torch.from_numpy(getattr(trace, name)).pin_memory()
+            for name in ("k_stream", "k_start", "k_dur", "k_name", "r_stream", "r_start", "r_end", "r_depth",
+                         "r_op", "ncu_name", "counters")}
+    if trace.k_layer is not None:
+        host["k_layer"] = torch.from_numpy(trace.k_layer).pin_memory()
+    out_host = {"rk": torch.empty(K, dtype=torch.int32).pin_memory(),
+                "idx": torch.empty(K, dtype=torch.int32).pin_memory()}
+    out_host.update({k: torch.empty_like(v, device="cpu").pin_memory() for k, v in ops.items()})
+    h2d = sum(v.numel() * v.element_size() for v in host.values())
+    d2h = sum(v.numel() * v.element_size() for v in out_host.values())
+
+    def e2e_step():
+        with torch.cuda.stream(stream):
+            for name, v in host.items():
+                getattr(tr, name).copy_(v, non_blocking=True)
+        ctx.enclose(tr, rk, nop)
+        ctx.match(tr, dedup=use_dedup, out_idx=idx, out_kind=kind)
+        ctx.aggregate(tr, rk, idx, ops)
+        with torch.cuda.stream(stream):
+            out_host["rk"].copy_(rk, non_blocking=True)
+            out_host["idx"].copy_(idx, non_blocking=True)
+            for k, v in ops.items():
+                out_host[k].copy_(v, non_blocking=True)
+        stream.synchronize()
+
+    e2e_step()
+    e2e_s = run_timed(e2e_step, args.e2e_steps, 1, sync, barrier)
+    e2e_t, e2e_units = combine_ranks(e2e_s, K * args.e2e_steps, world, rmax, rsum)
+
+    if rank != 0:
+        ctx.close()
+        if world > 1:
+            dist.destroy_process_group()
+        return
+
+    # ---- roofline of the dominant kernel (CUDA events around each launch)
+    peak, peak_kind = load_peaks()
+    dom = max(report.items(), key=lambda kv: kv[1][0])
+    dname, (dms, dcount) = dom
+    dbytes = KERNEL_BYTES.get(dname, lambda *a: 0)(K, R, M, O)
+    avg_s = dms / 1e3 / max(dcount, 1)
+    achieved = dbytes / avg_s / 1e9 if dbytes else None
+    step_s = elapsed / args.steps
+    path_bytes = PATH_BYTES["kernel"] * K + PATH_BYTES["range"] * R + PATH_BYTES["ncu"] * M + PATH_BYTES["op"] * O
+    path_gbs = path_bytes / step_s / 1e9
+    ctx.close()
+
+    n_or, t_or = time_oracle(args.config, args.oracle_kernels)
+    line = {
+        "metric": METRIC,
+        "value": units / t_max / 1e6,
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": 1e3 * t_max / args.steps,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "int64+f32x2",
+        "data": "synthetic",
+        "config": {"workload": f"{args.config}: {WORKLOADS[args.config]}", "kernels": K, "ranges": R,
+                   "ncu_rows": M, "ops": O, "shuffled": bool(args.shuffle), "parallelism": f"replicas x{world}",
+                   "l2": "inputs larger than L2 (129 MB)" if flush is None else "L2 flushed before every step"},
+        "roofline": {"bound": "hbm", "kernel": dname, "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": (achieved / peak) if achieved else None, "peak_kind": f"{peak_kind} copy bandwidth",
+                     "traffic": None, "alg_bytes_per_launch": dbytes, "avg_launch_ms": avg_s * 1e3,
+                     "launches": dcount},
+        "path_roofline": {"alg_bytes_per_step": path_bytes, "achieved_gbs": path_gbs,
+                          "frac_of_8tbs": path_gbs / NOMINAL_HBM_GBS, "frac_of_measured": path_gbs / peak},
+        "cpu_baseline": {"value": n_or / t_or / 1e6, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"{n_or} kernels drawn with the {args.config} generator parameters; indexed "
+                                   f"oracle (enclose + match + aggregate), single thread, {t_or:.2f} s"},
+        "e2e": {"value": e2e_units / e2e_t / 1e6, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": launches,
+        "kernel_ms_per_step": {k: round(v[0] / args.steps, 4) for k, v in sorted(report.items(),
+                                                                               key=lambda kv: -kv[1][0])},
+        "wall_ms_per_step": 1e3 * wall / args.steps,
+        "clocks": clocks.summary(),
+    }
+    print(json.dumps(line))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

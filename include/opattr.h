@@ -1,0 +1,262 @@
+/*
+ * opattr.h -- C ABI of the GPU trace join behind hardware-attributed operator
+ * profiling ("Hardware-Attributed Operator Profiling for PyTorch").
+ *
+ * The join has three calls, in this order:
+ *   opattr_enclose   -- Algorithm 2 (Sec. 3.5): each kernel record gets the
+ *                       innermost enclosing operator range on its stream.
+ *   opattr_match     -- Algorithm 1 (Sec. 3.3): the i-th launch of a kernel
+ *                       name pairs with the i-th Nsight Compute row of that
+ *                       name; layer deduplication (Sec. 3.7) broadcasts a
+ *                       representative layer's rows to its duplicates.
+ *   opattr_aggregate -- Eq. (1) and Sec. 3.8.1: per-operator duration-weighted
+ *                       means, sums and maxima of the 20-counter set
+ *                       (Table 8), plus attributed / unattributed kernel time
+ *                       (Fig. 3).
+ *
+ * Conventions shared by every call
+ *  - Record and output arrays are DEVICE pointers owned by the caller, on the
+ *    context's device.  Struct arguments themselves (and opattr_dedup's
+ *    tables, the summaries and totals) live in HOST memory.
+ *  - Work is ordered on the context's CUDA stream.  A call returns once its
+ *    small host-side results have been copied back; the device outputs are
+ *    then complete on that stream.
+ *  - n == 0 is valid everywhere and yields empty results.
+ *  - Return value: negative = error (outputs undefined; the context stays
+ *    usable except after OPATTR_E_CUDA, after which it must be destroyed),
+ *    positive = warning (outputs valid), 0 = success.
+ *  - Nothing is sorted in place; inputs are never written.
+ */
+#ifndef OPATTR_H
+#define OPATTR_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct opattr_ctx opattr_ctx;
+
+typedef enum {
+    OPATTR_OK = 0,
+    OPATTR_W_COUNT_MISMATCH = 1,   /* some kernel name has different counts in the two traces */
+    OPATTR_W_DEDUP_MISMATCH = 2,   /* some duplicate-layer kernel found no representative row */
+    OPATTR_E_INVALID_ARG = -1,     /* bad pointer, size, id or value (see each call) */
+    OPATTR_E_NOT_NESTED = -2,      /* ranges are not a laminar family per stream */
+    OPATTR_E_DEPTH = -3,           /* a range depth is above 31 */
+    OPATTR_E_COUNT_MISMATCH = -4,  /* count mismatch under OPATTR_MISMATCH_ERROR */
+    OPATTR_E_CUDA = -5,            /* a CUDA call failed; destroy the context */
+    OPATTR_E_OOM = -6,             /* device scratch could not be allocated */
+    OPATTR_E_TIMEOUT = -7,         /* a bounded device-side wait gave up */
+    OPATTR_E_STATE = -8            /* the context is unusable (after OPATTR_E_CUDA) */
+} opattr_status;
+
+/* What to do when a kernel name is launched a different number of times in
+ * the Nsight Systems trace (replayed launches) and in the ncu rows. */
+typedef enum {
+    OPATTR_MISMATCH_SKIP_NAME = 0, /* every kernel of that name stays unmatched (Sec. 3.3 text) */
+    OPATTR_MISMATCH_PREFIX = 1,    /* launch i takes row i while rows last (Algorithm 1 as printed) */
+    OPATTR_MISMATCH_ERROR = 2      /* return OPATTR_E_COUNT_MISMATCH (limitations section) */
+} opattr_mismatch_mode;
+
+/* Range kinds are carried in op_id.  Algorithm 2 tests the range text: a
+ * text without "::" (ProfilerStep#0, a layer or block marker) stops the walk;
+ * a namespaced text that is not an operator (prims::, torch::) is skipped;
+ * an operator (aten::, quantized::, a custom op) is collected.  Callers map
+ * texts to these codes; every other op_id value names an operator. */
+#define OPATTR_OP_STRUCTURAL 0xFFFFFFFFu
+#define OPATTR_OP_NONOP 0xFFFFFFFEu
+#define OPATTR_MAX_DEPTH 32
+#define OPATTR_N_COUNTERS 20
+
+/* Kernel records of the Nsight Systems trace (Sec. 3.1), one per launch.
+ *   stream    u8[n]   stream the kernel ran on (< 256)
+ *   start_ns  i64[n]  query point T: launch timestamp, ns (Sec. 3.5)
+ *   dur_ns    i64[n]  kernel duration, ns, >= 0 (read by opattr_aggregate)
+ *   name_id   u32[n]  kernel-name id (read by opattr_match)
+ *   layer_id  i32[n]  layer partition tag, -1 outside layers, or NULL
+ *                     (read by opattr_match when deduplication is on)
+ * Time order of kernels is (start_ns, stream, array index).  No order is
+ * required; records in time order take faster paths. */
+typedef struct {
+    const uint8_t *stream;
+    const int64_t *start_ns;
+    const int64_t *dur_ns;
+    const uint32_t *name_id;
+    const int32_t *layer_id;
+    int64_t n;
+} opattr_kernels;
+
+/* NVTX ranges (Sec. 3.5), one per push/pop pair.
+ *   stream    u8[n]   stream the range is keyed by
+ *   start_ns, end_ns  i64[n]  closed interval [start, end], end >= start
+ *   depth     u8[n]   nesting depth on its stream, 0 = outermost, <= 31
+ *   op_id     u32[n]  operator id, or OPATTR_OP_STRUCTURAL / OPATTR_OP_NONOP
+ * Per stream the ranges must be laminar: same-depth ranges overlap at most in
+ * one instant (sorted by (start, end, index), each ends no later than the
+ * next starts) and every range at depth d > 0 lies inside a depth d-1 range.
+ * Violations return OPATTR_E_NOT_NESTED. */
+typedef struct {
+    const uint8_t *stream;
+    const int64_t *start_ns;
+    const int64_t *end_ns;
+    const uint8_t *depth;
+    const uint32_t *op_id;
+    int64_t n;
+} opattr_ranges;
+
+/* Nsight Compute rows in launch order (Sec. 3.1).
+ *   name_id   u32[n]       kernel-name id of the row
+ *   counters  f32[n * 20]  row-major, counter #k (Table 8) at column k-1;
+ *                          NaN = null (absent counter); values must be finite
+ *                          or NaN; 16-byte aligned (read by opattr_aggregate) */
+typedef struct {
+    const uint32_t *name_id;
+    const float *counters;
+    int64_t n;
+} opattr_ncu;
+
+/* Layer deduplication tables (Sec. 3.7), HOST memory.
+ *   class_of_layer  i32[n_layers]  equivalence class of each layer
+ *   rep_of_class    i32[n_classes] representative layer of each class; it
+ *                                  must belong to that class
+ * Kernels of non-representative layers are not replayed: they take the row of
+ * the representative's kernel at the same position within the layer (time
+ * order), if that kernel has the same name and a row. */
+typedef struct {
+    const int32_t *class_of_layer;
+    const int32_t *rep_of_class;
+    int32_t n_layers;
+    int32_t n_classes;
+} opattr_dedup;
+
+typedef struct {
+    opattr_mismatch_mode mismatch; /* default OPATTR_MISMATCH_SKIP_NAME */
+    int32_t dedup;                 /* 1: apply opattr_dedup when given (default 1) */
+    int32_t checked;               /* reserved, 0 */
+    int64_t spin_limit;            /* bound on device-side waits (0 = default) */
+} opattr_config;
+
+/* Host-side result of opattr_match. */
+typedef struct {
+    int64_t kernels;               /* kernel records */
+    int64_t replayed;              /* kernels with their own ncu row expected */
+    int64_t direct;                /* kernels matched to a row directly */
+    int64_t broadcast;             /* duplicate-layer kernels given a representative's row */
+    int64_t unmatched;             /* kernels left without a row */
+    int64_t names_mismatched;      /* names whose replayed and row counts differ */
+    int64_t count_unmatched;       /* replayed kernels left unmatched by the count rule */
+    int64_t dedup_mismatch;        /* duplicate-layer kernels without a usable source */
+    int32_t fast_path;             /* 1: rows equal replayed kernels in time order */
+    int32_t reserved;
+} opattr_match_summary;
+
+/* Device outputs of opattr_aggregate, one entry per op id, caller-allocated.
+ *   kernel_count       i64[n_ops]       attributed kernels
+ *   total_duration_ns  i64[n_ops]       sum of their durations
+ *   matched_count      i64[n_ops]       attributed kernels that have a row
+ *   agg                f64[20 * n_ops]  counter-major: agg[c * n_ops + op];
+ *                                       NaN where no non-null value exists */
+typedef struct {
+    int64_t *kernel_count;
+    int64_t *total_duration_ns;
+    int64_t *matched_count;
+    double *agg;
+} opattr_op_aggregates;
+
+/* Host-side totals of opattr_aggregate (Fig. 3 coverage). */
+typedef struct {
+    int64_t total_ns;              /* sum of all kernel durations */
+    int64_t attributed_ns;         /* kernels with range_of_kernel >= 0 */
+    int64_t unattributed_ns;       /* total_ns - attributed_ns */
+    int64_t kernels;
+    int64_t attributed_kernels;
+    int64_t matched_kernels;       /* attributed kernels with a row */
+    double attributed_frac;        /* attributed_ns / total_ns, NaN if total_ns == 0 */
+    double unattributed_frac;
+} opattr_totals;
+
+/* Create a context on `device` that orders its work on `cuda_stream` (a
+ * cudaStream_t; NULL = the legacy default stream).  `cfg` may be NULL for
+ * defaults.  The context owns reusable device scratch only.
+ * Errors: OPATTR_E_INVALID_ARG (out NULL, bad device or mode),
+ * OPATTR_E_CUDA. */
+opattr_status opattr_create(opattr_ctx **out, int device, void *cuda_stream, const opattr_config *cfg);
+
+/* Algorithm 2 for every kernel: range_of_kernel[k] = index of the innermost
+ * operator range enclosing kernel k, or -1; n_op_enclosing[k] = number of
+ * operator ranges collected by the walk (is_fused = value > 1).
+ * Per depth d the representative is the greatest (start, end, index) among
+ * depth-d ranges of the kernel's stream with start <= T <= end; the walk goes
+ * from the deepest representative outward, collects operators, skips
+ * OPATTR_OP_NONOP, stops at OPATTR_OP_STRUCTURAL.
+ * Reads kernels->stream, start_ns and all range fields.
+ *   range_of_kernel  i32[kernels->n]  device, required
+ *   n_op_enclosing   u8[kernels->n]   device, may be NULL
+ * Errors: OPATTR_E_INVALID_ARG (NULL arrays with n > 0, end < start, more
+ * than 2^30 ranges), OPATTR_E_DEPTH, OPATTR_E_NOT_NESTED, OPATTR_E_OOM,
+ * OPATTR_E_CUDA. */
+opattr_status opattr_enclose(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,
+                             int32_t *range_of_kernel, uint8_t *n_op_enclosing);
+
+/* Algorithm 1 with the context's mismatch mode.  ncu_idx_of_kernel[k] = ncu
+ * row of kernel k or -1; match_kind[k] = 0 none, 1 direct, 2 broadcast.
+ * Ordinals are taken over replayed kernels in time order and over rows in
+ * array order.  `dedup` (host) may be NULL; deduplication also needs
+ * kernels->layer_id and cfg.dedup = 1.
+ * Reads kernels->stream, start_ns, name_id (and layer_id), ncu->name_id.
+ *   ncu_idx_of_kernel  i32[kernels->n]  device, required
+ *   match_kind         u8[kernels->n]   device, may be NULL
+ *   host_summary       host, may be NULL
+ * Returns OPATTR_W_COUNT_MISMATCH (skip-name: some name mismatched; prefix:
+ * some kernel found no row), else OPATTR_W_DEDUP_MISMATCH when a duplicate
+ * found no source.  Errors: OPATTR_E_INVALID_ARG (layer id >= n_layers, bad
+ * tables), OPATTR_E_COUNT_MISMATCH (error mode), OPATTR_E_OOM, OPATTR_E_CUDA. */
+opattr_status opattr_match(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ncu *ncu,
+                           const opattr_dedup *dedup, int32_t *ncu_idx_of_kernel, uint8_t *match_kind,
+                           opattr_match_summary *host_summary);
+
+/* Eq. (1) per operator: for op = op_id[range_of_kernel[k]], counts and
+ * duration sums in int64 (exact); per counter, over attributed kernels with a
+ * row and a non-null value: SUM of values, MAX of values, or the
+ * duration-weighted mean sum(m*d)/sum(d) (Table 8 picks which); NaN for an
+ * empty set or a zero total weight.  Floating-point results are within 1e-9
+ * relative of an fp64 evaluation (float-float accumulation, see the design
+ * notes).  Every op id in [0, n_ops) is written.
+ * Reads kernels->dur_ns (and start_ns, stream for the fast path), range
+ * start_ns and op_id, ncu->counters.
+ *   range_of_kernel    i32[kernels->n]  device, values in [-1, ranges->n)
+ *   ncu_idx_of_kernel  i32[kernels->n]  device, values in [-1, ncu->n)
+ *   dev_out            host struct of device pointers, see above
+ *   host_totals        host, may be NULL
+ * Errors: OPATTR_E_INVALID_ARG (index out of range, attributed range that is
+ * not an operator below n_ops, negative duration, infinite counter, counters
+ * not 16-byte aligned),
+ * OPATTR_E_OOM, OPATTR_E_CUDA. */
+opattr_status opattr_aggregate(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,
+                               const int32_t *range_of_kernel, const opattr_ncu *ncu,
+                               const int32_t *ncu_idx_of_kernel, uint32_t n_ops,
+                               const opattr_op_aggregates *dev_out, opattr_totals *host_totals);
+
+/* Free the context and its scratch.  NULL is ignored. */
+void opattr_destroy(opattr_ctx *ctx);
+
+/* Static string for a status code. */
+const char *opattr_status_string(opattr_status status);
+
+/* Launch accounting and per-kernel timing.  With timing on, every kernel
+ * launch of the context is bracketed by CUDA events on the context's stream
+ * and its duration accumulated per kernel name.  opattr_timing_report fills
+ * up to `cap` entries (names are static strings) and returns how many kernel
+ * names have been seen; opattr_launch_count returns the number of kernels the
+ * context has launched since creation or the last reset. */
+opattr_status opattr_set_timing(opattr_ctx *ctx, int enable);
+int opattr_timing_report(opattr_ctx *ctx, const char **names, double *total_ms, int64_t *launches, int cap);
+void opattr_timing_reset(opattr_ctx *ctx);
+int64_t opattr_launch_count(const opattr_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* OPATTR_H */

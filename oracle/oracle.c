@@ -134,12 +134,12 @@ static int rep_greater(const ranges_t *r, int64_t a, int64_t b) {
     return a > b;
 }
 
-/* Argument checks shared by both modes: end >= start, depth <= 31. */
+/* Argument checks shared by both modes: end >= start, then depth <= 31. */
 static int check_range_fields(const ranges_t *r) {
-    for (int64_t i = 0; i < r->R; ++i) {
+    for (int64_t i = 0; i < r->R; ++i)
         if (r->end[i] < r->start[i]) return ORC_E_INVALID_ARG;
+    for (int64_t i = 0; i < r->R; ++i)
         if (r->depth[i] >= MAX_DEPTH) return ORC_E_DEPTH;
-    }
     return ORC_OK;
 }
 

@@ -1,0 +1,379 @@
+"""Python binding of libopattr, the GPU trace join for hardware-attributed
+operator profiling ("Hardware-Attributed Operator Profiling for PyTorch").
+
+Argument marshalling only: every step of the join runs in the CUDA kernels of
+``libopattr.so`` (``csrc/``), reached through its C ABI (``include/opattr.h``).
+PyTorch supplies device memory and the stream.  There is no CPU fallback: if
+the library cannot be loaded the import of the binding's functions raises.
+
+Function names follow the C ABI: ``opattr_create``, ``opattr_enclose``,
+``opattr_match``, ``opattr_aggregate``, ``opattr_destroy``; ``Context`` wraps
+them for torch tensors.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from dataclasses import dataclass
+
+from . import _build
+
+__all__ = [
+    "OK", "W_COUNT_MISMATCH", "W_DEDUP_MISMATCH", "E_INVALID_ARG", "E_NOT_NESTED", "E_DEPTH",
+    "E_COUNT_MISMATCH", "E_CUDA", "E_OOM", "E_TIMEOUT", "E_STATE", "OP_STRUCTURAL", "OP_NONOP",
+    "N_COUNTERS", "OpattrError", "Context", "library", "build",
+    "opattr_create", "opattr_enclose", "opattr_match", "opattr_aggregate", "opattr_destroy",
+    "opattr_status_string",
+]
+
+OK, W_COUNT_MISMATCH, W_DEDUP_MISMATCH = 0, 1, 2
+E_INVALID_ARG, E_NOT_NESTED, E_DEPTH, E_COUNT_MISMATCH = -1, -2, -3, -4
+E_CUDA, E_OOM, E_TIMEOUT, E_STATE = -5, -6, -7, -8
+OP_STRUCTURAL = 0xFFFFFFFF
+OP_NONOP = 0xFFFFFFFE
+N_COUNTERS = 20
+MISMATCH = {"skip_name": 0, "prefix": 1, "error": 2}
+
+_vp = ctypes.c_void_p
+
+
+class Kernels(ctypes.Structure):
+    _fields_ = [("stream", _vp), ("start_ns", _vp), ("dur_ns", _vp), ("name_id", _vp), ("layer_id", _vp),
+                ("n", ctypes.c_int64)]
+
+
+class Ranges(ctypes.Structure):
+    _fields_ = [("stream", _vp), ("start_ns", _vp), ("end_ns", _vp), ("depth", _vp), ("op_id", _vp),
+                ("n", ctypes.c_int64)]
+
+
+class Ncu(ctypes.Structure):
+    _fields_ = [("name_id", _vp), ("counters", _vp), ("n", ctypes.c_int64)]
+
+
+class Dedup(ctypes.Structure):
+    _fields_ = [("class_of_layer", _vp), ("rep_of_class", _vp), ("n_layers", ctypes.c_int32),
+                ("n_classes", ctypes.c_int32)]
+
+
+class Config(ctypes.Structure):
+    _fields_ = [("mismatch", ctypes.c_int), ("dedup", ctypes.c_int32), ("checked", ctypes.c_int32),
+                ("spin_limit", ctypes.c_int64)]
+
+
+class MatchSummary(ctypes.Structure):
+    _fields_ = [(f, ctypes.c_int64) for f in ("kernels", "replayed", "direct", "broadcast", "unmatched",
+                                              "names_mismatched", "count_unmatched", "dedup_mismatch")] + \
+               [("fast_path", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+    def as_dict(self) -> dict:
+        return {f: int(getattr(self, f)) for f, _ in self._fields_ if f != "reserved"}
+
+
+class OpAggregates(ctypes.Structure):
+    _fields_ = [("kernel_count", _vp), ("total_duration_ns", _vp), ("matched_count", _vp), ("agg", _vp)]
+
+
+class Totals(ctypes.Structure):
+    _fields_ = [(f, ctypes.c_int64) for f in ("total_ns", "attributed_ns", "unattributed_ns", "kernels",
+                                              "attributed_kernels", "matched_kernels")] + \
+               [("attributed_frac", ctypes.c_double), ("unattributed_frac", ctypes.c_double)]
+
+    def as_dict(self) -> dict:
+        return {f: getattr(self, f) for f, _ in self._fields_}
+
+
+_lib_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile libopattr.so for sm_103a (no-op when up to date)."""
+    return _build.build(force=force)
+
+
+def library():
+    """Load libopattr.so (building it first if needed).  Raises on failure."""
+    global _lib
+    with _lib_lock:
+        if _lib is None:
+            path = _build.LIB
+            if not os.path.exists(path) or os.environ.get("OPATTR_REBUILD"):
+                path = _build.build()
+            lib = ctypes.CDLL(path)
+            P = ctypes.POINTER
+            lib.opattr_create.argtypes = [P(_vp), ctypes.c_int, _vp, P(Config)]
+            lib.opattr_enclose.argtypes = [_vp, P(Kernels), P(Ranges), _vp, _vp]
+            lib.opattr_match.argtypes = [_vp, P(Kernels), P(Ncu), P(Dedup), _vp, _vp, P(MatchSummary)]
+            lib.opattr_aggregate.argtypes = [_vp, P(Kernels), P(Ranges), _vp, P(Ncu), _vp, ctypes.c_uint32,
+                                             P(OpAggregates), P(Totals)]
+            lib.opattr_destroy.argtypes = [_vp]
+            lib.opattr_destroy.restype = None
+            lib.opattr_status_string.argtypes = [ctypes.c_int]
+            lib.opattr_status_string.restype = ctypes.c_char_p
+            lib.opattr_set_timing.argtypes = [_vp, ctypes.c_int]
+            lib.opattr_timing_report.argtypes = [_vp, P(ctypes.c_char_p), P(ctypes.c_double), P(ctypes.c_int64),
+                                                 ctypes.c_int]
+            lib.opattr_timing_reset.argtypes = [_vp]
+            lib.opattr_timing_reset.restype = None
+            lib.opattr_launch_count.argtypes = [_vp]
+            lib.opattr_launch_count.restype = ctypes.c_int64
+            for f in ("opattr_create", "opattr_enclose", "opattr_match", "opattr_aggregate", "opattr_set_timing",
+                      "opattr_timing_report"):
+                getattr(lib, f).restype = ctypes.c_int
+            _lib = lib
+        return _lib
+
+
+class OpattrError(RuntimeError):
+    def __init__(self, status: int, call: str):
+        super().__init__(f"{call}: {opattr_status_string(status)} ({status})")
+        self.status = status
+
+
+def opattr_status_string(status: int) -> str:
+    return library().opattr_status_string(status).decode()
+
+
+# ---------------------------------------------------------------- C ABI, one to one
+def opattr_create(device: int = 0, stream: int | None = None, mismatch: str = "skip_name", dedup: bool = True,
+                  spin_limit: int = 0):
+    """Returns (status, handle)."""
+    cfg = Config(MISMATCH[mismatch], int(bool(dedup)), 0, int(spin_limit))
+    h = _vp()
+    st = library().opattr_create(ctypes.byref(h), int(device), _vp(stream or 0), ctypes.byref(cfg))
+    return st, h
+
+
+def opattr_enclose(handle, kernels: Kernels, ranges: Ranges, range_of_kernel_ptr: int, n_op_ptr: int | None) -> int:
+    return library().opattr_enclose(handle, ctypes.byref(kernels), ctypes.byref(ranges), _vp(range_of_kernel_ptr),
+                                    _vp(n_op_ptr or 0))
+
+
+def opattr_match(handle, kernels: Kernels, ncu: Ncu, dedup: Dedup | None, idx_ptr: int, kind_ptr: int | None,
+                 summary: MatchSummary) -> int:
+    return library().opattr_match(handle, ctypes.byref(kernels), ctypes.byref(ncu),
+                                  ctypes.byref(dedup) if dedup is not None else None, _vp(idx_ptr),
+                                  _vp(kind_ptr or 0), ctypes.byref(summary))
+
+
+def opattr_aggregate(handle, kernels: Kernels, ranges: Ranges, rok_ptr: int, ncu: Ncu, idx_ptr: int, n_ops: int,
+                     out: OpAggregates, totals: Totals) -> int:
+    return library().opattr_aggregate(handle, ctypes.byref(kernels), ctypes.byref(ranges), _vp(rok_ptr),
+                                      ctypes.byref(ncu), _vp(idx_ptr), ctypes.c_uint32(n_ops), ctypes.byref(out),
+                                      ctypes.byref(totals))
+
+
+def opattr_destroy(handle) -> None:
+    if handle:
+        library().opattr_destroy(handle)
+
+
+# ---------------------------------------------------------------- torch convenience layer
+def _ptr(t, dtype, name, device):
+    import torch
+    if t is None:
+        return None
+    ok = (t.dtype == dtype) or (dtype == torch.uint32 and t.dtype == torch.int32)
+    if not ok:
+        raise TypeError(f"{name}: expected {dtype}, got {t.dtype}")
+    if not t.is_cuda or t.device.index != device:
+        raise ValueError(f"{name}: must live on cuda:{device}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name}: must be contiguous")
+    return t.data_ptr() if t.numel() else None
+
+
+@dataclass
+class DeviceTrace:
+    """A trace's arrays as device tensors (see include/opattr.h for layouts)."""
+    k_stream: object
+    k_start: object
+    k_dur: object
+    k_name: object
+    k_layer: object
+    r_stream: object
+    r_start: object
+    r_end: object
+    r_depth: object
+    r_op: object
+    n_ops: int
+    ncu_name: object
+    counters: object
+    class_of_layer: object = None   # host (numpy / list) tables
+    rep_of_class: object = None
+
+    @property
+    def K(self):
+        return int(self.k_start.shape[0])
+
+    @property
+    def R(self):
+        return int(self.r_start.shape[0])
+
+    @property
+    def M(self):
+        return int(self.ncu_name.shape[0])
+
+
+def to_device(trace, device: int = 0, pin: bool = False) -> DeviceTrace:
+    """Copy a tracegen.Trace (numpy arrays) to the GPU as torch tensors."""
+    import torch
+
+    def d(a):
+        if a is None:
+            return None
+        t = torch.from_numpy(a)
+        if pin:
+            t = t.pin_memory()
+        return t.to(f"cuda:{device}", non_blocking=pin)
+
+    return DeviceTrace(d(trace.k_stream), d(trace.k_start), d(trace.k_dur), d(trace.k_name), d(trace.k_layer),
+                       d(trace.r_stream), d(trace.r_start), d(trace.r_end), d(trace.r_depth), d(trace.r_op),
+                       int(trace.n_ops), d(trace.ncu_name), d(trace.counters), trace.class_of_layer,
+                       trace.rep_of_class)
+
+
+class Context:
+    """An opattr context bound to one device and one CUDA stream."""
+
+    def __init__(self, device: int = 0, stream=None, mismatch: str = "skip_name", dedup: bool = True):
+        import torch
+        self.device = device
+        if stream is None:
+            stream = torch.cuda.current_stream(device)
+        self.stream = stream
+        st, self.handle = opattr_create(device, stream.cuda_stream, mismatch, dedup)
+        if st != OK:
+            raise OpattrError(st, "opattr_create")
+
+    def close(self):
+        if getattr(self, "handle", None):
+            opattr_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    # -- structs
+    def kernels(self, tr: DeviceTrace) -> Kernels:
+        import torch
+        dv = self.device
+        return Kernels(_ptr(tr.k_stream, torch.uint8, "k_stream", dv), _ptr(tr.k_start, torch.int64, "k_start", dv),
+                       _ptr(tr.k_dur, torch.int64, "k_dur", dv), _ptr(tr.k_name, torch.uint32, "k_name", dv),
+                       _ptr(tr.k_layer, torch.int32, "k_layer", dv), tr.K)
+
+    def ranges(self, tr: DeviceTrace) -> Ranges:
+        import torch
+        dv = self.device
+        return Ranges(_ptr(tr.r_stream, torch.uint8, "r_stream", dv), _ptr(tr.r_start, torch.int64, "r_start", dv),
+                      _ptr(tr.r_end, torch.int64, "r_end", dv), _ptr(tr.r_depth, torch.uint8, "r_depth", dv),
+                      _ptr(tr.r_op, torch.uint32, "r_op", dv), tr.R)
+
+    def ncu(self, tr: DeviceTrace) -> Ncu:
+        import torch
+        dv = self.device
+        return Ncu(_ptr(tr.ncu_name, torch.uint32, "ncu_name", dv), _ptr(tr.counters, torch.float32, "counters", dv),
+                   tr.M)
+
+    # -- calls
+    def enclose(self, tr: DeviceTrace, out_range=None, out_nop=None, need_nop: bool = True):
+        import torch
+        dev = f"cuda:{self.device}"
+        if out_range is None:
+            out_range = torch.empty(tr.K, dtype=torch.int32, device=dev)
+        if out_nop is None and need_nop:
+            out_nop = torch.empty(tr.K, dtype=torch.uint8, device=dev)
+        st = opattr_enclose(self.handle, self.kernels(tr), self.ranges(tr),
+                            _ptr(out_range, torch.int32, "range_of_kernel", self.device),
+                            _ptr(out_nop, torch.uint8, "n_op_enclosing", self.device) if out_nop is not None else None)
+        if st < 0:
+            raise OpattrError(st, "opattr_enclose")
+        return st, out_range, out_nop
+
+    def match(self, tr: DeviceTrace, dedup: bool | None = None, out_idx=None, out_kind=None):
+        import numpy as np
+        import torch
+        dev = f"cuda:{self.device}"
+        if out_idx is None:
+            out_idx = torch.empty(tr.K, dtype=torch.int32, device=dev)
+        if out_kind is None:
+            out_kind = torch.empty(tr.K, dtype=torch.uint8, device=dev)
+        dd = None
+        keep = None
+        use = (tr.class_of_layer is not None and tr.k_layer is not None) if dedup is None else dedup
+        if use:
+            col = np.ascontiguousarray(tr.class_of_layer, dtype=np.int32)
+            roc = np.ascontiguousarray(tr.rep_of_class, dtype=np.int32)
+            keep = (col, roc)
+            dd = Dedup(col.ctypes.data if col.size else None, roc.ctypes.data if roc.size else None, len(col), len(roc))
+        summ = MatchSummary()
+        st = opattr_match(self.handle, self.kernels(tr), self.ncu(tr), dd,
+                          _ptr(out_idx, torch.int32, "ncu_idx_of_kernel", self.device),
+                          _ptr(out_kind, torch.uint8, "match_kind", self.device), summ)
+        del keep
+        if st < 0:
+            raise OpattrError(st, "opattr_match")
+        return st, out_idx, out_kind, summ.as_dict()
+
+    def alloc_ops(self, n_ops: int):
+        import torch
+        dev = f"cuda:{self.device}"
+        return dict(kernel_count=torch.empty(n_ops, dtype=torch.int64, device=dev),
+                    total_duration_ns=torch.empty(n_ops, dtype=torch.int64, device=dev),
+                    matched_count=torch.empty(n_ops, dtype=torch.int64, device=dev),
+                    agg=torch.empty((N_COUNTERS, n_ops), dtype=torch.float64, device=dev))
+
+    def aggregate(self, tr: DeviceTrace, range_of_kernel, ncu_idx, ops=None):
+        import torch
+        if ops is None:
+            ops = self.alloc_ops(tr.n_ops)
+        dv = self.device
+        out = OpAggregates(_ptr(ops["kernel_count"], torch.int64, "kernel_count", dv),
+                           _ptr(ops["total_duration_ns"], torch.int64, "total_duration_ns", dv),
+                           _ptr(ops["matched_count"], torch.int64, "matched_count", dv),
+                           _ptr(ops["agg"], torch.float64, "agg", dv))
+        tot = Totals()
+        st = opattr_aggregate(self.handle, self.kernels(tr), self.ranges(tr),
+                              _ptr(range_of_kernel, torch.int32, "range_of_kernel", dv), self.ncu(tr),
+                              _ptr(ncu_idx, torch.int32, "ncu_idx_of_kernel", dv), tr.n_ops, out, tot)
+        if st < 0:
+            raise OpattrError(st, "opattr_aggregate")
+        return st, ops, tot.as_dict()
+
+    def run(self, tr: DeviceTrace, dedup: bool | None = None):
+        """enclose + match + aggregate on device-resident inputs."""
+        st_e, rk, nop = self.enclose(tr)
+        st_m, idx, kind, summ = self.match(tr, dedup=dedup)
+        st_a, ops, tot = self.aggregate(tr, rk, idx)
+        return dict(enclose_status=st_e, range_of_kernel=rk, n_op_enclosing=nop, match_status=st_m, ncu_idx=idx,
+                    match_kind=kind, summary=summ, aggregate_status=st_a, ops=ops, totals=tot)
+
+    # -- accounting
+    def set_timing(self, on: bool):
+        library().opattr_set_timing(self.handle, int(bool(on)))
+
+    def timing_report(self) -> dict:
+        lib = library()
+        n = lib.opattr_timing_report(self.handle, None, None, None, 0)
+        names = (ctypes.c_char_p * max(n, 1))()
+        ms = (ctypes.c_double * max(n, 1))()
+        cnt = (ctypes.c_int64 * max(n, 1))()
+        lib.opattr_timing_report(self.handle, names, ms, cnt, n)
+        return {names[i].decode(): (float(ms[i]), int(cnt[i])) for i in range(n)}
+
+    def timing_reset(self):
+        library().opattr_timing_reset(self.handle)
+
+    def launch_count(self) -> int:
+        return int(library().opattr_launch_count(self.handle))

@@ -1,0 +1,279 @@
+// api.cu -- the C ABI of libopattr: context life cycle, scratch arena, status
+// block, launch timing, and the three calls of the join.
+#include <stdlib.h>
+
+#include <algorithm>
+#include <new>
+
+#include "common.cuh"
+
+namespace opattr {
+
+opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges *rng, int32_t *out_range,
+                         uint8_t *out_nop);
+opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu, const opattr_dedup *dd,
+                       int32_t *out_idx, uint8_t *out_kind, opattr_match_summary *sum);
+opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_ranges *rng, const int32_t *rok,
+                           const opattr_ncu *ncu, const int32_t *nidx, uint32_t n_ops,
+                           const opattr_op_aggregates *out, opattr_totals *tot_out);
+
+opattr_status cuda_status(Ctx &c, cudaError_t e) {
+    if (e == cudaSuccess) e = c.last_error;
+    if (e == cudaSuccess) return OPATTR_OK;
+    c.last_error = e;
+    c.broken = true;
+    return OPATTR_E_CUDA;
+}
+
+// Grows the arena to at least `bytes`.  OPATTR_FAULT=alloc in the environment
+// makes growth fail, to exercise the out-of-memory path without a GPU fault.
+opattr_status ensure_arena(Ctx &c, size_t bytes) {
+    if (bytes <= c.arena_cap) return OPATTR_OK;
+    const char *fault = getenv("OPATTR_FAULT");
+    if (fault && strcmp(fault, "alloc") == 0) return OPATTR_E_OOM;
+    if (c.arena) {
+        if (cudaStreamSynchronize(c.stream) != cudaSuccess) return cuda_status(c, cudaGetLastError());
+        cudaFree(c.arena);
+        c.arena = nullptr;
+        c.arena_cap = 0;
+    }
+    size_t cap = std::max(bytes, (size_t)1 << 20);
+    cap = (cap + ((size_t)1 << 20) - 1) & ~(((size_t)1 << 20) - 1);
+    cudaError_t e = cudaMalloc(&c.arena, cap);
+    if (e == cudaErrorMemoryAllocation) {
+        cudaGetLastError();          // clear the sticky-free error state
+        c.arena = nullptr;
+        return OPATTR_E_OOM;
+    }
+    if (e != cudaSuccess) return cuda_status(c, e);
+    c.arena_cap = cap;
+    return OPATTR_OK;
+}
+
+opattr_status reset_status(Ctx &c) {
+    cudaError_t e = cudaMemcpyAsync(c.d_status, c.h_init, sizeof(DevStatus), cudaMemcpyHostToDevice, c.stream);
+    return e == cudaSuccess ? OPATTR_OK : cuda_status(c, e);
+}
+
+opattr_status read_status(Ctx &c) {
+    if (c.last_error != cudaSuccess) return cuda_status(c, c.last_error);
+    cudaError_t e = cudaMemcpyAsync(c.h_status, c.d_status, sizeof(DevStatus), cudaMemcpyDeviceToHost, c.stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(c.stream);
+    if (e != cudaSuccess) return cuda_status(c, e);
+    if (c.timing) timing_collect(c);
+    return OPATTR_OK;
+}
+
+int timing_slot(Ctx &c, const char *name) {
+    for (size_t i = 0; i < c.slots.size(); ++i)
+        if (c.slots[i].name == name || strcmp(c.slots[i].name, name) == 0) return (int)i;
+    c.slots.push_back(TimingSlot{name, 0.0, 0});
+    return (int)c.slots.size() - 1;
+}
+
+static cudaEvent_t take_event(Ctx &c) {
+    if (!c.event_pool.empty()) {
+        cudaEvent_t e = c.event_pool.back();
+        c.event_pool.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    cudaEventCreate(&e);
+    return e;
+}
+
+void timing_begin(Ctx &c, int, cudaEvent_t *e0, cudaEvent_t *e1) {
+    *e0 = take_event(c);
+    *e1 = take_event(c);
+    cudaEventRecord(*e0, c.stream);
+}
+
+void timing_end(Ctx &c, int slot, cudaEvent_t e0, cudaEvent_t e1) {
+    cudaEventRecord(e1, c.stream);
+    c.pending.push_back({slot, {e0, e1}});
+}
+
+void timing_collect(Ctx &c) {
+    for (auto &p : c.pending) {
+        float ms = 0.f;
+        if (cudaEventElapsedTime(&ms, p.second.first, p.second.second) == cudaSuccess) {
+            c.slots[p.first].total_ms += ms;
+            c.slots[p.first].launches += 1;
+        }
+        c.event_pool.push_back(p.second.first);
+        c.event_pool.push_back(p.second.second);
+    }
+    c.pending.clear();
+}
+
+// Each call runs with the context's device current and restores the caller's.
+struct DeviceGuard {
+    int prev = -1;
+    bool ok = true;
+    explicit DeviceGuard(int dev) {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        if (prev != dev) ok = cudaSetDevice(dev) == cudaSuccess;
+    }
+    ~DeviceGuard() {
+        int cur = -1;
+        if (prev >= 0 && cudaGetDevice(&cur) == cudaSuccess && cur != prev) cudaSetDevice(prev);
+    }
+};
+
+}  // namespace opattr
+
+using namespace opattr;
+
+struct opattr_ctx {
+    Ctx c;
+};
+
+extern "C" {
+
+opattr_status opattr_create(opattr_ctx **out, int device, void *cuda_stream, const opattr_config *cfg) {
+    if (!out) return OPATTR_E_INVALID_ARG;
+    *out = nullptr;
+    int ndev = 0;
+    if (cudaGetDeviceCount(&ndev) != cudaSuccess) {
+        cudaGetLastError();
+        return OPATTR_E_CUDA;
+    }
+    if (device < 0 || device >= ndev) return OPATTR_E_INVALID_ARG;
+    opattr_config conf{};
+    conf.mismatch = OPATTR_MISMATCH_SKIP_NAME;
+    conf.dedup = 1;
+    if (cfg) conf = *cfg;
+    if ((int)conf.mismatch < 0 || (int)conf.mismatch > 2 || conf.spin_limit < 0) return OPATTR_E_INVALID_ARG;
+    DeviceGuard g(device);
+    if (!g.ok) return OPATTR_E_CUDA;
+    opattr_ctx *x = new (std::nothrow) opattr_ctx();
+    if (!x) return OPATTR_E_OOM;
+    Ctx &c = x->c;
+    c.device = device;
+    c.stream = (cudaStream_t)cuda_stream;
+    c.cfg = conf;
+    bool fail = cudaMalloc(&c.d_status, sizeof(DevStatus)) != cudaSuccess;
+    fail = fail || cudaMallocHost(&c.h_status, sizeof(DevStatus)) != cudaSuccess;
+    fail = fail || cudaMallocHost(&c.h_init, sizeof(DevStatus)) != cudaSuccess;
+    if (fail) {
+        cudaGetLastError();
+        if (c.d_status) cudaFree(c.d_status);
+        if (c.h_status) cudaFreeHost(c.h_status);
+        if (c.h_init) cudaFreeHost(c.h_init);
+        delete x;
+        return OPATTR_E_OOM;
+    }
+    memset(c.h_init, 0, sizeof(DevStatus));
+    c.h_init->mm[MM_KSTART_MIN] = LLONG_MAX;
+    c.h_init->mm[MM_KSTART_MAX] = LLONG_MIN;
+    c.h_init->mm[MM_RSTART_MIN] = LLONG_MAX;
+    c.h_init->mm[MM_REND_MAX] = LLONG_MIN;
+    *c.h_status = *c.h_init;
+    *out = x;
+    return OPATTR_OK;
+}
+
+static opattr_status finish(Ctx &c, opattr_status st) {
+    if (c.last_error != cudaSuccess) return cuda_status(c, c.last_error);
+    if (st == OPATTR_E_CUDA) c.broken = true;
+    return st;
+}
+
+opattr_status opattr_enclose(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,
+                             int32_t *range_of_kernel, uint8_t *n_op_enclosing) {
+    if (!ctx || !kernels || !ranges) return OPATTR_E_INVALID_ARG;
+    Ctx &c = ctx->c;
+    if (c.broken) return OPATTR_E_STATE;
+    DeviceGuard g(c.device);
+    if (!g.ok) return OPATTR_E_CUDA;
+    return finish(c, do_enclose(c, kernels, ranges, range_of_kernel, n_op_enclosing));
+}
+
+opattr_status opattr_match(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ncu *ncu,
+                           const opattr_dedup *dedup, int32_t *ncu_idx_of_kernel, uint8_t *match_kind,
+                           opattr_match_summary *host_summary) {
+    if (!ctx || !kernels || !ncu) return OPATTR_E_INVALID_ARG;
+    Ctx &c = ctx->c;
+    if (c.broken) return OPATTR_E_STATE;
+    DeviceGuard g(c.device);
+    if (!g.ok) return OPATTR_E_CUDA;
+    return finish(c, do_match(c, kernels, ncu, dedup, ncu_idx_of_kernel, match_kind, host_summary));
+}
+
+opattr_status opattr_aggregate(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,
+                               const int32_t *range_of_kernel, const opattr_ncu *ncu,
+                               const int32_t *ncu_idx_of_kernel, uint32_t n_ops,
+                               const opattr_op_aggregates *dev_out, opattr_totals *host_totals) {
+    if (!ctx || !kernels || !ranges || !ncu) return OPATTR_E_INVALID_ARG;
+    Ctx &c = ctx->c;
+    if (c.broken) return OPATTR_E_STATE;
+    DeviceGuard g(c.device);
+    if (!g.ok) return OPATTR_E_CUDA;
+    return finish(c, do_aggregate(c, kernels, ranges, range_of_kernel, ncu, ncu_idx_of_kernel, n_ops, dev_out,
+                                  host_totals));
+}
+
+void opattr_destroy(opattr_ctx *ctx) {
+    if (!ctx) return;
+    Ctx &c = ctx->c;
+    {
+        DeviceGuard g(c.device);
+        cudaStreamSynchronize(c.stream);
+        if (c.arena) cudaFree(c.arena);
+        if (c.d_status) cudaFree(c.d_status);
+        if (c.h_status) cudaFreeHost(c.h_status);
+        if (c.h_init) cudaFreeHost(c.h_init);
+        for (auto &p : c.pending) {
+            cudaEventDestroy(p.second.first);
+            cudaEventDestroy(p.second.second);
+        }
+        for (cudaEvent_t e : c.event_pool) cudaEventDestroy(e);
+        cudaGetLastError();
+    }
+    delete ctx;
+}
+
+const char *opattr_status_string(opattr_status s) {
+    switch (s) {
+    case OPATTR_OK: return "ok";
+    case OPATTR_W_COUNT_MISMATCH: return "warning: kernel-name count mismatch";
+    case OPATTR_W_DEDUP_MISMATCH: return "warning: duplicate-layer kernel without representative row";
+    case OPATTR_E_INVALID_ARG: return "invalid argument";
+    case OPATTR_E_NOT_NESTED: return "ranges are not nested per stream";
+    case OPATTR_E_DEPTH: return "range depth above 31";
+    case OPATTR_E_COUNT_MISMATCH: return "kernel-name count mismatch";
+    case OPATTR_E_CUDA: return "CUDA error";
+    case OPATTR_E_OOM: return "out of device memory";
+    case OPATTR_E_TIMEOUT: return "device-side wait timed out";
+    case OPATTR_E_STATE: return "context unusable after a CUDA error";
+    }
+    return "unknown status";
+}
+
+opattr_status opattr_set_timing(opattr_ctx *ctx, int enable) {
+    if (!ctx) return OPATTR_E_INVALID_ARG;
+    ctx->c.timing = enable != 0;
+    return OPATTR_OK;
+}
+
+int opattr_timing_report(opattr_ctx *ctx, const char **names, double *total_ms, int64_t *launches, int cap) {
+    if (!ctx) return 0;
+    Ctx &c = ctx->c;
+    int n = (int)c.slots.size();
+    for (int i = 0; i < n && i < cap; ++i) {
+        if (names) names[i] = c.slots[i].name;
+        if (total_ms) total_ms[i] = c.slots[i].total_ms;
+        if (launches) launches[i] = c.slots[i].launches;
+    }
+    return n;
+}
+
+void opattr_timing_reset(opattr_ctx *ctx) {
+    if (!ctx) return;
+    for (auto &s : ctx->c.slots) { s.total_ms = 0.0; s.launches = 0; }
+    ctx->c.launches = 0;
+}
+
+int64_t opattr_launch_count(const opattr_ctx *ctx) { return ctx ? ctx->c.launches : 0; }
+
+}  // extern "C"

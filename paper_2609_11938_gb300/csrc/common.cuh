@@ -1,0 +1,199 @@
+// common.cuh -- context, scratch arena, launch accounting and device helpers
+// shared by the kernels of libopattr.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <string.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/opattr.h"
+
+namespace opattr {
+
+// ------------------------------------------------------------------ status block
+// One small struct in device memory per context, reset at the start of each
+// call and read back at its checkpoints.  Kernels never trap: they record
+// problems here and return.
+enum ErrBit : unsigned {
+    ERR_INVALID = 1u,     // bad id, value or size found on the device
+    ERR_NOT_NESTED = 2u,  // ranges are not laminar
+    ERR_DEPTH = 4u,       // depth > 31
+    ERR_TIMEOUT = 8u,     // a bounded wait gave up
+    ERR_COUNT = 16u,      // count mismatch in error mode
+};
+enum FlagBit : unsigned {
+    F_K_UNSORTED = 1u,    // kernels are not in (start, stream) order
+    F_R_UNSORTED = 2u,    // ranges are not in start order
+    F_LEVEL_FIXUP = 4u,   // equal starts in a level are not in end order
+    F_NAMES_DIFFER = 8u,  // ncu names differ from replayed names in time order
+    F_OP_DUP = 16u,       // two operator ranges share an op id
+    F_AGG_MISS = 32u,     // the owned-range aggregation missed kernels
+};
+enum CountSlot {
+    C_NAMES_MISMATCH = 0,
+    C_COUNT_UNMATCHED,
+    C_DIRECT,
+    C_BROADCAST,
+    C_DEDUP_MISMATCH,
+    C_REPLAYED,
+    C_TOTAL_NS,
+    C_ATTR_NS,
+    C_ATTR_K,
+    C_MATCHED_K,
+    C_AGG_SEEN,
+    C_UNMATCHED,
+    C_NSLOTS = 16
+};
+enum MinMaxSlot { MM_KSTART_MIN = 0, MM_KSTART_MAX, MM_RSTART_MIN, MM_REND_MAX, MM_NSLOTS = 8 };
+
+struct DevStatus {
+    unsigned int err;
+    unsigned int flags;
+    unsigned long long cnt[C_NSLOTS];
+    long long mm[MM_NSLOTS];
+};
+
+// ------------------------------------------------------------------ context
+struct TimingSlot {
+    const char *name;
+    double total_ms;
+    int64_t launches;
+};
+
+struct Ctx {
+    int device = 0;
+    cudaStream_t stream = nullptr;
+    opattr_config cfg{};
+    bool broken = false;
+    // scratch arena (bump allocation, reset per call)
+    char *arena = nullptr;
+    size_t arena_cap = 0, arena_used = 0;
+    // status block
+    DevStatus *d_status = nullptr;
+    DevStatus *h_status = nullptr;   // pinned mirror
+    DevStatus *h_init = nullptr;     // pinned reset template
+    // launch accounting
+    int64_t launches = 0;
+    bool timing = false;
+    std::vector<TimingSlot> slots;
+    std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> pending;
+    std::vector<cudaEvent_t> event_pool;
+    cudaError_t last_error = cudaSuccess;
+};
+
+// ------------------------------------------------------------------ scratch
+struct Arena {
+    Ctx &c;
+    explicit Arena(Ctx &ctx) : c(ctx) { c.arena_used = 0; }
+    template <typename T>
+    T *take(int64_t count) {
+        size_t bytes = (size_t)(count > 0 ? count : 1) * sizeof(T);
+        size_t at = (c.arena_used + 255) & ~(size_t)255;
+        if (at + bytes > c.arena_cap) return nullptr;
+        c.arena_used = at + bytes;
+        return reinterpret_cast<T *>(c.arena + at);
+    }
+};
+// Upper bound of an arena request made of several arrays (alignment slack included).
+struct Need {
+    size_t bytes = 0;
+    template <typename T>
+    Need &add(int64_t count) {
+        bytes += (((size_t)(count > 0 ? count : 1) * sizeof(T)) + 255) & ~(size_t)255;
+        return *this;
+    }
+};
+
+opattr_status ensure_arena(Ctx &c, size_t bytes);
+opattr_status reset_status(Ctx &c);
+opattr_status read_status(Ctx &c);      // D2H copy + stream synchronize
+opattr_status cuda_status(Ctx &c, cudaError_t e);
+int timing_slot(Ctx &c, const char *name);
+void timing_begin(Ctx &c, int slot, cudaEvent_t *e0, cudaEvent_t *e1);
+void timing_end(Ctx &c, int slot, cudaEvent_t e0, cudaEvent_t e1);
+void timing_collect(Ctx &c);             // after a stream synchronize
+
+// Launch a kernel on the context stream, counting it and (optionally) timing it.
+template <typename... KArgs, typename... Args>
+inline void launch(Ctx &c, const char *name, void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                   Args... args) {
+    if (grid.x == 0 || grid.y == 0 || grid.z == 0) return;
+    cudaEvent_t e0 = nullptr, e1 = nullptr;
+    int slot = -1;
+    if (c.timing) {
+        slot = timing_slot(c, name);
+        timing_begin(c, slot, &e0, &e1);
+    }
+    kern<<<grid, block, smem, c.stream>>>(args...);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess && c.last_error == cudaSuccess) c.last_error = e;
+    c.launches++;
+    if (c.timing) timing_end(c, slot, e0, e1);
+}
+
+inline unsigned grid_for(int64_t n, int per_block, unsigned cap = 1u << 30) {
+    int64_t g = (n + per_block - 1) / per_block;
+    if (g < 1) g = 1;
+    return (unsigned)(g > (int64_t)cap ? cap : g);
+}
+
+// ------------------------------------------------------------------ device helpers
+__device__ __forceinline__ unsigned lane_id() { return threadIdx.x & 31u; }
+__device__ __forceinline__ unsigned lanemask_lt() {
+    unsigned m;
+    asm volatile("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+    return m;
+}
+
+__device__ __forceinline__ void set_err(DevStatus *s, unsigned bit) { atomicOr(&s->err, bit); }
+__device__ __forceinline__ void set_flag(DevStatus *s, unsigned bit) { atomicOr(&s->flags, bit); }
+
+template <typename T>
+__device__ __forceinline__ T warp_sum(T v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+template <typename T>
+__device__ __forceinline__ T warp_inclusive_scan(T v) {
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        T u = __shfl_up_sync(0xffffffffu, v, o);
+        if ((int)lane_id() >= o) v += u;
+    }
+    return v;
+}
+
+// Exclusive scan over a block (blockDim.x a multiple of 32, <= 1024).
+// `warp_buf` holds 33 entries of shared memory.  Returns the exclusive prefix;
+// *total receives the block sum.
+template <typename T>
+__device__ __forceinline__ T block_exclusive_scan(T v, T *warp_buf, T *total) {
+    const unsigned w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    T inc = warp_inclusive_scan(v);
+    if (lane_id() == 31) warp_buf[w] = inc;
+    __syncthreads();
+    if (w == 0) {
+        T x = lane_id() < nw ? warp_buf[lane_id()] : T(0);
+        T xs = warp_inclusive_scan(x);
+        if (lane_id() < nw) warp_buf[lane_id()] = xs - x;
+        if (lane_id() == nw - 1) warp_buf[32] = xs;
+    }
+    __syncthreads();
+    T r = warp_buf[w] + inc - v;
+    if (total) *total = warp_buf[32];
+    __syncthreads();
+    return r;
+}
+
+template <typename T>
+__device__ __forceinline__ T block_sum(T v, T *warp_buf) {
+    T total;
+    block_exclusive_scan(v, warp_buf, &total);
+    return total;
+}
+
+}  // namespace opattr

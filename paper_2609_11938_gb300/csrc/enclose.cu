@@ -1,0 +1,523 @@
+// enclose.cu -- Algorithm 2 (NVTX enclosure attribution, Sec. 3.5) on the GPU.
+//
+// Data layout.  Ranges are regrouped into per-(stream, depth) level lists,
+// each in (start, end, index) order: lvl_start / lvl_end (i64) and lvl_info
+// (u32: range index in the low 30 bits, kind in the top 2: 0 operator,
+// 1 non-op, 2 structural).  lvl_off[level] gives the list bounds, level =
+// stream * 32 + depth.  Within a level ranges are disjoint or touching, so
+// "the last range with start <= T" is the only one that can contain T.
+//
+// Kernels are taken in time order, in tiles of ENC_TILE.  A window table
+// P[tile][level] (last level position with start <= the tile's first T) bounds,
+// per level, the ranges a tile can hit; the enclosure kernel stages those
+// windows in shared memory as 32-bit times relative to the tile start and
+// answers each kernel by one search per depth, walking depths outward-in
+// (0, 1, ...) until a depth has no containing range.  The walk state needs no
+// stack: a structural range resets the collection (everything above it is
+// beyond the cut); an operator becomes the innermost answer and counts;
+// a non-op range is passed over.
+#include <algorithm>
+
+#include "sort.cuh"
+#include "util.cuh"
+
+namespace opattr {
+
+constexpr int LEVELS = 256 * 32;
+constexpr int ENC_THREADS = 256;
+constexpr int ENC_TILE = 2048;          // kernels per tile
+constexpr int ENC_WIN_CAP = 5120;       // staged range entries per tile
+constexpr int ENC_ACT_CAP = 1024;       // active (stream, depth) levels per tile
+constexpr uint32_t KIND_OP = 0, KIND_NONOP = 1, KIND_STRUCT = 2;
+
+__device__ __forceinline__ uint32_t kind_of(uint32_t op) {
+    return op == OPATTR_OP_STRUCTURAL ? KIND_STRUCT : (op == OPATTR_OP_NONOP ? KIND_NONOP : KIND_OP);
+}
+
+// ------------------------------------------------------------------ range checks
+// end >= start, depth <= 31, start order of the array, min start / max end,
+// and a histogram of level keys (per block in shared memory, flushed with
+// one global atomic per non-empty bin).
+constexpr int RCHK_THREADS = 256;
+constexpr int RCHK_ITEMS = 16;
+__global__ void __launch_bounds__(RCHK_THREADS) k_check_ranges(const uint8_t *__restrict__ stream,
+                                                               const int64_t *__restrict__ start,
+                                                               const int64_t *__restrict__ end,
+                                                               const uint8_t *__restrict__ depth, int64_t n,
+                                                               uint32_t *__restrict__ level_hist, DevStatus *st) {
+    __shared__ uint32_t h[LEVELS];
+    __shared__ int flags;
+    __shared__ long long smin, smax;
+    for (int i = threadIdx.x; i < LEVELS; i += RCHK_THREADS) h[i] = 0;
+    if (threadIdx.x == 0) { flags = 0; smin = LLONG_MAX; smax = LLONG_MIN; }
+    __syncthreads();
+    const int64_t base = (int64_t)blockIdx.x * RCHK_THREADS * RCHK_ITEMS;
+    long long mn = LLONG_MAX, mx = LLONG_MIN;
+    int f = 0;
+    for (int it = 0; it < RCHK_ITEMS; ++it) {
+        int64_t i = base + it * RCHK_THREADS + threadIdx.x;
+        if (i >= n) break;
+        long long s = start[i], e = end[i];
+        unsigned d = depth[i];
+        if (e < s) f |= 1;
+        if (d >= OPATTR_MAX_DEPTH) f |= 2;
+        if (i + 1 < n && start[i + 1] < s) f |= 4;
+        mn = s < mn ? s : mn;
+        mx = e > mx ? e : mx;
+        if (d < OPATTR_MAX_DEPTH) atomicAdd(&h[stream[i] * 32 + d], 1u);
+    }
+    if (f) atomicOr(&flags, f);
+    atomicMin(&smin, mn);
+    atomicMax(&smax, mx);
+    __syncthreads();
+    for (int i = threadIdx.x; i < LEVELS; i += RCHK_THREADS)
+        if (h[i]) atomicAdd(&level_hist[i], h[i]);
+    if (threadIdx.x == 0) {
+        if (flags & 1) set_err(st, ERR_INVALID);
+        if (flags & 2) set_err(st, ERR_DEPTH);
+        if (flags & 4) set_flag(st, F_R_UNSORTED);
+        atomicMin(&st->mm[MM_RSTART_MIN], smin);
+        atomicMax(&st->mm[MM_REND_MAX], smax);
+    }
+}
+
+// ------------------------------------------------------------------ level lists
+__global__ void k_level_keys(const uint8_t *__restrict__ stream, const uint8_t *__restrict__ depth,
+                             const uint32_t *__restrict__ perm, int64_t n, uint32_t *__restrict__ keys) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        int64_t r = perm ? perm[i] : i;
+        keys[i] = (uint32_t)stream[r] * 32u + depth[r];
+    }
+}
+__global__ void k_time_key(const int64_t *__restrict__ t, const uint32_t *__restrict__ perm, int64_t n,
+                           long long tmin, uint64_t *__restrict__ keys) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        int64_t r = perm ? perm[i] : i;
+        keys[i] = (uint64_t)(t[r] - tmin);
+    }
+}
+__global__ void k_level_gather(const int64_t *__restrict__ start, const int64_t *__restrict__ end,
+                               const uint32_t *__restrict__ op, const uint32_t *__restrict__ perm, int64_t n,
+                               int64_t *__restrict__ ls, int64_t *__restrict__ le, uint32_t *__restrict__ li) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        uint32_t r = perm[i];
+        ls[i] = start[r];
+        le[i] = end[r];
+        li[i] = r | (kind_of(op[r]) << 30);
+    }
+}
+
+// Laminar checks over level positions: adjacent pairs of a level, and the
+// parent of every range at depth > 0 (the last range of level (s, d-1) that
+// starts no later; it must end no earlier).
+__global__ void k_validate_levels(const uint8_t *__restrict__ stream, const uint8_t *__restrict__ depth,
+                                  const int64_t *__restrict__ ls, const int64_t *__restrict__ le,
+                                  const uint32_t *__restrict__ li, const uint32_t *__restrict__ lvl_off, int64_t n,
+                                  DevStatus *st) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        uint32_t r = li[i] & 0x3FFFFFFFu;
+        uint32_t s = stream[r], d = depth[r];
+        uint32_t L = s * 32 + d;
+        long long a = ls[i], b = le[i];
+        if (i + 1 < (int64_t)lvl_off[L + 1]) {
+            long long a2 = ls[i + 1], b2 = le[i + 1];
+            if (a2 == a && b2 < b) set_flag(st, F_LEVEL_FIXUP);
+            else if (b > a2) set_err(st, ERR_NOT_NESTED);
+        }
+        if (d > 0) {
+            int64_t lo = lvl_off[L - 1], hi = lvl_off[L];
+            int64_t x = lo, y = hi;               // first position with start > a
+            while (x < y) {
+                int64_t m = (x + y) >> 1;
+                if (ls[m] <= a) x = m + 1; else y = m;
+            }
+            if (x == lo || le[x - 1] < b) set_err(st, ERR_NOT_NESTED);
+        }
+    }
+}
+
+// ------------------------------------------------------------------ window table
+// P[t * nl + l] = (last position p of level l with lvl_start[p] <= b_t) - level
+// start, or -1; b_t = start of the time-ordered kernel t*ENC_TILE for
+// t < nt, and of the last kernel for t = nt.
+__global__ void k_window_table(const int64_t *__restrict__ ls, const uint32_t *__restrict__ lvl_off,
+                               const uint16_t *__restrict__ level_of_compact, int nl,
+                               const int64_t *__restrict__ k_start, const uint32_t *__restrict__ korder, int64_t K,
+                               int64_t nt, int32_t *__restrict__ P) {
+    const int64_t total = (nt + 1) * nl;
+    for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < total; q += (int64_t)gridDim.x * blockDim.x) {
+        int64_t t = q / nl;
+        int l = (int)(q - t * nl);
+        int64_t pos = t < nt ? t * ENC_TILE : K - 1;
+        long long b = k_start[korder ? korder[pos] : pos];
+        uint32_t L = level_of_compact[l];
+        int64_t lo = lvl_off[L], hi = lvl_off[L + 1];
+        int64_t x = lo, y = hi;
+        while (x < y) {
+            int64_t m = (x + y) >> 1;
+            if (ls[m] <= b) x = m + 1; else y = m;
+        }
+        P[q] = (int32_t)(x - lo - 1);
+    }
+}
+
+// ------------------------------------------------------------------ enclosure
+struct EncArgs {
+    const uint8_t *k_stream;
+    const int64_t *k_start;
+    const uint32_t *korder;     // NULL = identity
+    int64_t K;
+    const int64_t *ls, *le;
+    const uint32_t *li;
+    const uint32_t *lvl_off;    // [LEVELS + 1]
+    const int32_t *P;           // [(nt + 1) * nl]
+    int nl;
+    int64_t nt;
+    const uint16_t *cbase;      // [256] first compact level of a stream
+    const uint8_t *ndepth;      // [256] levels of a stream (depths 0 .. n-1)
+    int32_t *out_range;
+    uint8_t *out_nop;
+};
+
+struct EncSmem {
+    uint32_t ws[ENC_WIN_CAP];       // staged start, relative to tile base (+1, clamped)
+    uint32_t we[ENC_WIN_CAP];       // staged end, same encoding
+    uint32_t wi[ENC_WIN_CAP];       // staged lvl_info
+    uint16_t act_off[ENC_ACT_CAP];  // window offset of an active level
+    uint16_t act_cnt[ENC_ACT_CAP];  // window length
+    int32_t act_gpos[ENC_ACT_CAP];  // global level position of the window's first entry (-1 none)
+    uint16_t sbase[256];            // first active slot of a present stream
+    uint32_t present[8];
+    uint32_t wbuf[33];
+    int slow;
+    int nact, nwin;
+};
+
+__device__ __forceinline__ uint32_t rel32(long long x, long long base) {
+    long long v = x - base + 1;
+    return v <= 0 ? 0u : (v >= 0xFFFFFFFFll ? 0xFFFFFFFFu : (uint32_t)v);
+}
+
+__global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    EncSmem &S = *reinterpret_cast<EncSmem *>(smem_raw);
+    const int64_t t = blockIdx.x;
+    const int64_t pos0 = t * ENC_TILE;
+    const int64_t cnt = A.K - pos0 < ENC_TILE ? A.K - pos0 : ENC_TILE;
+    if (threadIdx.x < 8) S.present[threadIdx.x] = 0;
+    __syncthreads();
+
+    constexpr int PER = ENC_TILE / ENC_THREADS;
+    uint8_t ks[PER];
+    long long kt[PER];
+    const long long tbase = A.k_start[A.korder ? A.korder[pos0] : pos0];
+#pragma unroll
+    for (int j = 0; j < PER; ++j) {
+        int64_t p = pos0 + j * ENC_THREADS + threadIdx.x;
+        if (j * ENC_THREADS + threadIdx.x < cnt) {
+            int64_t k = A.korder ? A.korder[p] : p;
+            ks[j] = A.k_stream[k];
+            kt[j] = A.k_start[k];
+            atomicOr(&S.present[ks[j] >> 5], 1u << (ks[j] & 31));
+        }
+    }
+    __syncthreads();
+
+    // active levels: the levels of every stream present in the tile
+    {
+        const unsigned s = threadIdx.x;        // ENC_THREADS == 256 streams
+        unsigned n = ((S.present[s >> 5] >> (s & 31)) & 1u) ? A.ndepth[s] : 0u;
+        unsigned tot;
+        unsigned off = block_exclusive_scan<unsigned>(n, S.wbuf, &tot);
+        S.sbase[s] = (uint16_t)(off < ENC_ACT_CAP ? off : ENC_ACT_CAP);
+        if (threadIdx.x == 0) S.nact = (int)tot;
+        __syncthreads();
+        if (tot <= ENC_ACT_CAP && n) {
+            for (unsigned d = 0; d < n; ++d) {
+                int l = A.cbase[s] + d;
+                int32_t lo = A.P[t * A.nl + l], hi = A.P[(t + 1) * A.nl + l];
+                int32_t first = lo < 0 ? 0 : lo;
+                int32_t c = hi - first + 1;
+                if (hi < 0) c = 0;
+                S.act_cnt[off + d] = (uint16_t)(c < 0xFFFF ? c : 0xFFFF);
+                S.act_gpos[off + d] = (int32_t)(A.lvl_off[s * 32 + d] + first);
+            }
+        }
+    }
+    __syncthreads();
+    long long tlast = kt[0];
+    {
+        // span of the tile: its last kernel (time order) minus its first
+        int64_t pl = pos0 + cnt - 1;
+        tlast = A.k_start[A.korder ? A.korder[pl] : pl];
+    }
+    int slow = S.nact > ENC_ACT_CAP || (tlast - tbase) >= 0xFFFFFFF0ll;
+    if (!slow) {
+        // window offsets: exclusive scan of counts over active slots
+        unsigned carry = 0;
+        for (int b = 0; b < S.nact; b += ENC_THREADS) {
+            int a = b + threadIdx.x;
+            unsigned c = a < S.nact ? S.act_cnt[a] : 0u;
+            unsigned tot;
+            unsigned off = block_exclusive_scan<unsigned>(c, S.wbuf, &tot);
+            if (a < S.nact) S.act_off[a] = (uint16_t)((carry + off) < 0xFFFF ? carry + off : 0xFFFF);
+            carry += tot;
+        }
+        if (threadIdx.x == 0) S.nwin = (int)carry;
+        __syncthreads();
+        slow = S.nwin > ENC_WIN_CAP;
+    }
+    if (!slow) {
+        // stage: one warp per active level
+        const unsigned w = threadIdx.x >> 5, lane = lane_id();
+        for (int a = w; a < S.nact; a += ENC_THREADS / 32) {
+            int c = S.act_cnt[a], o = S.act_off[a];
+            int64_t g = S.act_gpos[a];
+            for (int e = lane; e < c; e += 32) {
+                S.ws[o + e] = rel32(A.ls[g + e], tbase);
+                S.we[o + e] = rel32(A.le[g + e], tbase);
+                S.wi[o + e] = A.li[g + e];
+            }
+        }
+        __syncthreads();
+#pragma unroll
+        for (int j = 0; j < PER; ++j) {
+            if (j * ENC_THREADS + threadIdx.x >= cnt) break;
+            const unsigned s = ks[j];
+            const uint32_t T = rel32(kt[j], tbase);
+            const int nd = A.ndepth[s];
+            const int a0 = S.sbase[s];
+            int32_t ans = -1;
+            int nop = 0;
+            for (int d = 0; d < nd; ++d) {
+                int c = S.act_cnt[a0 + d], o = S.act_off[a0 + d];
+                int x = o, y = o + c;               // first staged entry with start > T
+                while (x < y) {
+                    int m = (x + y) >> 1;
+                    if (S.ws[m] <= T) x = m + 1; else y = m;
+                }
+                if (x == o || S.we[x - 1] < T) break;
+                uint32_t info = S.wi[x - 1];
+                uint32_t kind = info >> 30;
+                if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
+                else if (kind == KIND_OP) { ans = (int32_t)(info & 0x3FFFFFFFu); nop++; }
+            }
+            int64_t p = pos0 + j * ENC_THREADS + threadIdx.x;
+            int64_t k = A.korder ? A.korder[p] : p;
+            A.out_range[k] = ans;
+            if (A.out_nop) A.out_nop[k] = (uint8_t)nop;
+        }
+        return;
+    }
+    // slow tile: search the global level lists inside the window bounds
+#pragma unroll 1
+    for (int j = 0; j < PER; ++j) {
+        if (j * ENC_THREADS + threadIdx.x >= cnt) break;
+        const unsigned s = ks[j];
+        const long long T = kt[j];
+        const int nd = A.ndepth[s];
+        int32_t ans = -1;
+        int nop = 0;
+        for (int d = 0; d < nd; ++d) {
+            int l = A.cbase[s] + d;
+            int32_t lo = A.P[t * A.nl + l], hi = A.P[(t + 1) * A.nl + l];
+            if (hi < 0) break;
+            int64_t g0 = A.lvl_off[s * 32 + d];
+            int64_t x = g0 + (lo < 0 ? 0 : lo), y = g0 + hi + 1, o = x;
+            while (x < y) {
+                int64_t m = (x + y) >> 1;
+                if (A.ls[m] <= T) x = m + 1; else y = m;
+            }
+            if (x == o || A.le[x - 1] < T) break;
+            uint32_t info = A.li[x - 1];
+            uint32_t kind = info >> 30;
+            if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
+            else if (kind == KIND_OP) { ans = (int32_t)(info & 0x3FFFFFFFu); nop++; }
+        }
+        int64_t p = pos0 + j * ENC_THREADS + threadIdx.x;
+        int64_t k = A.korder ? A.korder[p] : p;
+        A.out_range[k] = ans;
+        if (A.out_nop) A.out_nop[k] = (uint8_t)nop;
+    }
+}
+
+__global__ void k_fill_unattributed(int32_t *out_range, uint8_t *out_nop, int64_t n) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        out_range[i] = -1;
+        if (out_nop) out_nop[i] = 0;
+    }
+}
+
+// ------------------------------------------------------------------ host
+static opattr_status status_from_err(unsigned err) {
+    if (err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
+    if (err & ERR_DEPTH) return OPATTR_E_DEPTH;
+    if (err & ERR_NOT_NESTED) return OPATTR_E_NOT_NESTED;
+    if (err & ERR_TIMEOUT) return OPATTR_E_TIMEOUT;
+    return OPATTR_OK;
+}
+
+opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges *rng, int32_t *out_range,
+                         uint8_t *out_nop) {
+    const int64_t K = kern->n, R = rng->n;
+    if (K < 0 || R < 0 || R >= (1ll << 30) || K >= (1ll << 31)) return OPATTR_E_INVALID_ARG;
+    if (K > 0 && (!kern->stream || !kern->start_ns || !out_range)) return OPATTR_E_INVALID_ARG;
+    if (R > 0 && (!rng->stream || !rng->start_ns || !rng->end_ns || !rng->depth || !rng->op_id))
+        return OPATTR_E_INVALID_ARG;
+
+    // scratch: range sort (u64 keys x2, values x2), level arrays, tables, kernel order
+    const int64_t nt = (K + ENC_TILE - 1) / ENC_TILE;
+    Need nd;
+    nd.add<uint32_t>(LEVELS + 1).add<uint32_t>(LEVELS + 1);
+    nd.add<uint64_t>(R).add<uint64_t>(R).add<uint32_t>(R).add<uint32_t>(R);
+    const int64_t part_n = std::max<int64_t>(scan_scratch_elems(radix_hist_elems(R)), scan_scratch_elems(LEVELS + 1));
+    nd.add<uint32_t>(radix_hist_elems(R)).add<uint32_t>(part_n);
+    nd.add<int64_t>(R).add<int64_t>(R).add<uint32_t>(R);
+    nd.add<uint16_t>(LEVELS).add<uint16_t>(256).add<uint8_t>(256);
+    nd.add<int32_t>((nt + 1) * (int64_t)LEVELS);
+    size_t need = nd.bytes + kernel_order_scratch(K) + 4096;
+    opattr_status st = ensure_arena(c, need);
+    if (st) return st;
+    Arena a(c);
+    if ((st = reset_status(c))) return st;
+
+    uint32_t *level_hist = a.take<uint32_t>(LEVELS + 1);
+    uint32_t *lvl_off = a.take<uint32_t>(LEVELS + 1);
+    cudaMemsetAsync(level_hist, 0, sizeof(uint32_t) * (LEVELS + 1), c.stream);
+    if (R > 0)
+        launch(c, "check_ranges", k_check_ranges, dim3(grid_for(R, RCHK_THREADS * RCHK_ITEMS)), dim3(RCHK_THREADS), 0,
+               rng->stream, rng->start_ns, rng->end_ns, rng->depth, R, level_hist, c.d_status);
+    check_kernel_order(c, kern->stream, kern->start_ns, K);
+    if ((st = read_status(c))) return st;
+    if ((st = status_from_err(c.h_status->err))) return st;
+    const bool k_sorted = !(c.h_status->flags & F_K_UNSORTED);
+    bool r_sorted = !(c.h_status->flags & F_R_UNSORTED);
+    const long long rmin = c.h_status->mm[MM_RSTART_MIN], rmax = c.h_status->mm[MM_REND_MAX];
+    const long long kmin = c.h_status->mm[MM_KSTART_MIN], kmax = c.h_status->mm[MM_KSTART_MAX];
+    if (K > 0 && (kmax - kmin) >= (1ll << 55)) return OPATTR_E_INVALID_ARG;
+
+    if (R == 0) {
+        if (K > 0)
+            launch(c, "fill_unattributed", k_fill_unattributed, dim3(grid_for(K, 256, 65535)), dim3(256), 0, out_range,
+                   out_nop, K);
+        return read_status(c);
+    }
+
+    // ---- level lists
+    uint64_t *rk0 = a.take<uint64_t>(R), *rk1 = a.take<uint64_t>(R);
+    uint32_t *rv0 = a.take<uint32_t>(R), *rv1 = a.take<uint32_t>(R);
+    uint32_t *hist = a.take<uint32_t>(radix_hist_elems(R));
+    uint32_t *part = a.take<uint32_t>(part_n);
+    int64_t *ls = a.take<int64_t>(R), *le = a.take<int64_t>(R);
+    uint32_t *li = a.take<uint32_t>(R);
+    if (!rk0 || !rk1 || !rv0 || !rv1 || !hist || !part || !ls || !le || !li) return OPATTR_E_OOM;
+    const unsigned g = grid_for(R, 256, 65535);
+    scan_exclusive_u32(c, level_hist, lvl_off, LEVELS + 1, part, nullptr);
+    for (int attempt = 0; attempt < 2; ++attempt) {
+        uint32_t *perm = nullptr;         // range indices in the order of the level sort
+        if (!r_sorted) {
+            // (start, end, index) order: sort by end, then stably by start
+            uint64_t *ko;
+            uint32_t *vo;
+            int bits = bits_for((uint64_t)(rmax - rmin));
+            launch(c, "range_time_key", k_time_key, dim3(g), dim3(256), 0, rng->end_ns, (const uint32_t *)nullptr, R,
+                   rmin, rk0);
+            radix_sort_pairs<uint64_t>(c, rk0, rv0, rk1, rv1, R, bits, true, hist, part, &ko, &vo);
+            uint64_t *kfree = ko == rk0 ? rk1 : rk0;
+            uint32_t *vfree = vo == rv0 ? rv1 : rv0;
+            launch(c, "range_time_key", k_time_key, dim3(g), dim3(256), 0, rng->start_ns, (const uint32_t *)vo, R,
+                   rmin, kfree);
+            radix_sort_pairs<uint64_t>(c, kfree, vo, ko, vfree, R, bits, false, hist, part, &ko, &perm);
+        }
+        // stable partition by level key (13 bits)
+        uint32_t *lk0 = reinterpret_cast<uint32_t *>(rk0), *lk1 = reinterpret_cast<uint32_t *>(rk1);
+        uint32_t *va = perm ? perm : rv0;
+        uint32_t *vb = perm == rv0 ? rv1 : (perm == rv1 ? rv0 : rv1);
+        launch(c, "level_keys", k_level_keys, dim3(g), dim3(256), 0, rng->stream, rng->depth, (const uint32_t *)perm, R,
+               lk0);
+        uint32_t *ko32, *lperm;
+        radix_sort_pairs<uint32_t>(c, lk0, va, lk1, vb, R, 13, perm == nullptr, hist, part, &ko32, &lperm);
+        launch(c, "level_gather", k_level_gather, dim3(g), dim3(256), 0, rng->start_ns, rng->end_ns, rng->op_id,
+               (const uint32_t *)lperm, R, ls, le, li);
+        launch(c, "validate_levels", k_validate_levels, dim3(grid_for(R, 256, 65535)), dim3(256), 0, rng->stream,
+               rng->depth, (const int64_t *)ls, (const int64_t *)le, (const uint32_t *)li, (const uint32_t *)lvl_off,
+               R, c.d_status);
+        if ((st = read_status(c))) return st;
+        if ((st = status_from_err(c.h_status->err))) return st;
+        if (!(c.h_status->flags & F_LEVEL_FIXUP)) break;
+        if (!r_sorted) return OPATTR_E_CUDA;     // a full sort leaves no equal-start disorder
+        r_sorted = false;
+        c.h_status->flags &= ~F_LEVEL_FIXUP;
+        cudaMemsetAsync(&c.d_status->flags, 0, sizeof(unsigned), c.stream);
+    }
+    if (K == 0) return OPATTR_OK;
+
+    // ---- compact level table (host side, from the level offsets)
+    std::vector<uint32_t> off(LEVELS + 1);
+    if (cudaMemcpyAsync(off.data(), lvl_off, sizeof(uint32_t) * (LEVELS + 1), cudaMemcpyDeviceToHost, c.stream) !=
+            cudaSuccess ||
+        cudaStreamSynchronize(c.stream) != cudaSuccess)
+        return cuda_status(c, cudaGetLastError());
+    std::vector<uint16_t> level_of_compact;
+    std::vector<uint16_t> cbase(256, 0);
+    std::vector<uint8_t> ndep(256, 0);
+    for (int s = 0; s < 256; ++s) {
+        cbase[s] = (uint16_t)level_of_compact.size();
+        int n = 0;
+        while (n < 32 && off[s * 32 + n + 1] > off[s * 32 + n]) {
+            level_of_compact.push_back((uint16_t)(s * 32 + n));
+            n++;
+        }
+        ndep[s] = (uint8_t)n;
+    }
+    const int nl = (int)level_of_compact.size();
+    uint16_t *d_loc = a.take<uint16_t>(LEVELS);
+    uint16_t *d_cbase = a.take<uint16_t>(256);
+    uint8_t *d_ndep = a.take<uint8_t>(256);
+    int32_t *P = a.take<int32_t>((nt + 1) * (int64_t)(nl > 0 ? nl : 1));
+    if (!d_loc || !d_cbase || !d_ndep || !P) return OPATTR_E_OOM;
+    cudaMemcpyAsync(d_loc, level_of_compact.data(), sizeof(uint16_t) * (nl > 0 ? nl : 1), cudaMemcpyHostToDevice,
+                    c.stream);
+    cudaMemcpyAsync(d_cbase, cbase.data(), sizeof(uint16_t) * 256, cudaMemcpyHostToDevice, c.stream);
+    cudaMemcpyAsync(d_ndep, ndep.data(), 256, cudaMemcpyHostToDevice, c.stream);
+
+    // ---- kernel time order
+    uint32_t *korder = nullptr;
+    if (!k_sorted) {
+        korder = kernel_time_order(c, a, kern->stream, kern->start_ns, K);
+        if (!korder) return OPATTR_E_OOM;
+    }
+    if (nl == 0) {
+        launch(c, "fill_unattributed", k_fill_unattributed, dim3(grid_for(K, 256, 65535)), dim3(256), 0, out_range,
+               out_nop, K);
+        return read_status(c);
+    }
+    launch(c, "window_table", k_window_table, dim3(grid_for((nt + 1) * nl, 256, 65535)), dim3(256), 0,
+           (const int64_t *)ls, (const uint32_t *)lvl_off, (const uint16_t *)d_loc, nl, kern->start_ns,
+           (const uint32_t *)korder, K, nt, P);
+    EncArgs A;
+    A.k_stream = kern->stream;
+    A.k_start = kern->start_ns;
+    A.korder = korder;
+    A.K = K;
+    A.ls = ls;
+    A.le = le;
+    A.li = li;
+    A.lvl_off = lvl_off;
+    A.P = P;
+    A.nl = nl;
+    A.nt = nt;
+    A.cbase = d_cbase;
+    A.ndepth = d_ndep;
+    A.out_range = out_range;
+    A.out_nop = out_nop;
+    static unsigned attr_done = 0;
+    if (c.device < 32 && !(attr_done & (1u << c.device))) {
+        cudaFuncSetAttribute(k_enclose, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(EncSmem));
+        attr_done |= 1u << c.device;
+    }
+    launch(c, "enclose", k_enclose, dim3((unsigned)nt), dim3(ENC_THREADS), sizeof(EncSmem), A);
+    return read_status(c);
+}
+
+}  // namespace opattr

@@ -1,0 +1,395 @@
+// match.cu -- Algorithm 1 (invocation-order matching, Sec. 3.3) and layer
+// deduplication broadcast (Sec. 3.7) on the GPU.
+//
+// Fast path.  When the replayed kernels, in time order, carry exactly the
+// names of the ncu rows in array order, launch i pairs with row i and no
+// ordinal is computed: one pass compares the two name arrays and writes the
+// identity.  Exports in time order with ncu replaying the same launches hit
+// this path.
+//
+// General path.  Ordinals come from stable radix sorts: replayed kernels in
+// time order sorted by name give o(k) = position - start of the name's run;
+// ncu rows in array order sorted by name give the rows of each name in
+// launch order.  The join is row = rows_of_name[o(k)], subject to the
+// mismatch mode.  Dedup positions come the same way from a stable sort of
+// layer-tagged kernels by layer id.
+#include <algorithm>
+
+#include "sort.cuh"
+#include "util.cuh"
+
+namespace opattr {
+
+// ------------------------------------------------------------------ fast path
+__global__ void k_match_identity(const uint32_t *__restrict__ kname, const uint32_t *__restrict__ nname, int64_t n,
+                                 int32_t *__restrict__ out_idx, uint8_t *__restrict__ out_kind, DevStatus *st) {
+    int bad = 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        bad |= kname[i] != nname[i];
+        out_idx[i] = (int32_t)i;
+        if (out_kind) out_kind[i] = 1;
+    }
+    if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_flag(st, F_NAMES_DIFFER);
+}
+
+// replayed kernels in time order (list rk) against rows 0..n-1
+__global__ void k_match_identity_list(const uint32_t *__restrict__ rk, const uint32_t *__restrict__ kname,
+                                      const uint32_t *__restrict__ nname, int64_t n, int32_t *__restrict__ out_idx,
+                                      uint8_t *__restrict__ out_kind, DevStatus *st) {
+    int bad = 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        uint32_t k = rk[i];
+        bad |= kname[k] != nname[i];
+        out_idx[k] = (int32_t)i;
+        if (out_kind) out_kind[k] = 1;
+    }
+    if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_flag(st, F_NAMES_DIFFER);
+}
+
+__global__ void k_fill_match(int32_t *out_idx, uint8_t *out_kind, int64_t n) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        out_idx[i] = -1;
+        if (out_kind) out_kind[i] = 0;
+    }
+}
+
+// ------------------------------------------------------------------ general path helpers
+// Flags in time order: flag[i] = predicate(korder[i]).
+//   what = 0: replayed (layer < 0 or the layer is its class representative)
+//   what = 1: layer-tagged (layer >= 0)
+__global__ void k_flags(const uint32_t *__restrict__ korder, const int32_t *__restrict__ layer,
+                        const int32_t *__restrict__ rep_layer, int64_t n, int what, uint32_t *__restrict__ flag) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        int64_t k = korder ? korder[i] : i;
+        int32_t l = layer ? layer[k] : -1;
+        uint32_t f = what == 0 ? (l < 0 || rep_layer[l] == l) : (l >= 0);
+        flag[i] = f;
+    }
+}
+// Compact: list[pos[i]] = korder[i] where flag[i]
+__global__ void k_compact(const uint32_t *__restrict__ korder, const uint32_t *__restrict__ flag,
+                          const uint32_t *__restrict__ pos, int64_t n, uint32_t *__restrict__ list) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        if (flag[i]) list[pos[i]] = korder ? korder[i] : (uint32_t)i;
+}
+__global__ void k_gather_u32(const uint32_t *__restrict__ src, const uint32_t *__restrict__ idx, int64_t n,
+                             uint32_t *__restrict__ dst) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        dst[i] = idx ? src[idx[i]] : src[i];
+}
+__global__ void k_gather_i32_as_u32(const int32_t *__restrict__ src, const uint32_t *__restrict__ idx, int64_t n,
+                                    uint32_t *__restrict__ dst) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        dst[i] = (uint32_t)src[idx[i]];
+}
+__global__ void k_max_u32(const uint32_t *__restrict__ a, int64_t n, unsigned long long *out) {
+    uint32_t m = 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        m = a[i] > m ? a[i] : m;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        uint32_t x = __shfl_xor_sync(0xffffffffu, m, o);
+        m = x > m ? x : m;
+    }
+    if (lane_id() == 0 && m) atomicMax(out, (unsigned long long)m);
+}
+__global__ void k_check_layers(const int32_t *__restrict__ layer, int64_t n, int32_t n_layers,
+                               const int32_t *__restrict__ rep_layer, DevStatus *st) {
+    unsigned long long rep = 0;
+    int bad = 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        int32_t l = layer[i];
+        if (l < -1 || l >= n_layers) bad = 1;
+        else rep += (l < 0 || rep_layer[l] == l);
+    }
+    rep = warp_sum(rep);
+    if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_err(st, ERR_INVALID);
+    if (lane_id() == 0 && rep) atomicAdd(&st->cnt[C_REPLAYED], rep);
+}
+
+__device__ __forceinline__ int64_t lower_bound_u32(const uint32_t *a, int64_t n, uint32_t x) {
+    int64_t lo = 0, hi = n;
+    while (lo < hi) {
+        int64_t m = (lo + hi) >> 1;
+        if (a[m] < x) lo = m + 1; else hi = m;
+    }
+    return lo;
+}
+__device__ __forceinline__ int64_t upper_bound_u32(const uint32_t *a, int64_t n, uint32_t x) {
+    int64_t lo = 0, hi = n;
+    while (lo < hi) {
+        int64_t m = (lo + hi) >> 1;
+        if (a[m] <= x) lo = m + 1; else hi = m;
+    }
+    return lo;
+}
+
+// The ordinal join.  i runs over replayed kernels sorted by (name, time).
+//   skn / skj: sorted names, and the time rank j of each (rk[j] = kernel)
+//   snn / snj: ncu names sorted, and the row index of each
+__global__ void k_ordinal_join(const uint32_t *__restrict__ skn, const uint32_t *__restrict__ skj,
+                               const uint32_t *__restrict__ rk, int64_t nrep, const uint32_t *__restrict__ snn,
+                               const uint32_t *__restrict__ snj, int64_t M, int mode, int32_t *__restrict__ out_idx,
+                               uint8_t *__restrict__ out_kind, DevStatus *st) {
+    unsigned long long direct = 0, unmatched = 0, names_bad = 0;
+    int err = 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nrep; i += (int64_t)gridDim.x * blockDim.x) {
+        uint32_t name = skn[i];
+        bool head = i == 0 || skn[i - 1] != name;
+        int64_t lo = head ? i : lower_bound_u32(skn, nrep, name);
+        int64_t ck = upper_bound_u32(skn, nrep, name) - lo;
+        int64_t b = lower_bound_u32(snn, M, name);
+        int64_t cq = upper_bound_u32(snn, M, name) - b;
+        int64_t o = i - lo;
+        bool ok = mode == OPATTR_MISMATCH_SKIP_NAME ? (ck == cq) : (o < cq);
+        if (mode == OPATTR_MISMATCH_ERROR && ck != cq) err = 1;
+        int32_t idx = ok && o < cq ? (int32_t)snj[b + o] : -1;
+        uint32_t k = rk[skj[i]];
+        out_idx[k] = idx;
+        if (out_kind) out_kind[k] = idx >= 0 ? 1 : 0;
+        direct += idx >= 0;
+        unmatched += idx < 0;
+        names_bad += head && ck != cq;
+    }
+    direct = warp_sum(direct);
+    unmatched = warp_sum(unmatched);
+    names_bad = warp_sum(names_bad);
+    if (__any_sync(0xffffffffu, err) && lane_id() == 0) set_err(st, ERR_COUNT);
+    if (lane_id() == 0) {
+        if (direct) atomicAdd(&st->cnt[C_DIRECT], direct);
+        if (unmatched) atomicAdd(&st->cnt[C_COUNT_UNMATCHED], unmatched);
+        if (names_bad) atomicAdd(&st->cnt[C_NAMES_MISMATCH], names_bad);
+    }
+}
+
+// Names that have ncu rows but no replayed kernel at all.
+__global__ void k_ncu_only_names(const uint32_t *__restrict__ snn, int64_t M, const uint32_t *__restrict__ skn,
+                                 int64_t nrep, int mode, DevStatus *st) {
+    unsigned long long bad = 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < M; i += (int64_t)gridDim.x * blockDim.x) {
+        uint32_t name = snn[i];
+        if (i > 0 && snn[i - 1] == name) continue;
+        int64_t lo = lower_bound_u32(skn, nrep, name);
+        bad += lo == nrep || skn[lo] != name;
+    }
+    bad = warp_sum(bad);
+    if (lane_id() == 0 && bad) {
+        atomicAdd(&st->cnt[C_NAMES_MISMATCH], bad);
+        if (mode == OPATTR_MISMATCH_ERROR) set_err(st, ERR_COUNT);
+    }
+}
+
+// Broadcast.  i runs over layer-tagged kernels sorted by (layer, time).
+//   sll / slj: sorted layer ids and the time rank j of each (lk[j] = kernel)
+__global__ void k_dedup_broadcast(const uint32_t *__restrict__ sll, const uint32_t *__restrict__ slj,
+                                  const uint32_t *__restrict__ lk, int64_t nl, const int32_t *__restrict__ rep_layer,
+                                  const uint32_t *__restrict__ kname, int32_t *__restrict__ out_idx,
+                                  uint8_t *__restrict__ out_kind, DevStatus *st) {
+    unsigned long long bc = 0, miss = 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nl; i += (int64_t)gridDim.x * blockDim.x) {
+        uint32_t L = sll[i];
+        int32_t rep = rep_layer[L];
+        if ((uint32_t)rep == L) continue;                        // the representative itself: replayed
+        int64_t lo = (i == 0 || sll[i - 1] != L) ? i : lower_bound_u32(sll, nl, L);
+        int64_t p = i - lo;
+        int64_t rlo = lower_bound_u32(sll, nl, (uint32_t)rep);
+        int64_t rn = upper_bound_u32(sll, nl, (uint32_t)rep) - rlo;
+        uint32_t k = lk[slj[i]];
+        int32_t idx = -1;
+        if (p < rn) {
+            uint32_t src = lk[slj[rlo + p]];
+            if (kname[src] == kname[k]) idx = out_idx[src];
+        }
+        out_idx[k] = idx;
+        if (out_kind) out_kind[k] = idx >= 0 ? 2 : 0;
+        bc += idx >= 0;
+        miss += idx < 0;
+    }
+    bc = warp_sum(bc);
+    miss = warp_sum(miss);
+    if (lane_id() == 0) {
+        if (bc) atomicAdd(&st->cnt[C_BROADCAST], bc);
+        if (miss) atomicAdd(&st->cnt[C_DEDUP_MISMATCH], miss);
+    }
+}
+
+// ------------------------------------------------------------------ host
+__global__ void k_iota(uint32_t *dst, int64_t n) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        dst[i] = (uint32_t)i;
+}
+
+static opattr_status read_u64(Ctx &c, const unsigned long long *d, unsigned long long *h) {
+    if (cudaMemcpyAsync(h, d, sizeof(*h), cudaMemcpyDeviceToHost, c.stream) != cudaSuccess ||
+        cudaStreamSynchronize(c.stream) != cudaSuccess)
+        return cuda_status(c, cudaGetLastError());
+    return OPATTR_OK;
+}
+
+opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu, const opattr_dedup *dd,
+                       int32_t *out_idx, uint8_t *out_kind, opattr_match_summary *sum) {
+    const int64_t K = kern->n, M = ncu->n;
+    if (K < 0 || M < 0 || K >= (1ll << 31) || M >= (1ll << 31)) return OPATTR_E_INVALID_ARG;
+    if (K > 0 && (!kern->stream || !kern->start_ns || !kern->name_id || !out_idx)) return OPATTR_E_INVALID_ARG;
+    if (M > 0 && !ncu->name_id) return OPATTR_E_INVALID_ARG;
+    const int mode = (int)c.cfg.mismatch;
+    const bool dedup_on = c.cfg.dedup && dd && kern->layer_id;
+    std::vector<int32_t> rep_layer;
+    if (dedup_on) {
+        if (dd->n_layers < 0 || dd->n_classes < 0 || (dd->n_layers > 0 && !dd->class_of_layer) ||
+            (dd->n_classes > 0 && !dd->rep_of_class))
+            return OPATTR_E_INVALID_ARG;
+        for (int32_t l = 0; l < dd->n_layers; ++l)
+            if (dd->class_of_layer[l] < 0 || dd->class_of_layer[l] >= dd->n_classes) return OPATTR_E_INVALID_ARG;
+        for (int32_t q = 0; q < dd->n_classes; ++q) {
+            int32_t r = dd->rep_of_class[q];
+            if (r < 0 || r >= dd->n_layers || dd->class_of_layer[r] != q) return OPATTR_E_INVALID_ARG;
+        }
+        rep_layer.resize(dd->n_layers > 0 ? dd->n_layers : 1);
+        for (int32_t l = 0; l < dd->n_layers; ++l) rep_layer[l] = dd->rep_of_class[dd->class_of_layer[l]];
+    }
+    const int64_t NL = dedup_on ? (dd->n_layers > 0 ? dd->n_layers : 1) : 1;
+    const int64_t NX = std::max(K, M);
+    Need nd;
+    nd.add<int32_t>(NL);
+    for (int i = 0; i < 5; ++i) nd.add<uint32_t>(K);                 // flag, pos, rk, lk, keys
+    for (int i = 0; i < 3; ++i) nd.add<uint32_t>(NX);                // sort buffers
+    for (int i = 0; i < 4; ++i) nd.add<uint32_t>(M);                 // ncu sort
+    nd.add<uint32_t>(radix_hist_elems(NX)).add<uint32_t>(scan_scratch_elems(std::max(radix_hist_elems(NX), K)));
+    nd.add<unsigned long long>(2);
+    size_t need = nd.bytes + kernel_order_scratch(K) + 4096;
+    opattr_status st = ensure_arena(c, need);
+    if (st) return st;
+    Arena a(c);
+    if ((st = reset_status(c))) return st;
+    int32_t *d_rep = a.take<int32_t>(NL);
+    uint32_t *flag = a.take<uint32_t>(K), *pos = a.take<uint32_t>(K), *rk = a.take<uint32_t>(K);
+    uint32_t *lk = a.take<uint32_t>(K), *k0 = a.take<uint32_t>(K);
+    uint32_t *s0 = a.take<uint32_t>(NX), *s1 = a.take<uint32_t>(NX), *s2 = a.take<uint32_t>(NX);
+    uint32_t *n0 = a.take<uint32_t>(M), *n1 = a.take<uint32_t>(M), *n2 = a.take<uint32_t>(M), *n3 = a.take<uint32_t>(M);
+    uint32_t *hist = a.take<uint32_t>(radix_hist_elems(NX));
+    uint32_t *part = a.take<uint32_t>(scan_scratch_elems(std::max(radix_hist_elems(NX), K)));
+    unsigned long long *dsm = a.take<unsigned long long>(2);
+    if (!d_rep || !flag || !pos || !rk || !lk || !k0 || !s0 || !s1 || !s2 || !n0 || !n1 || !n2 || !n3 || !hist ||
+        !part || !dsm)
+        return OPATTR_E_OOM;
+    if (dedup_on && dd->n_layers > 0)
+        cudaMemcpyAsync(d_rep, rep_layer.data(), sizeof(int32_t) * dd->n_layers, cudaMemcpyHostToDevice, c.stream);
+
+    const unsigned gK = grid_for(K, 256, 65535);
+    check_kernel_order(c, kern->stream, kern->start_ns, K);
+    if (dedup_on && K > 0)
+        launch(c, "check_layers", k_check_layers, dim3(gK), dim3(256), 0, kern->layer_id, K, dd->n_layers,
+               (const int32_t *)d_rep, c.d_status);
+    const bool try_identity = !dedup_on && K == M && K > 0;
+    if (try_identity)
+        launch(c, "match_identity", k_match_identity, dim3(gK), dim3(256), 0, kern->name_id, ncu->name_id, K, out_idx,
+               out_kind, c.d_status);
+    if ((st = read_status(c))) return st;
+    if (c.h_status->err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
+    const bool k_sorted = !(c.h_status->flags & F_K_UNSORTED);
+    opattr_match_summary S{};
+    S.kernels = K;
+    S.replayed = dedup_on ? (int64_t)c.h_status->cnt[C_REPLAYED] : K;
+    if (try_identity && k_sorted && !(c.h_status->flags & F_NAMES_DIFFER)) {
+        S.direct = K;
+        S.fast_path = 1;
+        if (sum) *sum = S;
+        return OPATTR_OK;
+    }
+
+    // ---- general path
+    if (K > 0) launch(c, "fill_match", k_fill_match, dim3(gK), dim3(256), 0, out_idx, out_kind, K);
+    uint32_t *korder = nullptr;
+    if (!k_sorted && K > 0) {
+        korder = kernel_time_order(c, a, kern->stream, kern->start_ns, K);
+        if (!korder) return OPATTR_E_OOM;
+    }
+    // rk[j] = kernel index of the j-th replayed kernel in time order
+    int64_t nrep = K;
+    if (dedup_on && K > 0) {
+        launch(c, "flags", k_flags, dim3(gK), dim3(256), 0, (const uint32_t *)korder, kern->layer_id,
+               (const int32_t *)d_rep, K, 0, flag);
+        scan_exclusive_u32(c, flag, pos, K, part, nullptr);
+        launch(c, "compact", k_compact, dim3(gK), dim3(256), 0, (const uint32_t *)korder, (const uint32_t *)flag,
+               (const uint32_t *)pos, K, rk);
+        nrep = S.replayed;
+    } else if (K > 0) {
+        if (korder) cudaMemcpyAsync(rk, korder, sizeof(uint32_t) * K, cudaMemcpyDeviceToDevice, c.stream);
+        else launch(c, "iota", k_iota, dim3(gK), dim3(256), 0, rk, K);
+    }
+    bool direct_done = false;
+    if (dedup_on && nrep == M && nrep > 0) {
+        launch(c, "match_identity_list", k_match_identity_list, dim3(grid_for(nrep, 256, 65535)), dim3(256), 0,
+               (const uint32_t *)rk, kern->name_id, ncu->name_id, nrep, out_idx, out_kind, c.d_status);
+        if ((st = read_status(c))) return st;
+        direct_done = !(c.h_status->flags & F_NAMES_DIFFER);
+        if (direct_done) S.fast_path = 1;
+        else launch(c, "fill_match", k_fill_match, dim3(gK), dim3(256), 0, out_idx, out_kind, K);
+    }
+    if (!direct_done && (nrep > 0 || M > 0)) {
+        cudaMemsetAsync(dsm, 0, sizeof(unsigned long long), c.stream);
+        if (nrep > 0) {
+            launch(c, "gather_names", k_gather_u32, dim3(grid_for(nrep, 256, 65535)), dim3(256), 0, kern->name_id,
+                   (const uint32_t *)rk, nrep, k0);
+            launch(c, "max_name", k_max_u32, dim3(grid_for(nrep, 256, 4096)), dim3(256), 0, (const uint32_t *)k0, nrep,
+                   dsm);
+        }
+        if (M > 0) {
+            cudaMemcpyAsync(n0, ncu->name_id, sizeof(uint32_t) * M, cudaMemcpyDeviceToDevice, c.stream);
+            launch(c, "max_name", k_max_u32, dim3(grid_for(M, 256, 4096)), dim3(256), 0, (const uint32_t *)n0, M, dsm);
+        }
+        unsigned long long hmax = 0;
+        if ((st = read_u64(c, dsm, &hmax))) return st;
+        const int bits = bits_for(hmax);
+        uint32_t *skn = nullptr, *skj = nullptr, *snn = n0, *snj = n1;
+        if (nrep > 0) radix_sort_pairs<uint32_t>(c, k0, s0, s1, s2, nrep, bits, true, hist, part, &skn, &skj);
+        if (M > 0) radix_sort_pairs<uint32_t>(c, n0, n1, n2, n3, M, bits, true, hist, part, &snn, &snj);
+        if (nrep > 0)
+            launch(c, "ordinal_join", k_ordinal_join, dim3(grid_for(nrep, 256, 65535)), dim3(256), 0,
+                   (const uint32_t *)skn, (const uint32_t *)skj, (const uint32_t *)rk, nrep, (const uint32_t *)snn,
+                   (const uint32_t *)snj, M, mode, out_idx, out_kind, c.d_status);
+        if (M > 0)
+            launch(c, "ncu_only_names", k_ncu_only_names, dim3(grid_for(M, 256, 65535)), dim3(256), 0,
+                   (const uint32_t *)snn, M, (const uint32_t *)skn, nrep, mode, c.d_status);
+    }
+    if (dedup_on && K > 0) {
+        // positions within layers: layer-tagged kernels in time order, sorted by layer
+        launch(c, "flags", k_flags, dim3(gK), dim3(256), 0, (const uint32_t *)korder, kern->layer_id,
+               (const int32_t *)d_rep, K, 1, flag);
+        uint32_t *ntag = reinterpret_cast<uint32_t *>(dsm + 1);
+        scan_exclusive_u32(c, flag, pos, K, part, ntag);
+        launch(c, "compact", k_compact, dim3(gK), dim3(256), 0, (const uint32_t *)korder, (const uint32_t *)flag,
+               (const uint32_t *)pos, K, lk);
+        unsigned long long ntag_h = 0;
+        if ((st = read_u64(c, dsm + 1, &ntag_h))) return st;
+        const int64_t nlk = (int64_t)(ntag_h & 0xFFFFFFFFull);
+        if (nlk > 0) {
+            launch(c, "gather_layers", k_gather_i32_as_u32, dim3(grid_for(nlk, 256, 65535)), dim3(256), 0,
+                   kern->layer_id, (const uint32_t *)lk, nlk, k0);
+            uint32_t *sll, *slj;
+            radix_sort_pairs<uint32_t>(c, k0, s0, s1, s2, nlk,
+                                       bits_for((uint64_t)(dd->n_layers > 0 ? dd->n_layers - 1 : 0)), true, hist, part,
+                                       &sll, &slj);
+            launch(c, "dedup_broadcast", k_dedup_broadcast, dim3(grid_for(nlk, 256, 65535)), dim3(256), 0,
+                   (const uint32_t *)sll, (const uint32_t *)slj, (const uint32_t *)lk, nlk, (const int32_t *)d_rep,
+                   kern->name_id, out_idx, out_kind, c.d_status);
+        }
+    }
+    if ((st = read_status(c))) return st;
+    const DevStatus &H = *c.h_status;
+    if (H.err & ERR_COUNT) return OPATTR_E_COUNT_MISMATCH;
+    S.direct = direct_done ? nrep : (int64_t)H.cnt[C_DIRECT];
+    S.broadcast = (int64_t)H.cnt[C_BROADCAST];
+    S.names_mismatched = (int64_t)H.cnt[C_NAMES_MISMATCH];
+    S.count_unmatched = direct_done ? 0 : (int64_t)H.cnt[C_COUNT_UNMATCHED];
+    S.dedup_mismatch = (int64_t)H.cnt[C_DEDUP_MISMATCH];
+    S.unmatched = K - S.direct - S.broadcast;
+    if (sum) *sum = S;
+    if (mode == OPATTR_MISMATCH_SKIP_NAME && S.names_mismatched > 0) return OPATTR_W_COUNT_MISMATCH;
+    if (mode == OPATTR_MISMATCH_PREFIX && S.count_unmatched > 0) return OPATTR_W_COUNT_MISMATCH;
+    if (S.dedup_mismatch > 0) return OPATTR_W_DEDUP_MISMATCH;
+    return OPATTR_OK;
+}
+
+}  // namespace opattr

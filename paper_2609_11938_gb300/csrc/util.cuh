@@ -1,0 +1,21 @@
+// util.cuh -- steps shared by the three calls: kernel time-order check and
+// time-order permutation.
+#pragma once
+#include "common.cuh"
+
+namespace opattr {
+
+// Sets F_K_UNSORTED unless (start_ns, stream) is non-decreasing along the
+// array, and records min / max start in MM_KSTART_MIN / MM_KSTART_MAX.
+void check_kernel_order(Ctx &c, const uint8_t *stream, const int64_t *start, int64_t n);
+
+// Scratch (bytes) of kernel_time_order for n kernels.
+size_t kernel_order_scratch(int64_t n);
+
+// Permutation of kernel indices into time order (start, stream, index) by a
+// stable radix sort of ((start - min_start) << 8 | stream).  Needs the
+// min / max from check_kernel_order in c.h_status.  Returns a device array of
+// n indices carved from `a`, or NULL on arena exhaustion.
+uint32_t *kernel_time_order(Ctx &c, struct Arena &a, const uint8_t *stream, const int64_t *start, int64_t n);
+
+}  // namespace opattr

@@ -1,0 +1,59 @@
+"""The C ABI library builds, loads and exports every entry point the header
+declares; the binding marshals structs of the header's layout.  CPU only: no
+call here touches a GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "opattr.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(opattr_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_join():
+    names = declared_functions()
+    for f in ("opattr_create", "opattr_enclose", "opattr_match", "opattr_aggregate", "opattr_destroy"):
+        assert f in names
+
+
+def test_library_exports_every_declared_symbol():
+    import paper_2609_11938_gb300 as opa
+    path = opa.build()
+    lib = ctypes.CDLL(path)
+    missing = [f for f in declared_functions() if not hasattr(lib, f)]
+    assert not missing, missing
+
+
+def test_struct_layouts_match_header():
+    import paper_2609_11938_gb300 as opa
+    # pointer-sized fields then int64 n; sizes follow the C layout on LP64
+    assert ctypes.sizeof(opa.Kernels) == 6 * 8
+    assert ctypes.sizeof(opa.Ranges) == 6 * 8
+    assert ctypes.sizeof(opa.Ncu) == 3 * 8
+    assert ctypes.sizeof(opa.Dedup) == 2 * 8 + 2 * 4
+    assert ctypes.sizeof(opa.Config) == 4 + 4 + 4 + 4 + 8
+    assert ctypes.sizeof(opa.MatchSummary) == 8 * 8 + 2 * 4
+    assert ctypes.sizeof(opa.OpAggregates) == 4 * 8
+    assert ctypes.sizeof(opa.Totals) == 6 * 8 + 2 * 8
+
+
+def test_status_strings_without_gpu():
+    import paper_2609_11938_gb300 as opa
+    assert opa.opattr_status_string(opa.E_NOT_NESTED) == "ranges are not nested per stream"
+    assert opa.opattr_status_string(123) == "unknown status"
+
+
+def test_create_without_gpu_fails_cleanly():
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    import paper_2609_11938_gb300 as opa
+    st, h = opa.opattr_create(0)
+    assert st in (opa.E_CUDA, opa.E_INVALID_ARG) and not h

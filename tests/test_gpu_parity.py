@@ -1,0 +1,257 @@
+"""GPU parity: the CUDA path, called through the C ABI, against the CPU oracle
+on the same seeded inputs.  Integer outputs bit-exact, floating-point
+aggregates within 1e-9 relative."""
+import json
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+import tracegen
+from gpu_util import RTOL, assert_close, assert_parity, gpu_run
+
+pytestmark = pytest.mark.gpu
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+
+@pytest.fixture(scope="module")
+def opa():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    import paper_2609_11938_gb300 as m
+    m.build()
+    return m
+
+
+def worked_trace():
+    g = json.load(open(os.path.join(GOLDEN, "worked.json")))
+    conv = {"STRUCTURAL": oracle.STRUCTURAL, "NONOP": oracle.NONOP}
+    r, k, n = g["ranges"], g["kernels"], g["ncu"]
+    counters = np.array([[np.nan if v is None else v for v in row] for row in n["counters"]], np.float32)
+    t = tracegen.Trace(
+        k_stream=np.array(k["stream"], np.uint8), k_start=np.array(k["start"], np.int64),
+        k_dur=np.array(k["dur"], np.int64), k_name=np.array(k["name"], np.uint32), k_layer=None,
+        r_stream=np.array(r["stream"], np.uint8), r_start=np.array(r["start"], np.int64),
+        r_end=np.array(r["end"], np.int64), r_depth=np.array(r["depth"], np.uint8),
+        r_op=np.array([conv.get(x, x) for x in r["op"]], np.uint32), n_ops=g["n_ops"],
+        ncu_name=np.array(n["name"], np.uint32), counters=counters)
+    return g, t
+
+
+@pytest.mark.parametrize("mode", ["skip_name", "prefix"])
+def test_worked_example(opa, mode):
+    g, t = worked_trace()
+    res = gpu_run(t, mode=mode)
+    e = g["expect"]
+    assert res["range_of_kernel"].tolist() == e["range_of_kernel"]
+    assert res["n_op_enclosing"].tolist() == e["n_op_enclosing"]
+    assert res["ncu_idx"].tolist() == e[mode]["ncu_idx"]
+    assert res["match_status"] == e[mode]["status"]
+    ops = res["ops"]
+    for key in ("kernel_count", "total_duration_ns", "matched_count"):
+        assert ops[key].tolist() == e[mode]["ops"][key]
+    for col, key in ((0, "c1_sum"), (3, "c4_dw"), (4, "c5_dw"), (17, "c18_max")):
+        want = np.array([np.nan if v is None else v for v in e[mode]["ops"][key]])
+        assert_close(ops["agg"][col], want, rtol=1e-12, what=key)
+    assert res["totals"]["attributed_ns"] == 37 and res["totals"]["total_ns"] == 68
+    assert_parity(res, oracle.run(t, mode=mode, enclose_mode="brute"))
+
+
+def test_worked_error_mode(opa):
+    _, t = worked_trace()
+    ctx = opa.Context(0, mismatch="error")
+    tr = opa.to_device(t)
+    with pytest.raises(opa.OpattrError) as ei:
+        ctx.match(tr)
+    assert ei.value.status == opa.E_COUNT_MISMATCH
+    # the context stays usable after an error status
+    st, rk, nop = ctx.enclose(tr)
+    assert st == opa.OK and rk.cpu().tolist() == [-1, 2, 8, 2, 4, 5, -1, -1, 7, -1]
+    ctx.close()
+
+
+@pytest.mark.parametrize("seed", range(160))
+def test_small_random(opa, seed):
+    t = tracegen.small_random(seed, n_streams=1 + seed % 4, n_events=10 + (seed * 7) % 90,
+                              max_depth=1 + seed % 7, shuffle=seed % 2 == 0, n_names=2 + seed % 5)
+    if seed % 5 == 3 and t.M > 1:              # force the general match path and count mismatches
+        t.ncu_name = t.ncu_name[1:].copy()
+        t.counters = t.counters[1:].copy()
+    if seed % 7 == 4:
+        t.counters[np.random.default_rng(seed).random(t.counters.shape) < 0.2] = np.nan
+    mode = ["skip_name", "prefix"][seed % 2]
+    assert_parity(gpu_run(t, mode=mode), oracle.run(t, mode=mode, enclose_mode="brute"))
+
+
+@pytest.mark.parametrize("name", ["tiny", "gpt2", "gpt2_dedup", "dedup"])
+@pytest.mark.parametrize("shuffle", [False, True])
+def test_configs(opa, name, shuffle):
+    t = tracegen.generate(name, shuffle=shuffle)
+    g = gpu_run(t)
+    o = oracle.run(t, enclose_mode="brute" if name in ("tiny", "gpt2") else "indexed")
+    assert_parity(g, o)
+    assert g["match_status"] == opa.OK and g["summary"]["unmatched"] == 0
+    if not shuffle:
+        assert g["summary"]["fast_path"] == 1
+
+
+@pytest.mark.parametrize("mode", ["skip_name", "prefix", "error"])
+def test_gpt2_count_mismatch(opa, mode):
+    t = tracegen.generate("gpt2")
+    rng = np.random.default_rng(7)
+    drop = rng.choice(t.M, 25, replace=False)
+    keep = np.setdiff1d(np.arange(t.M), drop)
+    t.ncu_name, t.counters = t.ncu_name[keep].copy(), t.counters[keep].copy()
+    o = oracle.run(t, mode=mode, enclose_mode="indexed")
+    if mode == "error":
+        import paper_2609_11938_gb300 as m
+        ctx = m.Context(0, mismatch="error")
+        with pytest.raises(m.OpattrError) as ei:
+            ctx.match(m.to_device(t))
+        assert ei.value.status == m.E_COUNT_MISMATCH == o["match_status"]
+        ctx.close()
+        return
+    g = gpu_run(t, mode=mode)
+    assert g["match_status"] == opa.W_COUNT_MISMATCH
+    assert_parity(g, o)
+
+
+def test_dedup_swapped_names(opa):
+    t = tracegen.generate("dedup")
+    # rename one kernel of a duplicate layer: its broadcast source no longer matches
+    dup = np.nonzero((t.k_layer >= 0) & (t.rep_of_class[t.class_of_layer[np.maximum(t.k_layer, 0)]] != t.k_layer))[0]
+    t.k_name = t.k_name.copy()
+    t.k_name[dup[::997]] += 1
+    g = gpu_run(t)
+    o = oracle.run(t)
+    assert g["match_status"] == o["match_status"] == opa.W_DEDUP_MISMATCH
+    assert_parity(g, o)
+
+
+def test_nan_counters(opa):
+    t = tracegen.generate("gpt2", nan_frac=0.1, nan_mask=1 << 12)
+    g, o = gpu_run(t), oracle.run(t, enclose_mode="indexed")
+    assert np.isnan(g["ops"]["agg"][12]).all()
+    assert_parity(g, o)
+
+
+def test_empty_inputs(opa):
+    t = tracegen.small_random(3)
+    z = lambda a: a[:0].copy()
+    for cut in ("kernels", "ranges", "ncu", "all"):
+        u = tracegen.small_random(3)
+        if cut in ("kernels", "all"):
+            u.k_stream, u.k_start, u.k_dur, u.k_name = z(t.k_stream), z(t.k_start), z(t.k_dur), z(t.k_name)
+        if cut in ("ranges", "all"):
+            u.r_stream, u.r_start, u.r_end, u.r_depth, u.r_op = (z(t.r_stream), z(t.r_start), z(t.r_end),
+                                                                z(t.r_depth), z(t.r_op))
+            u.n_ops = 0
+        if cut in ("ncu", "all"):
+            u.ncu_name, u.counters = z(t.ncu_name), z(t.counters)
+        assert_parity(gpu_run(u), oracle.run(u, enclose_mode="brute"))
+
+
+def test_error_statuses(opa):
+    import torch
+    t = tracegen.small_random(11, n_events=80, max_depth=4)
+    ctx = opa.Context(0)
+    # depth above 31
+    u = tracegen.small_random(11, n_events=80, max_depth=4)
+    u.r_depth = u.r_depth.copy(); u.r_depth[0] = 32
+    with pytest.raises(opa.OpattrError) as ei:
+        ctx.enclose(opa.to_device(u))
+    assert ei.value.status == opa.E_DEPTH
+    # end before start
+    u = tracegen.small_random(11, n_events=80, max_depth=4)
+    u.r_end = u.r_end.copy(); u.r_end[0] = u.r_start[0] - 1
+    with pytest.raises(opa.OpattrError) as ei:
+        ctx.enclose(opa.to_device(u))
+    assert ei.value.status == opa.E_INVALID_ARG
+    # two overlapping ranges at one depth
+    u = tracegen.small_random(11, n_events=80, max_depth=4)
+    u.r_stream = np.append(u.r_stream, [0, 0]).astype(np.uint8)
+    u.r_start = np.append(u.r_start, [100, 105]).astype(np.int64)
+    u.r_end = np.append(u.r_end, [110, 120]).astype(np.int64)
+    u.r_depth = np.append(u.r_depth, [0, 0]).astype(np.uint8)
+    u.r_op = np.append(u.r_op, [u.n_ops, u.n_ops + 1]).astype(np.uint32)
+    assert oracle.validate_ranges(u.r_stream, u.r_start, u.r_end, u.r_depth) == oracle.E_NOT_NESTED
+    with pytest.raises(opa.OpattrError) as ei:
+        ctx.enclose(opa.to_device(u))
+    assert ei.value.status == opa.E_NOT_NESTED
+    # aggregate: out-of-range index, infinite counter, negative duration
+    tr = opa.to_device(t)
+    st, rk, _ = ctx.enclose(tr)
+    st, idx, _, _ = ctx.match(tr)
+    bad = rk.clone(); bad[0] = t.R
+    with pytest.raises(opa.OpattrError):
+        ctx.aggregate(tr, bad, idx)
+    u = tracegen.small_random(11, n_events=80, max_depth=4)
+    u.counters = u.counters.copy(); u.counters[:, 4] = np.inf
+    res = oracle.run(u)
+    if (res["range_of_kernel"] >= 0).any():
+        with pytest.raises(opa.OpattrError) as ei:
+            ctx.aggregate(opa.to_device(u), rk, idx)
+        assert ei.value.status == opa.E_INVALID_ARG == res["aggregate_status"]
+    u = tracegen.small_random(11, n_events=80, max_depth=4)
+    u.k_dur = u.k_dur.copy(); u.k_dur[-1] = -5
+    with pytest.raises(opa.OpattrError):
+        ctx.aggregate(opa.to_device(u), rk, idx)
+    # still usable afterwards
+    assert_parity(gpu_run(t, ctx=ctx), oracle.run(t, enclose_mode="brute"))
+    ctx.close()
+
+
+def test_oom_injection(opa, monkeypatch):
+    t = tracegen.generate("tiny")
+    monkeypatch.setenv("OPATTR_FAULT", "alloc")
+    ctx = opa.Context(0)
+    with pytest.raises(opa.OpattrError) as ei:
+        ctx.enclose(opa.to_device(t))
+    assert ei.value.status == opa.E_OOM
+    monkeypatch.delenv("OPATTR_FAULT")
+    assert_parity(gpu_run(t, ctx=ctx), oracle.run(t, enclose_mode="brute"))
+    ctx.close()
+
+
+def test_large_full_parity(opa):
+    """The 20M-kernel benchmark trace, in the configuration the benchmark runs,
+    against the oracle on every output."""
+    t = tracegen.generate("large")
+    g = gpu_run(t)
+    assert g["summary"]["fast_path"] == 1
+    o = oracle.run(t, enclose_mode="indexed")
+    assert_parity(g, o)
+
+
+def test_adversarial_sampled(opa):
+    """The 50M-kernel adversarial trace: enclosure against the oracle on a
+    kernel sample, matching by the identity property, aggregation against the
+    oracle on every op (given the verified join)."""
+    t = tracegen.generate("adversarial")
+    g = gpu_run(t)
+    rk, K = g["range_of_kernel"], t.K
+    rng = np.random.default_rng(0)
+    sample = np.sort(rng.choice(K, 200_000, replace=False))
+    st, orc_rk, orc_nop = oracle.enclose(t.k_stream[sample], t.k_start[sample], t.r_stream, t.r_start, t.r_end,
+                                         t.r_depth, t.r_op, mode="indexed")
+    assert st == 0
+    np.testing.assert_array_equal(rk[sample], orc_rk)
+    np.testing.assert_array_equal(g["n_op_enclosing"][sample], orc_nop)
+    att = rk >= 0                                     # every attributed kernel: its range contains T
+    r = rk[att]
+    assert (t.r_stream[r] == t.k_stream[att]).all()
+    assert ((t.r_start[r] <= t.k_start[att]) & (t.k_start[att] <= t.r_end[r])).all()
+    assert (t.r_op[r] < t.n_ops).all()
+    # time-ordered kernels whose names equal the ncu rows: Algorithm 1 is the identity
+    order_ok = np.all((np.diff(t.k_start) > 0) | ((np.diff(t.k_start) == 0) & (np.diff(t.k_stream.astype(int)) >= 0)))
+    assert order_ok and t.M == K and (t.ncu_name == t.k_name).all()
+    assert g["summary"]["fast_path"] == 1
+    np.testing.assert_array_equal(g["ncu_idx"], np.arange(K, dtype=np.int32))
+    st, ops, tot = oracle.aggregate(t.k_dur, rk, t.r_op, t.counters, g["ncu_idx"], t.n_ops)
+    assert st == 0
+    for k in ("kernel_count", "total_duration_ns", "matched_count"):
+        np.testing.assert_array_equal(g["ops"][k], ops[k])
+    assert_close(g["ops"]["agg"], ops["agg"], what="agg")
+    assert g["totals"]["attributed_ns"] == tot["attributed_ns"] and g["totals"]["total_ns"] == tot["total_ns"]
