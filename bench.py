@@ -190,6 +190,8 @@ def main():
     ap.add_argument("--shuffle", action="store_true", help="permute kernel and range arrays (general paths)")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--oracle-kernels", type=int, default=1_000_000)
+    ap.add_argument("--kernels", type=int, default=0,
+                    help="draw this many kernels with the config's generator parameters (profiling runs)")
     args = ap.parse_args()
     world, rank, local = dist_env()
     if args.warmup < 3:
@@ -247,6 +249,8 @@ def main():
 
     cfg = tracegen.config(args.config)
     cfg["seed"] = cfg["seed"] + 1000 * rank          # each rank attributes its own trace
+    if args.kernels and cfg.get("shape", 0) == 0:
+        cfg["n_kernels"] = args.kernels
     trace = tracegen.generate(cfg, shuffle=args.shuffle)
     K, R, M, O = trace.K, trace.R, trace.M, trace.n_ops
     use_dedup = bool(cfg.get("dedup")) and trace.k_layer is not None
@@ -368,7 +372,8 @@ def main():
         "vs_baseline": None,
         "dtype": "int64+f32x2",
         "data": "synthetic",
-        "config": {"workload": f"{args.config}: {WORKLOADS[args.config]}", "kernels": K, "ranges": R,
+        "config": {"workload": f"{args.config}: {WORKLOADS[args.config]}" + (
+                       f" [scaled to {K} kernels]" if args.kernels else ""), "kernels": K, "ranges": R,
                    "ncu_rows": M, "ops": O, "shuffled": bool(args.shuffle), "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2 (129 MB)" if flush is None else "L2 flushed before every step"},
         "roofline": {"bound": "hbm", "kernel": dname, "achieved": achieved, "peak": peak, "unit": "GB/s",

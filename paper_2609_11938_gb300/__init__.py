@@ -238,13 +238,14 @@ def to_device(trace, device: int = 0, pin: bool = False) -> DeviceTrace:
 class Context:
     """An opattr context bound to one device and one CUDA stream."""
 
-    def __init__(self, device: int = 0, stream=None, mismatch: str = "skip_name", dedup: bool = True):
+    def __init__(self, device: int = 0, stream=None, mismatch: str = "skip_name", dedup: bool = True,
+                 spin_limit: int = 0):
         import torch
         self.device = device
         if stream is None:
             stream = torch.cuda.current_stream(device)
         self.stream = stream
-        st, self.handle = opattr_create(device, stream.cuda_stream, mismatch, dedup)
+        st, self.handle = opattr_create(device, stream.cuda_stream, mismatch, dedup, spin_limit)
         if st != OK:
             raise OpattrError(st, "opattr_create")
 

@@ -18,6 +18,9 @@
 // by op id; one thread per op id walks its segment.
 //
 // Accumulation is float-float with exact int64 weights (ff.cuh).
+#include <stdlib.h>
+#include <string.h>
+
 #include <algorithm>
 
 #include "ff.cuh"
@@ -40,67 +43,113 @@ struct AggIn {
 };
 
 // One operator's running aggregate.
+//  kc, dsum       attributed kernels and their summed duration
+//  mc, dall       matched kernels (with a row) and their summed duration
+//  s[i]           SUM counters, float-float
+//  w[i], nanw[i]  DW counters: sum of m*d, float-float, and the duration of
+//                 matched kernels whose value was null (weight = dall - nanw)
+//  mx[i]          MAX counters
+constexpr int RENORM = 128;
+
+// Per-counter finishing steps, kept out of line: they run once per operator
+// and counter, and one copy keeps the kernel's instruction footprint small.
+__device__ __noinline__ double finish_sum(float hi, float lo) {
+    ff v{hi, lo};
+    ff_renorm(v);
+    return ff_to_f64(v);
+}
+__device__ __noinline__ double finish_dw(float hi, float lo, long long den) {
+    ff v{hi, lo};
+    ff_renorm(v);
+    return ff_div_i64_to_f64(v, den);
+}
+__device__ __noinline__ double finish_max(float x) { return f32_to_f64_bits(x); }
+constexpr unsigned ALL_COUNTERS = (1u << NC) - 1;
+
 struct Acc {
-    long long kc, dsum, mc;
+    int kc, mc;
+    long long dsum, dall;
     ff s[N_SUM];
     ff w[N_DW];
-    long long den[N_DW];
+    long long nanw[N_DW];
     float mx[N_MAX];
     unsigned seen;      // bit c: counter c had a non-null value
     int bad;            // an infinite counter was seen
+    int terms;          // accumulations since the last renormalisation
 
     __device__ __forceinline__ void init() {
-        kc = dsum = mc = 0;
+        kc = mc = 0;
+        dsum = dall = 0;
 #pragma unroll
         for (int i = 0; i < N_SUM; ++i) s[i] = ff{0.f, 0.f};
 #pragma unroll
-        for (int i = 0; i < N_DW; ++i) { w[i] = ff{0.f, 0.f}; den[i] = 0; }
+        for (int i = 0; i < N_DW; ++i) { w[i] = ff{0.f, 0.f}; nanw[i] = 0; }
 #pragma unroll
         for (int i = 0; i < N_MAX; ++i) mx[i] = -INFINITY;
         seen = 0;
         bad = 0;
+        terms = 0;
     }
 
-    __device__ __forceinline__ void add(const AggIn &A, int64_t k) {
-        const long long d = A.dur[k];
+    __device__ __forceinline__ static int sum_col(int i) {
+        return i == 0 ? 0 : i == 1 ? 1 : i == 2 ? 2 : i == 3 ? 10 : i == 4 ? 14 : 18;
+    }
+    __device__ __forceinline__ static int dw_col(int i) { return i < 7 ? 3 + i : (i < 10 ? 4 + i : 5 + i); }
+    __device__ __forceinline__ static int max_col(int i) { return i == 0 ? 17 : 19; }
+
+    // Adds one kernel: duration d, and its counter row when `matched`.
+    __device__ __forceinline__ void accumulate(long long d, bool matched, const float4 *row) {
         kc++;
         dsum += d;
-        const int32_t j = A.ncu_idx[k];
-        if (j < 0) return;
+        if (!matched) return;
         mc++;
-        const float4 *row = reinterpret_cast<const float4 *>(A.counters + (int64_t)j * NC);
+        dall += d;
         float v[NC];
 #pragma unroll
         for (int q = 0; q < NC / 4; ++q) {
-            float4 x = __ldg(row + q);
+            const float4 x = row[q];
             v[4 * q] = x.x; v[4 * q + 1] = x.y; v[4 * q + 2] = x.z; v[4 * q + 3] = x.w;
         }
-        const ff dd = ff_from_i64(d);
+        float z = 0.f;              // NaN iff some value is NaN or infinite
 #pragma unroll
-        for (int i = 0; i < N_SUM; ++i) {
-            const int c = i == 0 ? 0 : i == 1 ? 1 : i == 2 ? 2 : i == 3 ? 10 : i == 4 ? 14 : 18;
-            const unsigned u = __float_as_uint(v[c]);
-            if ((u & 0x7F800000u) == 0x7F800000u) { bad |= (u & 0x7FFFFFu) == 0; continue; }
-            seen |= 1u << c;
-            ff_add(s[i], v[c], 0.f);
+        for (int c = 0; c < NC; ++c) z = __fmaf_rn(v[c], 0.f, z);
+        unsigned valid = ALL_COUNTERS;
+        if (z != z) {
+            // rare: null (NaN) values take no part -- a zero value with a
+            // zero weight for the sums, -inf for the maxima -- and their
+            // durations leave the DW weights; infinite values are errors
+#pragma unroll
+            for (int c = 0; c < NC; ++c) {
+                if (isnan(v[c])) {
+                    valid &= ~(1u << c);
+                    v[c] = (c == 17 || c == 19) ? -INFINITY : 0.f;
+                } else if (isinf(v[c])) {
+                    bad = 1;
+                    valid &= ~(1u << c);
+                    v[c] = (c == 17 || c == 19) ? -INFINITY : 0.f;
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < N_DW; ++i)
+                if (!((valid >> dw_col(i)) & 1u)) nanw[i] += d;
         }
+        seen |= valid;
+        const ff dd = split_i64(d);
+#pragma unroll
+        for (int i = 0; i < N_SUM; ++i) ff_accum(s[i], v[sum_col(i)], 0.f);
 #pragma unroll
         for (int i = 0; i < N_DW; ++i) {
-            const int c = i < 7 ? 3 + i : (i < 10 ? 4 + i : 5 + i);   // 3..9, 11..13, 15..16
-            const unsigned u = __float_as_uint(v[c]);
-            if ((u & 0x7F800000u) == 0x7F800000u) { bad |= (u & 0x7FFFFFu) == 0; continue; }
-            seen |= 1u << c;
-            ff p = ff_mul_f(v[c], dd);
-            ff_add(w[i], p.hi, p.lo);
-            den[i] += d;
+            const ff p = mul_split(v[dw_col(i)], dd);
+            ff_accum(w[i], p.hi, p.lo);
         }
 #pragma unroll
-        for (int i = 0; i < N_MAX; ++i) {
-            const int c = i == 0 ? 17 : 19;
-            const unsigned u = __float_as_uint(v[c]);
-            if ((u & 0x7F800000u) == 0x7F800000u) { bad |= (u & 0x7FFFFFu) == 0; continue; }
-            seen |= 1u << c;
-            mx[i] = fmaxf(mx[i], v[c]);
+        for (int i = 0; i < N_MAX; ++i) mx[i] = fmaxf(mx[i], v[max_col(i)]);
+        if (++terms >= RENORM) {
+            terms = 0;
+#pragma unroll
+            for (int i = 0; i < N_SUM; ++i) ff_renorm(s[i]);
+#pragma unroll
+            for (int i = 0; i < N_DW; ++i) ff_renorm(w[i]);
         }
     }
 
@@ -112,20 +161,24 @@ struct Acc {
         const int64_t n = A.n_ops;
         const double qnan = __longlong_as_double(0x7FF8000000000000ll);
 #pragma unroll
-        for (int i = 0; i < N_SUM; ++i) {
-            const int c = i == 0 ? 0 : i == 1 ? 1 : i == 2 ? 2 : i == 3 ? 10 : i == 4 ? 14 : 18;
-            agg[(int64_t)c * n + op] = ((seen >> c) & 1u) ? ff_to_f64(s[i]) : qnan;
-        }
+        for (int i = 0; i < N_SUM; ++i)
+            agg[(int64_t)sum_col(i) * n + op] = ((seen >> sum_col(i)) & 1u) ? finish_sum(s[i].hi, s[i].lo) : qnan;
 #pragma unroll
         for (int i = 0; i < N_DW; ++i) {
-            const int c = i < 7 ? 3 + i : (i < 10 ? 4 + i : 5 + i);
-            agg[(int64_t)c * n + op] = (((seen >> c) & 1u) && den[i] > 0) ? ff_div_i64_to_f64(w[i], den[i]) : qnan;
+            const long long den = dall - nanw[i];
+            agg[(int64_t)dw_col(i) * n + op] =
+                (((seen >> dw_col(i)) & 1u) && den > 0) ? finish_dw(w[i].hi, w[i].lo, den) : qnan;
         }
 #pragma unroll
-        for (int i = 0; i < N_MAX; ++i) {
-            const int c = i == 0 ? 17 : 19;
-            agg[(int64_t)c * n + op] = ((seen >> c) & 1u) ? f32_to_f64_bits(mx[i]) : qnan;
-        }
+        for (int i = 0; i < N_MAX; ++i)
+            agg[(int64_t)max_col(i) * n + op] = ((seen >> max_col(i)) & 1u) ? finish_max(mx[i]) : qnan;
+    }
+
+    // Row fetched from global memory (general path).
+    __device__ __forceinline__ void add(const AggIn &A, int64_t k) {
+        const long long d = A.dur[k];
+        const int32_t j = A.ncu_idx[k];
+        accumulate(d, j >= 0, reinterpret_cast<const float4 *>(A.counters + (int64_t)(j >= 0 ? j : 0) * NC));
     }
 };
 
@@ -137,10 +190,11 @@ __global__ void k_agg_check_kernels(const int64_t *__restrict__ dur, const int32
                                     const int32_t *__restrict__ nidx, const uint32_t *__restrict__ r_op, int64_t K,
                                     int64_t R, int64_t M, int64_t n_ops, DevStatus *st) {
     unsigned long long tot = 0, att = 0, natt = 0, nmatch = 0;
-    int bad = 0;
+    int bad = 0, not_id = 0;
     for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < K; k += (int64_t)gridDim.x * blockDim.x) {
         long long d = dur[k];
         int32_t r = rok[k], j = nidx[k];
+        not_id |= j >= 0 && j != k;
         if (d < 0 || r < -1 || r >= R || j < -1 || j >= M) { bad = 1; continue; }
         tot += (unsigned long long)d;
         if (r >= 0) {
@@ -151,17 +205,13 @@ __global__ void k_agg_check_kernels(const int64_t *__restrict__ dur, const int32
             nmatch += j >= 0;
         }
     }
-    tot = warp_sum(tot);
-    att = warp_sum(att);
-    natt = warp_sum(natt);
-    nmatch = warp_sum(nmatch);
+    __shared__ unsigned long long red[33];
     if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_err(st, ERR_INVALID);
-    if (lane_id() == 0) {
-        if (tot) atomicAdd(&st->cnt[C_TOTAL_NS], tot);
-        if (att) atomicAdd(&st->cnt[C_ATTR_NS], att);
-        if (natt) atomicAdd(&st->cnt[C_ATTR_K], natt);
-        if (nmatch) atomicAdd(&st->cnt[C_MATCHED_K], nmatch);
-    }
+    if (__any_sync(0xffffffffu, not_id) && lane_id() == 0) set_flag(st, F_IDX_NOT_ID);
+    block_add_u64(tot, &st->cnt[C_TOTAL_NS], red);
+    block_add_u64(att, &st->cnt[C_ATTR_NS], red);
+    block_add_u64(natt, &st->cnt[C_ATTR_K], red);
+    block_add_u64(nmatch, &st->cnt[C_MATCHED_K], red);
 }
 
 // Per range: start order of the array; a bitmap of op ids held by operator
@@ -183,20 +233,25 @@ __global__ void k_agg_check_ranges(const int64_t *__restrict__ r_start, const ui
 }
 
 // ------------------------------------------------------------------ fast path
-constexpr int AGG_THREADS = 256;
-constexpr int AGG_TILE = 1024;               // kernels per tile
-constexpr int AGG_SLOTS = 512;               // owned ranges handled per pass
-constexpr int AGG_WARPS = AGG_THREADS / 32;
-constexpr int AGG_PER_WARP = AGG_TILE / AGG_WARPS;
+constexpr int AO_THREADS = 256;
+constexpr int AO_WARPS = AO_THREADS / 32;
+constexpr int AO_TILE = 1024;                    // kernels per tile
+constexpr int AO_PER_WARP = AO_TILE / AO_WARPS;  // 128
+constexpr int AO_OPEN = 192;                     // open ranges carried from tile to tile
+constexpr int AO_KEYS = 640;                     // group keys per pass: owned slots, then carried slots
+constexpr int AO_OWN = AO_KEYS - AO_OPEN;        // owned ranges per pass
+constexpr int AO_HASH = 512;                     // range id -> carried slot, open addressing
+constexpr unsigned AO_NONE = GROUP_NONE;
+constexpr int AO_LBUCKETS = 64;
 
-// band[t] = number of ranges with start <= T(t * AGG_TILE - 1), band[0] = 0,
+// band[t] = number of ranges with start <= T(t * AO_TILE - 1), band[0] = 0,
 // band[nt] = R: tile t owns ranges [band[t], band[t+1]).
 __global__ void k_band_table(const int64_t *__restrict__ k_start, int64_t K, const int64_t *__restrict__ r_start,
                              int64_t R, int64_t nt, int64_t *__restrict__ band) {
     for (int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; t <= nt; t += (int64_t)gridDim.x * blockDim.x) {
         if (t == 0) { band[0] = 0; continue; }
         if (t == nt) { band[nt] = R; continue; }
-        long long b = k_start[t * AGG_TILE - 1];
+        long long b = k_start[t * AO_TILE - 1];
         int64_t lo = 0, hi = R;
         while (lo < hi) {
             int64_t m = (lo + hi) >> 1;
@@ -208,117 +263,256 @@ __global__ void k_band_table(const int64_t *__restrict__ k_start, int64_t K, con
 
 struct OwnArgs {
     AggIn in;
+    int64_t M;
+    int identity;               // ncu_idx[k] is k or -1 for every kernel
     const int64_t *k_start;
     const int32_t *rok;
     int64_t K;
     const int64_t *r_end;
     const uint32_t *r_op;
     const int64_t *band;
+    int64_t nt, tiles_per_block;
+    long long wait_cycles;      // bound on the wait for a tile's bulk copy
+    int withhold_copy;          // fault injection: announce the first copy but never issue it
+    Acc *open_acc;              // [gridDim.x][2][AO_OPEN] carried accumulators (L2-resident scratch)
+    int32_t *open_range;        // [gridDim.x][2][AO_OPEN]
     DevStatus *st;
 };
 
 struct OwnSmem {
-    int32_t rok[AGG_TILE];
-    uint16_t klist[AGG_TILE];
-    uint16_t wcnt[AGG_WARPS][AGG_SLOTS];
-    uint16_t soff[AGG_SLOTS + 1];
+    float4 rows[AO_TILE * (NC / 4)];   // the tile's counter rows (bulk copy or gather)
+    int32_t rok[AO_TILE];
+    uint16_t klist[AO_TILE];
+    uint16_t wcnt[AO_WARPS][AO_KEYS];
+    uint16_t soff[AO_KEYS + 1];
+    uint16_t order[AO_KEYS];
+    uint32_t lcount[AO_LBUCKETS + 1];
+    int32_t hkey[AO_HASH];
+    int16_t hval[AO_HASH];
+    unsigned long long mbar;
     uint32_t wbuf[33];
-    unsigned long long seen;
-    int bad;
+    unsigned long long red[33];
+    long long max_end_in, max_end_out;
+    int nopen_in, nopen_out, ok;
 };
 
-__global__ void __launch_bounds__(AGG_THREADS) k_agg_owned(OwnArgs A) {
-    __shared__ OwnSmem S;
-    const int64_t t = blockIdx.x;
-    const int64_t k0 = t * AGG_TILE;
-    const int64_t kn = A.K - k0 < AGG_TILE ? A.K - k0 : AGG_TILE;
-    const int64_t k1 = k0 + kn;
-    const int64_t ra = A.band[t], rb = A.band[t + 1];
-    const long long t_next = k1 < A.K ? A.k_start[k1] : LLONG_MAX;
-    const unsigned w = threadIdx.x >> 5, lane = lane_id(), lt = lanemask_lt();
-    for (int i = threadIdx.x; i < AGG_TILE; i += AGG_THREADS) S.rok[i] = i < kn ? A.rok[k0 + i] : -1;
-    if (threadIdx.x == 0) { S.seen = 0; S.bad = 0; }
+// ---- bulk copy (TMA) helpers: one mbarrier per block, one copy per tile
+__device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ void mbar_init(unsigned long long *bar) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(smem_u32(bar)) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_copy_g2s(void *dst, const void *src, unsigned bytes, unsigned long long *bar) {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     smem_u32(dst)),
+                 "l"(src), "r"(bytes), "r"(smem_u32(bar))
+                 : "memory");
+}
+__device__ __forceinline__ bool mbar_test_wait(unsigned long long *bar, unsigned parity) {
+    unsigned ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Bounded wait (non-blocking polls): gives up after `limit` cycles.
+__device__ __forceinline__ bool mbar_wait(unsigned long long *bar, unsigned parity, long long limit) {
+    const long long t0 = clock64();
+    while (!mbar_test_wait(bar, parity))
+        if (clock64() - t0 > limit) return false;
+    return true;
+}
+
+template <typename KeyFn>
+__device__ __forceinline__ void group_by_key(OwnSmem &S, int nkeys, KeyFn key_of) {
+    block_group_by_key<AO_THREADS, AO_PER_WARP>(nkeys, key_of, &S.wcnt[0][0], AO_KEYS, S.soff, S.klist, S.wbuf);
+}
+
+__device__ __forceinline__ unsigned hash_slot(int32_t r) { return ((uint32_t)r * 2654435761u) >> 23; }   // 9 bits
+
+__device__ __forceinline__ int hash_find(const OwnSmem &S, int32_t r) {
+    unsigned h = hash_slot(r);
+    for (int probe = 0; probe < AO_HASH; ++probe) {
+        const int32_t k = S.hkey[h];
+        if (k == r) return S.hval[h];
+        if (k < 0) return -1;
+        h = (h + 1) & (AO_HASH - 1);
+    }
+    return -1;
+}
+
+// Persistent blocks: block b takes tiles [b * tpb, (b + 1) * tpb) in order.
+// A range still open at the end of a tile keeps its accumulator in the
+// block's carry table and picks up its kernels in the next tile.  After its
+// own tiles, the block keeps walking the following tiles -- owning nothing
+// there -- until every range it carries has ended.  Each tile's counter rows
+// arrive in shared memory with one bulk copy (identity row map) or a gather.
+__global__ void __launch_bounds__(AO_THREADS, 2) k_agg_owned(OwnArgs A) {
+    extern __shared__ __align__(128) unsigned char smem_raw[];
+    OwnSmem &S = *reinterpret_cast<OwnSmem *>(smem_raw);
+    const int64_t t_begin = (int64_t)blockIdx.x * A.tiles_per_block;
+    const int64_t t_end = t_begin + A.tiles_per_block < A.nt ? t_begin + A.tiles_per_block : A.nt;
+    Acc *acc_tab[2] = {A.open_acc + (size_t)blockIdx.x * 2 * AO_OPEN, A.open_acc + ((size_t)blockIdx.x * 2 + 1) * AO_OPEN};
+    int32_t *rng_tab[2] = {A.open_range + (size_t)blockIdx.x * 2 * AO_OPEN,
+                           A.open_range + ((size_t)blockIdx.x * 2 + 1) * AO_OPEN};
+    int cur = 0;
+    unsigned phase = 0;
     unsigned long long seen = 0;
     int bad = 0;
-
-    for (int64_t ca = ra; ca < rb; ca += AGG_SLOTS) {
-        const int64_t cb = rb - ca < AGG_SLOTS ? rb : ca + AGG_SLOTS;
-        const int nslot = (int)(cb - ca);
-        for (int i = threadIdx.x; i < AGG_WARPS * AGG_SLOTS; i += AGG_THREADS) (&S.wcnt[0][0])[i] = 0;
-        __syncthreads();
-        // stable in-tile ranking by slot: warp w owns kernels [w*128, w*128+128)
-        uint16_t rank[AGG_PER_WARP / 32];
-        int slot_of[AGG_PER_WARP / 32];
-#pragma unroll
-        for (int it = 0; it < AGG_PER_WARP / 32; ++it) {
-            int i = w * AGG_PER_WARP + it * 32 + lane;
-            int32_t r = S.rok[i];
-            int sl = (r >= ca && r < cb) ? (int)(r - ca) : AGG_SLOTS;
-            unsigned peers = __match_any_sync(0xffffffffu, sl);
-            unsigned before = sl < AGG_SLOTS ? S.wcnt[w][sl] : 0u;
-            __syncwarp();
-            if (sl < AGG_SLOTS && (peers & lt) == 0) S.wcnt[w][sl] = (uint16_t)(before + __popc(peers));
-            __syncwarp();
-            rank[it] = (uint16_t)(before + __popc(peers & lt));
-            slot_of[it] = sl;
-        }
-        __syncthreads();
-        // per slot: exclusive prefix over warps, then over slots
-        for (int b = 0; b < AGG_SLOTS; b += AGG_THREADS) {
-            int sl = b + threadIdx.x;
-            unsigned tot = 0;
-#pragma unroll
-            for (int q = 0; q < AGG_WARPS; ++q) {
-                unsigned x = S.wcnt[q][sl];
-                S.wcnt[q][sl] = (uint16_t)tot;
-                tot += x;
-            }
-            unsigned all;
-            unsigned ex = block_exclusive_scan<unsigned>(tot, S.wbuf, &all);
-            unsigned carry = b == 0 ? 0u : S.soff[b];
-            __syncthreads();
-            S.soff[sl] = (uint16_t)(carry + ex);
-            if (threadIdx.x == AGG_THREADS - 1) S.soff[b + AGG_THREADS] = (uint16_t)(carry + ex + tot);
-            __syncthreads();
-        }
-#pragma unroll
-        for (int it = 0; it < AGG_PER_WARP / 32; ++it) {
-            int sl = slot_of[it];
-            if (sl < AGG_SLOTS) {
-                int i = w * AGG_PER_WARP + it * 32 + lane;
-                S.klist[S.soff[sl] + S.wcnt[w][sl] + rank[it]] = (uint16_t)i;
-            }
-        }
-        __syncthreads();
-        // one thread per owned range: its kernels in this tile, then beyond it
-        for (int sl = threadIdx.x; sl < nslot; sl += AGG_THREADS) {
-            const int64_t r = ca + sl;
-            const uint32_t op = A.r_op[r];
-            if ((int64_t)op >= A.in.n_ops) continue;             // not an operator range
-            Acc acc;
-            acc.init();
-            for (int q = S.soff[sl]; q < S.soff[sl + 1]; ++q) acc.add(A.in, k0 + S.klist[q]);
-            const long long e = A.r_end[r];
-            if (e >= t_next) {
-                for (int64_t k = k1; k < A.K; ++k) {
-                    if (A.k_start[k] > e) break;
-                    if (A.rok[k] == (int32_t)r) acc.add(A.in, k);
-                }
-            }
-            acc.write(A.in, op);
-            seen += (unsigned long long)acc.kc;
-            bad |= acc.bad;
-        }
-        __syncthreads();
-    }
-    seen = warp_sum(seen);
-    if (lane == 0 && seen) atomicAdd(&S.seen, seen);
-    if (__any_sync(0xffffffffu, bad) && lane == 0) S.bad = 1;
-    __syncthreads();
     if (threadIdx.x == 0) {
-        if (S.seen) atomicAdd(&A.st->cnt[C_AGG_SEEN], S.seen);
-        if (S.bad) set_err(A.st, ERR_INVALID);
+        mbar_init(&S.mbar);
+        S.nopen_in = 0;
+        S.max_end_in = LLONG_MIN;
     }
+    __syncthreads();
+
+    for (int64_t t = t_begin; t < A.nt; ++t) {
+        const bool own = t < t_end;
+        if (!own && (S.nopen_in == 0 || A.k_start[t * AO_TILE] > S.max_end_in)) break;
+        const int64_t k0 = t * AO_TILE;
+        const int64_t kn = A.K - k0 < AO_TILE ? A.K - k0 : AO_TILE;
+        const int64_t k1 = k0 + kn;
+        const int64_t ra = own ? A.band[t] : 0, rb = own ? A.band[t + 1] : 0;
+        const long long t_next = k1 < A.K ? A.k_start[k1] : LLONG_MAX;
+        const int nin = S.nopen_in;
+        // ---- stage the tile: rows (bulk copy or gather), range ids, carried-range hash
+        int64_t nrows = A.identity ? (A.M - k0 < kn ? A.M - k0 : kn) : 0;
+        if (nrows < 0) nrows = 0;
+        if (threadIdx.x == 0 && nrows > 0) {
+            if (A.withhold_copy && t == t_begin)
+                asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(&S.mbar)),
+                             "r"((unsigned)(nrows * NC * 4))
+                             : "memory");
+            else
+                bulk_copy_g2s(S.rows, A.in.counters + k0 * NC, (unsigned)(nrows * NC * 4), &S.mbar);
+        }
+        for (int i = threadIdx.x; i < AO_TILE; i += AO_THREADS) S.rok[i] = i < kn ? A.rok[k0 + i] : -1;
+        if (!A.identity) {
+            for (int i = threadIdx.x; i < kn; i += AO_THREADS) {
+                const int32_t j = A.in.ncu_idx[k0 + i];
+                if (j < 0) continue;
+                const float4 *src = reinterpret_cast<const float4 *>(A.in.counters + (int64_t)j * NC);
+#pragma unroll
+                for (int q = 0; q < NC / 4; ++q) S.rows[i * (NC / 4) + q] = __ldg(src + q);
+            }
+        }
+        for (int i = threadIdx.x; i < AO_HASH; i += AO_THREADS) S.hkey[i] = -1;
+        if (threadIdx.x == 0) { S.nopen_out = 0; S.max_end_out = LLONG_MIN; S.ok = 1; }
+        __syncthreads();
+        for (int o = threadIdx.x; o < nin; o += AO_THREADS) {
+            const int32_t r = rng_tab[cur][o];
+            unsigned h = hash_slot(r);
+            for (int probe = 0; probe < AO_HASH && atomicCAS(&S.hkey[h], -1, r) != -1; ++probe)
+                h = (h + 1) & (AO_HASH - 1);
+            S.hval[h] = (int16_t)o;
+        }
+        if (threadIdx.x == 0 && nrows > 0) {
+            if (!mbar_wait(&S.mbar, phase, A.wait_cycles)) {
+                // give up on this launch, but let the copy land before the block exits
+                set_err(A.st, ERR_TIMEOUT);
+                mbar_wait(&S.mbar, phase, 64 * A.wait_cycles + (1ll << 24));
+                S.ok = 0;
+            }
+        }
+        if (nrows > 0) phase ^= 1u;
+        __syncthreads();
+        if (!S.ok) return;
+        // ---- passes over the owned ranges; the carried ranges join the first
+        bool first = true;
+        for (int64_t ca = ra; first || ca < rb; ca += AO_OWN, first = false) {
+            const int64_t cb = rb - ca < AO_OWN ? rb : ca + AO_OWN;
+            const int nown = cb > ca ? (int)(cb - ca) : 0;
+            const int ncar = first ? nin : 0;
+            if (nown == 0 && ncar == 0) break;
+            group_by_key(S, nown + ncar, [&](int i) -> unsigned {
+                const int32_t r = S.rok[i];
+                if (r < 0) return (unsigned)AO_NONE;
+                if (r >= ca && r < cb) return (unsigned)(r - ca);
+                if (ncar) {
+                    const int o = hash_find(S, r);
+                    if (o >= 0) return (unsigned)(nown + o);
+                }
+                return (unsigned)AO_NONE;
+            });
+            // ranges ordered by kernel count, longest first (counting sort on
+            // a capped length), dealt out snake-wise for balance
+            const int nact = nown + ncar;
+            for (int i = threadIdx.x; i <= AO_LBUCKETS; i += AO_THREADS) S.lcount[i] = 0;
+            __syncthreads();
+            for (int a = threadIdx.x; a < nact; a += AO_THREADS) {
+                const int len = S.soff[a + 1] - S.soff[a];
+                atomicAdd(&S.lcount[AO_LBUCKETS - 1 - (len < AO_LBUCKETS - 1 ? len : AO_LBUCKETS - 1)], 1u);
+            }
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                unsigned run = 0;
+                for (int b = 0; b < AO_LBUCKETS; ++b) { unsigned x = S.lcount[b]; S.lcount[b] = run; run += x; }
+            }
+            __syncthreads();
+            for (int a = threadIdx.x; a < nact; a += AO_THREADS) {
+                const int len = S.soff[a + 1] - S.soff[a];
+                const unsigned pos = atomicAdd(&S.lcount[AO_LBUCKETS - 1 - (len < AO_LBUCKETS - 1 ? len : AO_LBUCKETS - 1)], 1u);
+                S.order[pos] = (uint16_t)a;
+            }
+            __syncthreads();
+            for (int g = 0; g * AO_THREADS < nact; ++g) {
+                const int a = g * AO_THREADS + ((g & 1) ? AO_THREADS - 1 - (int)threadIdx.x : (int)threadIdx.x);
+                if (a >= nact) continue;
+                const int key = S.order[a];
+                int64_t r;
+                Acc acc;
+                if (key < nown) {
+                    r = ca + key;
+                    if ((int64_t)A.r_op[r] >= A.in.n_ops) continue;   // not an operator range
+                    acc.init();
+                } else {
+                    const int o = key - nown;
+                    r = rng_tab[cur][o];
+                    acc = acc_tab[cur][o];
+                }
+                for (int q = S.soff[key]; q < S.soff[key + 1]; ++q) {
+                    const int i = S.klist[q];
+                    const int64_t k = k0 + i;
+                    acc.accumulate(A.in.dur[k], A.in.ncu_idx[k] >= 0, &S.rows[i * (NC / 4)]);
+                }
+                const long long e = A.r_end[r];
+                if (e >= t_next) {
+                    const int o2 = atomicAdd(&S.nopen_out, 1);
+                    if (o2 < AO_OPEN) {
+                        acc_tab[cur ^ 1][o2] = acc;
+                        rng_tab[cur ^ 1][o2] = (int32_t)r;
+                        atomicMax(&S.max_end_out, e);
+                    } else {
+                        set_flag(A.st, F_AGG_MISS);             // carry table full: the general path redoes it
+                    }
+                    continue;
+                }
+                acc.write(A.in, A.r_op[r]);
+                seen += (unsigned long long)acc.kc;
+                bad |= acc.bad;
+            }
+            __syncthreads();
+        }
+        if (threadIdx.x == 0) {
+            S.nopen_in = S.nopen_out < AO_OPEN ? S.nopen_out : AO_OPEN;
+            S.max_end_in = S.max_end_out;
+        }
+        cur ^= 1;
+        __syncthreads();
+    }
+    // ranges still carried here ended before the next tile
+    for (int o = threadIdx.x; o < S.nopen_in; o += AO_THREADS) {
+        const Acc acc = acc_tab[cur][o];
+        acc.write(A.in, A.r_op[rng_tab[cur][o]]);
+        seen += (unsigned long long)acc.kc;
+        bad |= acc.bad;
+    }
+    if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_err(A.st, ERR_INVALID);
+    block_add_u64(seen, &A.st->cnt[C_AGG_SEEN], S.red);
 }
 
 // Op ids held by no operator range: empty records.
@@ -377,9 +571,24 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
         return OPATTR_E_INVALID_ARG;
     if ((reinterpret_cast<uintptr_t>(ncu->counters) & 15) != 0) return OPATTR_E_INVALID_ARG;
 
-    const int64_t nt = (K + AGG_TILE - 1) / AGG_TILE;
+    const int64_t nt = (K + AO_TILE - 1) / AO_TILE;   // tiles of the owned-range path
+    int sms = 0, per_sm = 0;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
+    {
+        static unsigned attr_done = 0;
+        if (c.device < 32 && !(attr_done & (1u << c.device))) {
+            cudaFuncSetAttribute(k_agg_owned, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(OwnSmem));
+            attr_done |= 1u << c.device;
+        }
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_agg_owned, AO_THREADS, sizeof(OwnSmem));
+        cudaGetLastError();
+    }
+    const int64_t max_grid = (int64_t)std::max(1, sms) * std::max(1, per_sm);
+    const int64_t tpb = std::max<int64_t>(1, (nt + max_grid - 1) / max_grid);
+    const int64_t ogrid = nt > 0 ? (nt + tpb - 1) / tpb : 1;
     Need nd;
     nd.add<unsigned>((O + 31) / 32 + 1).add<int64_t>(nt + 1);
+    nd.add<Acc>(ogrid * 2 * AO_OPEN).add<int32_t>(ogrid * 2 * AO_OPEN);
     for (int i = 0; i < 7; ++i) nd.add<uint32_t>(K);
     nd.add<uint32_t>(radix_hist_elems(K)).add<uint32_t>(scan_scratch_elems(std::max(radix_hist_elems(K), K)));
     opattr_status st = ensure_arena(c, nd.bytes + 4096);
@@ -388,15 +597,17 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     if ((st = reset_status(c))) return st;
     unsigned *bitmap = a.take<unsigned>((O + 31) / 32 + 1);
     int64_t *band = a.take<int64_t>(nt + 1);
-    if (!bitmap || !band) return OPATTR_E_OOM;
+    Acc *open_acc = a.take<Acc>(ogrid * 2 * AO_OPEN);
+    int32_t *open_range = a.take<int32_t>(ogrid * 2 * AO_OPEN);
+    if (!bitmap || !band || !open_acc || !open_range) return OPATTR_E_OOM;
     cudaMemsetAsync(bitmap, 0, sizeof(unsigned) * ((O + 31) / 32 + 1), c.stream);
     if (K > 0) {
-        launch(c, "agg_check_kernels", k_agg_check_kernels, dim3(grid_for(K, 256, 65535)), dim3(256), 0, kern->dur_ns,
+        launch(c, "agg_check_kernels", k_agg_check_kernels, dim3(grid_for(K, 256 * 8, REDUCE_GRID)), dim3(256), 0, kern->dur_ns,
                rok, nidx, rng->op_id, K, R, M, O, c.d_status);
         check_kernel_order(c, kern->stream, kern->start_ns, K);
     }
     if (R > 0)
-        launch(c, "agg_check_ranges", k_agg_check_ranges, dim3(grid_for(R, 256, 65535)), dim3(256), 0, rng->start_ns,
+        launch(c, "agg_check_ranges", k_agg_check_ranges, dim3(grid_for(R, 256 * 8, REDUCE_GRID)), dim3(256), 0, rng->start_ns,
                rng->op_id, R, O, bitmap, c.d_status);
     if ((st = read_status(c))) return st;
     if (c.h_status->err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
@@ -427,19 +638,31 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
                rng->start_ns, R, nt, band);
         OwnArgs A;
         A.in = in;
+        A.M = M;
+        A.identity = !(flags & F_IDX_NOT_ID);
         A.k_start = kern->start_ns;
         A.rok = rok;
         A.K = K;
         A.r_end = rng->end_ns;
         A.r_op = rng->op_id;
         A.band = band;
+        A.nt = nt;
+        A.tiles_per_block = tpb;
+        A.wait_cycles = c.cfg.spin_limit > 0 ? c.cfg.spin_limit : (1ll << 31);
+        {
+            const char *fault = getenv("OPATTR_FAULT");
+            A.withhold_copy = fault && strcmp(fault, "wait") == 0;
+        }
+        A.open_acc = open_acc;
+        A.open_range = open_range;
         A.st = c.d_status;
-        launch(c, "agg_owned", k_agg_owned, dim3((unsigned)nt), dim3(AGG_THREADS), 0, A);
+        launch(c, "agg_owned", k_agg_owned, dim3((unsigned)ogrid), dim3(AO_THREADS), sizeof(OwnSmem), A);
         launch(c, "agg_fill_unreferenced", k_agg_fill_unreferenced, dim3(grid_for(O, 256, 65535)), dim3(256), 0,
                (const unsigned *)bitmap, in);
         if ((st = read_status(c))) return st;
         if (c.h_status->err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
-        fast = c.h_status->cnt[C_AGG_SEEN] == c.h_status->cnt[C_ATTR_K];
+        if (c.h_status->err & ERR_TIMEOUT) return OPATTR_E_TIMEOUT;
+        fast = !(c.h_status->flags & F_AGG_MISS) && c.h_status->cnt[C_AGG_SEEN] == c.h_status->cnt[C_ATTR_K];
     }
     if (!fast) {
         uint32_t *flag = a.take<uint32_t>(K), *pos = a.take<uint32_t>(K), *keys = a.take<uint32_t>(K);

@@ -31,6 +31,7 @@ enum FlagBit : unsigned {
     F_NAMES_DIFFER = 8u,  // ncu names differ from replayed names in time order
     F_OP_DUP = 16u,       // two operator ranges share an op id
     F_AGG_MISS = 32u,     // the owned-range aggregation missed kernels
+    F_IDX_NOT_ID = 64u,   // some kernel's ncu row index is neither its own index nor -1
 };
 enum CountSlot {
     C_NAMES_MISMATCH = 0,
@@ -195,5 +196,75 @@ __device__ __forceinline__ T block_sum(T v, T *warp_buf) {
     block_exclusive_scan(v, warp_buf, &total);
     return total;
 }
+
+// Sum v over the block and add the total to *dst with one atomic.  Every
+// thread of the block must call it (it synchronises the block).
+__device__ __forceinline__ void block_add_u64(unsigned long long v, unsigned long long *dst,
+                                              unsigned long long *warp_buf) {
+    unsigned long long t = block_sum<unsigned long long>(v, warp_buf);
+    if (threadIdx.x == 0 && t) atomicAdd(dst, t);
+}
+
+// Stable grouping of a block's entries by key.  The block's warps own
+// consecutive runs of PER_WARP entries; entry i has key key_of(i) < nkeys or
+// GROUP_NONE.  On return soff[0..nkeys] hold the group offsets and klist the
+// entry indices grouped by key, in index order within a group.  wcnt is a
+// [warps][wstride] scratch of 16-bit counters (wstride >= nkeys).  Warps rank
+// their entries 32 at a time with __match_any_sync peer groups.  Every thread
+// of the block must call it; it ends with a barrier.
+constexpr unsigned GROUP_NONE = 0xFFFFu;
+template <int THREADS, int PER_WARP, typename KeyFn>
+__device__ __forceinline__ void block_group_by_key(int nkeys, KeyFn key_of, uint16_t *wcnt, int wstride,
+                                                   uint16_t *soff, uint16_t *klist, uint32_t *wbuf) {
+    constexpr int WARPS = THREADS / 32;
+    const unsigned w = threadIdx.x >> 5, lane = lane_id(), lt = lanemask_lt();
+    for (int q = 0; q < WARPS; ++q)
+        for (int k = threadIdx.x; k < nkeys; k += THREADS) wcnt[q * wstride + k] = 0;
+    __syncthreads();
+    uint16_t rank[PER_WARP / 32];
+    uint16_t key[PER_WARP / 32];
+#pragma unroll
+    for (int it = 0; it < PER_WARP / 32; ++it) {
+        const int i = w * PER_WARP + it * 32 + lane;
+        const unsigned k = key_of(i);
+        const unsigned peers = __match_any_sync(0xffffffffu, k);
+        const unsigned before = k != GROUP_NONE ? wcnt[w * wstride + k] : 0u;
+        __syncwarp();
+        if (k != GROUP_NONE && (peers & lt) == 0) wcnt[w * wstride + k] = (uint16_t)(before + __popc(peers));
+        __syncwarp();
+        rank[it] = (uint16_t)(before + __popc(peers & lt));
+        key[it] = (uint16_t)k;
+    }
+    __syncthreads();
+    unsigned carry = 0;
+    for (int b = 0; b < nkeys; b += THREADS) {
+        const int k = b + threadIdx.x;
+        unsigned tot = 0;
+        if (k < nkeys) {
+#pragma unroll
+            for (int q = 0; q < WARPS; ++q) {
+                unsigned x = wcnt[q * wstride + k];
+                wcnt[q * wstride + k] = (uint16_t)tot;
+                tot += x;
+            }
+        }
+        unsigned all;
+        const unsigned ex = block_exclusive_scan<unsigned>(tot, wbuf, &all);
+        if (k < nkeys) soff[k] = (uint16_t)(carry + ex);
+        carry += all;
+    }
+    if (threadIdx.x == 0) soff[nkeys] = (uint16_t)carry;
+    __syncthreads();
+#pragma unroll
+    for (int it = 0; it < PER_WARP / 32; ++it) {
+        const unsigned k = key[it];
+        if (k != GROUP_NONE) klist[soff[k] + wcnt[w * wstride + k] + rank[it]] = (uint16_t)(w * PER_WARP + it * 32 + lane);
+    }
+    __syncthreads();
+}
+
+// Blocks for grid-stride reductions: enough to fill the GPU, few enough that
+// one atomic per block stays cheap.
+constexpr unsigned REDUCE_GRID = 2048;
 
 }  // namespace opattr

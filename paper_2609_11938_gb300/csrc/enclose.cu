@@ -26,8 +26,9 @@ namespace opattr {
 constexpr int LEVELS = 256 * 32;
 constexpr int ENC_THREADS = 256;
 constexpr int ENC_TILE = 2048;          // kernels per tile
-constexpr int ENC_WIN_CAP = 5120;       // staged range entries per tile
-constexpr int ENC_ACT_CAP = 1024;       // active (stream, depth) levels per tile
+constexpr int ENC_WIN_CAP = 3072;       // staged range entries per tile
+constexpr int ENC_ACT_CAP = 2048;       // active (stream, depth) levels per tile
+constexpr int ENC_CHUNK = ENC_TILE / ENC_THREADS;   // consecutive same-stream kernels per thread
 constexpr uint32_t KIND_OP = 0, KIND_NONOP = 1, KIND_STRUCT = 2;
 
 __device__ __forceinline__ uint32_t kind_of(uint32_t op) {
@@ -174,6 +175,7 @@ struct EncArgs {
     int nl;
     int64_t nt;
     const uint16_t *cbase;      // [256] first compact level of a stream
+    const uint16_t *level_of_compact;   // [nl] level key (stream * 32 + depth) of a compact level
     const uint8_t *ndepth;      // [256] levels of a stream (depths 0 .. n-1)
     int32_t *out_range;
     uint8_t *out_nop;
@@ -187,6 +189,11 @@ struct EncSmem {
     uint16_t act_cnt[ENC_ACT_CAP];  // window length
     int32_t act_gpos[ENC_ACT_CAP];  // global level position of the window's first entry (-1 none)
     uint16_t sbase[256];            // first active slot of a present stream
+    uint32_t kt[ENC_TILE];          // the tile's kernel times, relative to the tile base (+1, clamped)
+    uint8_t ks[ENC_TILE];           // the tile's kernel streams
+    uint16_t klist[ENC_TILE];       // tile positions grouped by stream
+    uint16_t wcnt[ENC_THREADS / 32][256];
+    uint16_t soff[257];
     uint32_t present[8];
     uint32_t wbuf[33];
     int slow;
@@ -207,19 +214,14 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
     if (threadIdx.x < 8) S.present[threadIdx.x] = 0;
     __syncthreads();
 
-    constexpr int PER = ENC_TILE / ENC_THREADS;
-    uint8_t ks[PER];
-    long long kt[PER];
     const long long tbase = A.k_start[A.korder ? A.korder[pos0] : pos0];
-#pragma unroll
-    for (int j = 0; j < PER; ++j) {
-        int64_t p = pos0 + j * ENC_THREADS + threadIdx.x;
-        if (j * ENC_THREADS + threadIdx.x < cnt) {
-            int64_t k = A.korder ? A.korder[p] : p;
-            ks[j] = A.k_stream[k];
-            kt[j] = A.k_start[k];
-            atomicOr(&S.present[ks[j] >> 5], 1u << (ks[j] & 31));
-        }
+    for (int j = threadIdx.x; j < cnt; j += ENC_THREADS) {
+        const int64_t p = pos0 + j;
+        const int64_t k = A.korder ? A.korder[p] : p;
+        const unsigned s = A.k_stream[k];
+        S.ks[j] = (uint8_t)s;
+        S.kt[j] = rel32(A.k_start[k], tbase);
+        atomicOr(&S.present[s >> 5], 1u << (s & 31));
     }
     __syncthreads();
 
@@ -231,26 +233,27 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
         unsigned off = block_exclusive_scan<unsigned>(n, S.wbuf, &tot);
         S.sbase[s] = (uint16_t)(off < ENC_ACT_CAP ? off : ENC_ACT_CAP);
         if (threadIdx.x == 0) S.nact = (int)tot;
-        __syncthreads();
         if (tot <= ENC_ACT_CAP && n) {
-            for (unsigned d = 0; d < n; ++d) {
-                int l = A.cbase[s] + d;
-                int32_t lo = A.P[t * A.nl + l], hi = A.P[(t + 1) * A.nl + l];
-                int32_t first = lo < 0 ? 0 : lo;
+            const unsigned cb = A.cbase[s];
+            for (unsigned d = 0; d < n; ++d) S.act_off[off + d] = (uint16_t)(cb + d);   // compact level, for now
+        }
+        __syncthreads();
+        // window bounds of every active level, one thread per level
+        if (tot <= ENC_ACT_CAP) {
+            for (unsigned a = threadIdx.x; a < tot; a += ENC_THREADS) {
+                const int l = S.act_off[a];
+                const int32_t lo = A.P[t * A.nl + l], hi = A.P[(t + 1) * A.nl + l];
+                const int32_t first = lo < 0 ? 0 : lo;
                 int32_t c = hi - first + 1;
                 if (hi < 0) c = 0;
-                S.act_cnt[off + d] = (uint16_t)(c < 0xFFFF ? c : 0xFFFF);
-                S.act_gpos[off + d] = (int32_t)(A.lvl_off[s * 32 + d] + first);
+                S.act_cnt[a] = (uint16_t)(c < 0xFFFF ? c : 0xFFFF);
+                S.act_gpos[a] = (int32_t)(A.lvl_off[A.level_of_compact[l]] + first);
             }
         }
     }
     __syncthreads();
-    long long tlast = kt[0];
-    {
-        // span of the tile: its last kernel (time order) minus its first
-        int64_t pl = pos0 + cnt - 1;
-        tlast = A.k_start[A.korder ? A.korder[pl] : pl];
-    }
+    // span of the tile: its last kernel (time order) minus its first
+    const long long tlast = A.k_start[A.korder ? A.korder[pos0 + cnt - 1] : pos0 + cnt - 1];
     int slow = S.nact > ENC_ACT_CAP || (tlast - tbase) >= 0xFFFFFFF0ll;
     if (!slow) {
         // window offsets: exclusive scan of counts over active slots
@@ -279,42 +282,89 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
                 S.wi[o + e] = A.li[g + e];
             }
         }
-        __syncthreads();
+        // kernels grouped by stream, so a warp's lanes share windows and
+        // loop trip counts
+        block_group_by_key<ENC_THREADS, ENC_TILE / (ENC_THREADS / 32)>(
+            256, [&](int j) -> unsigned { return j < cnt ? (unsigned)S.ks[j] : GROUP_NONE; }, &S.wcnt[0][0], 256,
+            S.soff, S.klist, S.wbuf);
+        // Each thread sweeps ENC_CHUNK consecutive kernels of one stream in
+        // time order.  Per depth it keeps the window position of the last
+        // range starting at or before the current kernel; positions only move
+        // forward, so after one search per depth the sweep advances them by
+        // comparison.
+        constexpr int RD = 8;                     // depths whose positions stay in registers
+        int cur_s = -1, nd = 0, a0 = 0;
+        int pr[RD];                               // window position + 1 (0 none, -1 not searched yet)
 #pragma unroll
-        for (int j = 0; j < PER; ++j) {
-            if (j * ENC_THREADS + threadIdx.x >= cnt) break;
-            const unsigned s = ks[j];
-            const uint32_t T = rel32(kt[j], tbase);
-            const int nd = A.ndepth[s];
-            const int a0 = S.sbase[s];
+        for (int d = 0; d < RD; ++d) pr[d] = -1;
+        for (int u = 0; u < ENC_CHUNK; ++u) {
+            const int idx = threadIdx.x * ENC_CHUNK + u;
+            if (idx >= cnt) break;
+            const int j = S.klist[idx];
+            const int64_t k = A.korder ? A.korder[pos0 + j] : pos0 + j;
+            const int s = S.ks[j];
+            const uint32_t T = S.kt[j];
+            if (s != cur_s) {
+                cur_s = s;
+                nd = A.ndepth[s];
+                a0 = S.sbase[s];
+#pragma unroll
+                for (int d = 0; d < RD; ++d) pr[d] = -1;
+            }
             int32_t ans = -1;
             int nop = 0;
-            for (int d = 0; d < nd; ++d) {
-                int c = S.act_cnt[a0 + d], o = S.act_off[a0 + d];
-                int x = o, y = o + c;               // first staged entry with start > T
+            bool alive = true;
+#pragma unroll
+            for (int d = 0; d < RD; ++d) {
+                if (alive && d < nd) {
+                    const int c = S.act_cnt[a0 + d], o = S.act_off[a0 + d];
+                    int p;                          // last window position with start <= T, or -1
+                    if (pr[d] < 0) {
+                        int x = o, y = o + c;
+                        while (x < y) {
+                            const int m = (x + y) >> 1;
+                            if (S.ws[m] <= T) x = m + 1; else y = m;
+                        }
+                        p = x - o - 1;
+                    } else {
+                        p = pr[d] - 1;
+                        while (p + 1 < c && S.ws[o + p + 1] <= T) ++p;
+                    }
+                    pr[d] = p + 1;
+                    if (p < 0 || S.we[o + p] < T) {
+                        alive = false;
+                    } else {
+                        const uint32_t info = S.wi[o + p];
+                        const uint32_t kind = info >> 30;
+                        if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
+                        else if (kind == KIND_OP) { ans = (int32_t)(info & 0x3FFFFFFFu); nop++; }
+                    }
+                }
+            }
+            for (int d = RD; alive && d < nd; ++d) {   // deeper levels: one search each
+                const int c = S.act_cnt[a0 + d], o = S.act_off[a0 + d];
+                int x = o, y = o + c;
                 while (x < y) {
-                    int m = (x + y) >> 1;
+                    const int m = (x + y) >> 1;
                     if (S.ws[m] <= T) x = m + 1; else y = m;
                 }
                 if (x == o || S.we[x - 1] < T) break;
-                uint32_t info = S.wi[x - 1];
-                uint32_t kind = info >> 30;
+                const uint32_t info = S.wi[x - 1];
+                const uint32_t kind = info >> 30;
                 if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
                 else if (kind == KIND_OP) { ans = (int32_t)(info & 0x3FFFFFFFu); nop++; }
             }
-            int64_t p = pos0 + j * ENC_THREADS + threadIdx.x;
-            int64_t k = A.korder ? A.korder[p] : p;
             A.out_range[k] = ans;
             if (A.out_nop) A.out_nop[k] = (uint8_t)nop;
         }
         return;
     }
     // slow tile: search the global level lists inside the window bounds
-#pragma unroll 1
-    for (int j = 0; j < PER; ++j) {
-        if (j * ENC_THREADS + threadIdx.x >= cnt) break;
-        const unsigned s = ks[j];
-        const long long T = kt[j];
+    for (int j = threadIdx.x; j < cnt; j += ENC_THREADS) {
+        const int64_t p = pos0 + j;
+        const int64_t k = A.korder ? A.korder[p] : p;
+        const unsigned s = A.k_stream[k];
+        const long long T = A.k_start[k];
         const int nd = A.ndepth[s];
         int32_t ans = -1;
         int nop = 0;
@@ -334,8 +384,6 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
             if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
             else if (kind == KIND_OP) { ans = (int32_t)(info & 0x3FFFFFFFu); nop++; }
         }
-        int64_t p = pos0 + j * ENC_THREADS + threadIdx.x;
-        int64_t k = A.korder ? A.korder[p] : p;
         A.out_range[k] = ans;
         if (A.out_nop) A.out_nop[k] = (uint8_t)nop;
     }
@@ -508,6 +556,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     A.nl = nl;
     A.nt = nt;
     A.cbase = d_cbase;
+    A.level_of_compact = d_loc;
     A.ndepth = d_ndep;
     A.out_range = out_range;
     A.out_nop = out_nop;

@@ -3,16 +3,17 @@
 //
 // GB300 issues fp64 FMA/add at ~0.5 T instr/s and f32<->f64 / i64->f32
 // conversions at ~0.6 T/s, against ~35 T/s for fp32 FMA.  The per-kernel work
-// therefore stays in fp32 pairs: a value is hi + lo with |lo| <= ulp(hi)/2,
-// about 48 significant bits.  Products use the FMA error term (Dekker's
-// product), sums use Knuth's two-sum followed by Dekker's fast two-sum
-// renormalisation.  Weights (durations) and weight sums stay exact in int64.
-// The final doubles are assembled from the pair with integer operations only.
+// therefore stays in fp32 pairs: a value is hi + lo, about 48 significant
+// bits.  Products use the FMA error term (Dekker's product); sums use Knuth's
+// two-sum into a running (hi, lo) pair whose lo collects the rounding errors
+// and is folded back into hi (Dekker's fast two-sum) every RENORM terms and
+// at the end.  Weights (durations) and weight sums stay exact in int64.  The
+// final doubles are assembled from the pair with integer operations only.
 //
-// Accuracy: each accumulation step adds a relative error of about 2^-47 of
-// the running sum, so n terms stay within n * 2^-47 (1e-9 up to ~140k terms
-// per operator; the long-op path splits sums into blocks).  Every helper
-// assumes finite inputs; NaN and infinity are filtered before.
+// Accuracy: a step adds a relative error of about 2^-47 of the running sum,
+// so n terms stay within n * 2^-47 (1e-9 for up to ~1.4e5 terms per
+// operator).  Helpers assume finite inputs; NaN and infinity are filtered
+// before.
 #pragma once
 #include <stdint.h>
 
@@ -29,39 +30,46 @@ __device__ __forceinline__ ff two_sum(float a, float b) {
     float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
     return ff{s, e};
 }
-// s + e == a + b exactly when |a| >= |b| (Dekker fast two-sum)
+// s + e == a + b exactly when |a| >= |b| or a == 0 (Dekker fast two-sum)
 __device__ __forceinline__ ff fast_two_sum(float a, float b) {
     float s = __fadd_rn(a, b);
     float e = __fsub_rn(b, __fsub_rn(s, a));
     return ff{s, e};
 }
-// acc += (xh + xl)
-__device__ __forceinline__ void ff_add(ff &acc, float xh, float xl) {
+// acc.hi + acc.lo += xh + xl, leaving lo unnormalised (see renorm)
+__device__ __forceinline__ void ff_accum(ff &acc, float xh, float xl) {
     ff s = two_sum(acc.hi, xh);
-    float e = __fadd_rn(s.lo, __fadd_rn(acc.lo, xl));
-    acc = fast_two_sum(s.hi, e);
+    acc.hi = s.hi;
+    acc.lo = __fadd_rn(acc.lo, __fadd_rn(s.lo, xl));
 }
-// m * (dh + dl) as a pair (product error from the FMA, m*dl rounded once)
-__device__ __forceinline__ ff ff_mul_f(float m, ff d) {
-    float p = __fmul_rn(m, d.hi);
-    float pe = __fmaf_rn(m, d.hi, -p);
-    float pl = __fmaf_rn(m, d.lo, pe);
-    return ff{p, pl};
+__device__ __forceinline__ void ff_renorm(ff &acc) {
+    // |acc.lo| stays far below |acc.hi| between renormalisations unless the
+    // running sum cancelled; two_sum keeps the pair exact either way
+    acc = two_sum(acc.hi, acc.lo);
 }
 
-// Non-negative int64 as a pair: exact below 2^48, else within 2^-48.
-__device__ __forceinline__ ff ff_from_i64(long long d) {
+// Non-negative int64 as a normalised pair hi + lo (|lo| <= ulp(hi) / 2):
+// exact below 2^48, within 2^-48 relative above.
+__device__ __forceinline__ ff split_i64(long long d) {
     unsigned long long u = (unsigned long long)d;
+    if (u < (1ull << 24)) return ff{__uint2float_rn((unsigned)u), 0.f};
     if (u < (1ull << 48)) {
-        float a = __uint2float_rn((unsigned)(u >> 24)) * 16777216.0f;   // exact: < 2^24 times 2^24
-        float b = __uint2float_rn((unsigned)(u & 0xFFFFFFu));            // exact: < 2^24
+        float a = __uint2float_rn((unsigned)(u >> 24)) * 16777216.0f;   // exact: the high 24 bits
+        float b = __uint2float_rn((unsigned)(u & 0xFFFFFFu));            // exact: the low 24 bits
         return two_sum(a, b);
     }
     int s = 64 - __clzll(u) - 24;
     unsigned long long A = u >> s, B = u - (A << s);
-    float a = ldexpf(__uint2float_rn((unsigned)A), s);
-    float b = __ull2float_rn(B);
-    return two_sum(a, b);
+    return two_sum(ldexpf(__uint2float_rn((unsigned)A), s), __ull2float_rn(B));
+}
+
+// m * (d.hi + d.lo) for a normalised d, as a pair: the first product exact
+// through its FMA error, the second (2^-24 smaller) rounded once
+__device__ __forceinline__ ff mul_split(float m, ff d) {
+    float p = __fmul_rn(m, d.hi);
+    float pe = __fmaf_rn(m, d.hi, -p);
+    float pl = __fmaf_rn(m, d.lo, pe);
+    return ff{p, pl};
 }
 
 // A finite float as a signed integer significand m and exponent e: x = m * 2^e.
@@ -102,32 +110,40 @@ __device__ __forceinline__ double f32_to_f64_bits(float x) {
     return i64_scaled_to_f64((long long)m, e);
 }
 
-// hi + lo as the nearest double (within one ulp when |lo| <= ulp(hi)).
+// hi + lo as a double for a normalised pair (|lo| <= ulp(hi) / 2): hi's 24
+// significand bits followed by lo's bits, truncated below 2^-53 of hi
+// (within one double ulp).
 __device__ __forceinline__ double ff_to_f64(ff v) {
-    int eh, el;
-    int mh = f32_decompose(v.hi, &eh);
+    const unsigned uh = __float_as_uint(v.hi);
+    const int exh = (int)((uh >> 23) & 0xFF);
+    if (exh == 0) return f32_to_f64_bits(v.hi);       // zero or subnormal hi: a normalised lo is negligible
+    int el;
     int ml = f32_decompose(v.lo, &el);
-    if (mh == 0) return f32_to_f64_bits(v.lo);
-    const int F = eh - 38;
-    long long acc = (long long)mh << 38;
-    int sh = el - F;
-    if (ml != 0) {
-        if (sh >= 0 && sh <= 38) acc += (long long)ml << sh;
-        else if (sh < 0 && sh > -63) acc += ((long long)ml) >> (-sh);
-    }
-    return i64_scaled_to_f64(acc, F);
+    if (uh >> 31) ml = -ml;                            // work on |hi|; lo enters with the relative sign
+    // value = (mh * 2^29 + ml * 2^(el - (exh - 150) + 29)) * 2^(exh - 150 - 29)
+    long long m = (long long)((uh & 0x7FFFFFu) | 0x800000u) << 29;
+    const int sh = el - (exh - 150) + 29;
+    if (ml != 0 && sh > -40) m += sh >= 0 ? ((long long)ml << sh) : ((long long)ml >> (-sh));
+    // m is within a factor 2 of 2^52; renormalise by at most one bit
+    int E = exh - 150 - 29 + 52;       // exponent of bit 52
+    if (m >= (1ll << 53)) { m >>= 1; E++; }
+    else if (m < (1ll << 52)) { m <<= 1; E--; }
+    const unsigned long long bits = ((unsigned long long)(uh >> 31) << 63) | ((unsigned long long)(E + 1023) << 52) |
+                                    ((unsigned long long)m & ((1ull << 52) - 1));
+    return __longlong_as_double((long long)bits);
 }
 
-// (n.hi + n.lo) / D for an int64 D > 0, as the nearest double (within a few
-// units of 2^-46 relative).
+// (n.hi + n.lo) / D for an int64 D > 0, as a double within a few units of
+// 2^-46 relative: q1 from an approximate reciprocal, then one correction from
+// the exact residual.
 __device__ __forceinline__ double ff_div_i64_to_f64(ff n, long long D) {
-    ff d = ff_from_i64(D);
-    float q1 = __fdiv_rn(n.hi, d.hi);
-    float p = __fmul_rn(q1, d.hi);
-    float pe = __fmaf_rn(q1, d.hi, -p);
-    float p2 = __fmul_rn(q1, d.lo);
-    float r = __fadd_rn(__fsub_rn(__fsub_rn(__fsub_rn(n.hi, p), pe), p2), n.lo);
-    float q2 = __fdiv_rn(r, d.hi);
+    const ff d = split_i64(D);
+    float inv;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(inv) : "f"(d.hi));
+    const float q1 = __fmul_rn(n.hi, inv);
+    const float r0 = __fmaf_rn(-q1, d.hi, n.hi);            // exact residual of the leading quotient
+    const float r = __fadd_rn(__fmaf_rn(-q1, d.lo, r0), n.lo);
+    const float q2 = __fmul_rn(r, inv);
     return ff_to_f64(fast_two_sum(q1, q2));
 }
 

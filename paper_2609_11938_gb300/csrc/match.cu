@@ -91,7 +91,13 @@ __global__ void k_max_u32(const uint32_t *__restrict__ a, int64_t n, unsigned lo
         uint32_t x = __shfl_xor_sync(0xffffffffu, m, o);
         m = x > m ? x : m;
     }
-    if (lane_id() == 0 && m) atomicMax(out, (unsigned long long)m);
+    __shared__ uint32_t sm[32];
+    if (lane_id() == 0) sm[threadIdx.x >> 5] = m;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (unsigned w = 1; w < blockDim.x / 32; ++w) m = sm[w] > m ? sm[w] : m;
+        if (m) atomicMax(out, (unsigned long long)m);
+    }
 }
 __global__ void k_check_layers(const int32_t *__restrict__ layer, int64_t n, int32_t n_layers,
                                const int32_t *__restrict__ rep_layer, DevStatus *st) {
@@ -102,9 +108,9 @@ __global__ void k_check_layers(const int32_t *__restrict__ layer, int64_t n, int
         if (l < -1 || l >= n_layers) bad = 1;
         else rep += (l < 0 || rep_layer[l] == l);
     }
-    rep = warp_sum(rep);
+    __shared__ unsigned long long red[33];
     if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_err(st, ERR_INVALID);
-    if (lane_id() == 0 && rep) atomicAdd(&st->cnt[C_REPLAYED], rep);
+    block_add_u64(rep, &st->cnt[C_REPLAYED], red);
 }
 
 __device__ __forceinline__ int64_t lower_bound_u32(const uint32_t *a, int64_t n, uint32_t x) {
@@ -151,15 +157,11 @@ __global__ void k_ordinal_join(const uint32_t *__restrict__ skn, const uint32_t 
         unmatched += idx < 0;
         names_bad += head && ck != cq;
     }
-    direct = warp_sum(direct);
-    unmatched = warp_sum(unmatched);
-    names_bad = warp_sum(names_bad);
+    __shared__ unsigned long long red[33];
     if (__any_sync(0xffffffffu, err) && lane_id() == 0) set_err(st, ERR_COUNT);
-    if (lane_id() == 0) {
-        if (direct) atomicAdd(&st->cnt[C_DIRECT], direct);
-        if (unmatched) atomicAdd(&st->cnt[C_COUNT_UNMATCHED], unmatched);
-        if (names_bad) atomicAdd(&st->cnt[C_NAMES_MISMATCH], names_bad);
-    }
+    block_add_u64(direct, &st->cnt[C_DIRECT], red);
+    block_add_u64(unmatched, &st->cnt[C_COUNT_UNMATCHED], red);
+    block_add_u64(names_bad, &st->cnt[C_NAMES_MISMATCH], red);
 }
 
 // Names that have ncu rows but no replayed kernel at all.
@@ -172,11 +174,9 @@ __global__ void k_ncu_only_names(const uint32_t *__restrict__ snn, int64_t M, co
         int64_t lo = lower_bound_u32(skn, nrep, name);
         bad += lo == nrep || skn[lo] != name;
     }
-    bad = warp_sum(bad);
-    if (lane_id() == 0 && bad) {
-        atomicAdd(&st->cnt[C_NAMES_MISMATCH], bad);
-        if (mode == OPATTR_MISMATCH_ERROR) set_err(st, ERR_COUNT);
-    }
+    __shared__ unsigned long long red[33];
+    if (__any_sync(0xffffffffu, bad != 0) && lane_id() == 0 && mode == OPATTR_MISMATCH_ERROR) set_err(st, ERR_COUNT);
+    block_add_u64(bad, &st->cnt[C_NAMES_MISMATCH], red);
 }
 
 // Broadcast.  i runs over layer-tagged kernels sorted by (layer, time).
@@ -205,12 +205,9 @@ __global__ void k_dedup_broadcast(const uint32_t *__restrict__ sll, const uint32
         bc += idx >= 0;
         miss += idx < 0;
     }
-    bc = warp_sum(bc);
-    miss = warp_sum(miss);
-    if (lane_id() == 0) {
-        if (bc) atomicAdd(&st->cnt[C_BROADCAST], bc);
-        if (miss) atomicAdd(&st->cnt[C_DEDUP_MISMATCH], miss);
-    }
+    __shared__ unsigned long long red[33];
+    block_add_u64(bc, &st->cnt[C_BROADCAST], red);
+    block_add_u64(miss, &st->cnt[C_DEDUP_MISMATCH], red);
 }
 
 // ------------------------------------------------------------------ host
@@ -276,7 +273,7 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     if (dedup_on && dd->n_layers > 0)
         cudaMemcpyAsync(d_rep, rep_layer.data(), sizeof(int32_t) * dd->n_layers, cudaMemcpyHostToDevice, c.stream);
 
-    const unsigned gK = grid_for(K, 256, 65535);
+    const unsigned gK = grid_for(K, 256, REDUCE_GRID);
     check_kernel_order(c, kern->stream, kern->start_ns, K);
     if (dedup_on && K > 0)
         launch(c, "check_layers", k_check_layers, dim3(gK), dim3(256), 0, kern->layer_id, K, dd->n_layers,
@@ -320,7 +317,7 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     }
     bool direct_done = false;
     if (dedup_on && nrep == M && nrep > 0) {
-        launch(c, "match_identity_list", k_match_identity_list, dim3(grid_for(nrep, 256, 65535)), dim3(256), 0,
+        launch(c, "match_identity_list", k_match_identity_list, dim3(grid_for(nrep, 256, REDUCE_GRID)), dim3(256), 0,
                (const uint32_t *)rk, kern->name_id, ncu->name_id, nrep, out_idx, out_kind, c.d_status);
         if ((st = read_status(c))) return st;
         direct_done = !(c.h_status->flags & F_NAMES_DIFFER);
@@ -330,7 +327,7 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     if (!direct_done && (nrep > 0 || M > 0)) {
         cudaMemsetAsync(dsm, 0, sizeof(unsigned long long), c.stream);
         if (nrep > 0) {
-            launch(c, "gather_names", k_gather_u32, dim3(grid_for(nrep, 256, 65535)), dim3(256), 0, kern->name_id,
+            launch(c, "gather_names", k_gather_u32, dim3(grid_for(nrep, 256, REDUCE_GRID)), dim3(256), 0, kern->name_id,
                    (const uint32_t *)rk, nrep, k0);
             launch(c, "max_name", k_max_u32, dim3(grid_for(nrep, 256, 4096)), dim3(256), 0, (const uint32_t *)k0, nrep,
                    dsm);
@@ -346,11 +343,11 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
         if (nrep > 0) radix_sort_pairs<uint32_t>(c, k0, s0, s1, s2, nrep, bits, true, hist, part, &skn, &skj);
         if (M > 0) radix_sort_pairs<uint32_t>(c, n0, n1, n2, n3, M, bits, true, hist, part, &snn, &snj);
         if (nrep > 0)
-            launch(c, "ordinal_join", k_ordinal_join, dim3(grid_for(nrep, 256, 65535)), dim3(256), 0,
+            launch(c, "ordinal_join", k_ordinal_join, dim3(grid_for(nrep, 256, REDUCE_GRID)), dim3(256), 0,
                    (const uint32_t *)skn, (const uint32_t *)skj, (const uint32_t *)rk, nrep, (const uint32_t *)snn,
                    (const uint32_t *)snj, M, mode, out_idx, out_kind, c.d_status);
         if (M > 0)
-            launch(c, "ncu_only_names", k_ncu_only_names, dim3(grid_for(M, 256, 65535)), dim3(256), 0,
+            launch(c, "ncu_only_names", k_ncu_only_names, dim3(grid_for(M, 256, REDUCE_GRID)), dim3(256), 0,
                    (const uint32_t *)snn, M, (const uint32_t *)skn, nrep, mode, c.d_status);
     }
     if (dedup_on && K > 0) {
@@ -365,13 +362,13 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
         if ((st = read_u64(c, dsm + 1, &ntag_h))) return st;
         const int64_t nlk = (int64_t)(ntag_h & 0xFFFFFFFFull);
         if (nlk > 0) {
-            launch(c, "gather_layers", k_gather_i32_as_u32, dim3(grid_for(nlk, 256, 65535)), dim3(256), 0,
+            launch(c, "gather_layers", k_gather_i32_as_u32, dim3(grid_for(nlk, 256, REDUCE_GRID)), dim3(256), 0,
                    kern->layer_id, (const uint32_t *)lk, nlk, k0);
             uint32_t *sll, *slj;
             radix_sort_pairs<uint32_t>(c, k0, s0, s1, s2, nlk,
                                        bits_for((uint64_t)(dd->n_layers > 0 ? dd->n_layers - 1 : 0)), true, hist, part,
                                        &sll, &slj);
-            launch(c, "dedup_broadcast", k_dedup_broadcast, dim3(grid_for(nlk, 256, 65535)), dim3(256), 0,
+            launch(c, "dedup_broadcast", k_dedup_broadcast, dim3(grid_for(nlk, 256, REDUCE_GRID)), dim3(256), 0,
                    (const uint32_t *)sll, (const uint32_t *)slj, (const uint32_t *)lk, nlk, (const int32_t *)d_rep,
                    kern->name_id, out_idx, out_kind, c.d_status);
         }

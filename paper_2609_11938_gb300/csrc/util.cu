@@ -5,31 +5,45 @@
 namespace opattr {
 
 constexpr int CHK_THREADS = 256;
-constexpr int CHK_ITEMS = 8;
 
-// Each thread checks CHK_ITEMS consecutive pairs (i, i+1); loads are
-// coalesced across the block.
+// Grid-stride over groups of four consecutive kernels (16-byte loads when
+// the arrays allow), comparing each (start, stream) with its successor; min /
+// max and the order flag are reduced per block and published with one atomic
+// each.
 __global__ void __launch_bounds__(CHK_THREADS) k_check_kernel_order(const uint8_t *__restrict__ stream,
                                                                     const int64_t *__restrict__ start, int64_t n,
-                                                                    DevStatus *st) {
+                                                                    int vec, DevStatus *st) {
     __shared__ long long smin[CHK_THREADS / 32], smax[CHK_THREADS / 32];
-    __shared__ int bad;
-    if (threadIdx.x == 0) bad = 0;
-    __syncthreads();
-    const int64_t base = (int64_t)blockIdx.x * CHK_THREADS * CHK_ITEMS;
+    __shared__ int sbad[CHK_THREADS / 32];
     long long mn = LLONG_MAX, mx = LLONG_MIN;
     int unsorted = 0;
+    const int64_t ngroups = (n + 3) / 4;
+    for (int64_t g = (int64_t)blockIdx.x * CHK_THREADS + threadIdx.x; g < ngroups;
+         g += (int64_t)gridDim.x * CHK_THREADS) {
+        const int64_t i0 = g * 4;
+        long long t[5];
+        unsigned s[5];
+        if (vec && i0 + 4 <= n) {
+            const longlong2 a = reinterpret_cast<const longlong2 *>(start)[g * 2];
+            const longlong2 b = reinterpret_cast<const longlong2 *>(start)[g * 2 + 1];
+            const uchar4 q = reinterpret_cast<const uchar4 *>(stream)[g];
+            t[0] = a.x; t[1] = a.y; t[2] = b.x; t[3] = b.y;
+            s[0] = q.x; s[1] = q.y; s[2] = q.z; s[3] = q.w;
+        } else {
 #pragma unroll
-    for (int it = 0; it < CHK_ITEMS; ++it) {
-        int64_t i = base + it * CHK_THREADS + threadIdx.x;
-        if (i < n) {
-            long long t = start[i];
-            mn = t < mn ? t : mn;
-            mx = t > mx ? t : mx;
-            if (i + 1 < n) {
-                long long u = start[i + 1];
-                unsorted |= (u < t) || (u == t && stream[i + 1] < stream[i]);
+            for (int u = 0; u < 4; ++u) {
+                t[u] = i0 + u < n ? start[i0 + u] : LLONG_MAX;
+                s[u] = i0 + u < n ? stream[i0 + u] : 255u;
             }
+        }
+        t[4] = i0 + 4 < n ? start[i0 + 4] : LLONG_MAX;
+        s[4] = i0 + 4 < n ? stream[i0 + 4] : 255u;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            if (i0 + u >= n) break;
+            mn = t[u] < mn ? t[u] : mn;
+            mx = t[u] > mx ? t[u] : mx;
+            if (i0 + u + 1 < n) unsorted |= (t[u + 1] < t[u]) || (t[u + 1] == t[u] && s[u + 1] < s[u]);
         }
     }
 #pragma unroll
@@ -38,16 +52,20 @@ __global__ void __launch_bounds__(CHK_THREADS) k_check_kernel_order(const uint8_
         mn = a < mn ? a : mn;
         mx = b > mx ? b : mx;
     }
-    if (unsorted) bad = 1;
-    if (lane_id() == 0) { smin[threadIdx.x >> 5] = mn; smax[threadIdx.x >> 5] = mx; }
+    unsorted = __any_sync(0xffffffffu, unsorted);
+    if (lane_id() == 0) {
+        smin[threadIdx.x >> 5] = mn;
+        smax[threadIdx.x >> 5] = mx;
+        sbad[threadIdx.x >> 5] = unsorted;
+    }
     __syncthreads();
     if (threadIdx.x == 0) {
-        for (int w = 1; w < CHK_THREADS / 32; ++w) {
+        int bad = 0;
+        for (int w = 0; w < CHK_THREADS / 32; ++w) {
             mn = smin[w] < mn ? smin[w] : mn;
             mx = smax[w] > mx ? smax[w] : mx;
+            bad |= sbad[w];
         }
-        mn = smin[0] < mn ? smin[0] : mn;
-        mx = smax[0] > mx ? smax[0] : mx;
         atomicMin(&st->mm[MM_KSTART_MIN], mn);
         atomicMax(&st->mm[MM_KSTART_MAX], mx);
         if (bad) set_flag(st, F_K_UNSORTED);
@@ -56,8 +74,9 @@ __global__ void __launch_bounds__(CHK_THREADS) k_check_kernel_order(const uint8_
 
 void check_kernel_order(Ctx &c, const uint8_t *stream, const int64_t *start, int64_t n) {
     if (n <= 0) return;
-    launch(c, "check_kernel_order", k_check_kernel_order, dim3(grid_for(n, CHK_THREADS * CHK_ITEMS)),
-           dim3(CHK_THREADS), 0, stream, start, n, c.d_status);
+    const int vec = ((reinterpret_cast<uintptr_t>(start) & 15) == 0) && ((reinterpret_cast<uintptr_t>(stream) & 3) == 0);
+    launch(c, "check_kernel_order", k_check_kernel_order, dim3(grid_for(n, CHK_THREADS * 16, REDUCE_GRID)),
+           dim3(CHK_THREADS), 0, stream, start, n, vec, c.d_status);
 }
 
 __global__ void k_time_keys(const uint8_t *__restrict__ stream, const int64_t *__restrict__ start, int64_t n,

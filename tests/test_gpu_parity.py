@@ -215,6 +215,26 @@ def test_oom_injection(opa, monkeypatch):
     ctx.close()
 
 
+def test_bounded_wait_timeout(opa, monkeypatch):
+    """The aggregation's wait for a tile's bulk copy is bounded.  With the copy
+    withheld (announced to the barrier, never issued) the wait runs out: the
+    call returns E_TIMEOUT and the device and context stay usable."""
+    t = tracegen.generate("gpt2")
+    ctx = opa.Context(0, spin_limit=20000)
+    tr = opa.to_device(t)
+    st, rk, _ = ctx.enclose(tr)
+    st, idx, _, _ = ctx.match(tr)
+    monkeypatch.setenv("OPATTR_FAULT", "wait")
+    with pytest.raises(opa.OpattrError) as ei:
+        ctx.aggregate(tr, rk, idx)
+    assert ei.value.status == opa.E_TIMEOUT
+    monkeypatch.delenv("OPATTR_FAULT")
+    st, ops, tot = ctx.aggregate(tr, rk, idx)        # same context, short bound, real copies
+    assert st == opa.OK
+    ctx.close()
+    assert_parity(gpu_run(t), oracle.run(t, enclose_mode="indexed"))
+
+
 def test_large_full_parity(opa):
     """The 20M-kernel benchmark trace, in the configuration the benchmark runs,
     against the oracle on every output."""
