@@ -256,6 +256,30 @@ int opattr_timing_report(opattr_ctx *ctx, const char **names, double *total_ms, 
 void opattr_timing_reset(opattr_ctx *ctx);
 int64_t opattr_launch_count(const opattr_ctx *ctx);
 
+/* No-allocation variant of opattr_match.  The paper has no counterpart: it
+ * exists for callers that cannot allocate device memory -- an attribution
+ * pass running inside the profiled application (an injection library or a
+ * profiler callback) must leave that application's device memory untouched,
+ * and some hosts own all device memory through a caching allocator or forbid
+ * allocation on a hot path.
+ *   Same inputs, outputs, ordering and status codes as opattr_match with
+ *   layer deduplication off, on the stream `cuda_stream` of the current
+ *   device, with `mismatch` in place of the context's mode.  No context.
+ *   All scratch (about 6 MB) lives in one fixed device array inside the
+ *   library; every GPU that loads the library holds it until exit.
+ *   kernels->n and ncu->n must each be at most OPATTR_MATCH_NOALLOC_MAX,
+ *   else OPATTR_E_INVALID_ARG.
+ *   The first call on a device looks up the array's device address; make
+ *   that first call before any stream capture.
+ *   Calls share the array.  Host threads are serialised inside the call, and
+ *   each call finishes its device work before it returns; a caller that lets
+ *   other work on the GPU touch the same memory concurrently races.
+ *   Allocates nothing: no cudaMalloc, cudaFree or pinned host memory. */
+#define OPATTR_MATCH_NOALLOC_MAX 65536
+opattr_status opattr_match_noalloc(const opattr_kernels *kernels, const opattr_ncu *ncu,
+                                   opattr_mismatch_mode mismatch, int32_t *ncu_idx_of_kernel, uint8_t *match_kind,
+                                   opattr_match_summary *host_summary, void *cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -24,7 +24,7 @@ __all__ = [
     "E_COUNT_MISMATCH", "E_CUDA", "E_OOM", "E_TIMEOUT", "E_STATE", "OP_STRUCTURAL", "OP_NONOP",
     "N_COUNTERS", "OpattrError", "Context", "library", "build",
     "opattr_create", "opattr_enclose", "opattr_match", "opattr_aggregate", "opattr_destroy",
-    "opattr_status_string",
+    "opattr_status_string", "opattr_match_noalloc", "MATCH_NOALLOC_MAX",
 ]
 
 OK, W_COUNT_MISMATCH, W_DEDUP_MISMATCH = 0, 1, 2
@@ -33,6 +33,7 @@ E_CUDA, E_OOM, E_TIMEOUT, E_STATE = -5, -6, -7, -8
 OP_STRUCTURAL = 0xFFFFFFFF
 OP_NONOP = 0xFFFFFFFE
 N_COUNTERS = 20
+MATCH_NOALLOC_MAX = 65536
 MISMATCH = {"skip_name": 0, "prefix": 1, "error": 2}
 
 _vp = ctypes.c_void_p
@@ -119,6 +120,8 @@ def library():
             lib.opattr_timing_reset.restype = None
             lib.opattr_launch_count.argtypes = [_vp]
             lib.opattr_launch_count.restype = ctypes.c_int64
+            lib.opattr_match_noalloc.argtypes = [P(Kernels), P(Ncu), ctypes.c_int, _vp, _vp, P(MatchSummary), _vp]
+            lib.opattr_match_noalloc.restype = ctypes.c_int
             for f in ("opattr_create", "opattr_enclose", "opattr_match", "opattr_aggregate", "opattr_set_timing",
                       "opattr_timing_report"):
                 getattr(lib, f).restype = ctypes.c_int
@@ -163,6 +166,15 @@ def opattr_aggregate(handle, kernels: Kernels, ranges: Ranges, rok_ptr: int, ncu
     return library().opattr_aggregate(handle, ctypes.byref(kernels), ctypes.byref(ranges), _vp(rok_ptr),
                                       ctypes.byref(ncu), _vp(idx_ptr), ctypes.c_uint32(n_ops), ctypes.byref(out),
                                       ctypes.byref(totals))
+
+
+def opattr_match_noalloc(kernels: Kernels, ncu: Ncu, mismatch: str, idx_ptr: int, kind_ptr: int | None,
+                         summary: MatchSummary, stream: int | None) -> int:
+    """opattr_match without a context and without any device allocation, for
+    callers that must not allocate (see include/opattr.h); inputs of at most
+    OPATTR_MATCH_NOALLOC_MAX kernels and rows."""
+    return library().opattr_match_noalloc(ctypes.byref(kernels), ctypes.byref(ncu), MISMATCH[mismatch],
+                                          _vp(idx_ptr), _vp(kind_ptr or 0), ctypes.byref(summary), _vp(stream or 0))
 
 
 def opattr_destroy(handle) -> None:

@@ -29,6 +29,7 @@ opattr_status cuda_status(Ctx &c, cudaError_t e) {
 // makes growth fail, to exercise the out-of-memory path without a GPU fault.
 opattr_status ensure_arena(Ctx &c, size_t bytes) {
     if (bytes <= c.arena_cap) return OPATTR_OK;
+    if (c.arena_fixed) return OPATTR_E_OOM;
     const char *fault = getenv("OPATTR_FAULT");
     if (fault && strcmp(fault, "alloc") == 0) return OPATTR_E_OOM;
     if (c.arena) {

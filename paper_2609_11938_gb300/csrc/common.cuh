@@ -72,6 +72,7 @@ struct Ctx {
     // scratch arena (bump allocation, reset per call)
     char *arena = nullptr;
     size_t arena_cap = 0, arena_used = 0;
+    bool arena_fixed = false;        // the arena is caller-provided memory: never grow or free it
     // status block
     DevStatus *d_status = nullptr;
     DevStatus *h_status = nullptr;   // pinned mirror
