@@ -189,20 +189,35 @@ struct Acc {
 __global__ void k_agg_check_kernels(const int64_t *__restrict__ dur, const int32_t *__restrict__ rok,
                                     const int32_t *__restrict__ nidx, const uint32_t *__restrict__ r_op, int64_t K,
                                     int64_t R, int64_t M, int64_t n_ops, DevStatus *st) {
+    constexpr int U = 4;                    // kernels per thread per round, loads issued together
     unsigned long long tot = 0, att = 0, natt = 0, nmatch = 0;
     int bad = 0, not_id = 0;
-    for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < K; k += (int64_t)gridDim.x * blockDim.x) {
-        long long d = dur[k];
-        int32_t r = rok[k], j = nidx[k];
-        not_id |= j >= 0 && j != k;
-        if (d < 0 || r < -1 || r >= R || j < -1 || j >= M) { bad = 1; continue; }
-        tot += (unsigned long long)d;
-        if (r >= 0) {
-            uint32_t op = r_op[r];
-            if ((int64_t)op >= n_ops) { bad = 1; continue; }
-            att += (unsigned long long)d;
-            natt++;
-            nmatch += j >= 0;
+    for (int64_t base = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * U; base < K;
+         base += (int64_t)gridDim.x * blockDim.x * U) {
+        long long d[U];
+        int32_t r[U], j[U];
+        uint32_t op[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const bool in = base + u < K;
+            d[u] = in ? dur[base + u] : 0;
+            r[u] = in ? rok[base + u] : -1;
+            j[u] = in ? nidx[base + u] : -1;
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) op[u] = (r[u] >= 0 && r[u] < R) ? r_op[r[u]] : 0u;
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            if (base + u >= K) continue;
+            not_id |= j[u] >= 0 && j[u] != base + u;
+            if (d[u] < 0 || r[u] < -1 || r[u] >= R || j[u] < -1 || j[u] >= M) { bad = 1; continue; }
+            tot += (unsigned long long)d[u];
+            if (r[u] >= 0) {
+                if ((int64_t)op[u] >= n_ops) { bad = 1; continue; }
+                att += (unsigned long long)d[u];
+                natt++;
+                nmatch += j[u] >= 0;
+            }
         }
     }
     __shared__ unsigned long long red[33];
@@ -602,7 +617,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     if (!bitmap || !band || !open_acc || !open_range) return OPATTR_E_OOM;
     cudaMemsetAsync(bitmap, 0, sizeof(unsigned) * ((O + 31) / 32 + 1), c.stream);
     if (K > 0) {
-        launch(c, "agg_check_kernels", k_agg_check_kernels, dim3(grid_for(K, 256 * 8, REDUCE_GRID)), dim3(256), 0, kern->dur_ns,
+        launch(c, "agg_check_kernels", k_agg_check_kernels, dim3(grid_for(K, 256 * 16, REDUCE_GRID)), dim3(256), 0, kern->dur_ns,
                rok, nidx, rng->op_id, K, R, M, O, c.d_status);
         check_kernel_order(c, kern->stream, kern->start_ns, K);
     }

@@ -9,7 +9,7 @@
 #include <string>
 #include <vector>
 
-#include "../../include/opattr.h"
+#include "opattr.h"
 
 namespace opattr {
 

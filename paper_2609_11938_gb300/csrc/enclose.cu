@@ -215,13 +215,28 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
     __syncthreads();
 
     const long long tbase = A.k_start[A.korder ? A.korder[pos0] : pos0];
-    for (int j = threadIdx.x; j < cnt; j += ENC_THREADS) {
-        const int64_t p = pos0 + j;
-        const int64_t k = A.korder ? A.korder[p] : p;
-        const unsigned s = A.k_stream[k];
-        S.ks[j] = (uint8_t)s;
-        S.kt[j] = rel32(A.k_start[k], tbase);
-        atomicOr(&S.present[s >> 5], 1u << (s & 31));
+    {
+        // all loads first, so they are in flight together
+        constexpr int PER = ENC_TILE / ENC_THREADS;
+        unsigned sv[PER];
+        long long tv[PER];
+#pragma unroll
+        for (int u = 0; u < PER; ++u) {
+            const int j = u * ENC_THREADS + threadIdx.x;
+            const int64_t p = pos0 + (j < cnt ? j : 0);
+            const int64_t k = A.korder ? A.korder[p] : p;
+            sv[u] = A.k_stream[k];
+            tv[u] = A.k_start[k];
+        }
+#pragma unroll
+        for (int u = 0; u < PER; ++u) {
+            const int j = u * ENC_THREADS + threadIdx.x;
+            if (j < cnt) {
+                S.ks[j] = (uint8_t)sv[u];
+                S.kt[j] = rel32(tv[u], tbase);
+                atomicOr(&S.present[sv[u] >> 5], 1u << (sv[u] & 31));
+            }
+        }
     }
     __syncthreads();
 
@@ -271,16 +286,21 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
         slow = S.nwin > ENC_WIN_CAP;
     }
     if (!slow) {
-        // stage: one warp per active level
-        const unsigned w = threadIdx.x >> 5, lane = lane_id();
-        for (int a = w; a < S.nact; a += ENC_THREADS / 32) {
-            int c = S.act_cnt[a], o = S.act_off[a];
-            int64_t g = S.act_gpos[a];
-            for (int e = lane; e < c; e += 32) {
-                S.ws[o + e] = rel32(A.ls[g + e], tbase);
-                S.we[o + e] = rel32(A.le[g + e], tbase);
-                S.wi[o + e] = A.li[g + e];
+        // stage the windows: one thread per staged entry (its level found by a
+        // search over the window offsets), so all loads of a round are in flight
+        // together
+        const int nact = S.nact, nwin = S.nwin;
+        for (int e = threadIdx.x; e < nwin; e += ENC_THREADS) {
+            int x = 0, y = nact;                   // last active level with offset <= e
+            while (y - x > 1) {
+                const int m = (x + y) >> 1;
+                if (S.act_off[m] <= e) x = m; else y = m;
             }
+            while (x + 1 < nact && S.act_off[x + 1] <= e && S.act_cnt[x] == 0) ++x;
+            const int64_t g = S.act_gpos[x] + (e - S.act_off[x]);
+            S.ws[e] = rel32(A.ls[g], tbase);
+            S.we[e] = rel32(A.le[g], tbase);
+            S.wi[e] = A.li[g];
         }
         // kernels grouped by stream, so a warp's lanes share windows and
         // loop trip counts

@@ -23,11 +23,23 @@ namespace opattr {
 // ------------------------------------------------------------------ fast path
 __global__ void k_match_identity(const uint32_t *__restrict__ kname, const uint32_t *__restrict__ nname, int64_t n,
                                  int32_t *__restrict__ out_idx, uint8_t *__restrict__ out_kind, DevStatus *st) {
+    constexpr int U = 4;                    // elements per thread per round, loads issued together
     int bad = 0;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-        bad |= kname[i] != nname[i];
-        out_idx[i] = (int32_t)i;
-        if (out_kind) out_kind[i] = 1;
+    for (int64_t base = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * U; base < n;
+         base += (int64_t)gridDim.x * blockDim.x * U) {
+        uint32_t a[U], b[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            a[u] = base + u < n ? kname[base + u] : 0u;
+            b[u] = base + u < n ? nname[base + u] : 0u;
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            if (base + u >= n) continue;
+            bad |= a[u] != b[u];
+            out_idx[base + u] = (int32_t)(base + u);
+            if (out_kind) out_kind[base + u] = 1;
+        }
     }
     if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_flag(st, F_NAMES_DIFFER);
 }
@@ -280,7 +292,8 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
                (const int32_t *)d_rep, c.d_status);
     const bool try_identity = !dedup_on && K == M && K > 0;
     if (try_identity)
-        launch(c, "match_identity", k_match_identity, dim3(gK), dim3(256), 0, kern->name_id, ncu->name_id, K, out_idx,
+        launch(c, "match_identity", k_match_identity, dim3(grid_for(K, 256 * 16, REDUCE_GRID)), dim3(256), 0,
+               kern->name_id, ncu->name_id, K, out_idx,
                out_kind, c.d_status);
     if ((st = read_status(c))) return st;
     if (c.h_status->err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
