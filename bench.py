@@ -55,6 +55,33 @@ WORKLOADS = {
 }
 
 
+def source_digest():
+    """Digest of the CUDA sources (csrc/*.cu, *.cuh), to tie recorded ncu figures to the code they came from."""
+    import glob
+    import hashlib
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_11938_gb300", "csrc")
+    for p in sorted(glob.glob(os.path.join(csrc, "*.cu")) + glob.glob(os.path.join(csrc, "*.cuh"))):
+        h.update(os.path.basename(p).encode())
+        with open(p, "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel, workload, kernels):
+    """DRAM bytes per launch from profiles/traffic.txt, or None if absent or taken on other sources."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.txt")) as f:
+            lines = [ln.split() for ln in f if ln.strip() and not ln.startswith("#")]
+    except OSError:
+        return None
+    digest = source_digest()
+    for ln in lines:
+        if len(ln) == 5 and ln[0] == kernel and ln[1] == workload and int(ln[2]) == kernels and ln[3] == digest:
+            return int(ln[4])
+    return None
+
+
 def load_peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -378,7 +405,8 @@ def main():
                    "l2": "inputs larger than L2 (129 MB)" if flush is None else "L2 flushed before every step"},
         "roofline": {"bound": "hbm", "kernel": dname, "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": (achieved / peak) if achieved else None, "peak_kind": f"{peak_kind} copy bandwidth",
-                     "traffic": None, "alg_bytes_per_launch": dbytes, "avg_launch_ms": avg_s * 1e3,
+                     "traffic": recorded_traffic(dname, args.config, K), "alg_bytes_per_launch": dbytes,
+                     "avg_launch_ms": avg_s * 1e3,
                      "launches": dcount},
         "path_roofline": {"alg_bytes_per_step": path_bytes, "achieved_gbs": path_gbs,
                           "frac_of_8tbs": path_gbs / NOMINAL_HBM_GBS, "frac_of_measured": path_gbs / peak},
