@@ -32,15 +32,15 @@ PATH_BYTES = dict(kernel=29, range=22, ncu=84, op=184)
 
 # Per-launch algorithmic bytes of the kernels that can dominate a step.
 KERNEL_BYTES = {
-    "agg_owned": lambda K, R, M, O: 96 * K + 12 * R + 184 * O,
+    "agg_ops": lambda K, R, M, O: 96 * K + 188 * O,
     "enclose": lambda K, R, M, O: 14 * K + 20 * R,
+    "agg_fill": lambda K, R, M, O: 28 * K,
+    "agg_count": lambda K, R, M, O: 20 * K + 4 * O,
     "match_identity": lambda K, R, M, O: 13 * K,
-    "agg_check_kernels": lambda K, R, M, O: 20 * K,
     "check_kernel_order": lambda K, R, M, O: 9 * K,
     "check_ranges": lambda K, R, M, O: 18 * R,
     "level_gather": lambda K, R, M, O: 44 * R,
     "validate_levels": lambda K, R, M, O: 22 * R,
-    "agg_check_ranges": lambda K, R, M, O: 12 * R,
     "window_table": lambda K, R, M, O: 0,
 }
 

@@ -135,7 +135,8 @@ typedef struct {
     opattr_mismatch_mode mismatch; /* default OPATTR_MISMATCH_SKIP_NAME */
     int32_t dedup;                 /* 1: apply opattr_dedup when given (default 1) */
     int32_t checked;               /* reserved, 0 */
-    int64_t spin_limit;            /* bound on device-side waits (0 = default) */
+    int64_t spin_limit;            /* bound on device-side waits (0 = default); the current
+                                      kernels have none, so it is checked (>= 0) and unused */
 } opattr_config;
 
 /* Host-side result of opattr_match. */

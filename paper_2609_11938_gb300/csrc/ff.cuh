@@ -133,6 +133,47 @@ __device__ __forceinline__ double ff_to_f64(ff v) {
     return __longlong_as_double((long long)bits);
 }
 
+// hi + lo as a double for a normalised pair, with 32-bit integer operations:
+// hi's bits widened to a double, lo added to its 52-bit fraction as a signed
+// integer (exact while lo's bits reach no lower than 2^-52 of hi, else
+// truncated within one unit).  A normalised lo cannot carry the fraction out
+// of its binade; it can borrow out of it only when hi is a power of two, and
+// then one unit of the lower binade is half as large, so lo counts twice.
+// A zero hi gives +0; a subnormal hi takes ff_to_f64.
+__device__ __forceinline__ double ff_to_f64_fast(ff v) {
+    const unsigned uh = __float_as_uint(v.hi), ul = __float_as_uint(v.lo);
+    const unsigned exh = (uh >> 23) & 0xFFu, exl = (ul >> 23) & 0xFFu;
+    if (exh == 0) return (uh << 1) == 0 ? 0.0 : ff_to_f64(v);
+    const unsigned mh = uh & 0x7FFFFFu;
+    const unsigned ml = (ul & 0x7FFFFFu) | (exl ? 0x800000u : 0u);
+    const int s = (int)(exl ? exl : 1u) - (int)exh + 29;               // lo's unit against 2^-52 of hi
+    const bool relneg = ((uh ^ ul) >> 31) != 0;
+    unsigned d = s >= 0 ? (s < 32 ? ml << s : 0u) : (-s < 32 ? ml >> -s : 0u);
+    if (mh == 0 && relneg) d <<= 1;
+    const unsigned long long pat = ((unsigned long long)(((exh + 896u) << 20) | (mh >> 3)) << 32) | (mh << 29);
+    const unsigned long long r = relneg ? pat - d : pat + d;
+    return __longlong_as_double((long long)(r | ((unsigned long long)(uh >> 31) << 63)));
+}
+
+// 1 / D for an int64 D > 0 as a normalised pair within about 2^-46 relative:
+// an approximate reciprocal r, then r (1 + e) with e = 1 - D r.
+__device__ __forceinline__ ff ff_recip_i64(long long D) {
+    const ff d = split_i64(D);
+    float r;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(d.hi));
+    const float e = __fsub_rn(__fmaf_rn(-d.hi, r, 1.0f), __fmul_rn(d.lo, r));
+    return fast_two_sum(r, __fmul_rn(r, e));
+}
+
+// a * b as a double, a a pair (lo need not be normalised), b a normalised pair.
+__device__ __forceinline__ double ff_mul_to_f64(ff a, ff b) {
+    const float p = __fmul_rn(a.hi, b.hi);
+    float e = __fmaf_rn(a.hi, b.hi, -p);
+    e = __fmaf_rn(a.hi, b.lo, e);
+    e = __fmaf_rn(a.lo, b.hi, e);
+    return ff_to_f64_fast(fast_two_sum(p, e));
+}
+
 // (n.hi + n.lo) / D for an int64 D > 0, as a double within a few units of
 // 2^-46 relative: q1 from an approximate reciprocal, then one correction from
 // the exact residual.

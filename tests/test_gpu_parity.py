@@ -215,23 +215,86 @@ def test_oom_injection(opa, monkeypatch):
     ctx.close()
 
 
-def test_bounded_wait_timeout(opa, monkeypatch):
-    """The aggregation's wait for a tile's bulk copy is bounded.  With the copy
-    withheld (announced to the barrier, never issued) the wait runs out: the
-    call returns E_TIMEOUT and the device and context stay usable."""
-    t = tracegen.generate("gpt2")
-    ctx = opa.Context(0, spin_limit=20000)
-    tr = opa.to_device(t)
-    st, rk, _ = ctx.enclose(tr)
-    st, idx, _, _ = ctx.match(tr)
-    monkeypatch.setenv("OPATTR_FAULT", "wait")
-    with pytest.raises(opa.OpattrError) as ei:
-        ctx.aggregate(tr, rk, idx)
-    assert ei.value.status == opa.E_TIMEOUT
-    monkeypatch.delenv("OPATTR_FAULT")
-    st, ops, tot = ctx.aggregate(tr, rk, idx)        # same context, short bound, real copies
-    assert st == opa.OK
+def _agg_inputs(seed, K, seg_lens, n_small_ops, nan_frac=0.0):
+    """Aggregation-only inputs: ops 0..len(seg_lens)-1 get seg_lens[i] kernels,
+    the rest of the kernels fall on n_small_ops more ops or stay unattributed;
+    kernel order is shuffled so that every op's kernels are scattered."""
+    rng = np.random.default_rng(seed)
+    n_ops = len(seg_lens) + n_small_ops
+    op_of = np.full(K, -1, np.int64)
+    pos = 0
+    for i, n in enumerate(seg_lens):
+        op_of[pos:pos + n] = i
+        pos += n
+    rest = K - pos
+    op_of[pos:] = np.where(rng.random(rest) < 0.9, len(seg_lens) + rng.integers(0, n_small_ops, rest), -1)
+    op_of = op_of[rng.permutation(K)]
+    # one range per op id plus a few ranges sharing op ids (duplicates aggregate together)
+    r_op = np.concatenate([np.arange(n_ops), rng.integers(0, n_ops, 64)]).astype(np.uint32)
+    dup_of_op = {int(r_op[n_ops + q]): n_ops + q for q in range(64)}
+    rk = np.where(op_of >= 0, op_of, -1).astype(np.int32)
+    for k in np.nonzero(op_of >= 0)[0][::7]:              # some kernels through the duplicate ranges
+        if int(op_of[k]) in dup_of_op:
+            rk[k] = dup_of_op[int(op_of[k])]
+    dur = rng.lognormal(np.log(8000), 1.2, K).astype(np.int64)
+    M = K
+    counters = rng.uniform(0, 100, (M, 20)).astype(np.float32)
+    if nan_frac:
+        counters[rng.random((M, 20)) < nan_frac] = np.nan
+    idx = np.where(rng.random(K) < 0.95, np.arange(K), -1).astype(np.int32)
+    R = len(r_op)
+    t = tracegen.Trace(np.zeros(K, np.uint8), np.arange(K, dtype=np.int64), dur, np.zeros(K, np.uint32), None,
+                       np.zeros(R, np.uint8), np.arange(R, dtype=np.int64), np.arange(R, dtype=np.int64),
+                       np.zeros(R, np.uint8), r_op, n_ops, np.zeros(M, np.uint32), counters)
+    return t, rk, idx
+
+
+def _gpu_aggregate(opa, t, rk, idx, ctx=None):
+    import torch
+    own = ctx is None
+    ctx = ctx or opa.Context(0)
+    try:
+        tr = opa.to_device(t)
+        st, ops, tot = ctx.aggregate(tr, torch.from_numpy(rk).cuda(), torch.from_numpy(idx).cuda())
+        return st, {k: v.cpu().numpy() for k, v in ops.items()}, tot
+    finally:
+        if own:
+            ctx.close()
+
+
+def _check_aggregate(g, o):
+    gst, gops, gtot = g
+    ost, oops, otot = o
+    assert gst == ost
+    for k in ("kernel_count", "total_duration_ns", "matched_count"):
+        np.testing.assert_array_equal(gops[k], oops[k])
+    for c in range(20):
+        assert_close(gops["agg"][c], oops["agg"][c], what=f"counter {c}")
+    for k in ("total_ns", "attributed_ns", "kernels", "attributed_kernels", "matched_kernels"):
+        assert gtot[k] == otot[k], k
+
+
+@pytest.mark.parametrize("nan_frac", [0.0, 0.02])
+def test_aggregate_segment_lengths(opa, nan_frac):
+    """Ops whose kernels are walked by selection (<= 48), after an in-place
+    sort (49 .. 16384) and in list order (above), with kernels scattered over
+    the array, duplicate op ids and null counters: against the oracle."""
+    seg_lens = [1, 2, 48, 49, 300, 5000, 16384, 16385, 40000]
+    t, rk, idx = _agg_inputs(7, 200_000, seg_lens, 20_000, nan_frac)
+    o = oracle.aggregate(t.k_dur, rk, t.r_op, t.counters, idx, t.n_ops)
+    _check_aggregate(_gpu_aggregate(opa, t, rk, idx), o)
+
+
+def test_aggregate_reproducible(opa):
+    """Two runs give bit-identical records although the fill pass orders each
+    op's kernel list by atomics: segments are walked in ascending index."""
+    t, rk, idx = _agg_inputs(8, 300_000, [3000, 700], 40_000)
+    ctx = opa.Context(0)
+    a = _gpu_aggregate(opa, t, rk, idx, ctx)[1]
+    b = _gpu_aggregate(opa, t, rk, idx, ctx)[1]
     ctx.close()
+    for k in a:
+        assert np.array_equal(a[k].view(np.int64), b[k].view(np.int64)), k
     assert_parity(gpu_run(t), oracle.run(t, enclose_mode="indexed"))
 
 
