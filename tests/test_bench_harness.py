@@ -65,7 +65,7 @@ def test_two_gloo_ranks_combine():
     (r0, e0, t0, u0, c0), (r1, e1, t1, u1, c1) = res
     assert c0 == c1 == 8                              # 3 warm-up + 5 timed steps on each rank
     assert t0 == t1 == pytest.approx(max(e0, e1))     # max over ranks, same on every rank
-    assert e1 > e0                                    # the slower rank dominates
+    assert min(e0, e1) >= 5 * 0.02 * 0.95             # the closing barrier holds rank 0 until rank 1 is done
     assert u0 == u1 == 3000                           # units of both ranks
 
 
