@@ -328,7 +328,8 @@ __global__ void k_agg_count(const int64_t *__restrict__ dur, const int32_t *__re
                     nmatch += j[u] >= 0;
                 }
             }
-            const unsigned key = valid && r[u] >= 0 ? op[u] : 0xFFFFFFFFu;
+            // counted exactly as k_agg_fill places it: by range and op id alone
+            const unsigned key = (k < K && r[u] >= 0 && r[u] < R && (int64_t)op[u] < n_ops) ? op[u] : 0xFFFFFFFFu;
             const unsigned peers = __match_any_sync(0xffffffffu, key);
             if (key != 0xFFFFFFFFu && (peers & lanemask_lt()) == 0) atomicAdd(&cnt[key], (unsigned)__popc(peers));
         }
@@ -342,41 +343,50 @@ __global__ void k_agg_count(const int64_t *__restrict__ dur, const int32_t *__re
 }
 
 // ------------------------------------------------------------------ fill
-// list[off[op] + slot] = k for each valid attributed kernel; slots are taken
-// by atomics on cur[op] (zeroed), so a segment's order is arbitrary.
-__global__ void k_agg_fill(const int64_t *__restrict__ dur, const int32_t *__restrict__ rok,
-                           const int32_t *__restrict__ nidx, const uint32_t *__restrict__ r_op, int64_t K, int64_t R,
-                           int64_t M, int64_t n_ops, const uint32_t *__restrict__ off, uint32_t *__restrict__ cur,
+// list[off[op] + slot] = k for each attributed kernel with a valid range and
+// op id (the kernels k_agg_count counted); slots are taken by atomics on
+// cur[op] (zeroed).  Each warp fills a run of AF_RUN consecutive kernels 32 at
+// a time in index order, so an op whose kernels all lie in one run gets them
+// in ascending order; the ops pass sorts the few segments that do not.
+constexpr int AF_RUN = 2048;
+
+__global__ void k_agg_fill(const int32_t *__restrict__ rok, const uint32_t *__restrict__ r_op, int64_t K, int64_t R,
+                           int64_t n_ops, const uint32_t *__restrict__ off, uint32_t *__restrict__ cur,
                            uint32_t *__restrict__ list) {
-    for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k - threadIdx.x < K;
-         k += (int64_t)gridDim.x * blockDim.x) {
-        unsigned key = 0xFFFFFFFFu;
-        if (k < K) {
-            const int32_t r = rok[k], j = nidx[k];
-            const long long d = dur[k];
-            if (r >= 0 && r < R && d >= 0 && j >= -1 && j < M) {
+    const unsigned lane = lane_id();
+    const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / 32;
+    const int64_t nwarps = (int64_t)gridDim.x * blockDim.x / 32;
+    for (int64_t k0 = warp * AF_RUN; k0 < K; k0 += nwarps * AF_RUN) {
+        const int64_t k1 = k0 + AF_RUN < K ? k0 + AF_RUN : K;
+        int32_t r_next = k0 + lane < k1 ? rok[k0 + lane] : -1;
+        for (int64_t kb = k0; kb < k1; kb += 32) {
+            const int64_t k = kb + lane;
+            const int32_t r = r_next;
+            r_next = k + 32 < k1 ? rok[k + 32] : -1;           // the next group's ranges, loaded early
+            unsigned key = 0xFFFFFFFFu;
+            if (r >= 0 && r < R) {
                 const uint32_t op = r_op[r];
                 if ((int64_t)op < n_ops) key = op;
             }
+            const unsigned peers = __match_any_sync(0xffffffffu, key);
+            const int leader = __ffs(peers) - 1;
+            unsigned base = 0;
+            if (key != 0xFFFFFFFFu && (int)lane == leader) base = atomicAdd(&cur[key], (unsigned)__popc(peers));
+            base = __shfl_sync(0xffffffffu, base, leader);
+            if (key != 0xFFFFFFFFu) list[off[key] + base + __popc(peers & lanemask_lt())] = (uint32_t)k;
         }
-        const unsigned peers = __match_any_sync(0xffffffffu, key);
-        if (key == 0xFFFFFFFFu) continue;
-        const int leader = __ffs(peers) - 1;
-        unsigned base = 0;
-        if ((int)lane_id() == leader) base = atomicAdd(&cur[key], (unsigned)__popc(peers));
-        base = __shfl_sync(peers, base, leader);
-        list[off[key] + base + __popc(peers & lanemask_lt())] = (uint32_t)k;
     }
 }
 
 // ------------------------------------------------------------------ long segments
-// Segments longer than AG_SELECT_MAX are sorted by kernel index before the ops
+// Segments longer than AG_SHORT_MAX are sorted by kernel index before the ops
 // pass, one block per segment: up to SL_SMEM entries by a bitonic sort in
 // shared memory; longer ones in SL_SMEM runs sorted that way, then merged
 // pairwise through `tmp` (merge path: each thread merges an equal share of
 // the output after a binary search on its diagonal).
 constexpr int SL_THREADS = 256;
 constexpr int SL_SMEM = 8192;
+constexpr uint32_t AG_SHORT_MAX = 64;           // segments up to this length: sorted by one warp; longer: one block
 
 __global__ void k_agg_long_list(const uint32_t *__restrict__ off, int64_t n_ops, uint32_t limit,
                                 uint32_t *__restrict__ longs, unsigned *__restrict__ nlong) {
@@ -464,42 +474,27 @@ __global__ void __launch_bounds__(SL_THREADS) k_agg_sort_long(const uint32_t *__
 // similar length; warps share nothing and never wait for each other.  The
 // grid is what stays resident and takes the chunks in order, so the kernels
 // and outputs the GPU works on at any moment form one window that stays in
-// L2.  A segment is walked in ascending kernel index: a short one by repeated
-// minimum search over the segment (it stays in L1), a long one in order after
-// k_agg_sort_long.  The next kernel's duration and row index are loaded before
-// the current kernel is added.
+// L2.  Segments are walked in ascending kernel index: a short one is checked
+// and, in the rare case the fill left it out of order, insertion-sorted in
+// place by its thread; long ones were sorted by k_agg_sort_long.  The next
+// kernel's duration and row index are loaded before the current kernel is
+// added.
 constexpr int AG_THREADS = 128;
 constexpr int AG_WARPS = AG_THREADS / 32;
-constexpr int AG_CHUNK = 64;                    // op ids per warp and chunk
+constexpr int AG_CHUNK = 128;                   // op ids per warp and chunk
 constexpr int AG_LBUCKETS = 32;
-constexpr uint32_t AG_SELECT_MAX = 48;          // segments up to this length: selection order; longer: sorted
-
-// Next kernel of a segment in ascending index, at or above `from`.
-__device__ __forceinline__ uint32_t seg_next(const uint32_t *seg, uint32_t len, uint32_t from, bool sorted, uint32_t t) {
-    if (sorted) return seg[t];
-    uint32_t best = 0xFFFFFFFFu;
-    for (uint32_t u = 0; u < len; ++u) {
-        const uint32_t x = seg[u];
-        best = (x >= from && x < best) ? x : best;
-    }
-    return best;
-}
 
 // An op whose fast sums saw a null or infinite value: the segment again, in
 // the same order, with Acc.  Returns 1 if a value was infinite.
-__device__ __noinline__ int op_careful(const uint32_t *seg, uint32_t len, bool sorted, AggIn A, int64_t o) {
+__device__ __noinline__ int op_careful(const uint32_t *seg, uint32_t len, AggIn A, int64_t o) {
     Acc acc;
     acc.init();
-    uint32_t k = 0;
-    for (uint32_t t = 0; t < len; ++t) {
-        k = seg_next(seg, len, t == 0 ? 0u : k + 1, sorted, t);
-        acc.add(A, k);
-    }
+    for (uint32_t t = 0; t < len; ++t) acc.add(A, seg[t]);
     acc.write(A, o);
     return acc.bad;
 }
 
-__global__ void __launch_bounds__(AG_THREADS) k_agg_ops(const uint32_t *__restrict__ off, const uint32_t *__restrict__ list,
+__global__ void __launch_bounds__(AG_THREADS) k_agg_ops(const uint32_t *__restrict__ off, uint32_t *__restrict__ list,
                                                           AggIn A, DevStatus *st) {
     __shared__ uint32_t lcount_s[AG_WARPS][AG_LBUCKETS];
     __shared__ uint8_t order_s[AG_WARPS][AG_CHUNK];
@@ -546,22 +541,32 @@ __global__ void __launch_bounds__(AG_THREADS) k_agg_ops(const uint32_t *__restri
             if (i >= nchunk) continue;
             const int64_t o = o0 + order[i];
             const uint32_t s0 = off[o], len = off[o + 1] - s0;
-            const uint32_t *seg = list + s0;
-            const bool sorted = len <= 1 || len > AG_SELECT_MAX;     // long segments were sorted before
+            uint32_t *seg = list + s0;
+            if (len <= AG_SHORT_MAX) {                   // ascending unless the fill met the op in two runs
+                bool up = true;
+                for (uint32_t t = 1; t < len; ++t) up &= seg[t - 1] < seg[t];
+                if (!up) {
+                    for (uint32_t t = 1; t < len; ++t) {
+                        const uint32_t x = seg[t];
+                        uint32_t u = t;
+                        for (; u > 0 && seg[u - 1] > x; --u) seg[u] = seg[u - 1];
+                        seg[u] = x;
+                    }
+                }
+            }
             AccF acc;
             acc.init();
             if (len > 0) {
-                uint32_t k = seg_next(seg, len, 0, sorted, 0);
-                long long d = A.dur[k];
-                int32_t j = A.ncu_idx[k];
+                uint32_t kn = seg[0];
+                long long d = A.dur[kn];
+                int32_t j = A.ncu_idx[kn];
                 for (uint32_t t = 0; t < len; ++t) {
                     long long d2 = 0;
                     int32_t j2 = -1;
                     if (t + 1 < len) {
-                        const uint32_t k2 = seg_next(seg, len, k + 1, sorted, t + 1);
-                        d2 = A.dur[k2];
-                        j2 = A.ncu_idx[k2];
-                        k = k2;
+                        kn = seg[t + 1];
+                        d2 = A.dur[kn];
+                        j2 = A.ncu_idx[kn];
                     }
                     acc.accumulate(d, j >= 0,
                                    reinterpret_cast<const float4 *>(A.counters + (int64_t)(j >= 0 ? j : 0) * NC));
@@ -570,7 +575,7 @@ __global__ void __launch_bounds__(AG_THREADS) k_agg_ops(const uint32_t *__restri
                 }
             }
             if (acc.clean()) acc.write(A, o, (int)len);
-            else bad |= op_careful(seg, len, sorted, A, o);
+            else bad |= op_careful(seg, len, A, o);
         }
         __syncwarp();
     }
@@ -630,16 +635,16 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     if (O > 0) {
         scan_exclusive_u32(c, cnt, off, O + 1, part, nullptr);
         if (K > 0)
-            launch(c, "agg_fill", k_agg_fill, dim3(grid_for(K, 256, 65535)), dim3(256), 0, kern->dur_ns, rok, nidx,
-                   rng->op_id, K, R, M, O, (const uint32_t *)off, cur, list);
+            launch(c, "agg_fill", k_agg_fill, dim3(grid_for(K, 256 / 32 * AF_RUN, 65535)), dim3(256), 0, rok,
+                   rng->op_id, K, R, O, (const uint32_t *)off, cur, list);
         launch(c, "agg_long_list", k_agg_long_list, dim3(grid_for(O, 256, 4096)), dim3(256), 0, (const uint32_t *)off,
-               O, AG_SELECT_MAX, longs, nlong);
+               O, AG_SHORT_MAX, longs, nlong);
         int sms = 0;
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
         launch(c, "agg_sort_long", k_agg_sort_long, dim3(2 * std::max(1, sms)), dim3(SL_THREADS), 0, (const uint32_t *)off,
                (const uint32_t *)longs, (const unsigned *)nlong, list, tmp);
         launch(c, "agg_ops", k_agg_ops, dim3(ops_grid(c, O)), dim3(AG_THREADS), 0,
-               (const uint32_t *)off, (const uint32_t *)list, in, c.d_status);
+               (const uint32_t *)off, list, in, c.d_status);
     }
     if ((st = read_status(c))) return st;
     if (c.h_status->err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
