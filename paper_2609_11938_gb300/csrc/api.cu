@@ -156,11 +156,13 @@ opattr_status opattr_create(opattr_ctx **out, int device, void *cuda_stream, con
     bool fail = cudaMalloc(&c.d_status, sizeof(DevStatus)) != cudaSuccess;
     fail = fail || cudaMallocHost(&c.h_status, sizeof(DevStatus)) != cudaSuccess;
     fail = fail || cudaMallocHost(&c.h_init, sizeof(DevStatus)) != cudaSuccess;
+    fail = fail || cudaMallocHost(&c.h_levels, sizeof(uint32_t) * (N_LEVELS + 1)) != cudaSuccess;
     if (fail) {
         cudaGetLastError();
         if (c.d_status) cudaFree(c.d_status);
         if (c.h_status) cudaFreeHost(c.h_status);
         if (c.h_init) cudaFreeHost(c.h_init);
+        if (c.h_levels) cudaFreeHost(c.h_levels);
         delete x;
         return OPATTR_E_OOM;
     }
@@ -224,6 +226,7 @@ void opattr_destroy(opattr_ctx *ctx) {
         if (c.d_status) cudaFree(c.d_status);
         if (c.h_status) cudaFreeHost(c.h_status);
         if (c.h_init) cudaFreeHost(c.h_init);
+        if (c.h_levels) cudaFreeHost(c.h_levels);
         for (auto &p : c.pending) {
             cudaEventDestroy(p.second.first);
             cudaEventDestroy(p.second.second);

@@ -64,6 +64,8 @@ struct TimingSlot {
     int64_t launches;
 };
 
+constexpr int N_LEVELS = 256 * 32;   // (stream, depth) levels of the enclosure
+
 struct Ctx {
     int device = 0;
     cudaStream_t stream = nullptr;
@@ -77,6 +79,7 @@ struct Ctx {
     DevStatus *d_status = nullptr;
     DevStatus *h_status = nullptr;   // pinned mirror
     DevStatus *h_init = nullptr;     // pinned reset template
+    uint32_t *h_levels = nullptr;    // pinned host copy of the enclosure's level offsets [N_LEVELS + 1]
     // launch accounting
     int64_t launches = 0;
     bool timing = false;

@@ -23,7 +23,7 @@
 
 namespace opattr {
 
-constexpr int LEVELS = 256 * 32;
+constexpr int LEVELS = N_LEVELS;
 constexpr int ENC_THREADS = 256;
 constexpr int ENC_TILE = 2048;          // kernels per tile
 constexpr int ENC_WIN_CAP = 3072;       // staged range entries per tile
@@ -451,15 +451,22 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
 
     uint32_t *level_hist = a.take<uint32_t>(LEVELS + 1);
     uint32_t *lvl_off = a.take<uint32_t>(LEVELS + 1);
+    uint32_t *part = a.take<uint32_t>(part_n);
+    if (!level_hist || !lvl_off || !part) return OPATTR_E_OOM;
     cudaMemsetAsync(level_hist, 0, sizeof(uint32_t) * (LEVELS + 1), c.stream);
     if (R > 0)
         launch(c, "check_ranges", k_check_ranges, dim3(grid_for(R, RCHK_THREADS * RCHK_ITEMS)), dim3(RCHK_THREADS), 0,
                rng->stream, rng->start_ns, rng->end_ns, rng->depth, R, level_hist, c.d_status);
     check_kernel_order(c, kern->stream, kern->start_ns, K);
+    // the level offsets come back with the status: one synchronisation for both
+    scan_exclusive_u32(c, level_hist, lvl_off, LEVELS + 1, part, nullptr);
+    if (cudaMemcpyAsync(c.h_levels, lvl_off, sizeof(uint32_t) * (LEVELS + 1), cudaMemcpyDeviceToHost, c.stream) !=
+        cudaSuccess)
+        return cuda_status(c, cudaGetLastError());
     if ((st = read_status(c))) return st;
     if ((st = status_from_err(c.h_status->err))) return st;
     const bool k_sorted = !(c.h_status->flags & F_K_UNSORTED);
-    bool r_sorted = !(c.h_status->flags & F_R_UNSORTED);
+    const bool r_sorted = !(c.h_status->flags & F_R_UNSORTED);
     const long long rmin = c.h_status->mm[MM_RSTART_MIN], rmax = c.h_status->mm[MM_REND_MAX];
     const long long kmin = c.h_status->mm[MM_KSTART_MIN], kmax = c.h_status->mm[MM_KSTART_MAX];
     if (K > 0 && (kmax - kmin) >= (1ll << 55)) return OPATTR_E_INVALID_ARG;
@@ -471,19 +478,56 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
         return read_status(c);
     }
 
-    // ---- level lists
+    // ---- compact level table (host side, from the level offsets)
+    const uint32_t *off = c.h_levels;
+    std::vector<uint16_t> level_of_compact;
+    std::vector<uint16_t> cbase(256, 0);
+    std::vector<uint8_t> ndep(256, 0);
+    for (int s = 0; s < 256; ++s) {
+        cbase[s] = (uint16_t)level_of_compact.size();
+        int n = 0;
+        while (n < 32 && off[s * 32 + n + 1] > off[s * 32 + n]) {
+            level_of_compact.push_back((uint16_t)(s * 32 + n));
+            n++;
+        }
+        ndep[s] = (uint8_t)n;
+    }
+    const int nl = (int)level_of_compact.size();
+
     uint64_t *rk0 = a.take<uint64_t>(R), *rk1 = a.take<uint64_t>(R);
     uint32_t *rv0 = a.take<uint32_t>(R), *rv1 = a.take<uint32_t>(R);
     uint32_t *hist = a.take<uint32_t>(radix_hist_elems(R));
-    uint32_t *part = a.take<uint32_t>(part_n);
     int64_t *ls = a.take<int64_t>(R), *le = a.take<int64_t>(R);
     uint32_t *li = a.take<uint32_t>(R);
-    if (!rk0 || !rk1 || !rv0 || !rv1 || !hist || !part || !ls || !le || !li) return OPATTR_E_OOM;
+    uint16_t *d_loc = a.take<uint16_t>(LEVELS);
+    uint16_t *d_cbase = a.take<uint16_t>(256);
+    uint8_t *d_ndep = a.take<uint8_t>(256);
+    int32_t *P = a.take<int32_t>((nt + 1) * (int64_t)(nl > 0 ? nl : 1));
+    if (!rk0 || !rk1 || !rv0 || !rv1 || !hist || !ls || !le || !li || !d_loc || !d_cbase || !d_ndep || !P)
+        return OPATTR_E_OOM;
+    cudaMemcpyAsync(d_loc, level_of_compact.data(), sizeof(uint16_t) * (nl > 0 ? nl : 1), cudaMemcpyHostToDevice,
+                    c.stream);
+    cudaMemcpyAsync(d_cbase, cbase.data(), sizeof(uint16_t) * 256, cudaMemcpyHostToDevice, c.stream);
+    cudaMemcpyAsync(d_ndep, ndep.data(), 256, cudaMemcpyHostToDevice, c.stream);
+
+    // ---- kernel time order
+    uint32_t *korder = nullptr;
+    if (!k_sorted && K > 0) {
+        korder = kernel_time_order(c, a, kern->stream, kern->start_ns, K);
+        if (!korder) return OPATTR_E_OOM;
+    }
+
+    // ---- level lists, their validation, the windows and the enclosure, without
+    // a synchronisation in between: a failed validation is reported at the end
+    // (the enclosure reads only positions found by searches inside the level
+    // lists, so non-laminar ranges give wrong answers but no stray access).
+    // If ranges with equal starts were not in (start, end, index) order within
+    // a level, the whole pass runs again on fully sorted ranges.
     const unsigned g = grid_for(R, 256, 65535);
-    scan_exclusive_u32(c, level_hist, lvl_off, LEVELS + 1, part, nullptr);
     for (int attempt = 0; attempt < 2; ++attempt) {
+        const bool full_sort = !r_sorted || attempt > 0;
         uint32_t *perm = nullptr;         // range indices in the order of the level sort
-        if (!r_sorted) {
+        if (full_sort) {
             // (start, end, index) order: sort by end, then stably by start
             uint64_t *ko;
             uint32_t *vo;
@@ -510,83 +554,45 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
         launch(c, "validate_levels", k_validate_levels, dim3(grid_for(R, 256, 65535)), dim3(256), 0, rng->stream,
                rng->depth, (const int64_t *)ls, (const int64_t *)le, (const uint32_t *)li, (const uint32_t *)lvl_off,
                R, c.d_status);
+        if (K > 0 && nl == 0)
+            launch(c, "fill_unattributed", k_fill_unattributed, dim3(grid_for(K, 256, 65535)), dim3(256), 0, out_range,
+                   out_nop, K);
+        if (K > 0 && nl > 0) {
+            launch(c, "window_table", k_window_table, dim3(grid_for((nt + 1) * nl, 256, 65535)), dim3(256), 0,
+                   (const int64_t *)ls, (const uint32_t *)lvl_off, (const uint16_t *)d_loc, nl, kern->start_ns,
+                   (const uint32_t *)korder, K, nt, P);
+            EncArgs A;
+            A.k_stream = kern->stream;
+            A.k_start = kern->start_ns;
+            A.korder = korder;
+            A.K = K;
+            A.ls = ls;
+            A.le = le;
+            A.li = li;
+            A.lvl_off = lvl_off;
+            A.P = P;
+            A.nl = nl;
+            A.nt = nt;
+            A.cbase = d_cbase;
+            A.level_of_compact = d_loc;
+            A.ndepth = d_ndep;
+            A.out_range = out_range;
+            A.out_nop = out_nop;
+            static unsigned attr_done = 0;
+            if (c.device < 32 && !(attr_done & (1u << c.device))) {
+                cudaFuncSetAttribute(k_enclose, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(EncSmem));
+                attr_done |= 1u << c.device;
+            }
+            launch(c, "enclose", k_enclose, dim3((unsigned)nt), dim3(ENC_THREADS), sizeof(EncSmem), A);
+        }
         if ((st = read_status(c))) return st;
         if ((st = status_from_err(c.h_status->err))) return st;
-        if (!(c.h_status->flags & F_LEVEL_FIXUP)) break;
-        if (!r_sorted) return OPATTR_E_CUDA;     // a full sort leaves no equal-start disorder
-        r_sorted = false;
+        if (!(c.h_status->flags & F_LEVEL_FIXUP)) return OPATTR_OK;
+        if (full_sort) return OPATTR_E_CUDA;      // a full sort leaves no equal-start disorder
         c.h_status->flags &= ~F_LEVEL_FIXUP;
         cudaMemsetAsync(&c.d_status->flags, 0, sizeof(unsigned), c.stream);
     }
-    if (K == 0) return OPATTR_OK;
-
-    // ---- compact level table (host side, from the level offsets)
-    std::vector<uint32_t> off(LEVELS + 1);
-    if (cudaMemcpyAsync(off.data(), lvl_off, sizeof(uint32_t) * (LEVELS + 1), cudaMemcpyDeviceToHost, c.stream) !=
-            cudaSuccess ||
-        cudaStreamSynchronize(c.stream) != cudaSuccess)
-        return cuda_status(c, cudaGetLastError());
-    std::vector<uint16_t> level_of_compact;
-    std::vector<uint16_t> cbase(256, 0);
-    std::vector<uint8_t> ndep(256, 0);
-    for (int s = 0; s < 256; ++s) {
-        cbase[s] = (uint16_t)level_of_compact.size();
-        int n = 0;
-        while (n < 32 && off[s * 32 + n + 1] > off[s * 32 + n]) {
-            level_of_compact.push_back((uint16_t)(s * 32 + n));
-            n++;
-        }
-        ndep[s] = (uint8_t)n;
-    }
-    const int nl = (int)level_of_compact.size();
-    uint16_t *d_loc = a.take<uint16_t>(LEVELS);
-    uint16_t *d_cbase = a.take<uint16_t>(256);
-    uint8_t *d_ndep = a.take<uint8_t>(256);
-    int32_t *P = a.take<int32_t>((nt + 1) * (int64_t)(nl > 0 ? nl : 1));
-    if (!d_loc || !d_cbase || !d_ndep || !P) return OPATTR_E_OOM;
-    cudaMemcpyAsync(d_loc, level_of_compact.data(), sizeof(uint16_t) * (nl > 0 ? nl : 1), cudaMemcpyHostToDevice,
-                    c.stream);
-    cudaMemcpyAsync(d_cbase, cbase.data(), sizeof(uint16_t) * 256, cudaMemcpyHostToDevice, c.stream);
-    cudaMemcpyAsync(d_ndep, ndep.data(), 256, cudaMemcpyHostToDevice, c.stream);
-
-    // ---- kernel time order
-    uint32_t *korder = nullptr;
-    if (!k_sorted) {
-        korder = kernel_time_order(c, a, kern->stream, kern->start_ns, K);
-        if (!korder) return OPATTR_E_OOM;
-    }
-    if (nl == 0) {
-        launch(c, "fill_unattributed", k_fill_unattributed, dim3(grid_for(K, 256, 65535)), dim3(256), 0, out_range,
-               out_nop, K);
-        return read_status(c);
-    }
-    launch(c, "window_table", k_window_table, dim3(grid_for((nt + 1) * nl, 256, 65535)), dim3(256), 0,
-           (const int64_t *)ls, (const uint32_t *)lvl_off, (const uint16_t *)d_loc, nl, kern->start_ns,
-           (const uint32_t *)korder, K, nt, P);
-    EncArgs A;
-    A.k_stream = kern->stream;
-    A.k_start = kern->start_ns;
-    A.korder = korder;
-    A.K = K;
-    A.ls = ls;
-    A.le = le;
-    A.li = li;
-    A.lvl_off = lvl_off;
-    A.P = P;
-    A.nl = nl;
-    A.nt = nt;
-    A.cbase = d_cbase;
-    A.level_of_compact = d_loc;
-    A.ndepth = d_ndep;
-    A.out_range = out_range;
-    A.out_nop = out_nop;
-    static unsigned attr_done = 0;
-    if (c.device < 32 && !(attr_done & (1u << c.device))) {
-        cudaFuncSetAttribute(k_enclose, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(EncSmem));
-        attr_done |= 1u << c.device;
-    }
-    launch(c, "enclose", k_enclose, dim3((unsigned)nt), dim3(ENC_THREADS), sizeof(EncSmem), A);
-    return read_status(c);
+    return OPATTR_E_CUDA;
 }
 
 }  // namespace opattr
