@@ -55,15 +55,14 @@ WORKLOADS = {
 }
 
 
-def source_digest():
-    """Digest of the CUDA sources (csrc/*.cu, *.cuh), to tie recorded ncu figures to the code they came from."""
-    import glob
+def source_digest(files):
+    """Digest of the named CUDA sources (csrc/ file names), to tie recorded ncu figures to the code they came from."""
     import hashlib
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_11938_gb300", "csrc")
-    for p in sorted(glob.glob(os.path.join(csrc, "*.cu")) + glob.glob(os.path.join(csrc, "*.cuh"))):
-        h.update(os.path.basename(p).encode())
-        with open(p, "rb") as f:
+    for name in sorted(files):
+        h.update(name.encode())
+        with open(os.path.join(csrc, name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
 
@@ -75,10 +74,13 @@ def recorded_traffic(kernel, workload, kernels):
             lines = [ln.split() for ln in f if ln.strip() and not ln.startswith("#")]
     except OSError:
         return None
-    digest = source_digest()
     for ln in lines:
-        if len(ln) == 5 and ln[0] == kernel and ln[1] == workload and int(ln[2]) == kernels and ln[3] == digest:
-            return int(ln[4])
+        if len(ln) == 6 and ln[0] == kernel and ln[1] == workload and int(ln[2]) == kernels:
+            try:
+                if ln[4] == source_digest(ln[3].split(",")):
+                    return int(ln[5])
+            except OSError:
+                return None
     return None
 
 

@@ -476,9 +476,10 @@ __global__ void __launch_bounds__(SL_THREADS) k_agg_sort_long(const uint32_t *__
 // and outputs the GPU works on at any moment form one window that stays in
 // L2.  Segments are walked in ascending kernel index: a short one is checked
 // and, in the rare case the fill left it out of order, insertion-sorted in
-// place by its thread; long ones were sorted by k_agg_sort_long.  The next
-// kernel's duration and row index are loaded before the current kernel is
-// added.
+// place by its thread; long ones were sorted by k_agg_sort_long.  While a
+// kernel is added, the counter rows and durations of the next two arrive in
+// per-thread shared-memory slots by asynchronous copy (cp.async), with their
+// row indices loaded a step earlier still.
 constexpr int AG_THREADS = 128;
 constexpr int AG_WARPS = AG_THREADS / 32;
 constexpr int AG_CHUNK = 128;                   // op ids per warp and chunk
@@ -494,10 +495,26 @@ __device__ __noinline__ int op_careful(const uint32_t *seg, uint32_t len, AggIn 
     return acc.bad;
 }
 
+__device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ void cp_async16(void *dst, const void *src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async8(void *dst, const void *src) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
 __global__ void __launch_bounds__(AG_THREADS) k_agg_ops(const uint32_t *__restrict__ off, uint32_t *__restrict__ list,
                                                           AggIn A, DevStatus *st) {
     __shared__ uint32_t lcount_s[AG_WARPS][AG_LBUCKETS];
     __shared__ uint8_t order_s[AG_WARPS][AG_CHUNK];
+    // two in-flight kernels per thread: counter row and duration, by async copy
+    __shared__ __align__(16) float4 rowbuf[2][AG_THREADS][NC / 4];
+    __shared__ long long durbuf[2][AG_THREADS];
     uint32_t *lcount = lcount_s[threadIdx.x / 32];
     uint8_t *order = order_s[threadIdx.x / 32];
     const unsigned lane = lane_id();
@@ -557,22 +574,39 @@ __global__ void __launch_bounds__(AG_THREADS) k_agg_ops(const uint32_t *__restri
             AccF acc;
             acc.init();
             if (len > 0) {
-                uint32_t kn = seg[0];
-                long long d = A.dur[kn];
-                int32_t j = A.ncu_idx[kn];
-                for (uint32_t t = 0; t < len; ++t) {
-                    long long d2 = 0;
-                    int32_t j2 = -1;
-                    if (t + 1 < len) {
-                        kn = seg[t + 1];
-                        d2 = A.dur[kn];
-                        j2 = A.ncu_idx[kn];
+                // kernel t's row and duration land in slot t & 1 while kernel
+                // t - 1 is added; row indices are loaded one step further ahead
+                const unsigned me = threadIdx.x;
+                auto issue = [&](uint32_t t, uint32_t k, int32_t j) {
+                    if (t < len) {
+                        cp_async8(&durbuf[t & 1][me], A.dur + k);
+                        if (j >= 0) {
+                            const float4 *src = reinterpret_cast<const float4 *>(A.counters + (int64_t)j * NC);
+#pragma unroll
+                            for (int q = 0; q < NC / 4; ++q) cp_async16(&rowbuf[t & 1][me][q], src + q);
+                        }
                     }
-                    acc.accumulate(d, j >= 0,
-                                   reinterpret_cast<const float4 *>(A.counters + (int64_t)(j >= 0 ? j : 0) * NC));
-                    d = d2;
-                    j = j2;
+                    cp_async_commit();
+                };
+                const uint32_t k0 = seg[0], k1 = len > 1 ? seg[1] : 0u;
+                const int32_t j0 = A.ncu_idx[k0], j1 = len > 1 ? A.ncu_idx[k1] : -1;
+                uint32_t k2 = len > 2 ? seg[2] : 0u;
+                int32_t j2 = len > 2 ? A.ncu_idx[k2] : -1;
+                issue(0, k0, j0);
+                issue(1, k1, j1);
+                int32_t js0 = j0, js1 = j1;           // row index of the kernel in each slot
+                for (uint32_t t = 0; t < len; ++t) {
+                    const uint32_t k3 = t + 3 < len ? seg[t + 3] : 0u;
+                    const int32_t j3 = t + 3 < len ? A.ncu_idx[k3] : -1;
+                    cp_async_wait<1>();
+                    const int32_t j = (t & 1) ? js1 : js0;
+                    acc.accumulate(durbuf[t & 1][me], j >= 0, rowbuf[t & 1][me]);
+                    issue(t + 2, k2, j2);
+                    if (t & 1) js1 = j2; else js0 = j2;
+                    k2 = k3;
+                    j2 = j3;
                 }
+                cp_async_wait<0>();
             }
             if (acc.clean()) acc.write(A, o, (int)len);
             else bad |= op_careful(seg, len, A, o);
