@@ -345,19 +345,20 @@ __global__ void k_agg_count(const int64_t *__restrict__ dur, const int32_t *__re
 // ------------------------------------------------------------------ fill
 // list[off[op] + slot] = k for each attributed kernel with a valid range and
 // op id (the kernels k_agg_count counted); slots are taken by atomics on
-// cur[op] (zeroed).  Each warp fills a run of AF_RUN consecutive kernels 32 at
-// a time in index order, so an op whose kernels all lie in one run gets them
-// in ascending order; the ops pass sorts the few segments that do not.
+// cur[op] (zeroed).  Each warp fills a run of `run` consecutive kernels (a
+// multiple of 32, up to AF_RUN) 32 at a time in index order, so an op whose
+// kernels all lie in one run gets them in ascending order; the ops pass sorts
+// the few segments that do not.
 constexpr int AF_RUN = 2048;
 
 __global__ void k_agg_fill(const int32_t *__restrict__ rok, const uint32_t *__restrict__ r_op, int64_t K, int64_t R,
                            int64_t n_ops, const uint32_t *__restrict__ off, uint32_t *__restrict__ cur,
-                           uint32_t *__restrict__ list) {
+                           uint32_t *__restrict__ list, int64_t run) {
     const unsigned lane = lane_id();
     const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / 32;
     const int64_t nwarps = (int64_t)gridDim.x * blockDim.x / 32;
-    for (int64_t k0 = warp * AF_RUN; k0 < K; k0 += nwarps * AF_RUN) {
-        const int64_t k1 = k0 + AF_RUN < K ? k0 + AF_RUN : K;
+    for (int64_t k0 = warp * run; k0 < K; k0 += nwarps * run) {
+        const int64_t k1 = k0 + run < K ? k0 + run : K;
         int32_t r_next = k0 + lane < k1 ? rok[k0 + lane] : -1;
         for (int64_t kb = k0; kb < k1; kb += 32) {
             const int64_t k = kb + lane;
@@ -668,9 +669,16 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     in.out = *out;
     if (O > 0) {
         scan_exclusive_u32(c, cnt, off, O + 1, part, nullptr);
-        if (K > 0)
-            launch(c, "agg_fill", k_agg_fill, dim3(grid_for(K, 256 / 32 * AF_RUN, 65535)), dim3(256), 0, rok,
-                   rng->op_id, K, R, O, (const uint32_t *)off, cur, list);
+        if (K > 0) {
+            // runs long enough to keep most segments in one warp, short enough
+            // that small traces still spread over the GPU (64 warps per SM)
+            int sms = 0;
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
+            const int64_t warps = (int64_t)std::max(1, sms) * 64;
+            const int64_t run = std::min<int64_t>(AF_RUN, std::max<int64_t>(32, ((K + warps - 1) / warps + 31) / 32 * 32));
+            launch(c, "agg_fill", k_agg_fill, dim3(grid_for(K, 256 / 32 * run, 65535)), dim3(256), 0, rok,
+                   rng->op_id, K, R, O, (const uint32_t *)off, cur, list, run);
+        }
         launch(c, "agg_long_list", k_agg_long_list, dim3(grid_for(O, 256, 4096)), dim3(256), 0, (const uint32_t *)off,
                O, AG_SHORT_MAX, longs, nlong);
         int sms = 0;
