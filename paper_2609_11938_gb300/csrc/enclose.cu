@@ -317,6 +317,13 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
         int pr[RD];                               // window position + 1 (0 none, -1 not searched yet)
 #pragma unroll
         for (int d = 0; d < RD; ++d) pr[d] = -1;
+        // The last walk's answer holds for a later kernel of the stream while
+        // no range of a depth the walk looked at starts in between and every
+        // range it found still contains the kernel: the walk would visit the
+        // same ranges with the same results.
+        int32_t ans = -1;
+        int nop = 0;
+        uint32_t reuse_below = 0, reuse_upto = 0;    // valid for next_start > T and T <= min_end
         for (int u = 0; u < ENC_CHUNK; ++u) {
             const int idx = threadIdx.x * ENC_CHUNK + u;
             if (idx >= cnt) break;
@@ -330,49 +337,60 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
                 a0 = S.sbase[s];
 #pragma unroll
                 for (int d = 0; d < RD; ++d) pr[d] = -1;
+                reuse_below = 0;
             }
-            int32_t ans = -1;
-            int nop = 0;
-            bool alive = true;
+            if (!(T < reuse_below && T <= reuse_upto)) {
+                ans = -1;
+                nop = 0;
+                bool alive = true;
+                uint32_t next_start = 0xFFFFFFFFu, min_end = 0xFFFFFFFFu;
 #pragma unroll
-            for (int d = 0; d < RD; ++d) {
-                if (alive && d < nd) {
-                    const int c = S.act_cnt[a0 + d], o = S.act_off[a0 + d];
-                    int p;                          // last window position with start <= T, or -1
-                    if (pr[d] < 0) {
-                        int x = o, y = o + c;
-                        while (x < y) {
-                            const int m = (x + y) >> 1;
-                            if (S.ws[m] <= T) x = m + 1; else y = m;
+                for (int d = 0; d < RD; ++d) {
+                    if (alive && d < nd) {
+                        const int c = S.act_cnt[a0 + d], o = S.act_off[a0 + d];
+                        int p;                          // last window position with start <= T, or -1
+                        if (pr[d] < 0) {
+                            int x = o, y = o + c;
+                            while (x < y) {
+                                const int m = (x + y) >> 1;
+                                if (S.ws[m] <= T) x = m + 1; else y = m;
+                            }
+                            p = x - o - 1;
+                        } else {
+                            p = pr[d] - 1;
+                            while (p + 1 < c && S.ws[o + p + 1] <= T) ++p;
                         }
-                        p = x - o - 1;
-                    } else {
-                        p = pr[d] - 1;
-                        while (p + 1 < c && S.ws[o + p + 1] <= T) ++p;
-                    }
-                    pr[d] = p + 1;
-                    if (p < 0 || S.we[o + p] < T) {
-                        alive = false;
-                    } else {
-                        const uint32_t info = S.wi[o + p];
-                        const uint32_t kind = info >> 30;
-                        if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
-                        else if (kind == KIND_OP) { ans = (int32_t)(info & 0x3FFFFFFFu); nop++; }
+                        pr[d] = p + 1;
+                        if (p + 1 < c) next_start = min(next_start, S.ws[o + p + 1]);
+                        if (p < 0 || S.we[o + p] < T) {
+                            alive = false;
+                        } else {
+                            const uint32_t e = S.we[o + p];
+                            min_end = min(min_end, e);
+                            const uint32_t info = S.wi[o + p];
+                            const uint32_t kind = info >> 30;
+                            if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
+                            else if (kind == KIND_OP) { ans = (int32_t)(info & 0x3FFFFFFFu); nop++; }
+                        }
                     }
                 }
-            }
-            for (int d = RD; alive && d < nd; ++d) {   // deeper levels: one search each
-                const int c = S.act_cnt[a0 + d], o = S.act_off[a0 + d];
-                int x = o, y = o + c;
-                while (x < y) {
-                    const int m = (x + y) >> 1;
-                    if (S.ws[m] <= T) x = m + 1; else y = m;
+                bool deep = false;
+                for (int d = RD; alive && d < nd; ++d) {   // deeper levels: one search each
+                    deep = true;
+                    const int c = S.act_cnt[a0 + d], o = S.act_off[a0 + d];
+                    int x = o, y = o + c;
+                    while (x < y) {
+                        const int m = (x + y) >> 1;
+                        if (S.ws[m] <= T) x = m + 1; else y = m;
+                    }
+                    if (x == o || S.we[x - 1] < T) break;
+                    const uint32_t info = S.wi[x - 1];
+                    const uint32_t kind = info >> 30;
+                    if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
+                    else if (kind == KIND_OP) { ans = (int32_t)(info & 0x3FFFFFFFu); nop++; }
                 }
-                if (x == o || S.we[x - 1] < T) break;
-                const uint32_t info = S.wi[x - 1];
-                const uint32_t kind = info >> 30;
-                if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
-                else if (kind == KIND_OP) { ans = (int32_t)(info & 0x3FFFFFFFu); nop++; }
+                reuse_below = deep ? 0u : next_start;
+                reuse_upto = min_end;
             }
             A.out_range[k] = ans;
             if (A.out_nop) A.out_nop[k] = (uint8_t)nop;
