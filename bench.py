@@ -8,6 +8,7 @@ bounded sample of the same workload instead.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import os
 import statistics
@@ -219,6 +220,10 @@ def main():
     ap.add_argument("--shuffle", action="store_true", help="permute kernel and range arrays (general paths)")
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--oracle-kernels", type=int, default=1_000_000)
+    ap.add_argument("--per-stream-ncu", action="store_true",
+                    help="ncu rows as per-stream replay runs, matched per (name, stream)")
+    ap.add_argument("--launch-lag", type=int, default=0,
+                    help="enclosure queries at start - U[0, LAG) ns (host launch times)")
     ap.add_argument("--kernels", type=int, default=0,
                     help="draw this many kernels with the config's generator parameters (profiling runs)")
     args = ap.parse_args()
@@ -281,9 +286,15 @@ def main():
     if args.kernels and cfg.get("shape", 0) == 0:
         cfg["n_kernels"] = args.kernels
     trace = tracegen.generate(cfg, shuffle=args.shuffle)
+    if args.per_stream_ncu:
+        trace = tracegen.per_stream_runs(trace)
     K, R, M, O = trace.K, trace.R, trace.M, trace.n_ops
     use_dedup = bool(cfg.get("dedup")) and trace.k_layer is not None
     tr = opa.to_device(trace, dev)
+    tq = tr                                           # what the enclosure queries at
+    if args.launch_lag > 0:
+        lag = np.random.default_rng(cfg["seed"]).integers(0, args.launch_lag, K)
+        tq = dataclasses.replace(tr, k_start=torch.from_numpy(trace.k_start - lag).to(f"cuda:{dev}"))
     torch.cuda.synchronize(dev)
     stream = torch.cuda.Stream(dev)
     ctx = opa.Context(dev, stream=stream)
@@ -303,7 +314,7 @@ def main():
         if flush is not None:
             with torch.cuda.stream(stream):
                 flush.fill_(1.0)
-        ctx.enclose(tr, rk, nop)
+        ctx.enclose(tq, rk, nop)
         ctx.match(tr, dedup=use_dedup, out_idx=idx, out_kind=kind)
         ctx.aggregate(tr, rk, idx, ops)
 
@@ -345,17 +356,23 @@ def main():
                          "r_op", "ncu_name", "counters")}
     if trace.k_layer is not None:
         host["k_layer"] = torch.from_numpy(trace.k_layer).pin_memory()
+    if tq is not tr:
+        launch_host = tq.k_start.cpu().pin_memory()
     out_host = {"rk": torch.empty(K, dtype=torch.int32).pin_memory(),
                 "idx": torch.empty(K, dtype=torch.int32).pin_memory()}
     out_host.update({k: torch.empty_like(v, device="cpu").pin_memory() for k, v in ops.items()})
     h2d = sum(v.numel() * v.element_size() for v in host.values())
+    if tq is not tr:
+        h2d += launch_host.numel() * launch_host.element_size()
     d2h = sum(v.numel() * v.element_size() for v in out_host.values())
 
     def e2e_step():
         with torch.cuda.stream(stream):
             for name, v in host.items():
                 getattr(tr, name).copy_(v, non_blocking=True)
-        ctx.enclose(tr, rk, nop)
+            if tq is not tr:
+                tq.k_start.copy_(launch_host, non_blocking=True)
+        ctx.enclose(tq, rk, nop)
         ctx.match(tr, dedup=use_dedup, out_idx=idx, out_kind=kind)
         ctx.aggregate(tr, rk, idx, ops)
         with torch.cuda.stream(stream):
@@ -403,7 +420,8 @@ def main():
         "data": "synthetic",
         "config": {"workload": f"{args.config}: {WORKLOADS[args.config]}" + (
                        f" [scaled to {K} kernels]" if args.kernels else ""), "kernels": K, "ranges": R,
-                   "ncu_rows": M, "ops": O, "shuffled": bool(args.shuffle), "parallelism": f"replicas x{world}",
+                   "ncu_rows": M, "ops": O, "shuffled": bool(args.shuffle), "per_stream_ncu": bool(args.per_stream_ncu),
+                   "launch_lag_ns": args.launch_lag, "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2 (129 MB)" if flush is None else "L2 flushed before every step"},
         "roofline": {"bound": "hbm", "kernel": dname, "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": (achieved / peak) if achieved else None, "peak_kind": f"{peak_kind} copy bandwidth",

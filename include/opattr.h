@@ -110,11 +110,19 @@ typedef struct {
  *   name_id   u32[n]       kernel-name id of the row
  *   counters  f32[n * 20]  row-major, counter #k (Table 8) at column k-1;
  *                          NaN = null (absent counter); values must be finite
- *                          or NaN; 16-byte aligned (read by opattr_aggregate) */
+ *                          or NaN; 16-byte aligned (read by opattr_aggregate)
+ *   stream    u8[n]        stream of the row, or NULL.  Nsight Compute replays
+ *                          one stream per run when a workload is multi-stream
+ *                          (limitations paragraph of Sec. 6); with the rows of
+ *                          those runs tagged here, opattr_match takes ordinals
+ *                          per (name, stream) instead of per name, and name ids
+ *                          must then be below 2^24.  Rows of one stream keep
+ *                          their launch order; runs may come in any order. */
 typedef struct {
     const uint32_t *name_id;
     const float *counters;
     int64_t n;
+    const uint8_t *stream;
 } opattr_ncu;
 
 /* Layer deduplication tables (Sec. 3.7), HOST memory.
@@ -204,16 +212,20 @@ opattr_status opattr_enclose(opattr_ctx *ctx, const opattr_kernels *kernels, con
 /* Algorithm 1 with the context's mismatch mode.  ncu_idx_of_kernel[k] = ncu
  * row of kernel k or -1; match_kind[k] = 0 none, 1 direct, 2 broadcast.
  * Ordinals are taken over replayed kernels in time order and over rows in
- * array order.  `dedup` (host) may be NULL; deduplication also needs
- * kernels->layer_id and cfg.dedup = 1.
- * Reads kernels->stream, start_ns, name_id (and layer_id), ncu->name_id.
+ * array order, per name -- or per (name, stream) when ncu->stream is given:
+ * then a kernel's "name" everywhere below (counts, ordinals, mismatch modes,
+ * the duplicate-layer name check) is the pair.  `dedup` (host) may be NULL;
+ * deduplication also needs kernels->layer_id and cfg.dedup = 1.
+ * Reads kernels->stream, start_ns, name_id (and layer_id), ncu->name_id (and
+ * ncu->stream).
  *   ncu_idx_of_kernel  i32[kernels->n]  device, required
  *   match_kind         u8[kernels->n]   device, may be NULL
  *   host_summary       host, may be NULL
  * Returns OPATTR_W_COUNT_MISMATCH (skip-name: some name mismatched; prefix:
  * some kernel found no row), else OPATTR_W_DEDUP_MISMATCH when a duplicate
  * found no source.  Errors: OPATTR_E_INVALID_ARG (layer id >= n_layers, bad
- * tables), OPATTR_E_COUNT_MISMATCH (error mode), OPATTR_E_OOM, OPATTR_E_CUDA. */
+ * tables, a name id >= 2^24 with ncu->stream), OPATTR_E_COUNT_MISMATCH (error
+ * mode), OPATTR_E_OOM, OPATTR_E_CUDA. */
 opattr_status opattr_match(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ncu *ncu,
                            const opattr_dedup *dedup, int32_t *ncu_idx_of_kernel, uint8_t *match_kind,
                            opattr_match_summary *host_summary);
@@ -269,7 +281,8 @@ int64_t opattr_launch_count(const opattr_ctx *ctx);
  *   All scratch (about 6 MB) lives in one fixed device array inside the
  *   library; every GPU that loads the library holds it until exit.
  *   kernels->n and ncu->n must each be at most OPATTR_MATCH_NOALLOC_MAX,
- *   else OPATTR_E_INVALID_ARG.
+ *   else OPATTR_E_INVALID_ARG; per-stream ordinals are not available here
+ *   (ncu->stream must be NULL, else OPATTR_E_INVALID_ARG).
  *   The first call on a device looks up the array's device address; make
  *   that first call before any stream capture.
  *   Calls share the array.  Host threads are serialised inside the call, and

@@ -128,12 +128,23 @@ def enclose(k_stream, k_start, r_stream, r_start, r_end, r_depth, r_op, mode: st
 
 
 def match(k_stream, k_start, k_name, ncu_name, k_layer=None, class_of_layer=None, rep_of_class=None,
-          mode: str = "skip_name", dedup: bool = False, brute: bool = False):
-    """Returns (status, ncu_idx i32[K], match_kind u8[K], summary dict)."""
+          mode: str = "skip_name", dedup: bool = False, brute: bool = False, ncu_stream=None):
+    """Returns (status, ncu_idx i32[K], match_kind u8[K], summary dict).
+
+    With ncu_stream (the stream of each ncu row, from per-stream replay runs),
+    Algorithm 1's key is the pair (name, stream) rather than the name: kernels
+    and rows are keyed name * 256 + stream (names below 2^24), and everything
+    the algorithm does with names it does with those keys."""
     lib = _lib()
     ks, kt, kn = _c(k_stream, np.uint8), _c(k_start, np.int64), _c(k_name, np.uint32)
     kl = _c(k_layer, np.int32)
     nn = _c(ncu_name, np.uint32)
+    if ncu_stream is not None and len(nn) > 0:
+        if (kn >= (1 << 24)).any() or (nn >= (1 << 24)).any():
+            return E_INVALID_ARG, np.full(len(kt), -1, np.int32), np.zeros(len(kt), np.uint8), \
+                dict(zip(SUMMARY_FIELDS, [0] * len(SUMMARY_FIELDS)))
+        kn = (kn.astype(np.uint32) << np.uint32(8)) | ks.astype(np.uint32)
+        nn = (nn.astype(np.uint32) << np.uint32(8)) | _c(ncu_stream, np.uint8).astype(np.uint32)
     col = _c(class_of_layer, np.int32) if class_of_layer is not None else np.zeros(1, np.int32)
     roc = _c(rep_of_class, np.int32) if rep_of_class is not None else np.zeros(1, np.int32)
     n_layers = 0 if class_of_layer is None else len(col)
@@ -180,7 +191,8 @@ def run(trace, mode: str = "skip_name", enclose_mode: str = "indexed", dedup: bo
         dedup = bool(trace.config.get("dedup")) and trace.k_layer is not None
     use_dedup = dedup
     st_m, idx, kind, summ = match(trace.k_stream, trace.k_start, trace.k_name, trace.ncu_name, trace.k_layer,
-                                  trace.class_of_layer, trace.rep_of_class, mode=mode, dedup=use_dedup)
+                                  trace.class_of_layer, trace.rep_of_class, mode=mode, dedup=use_dedup,
+                                  ncu_stream=getattr(trace, "ncu_stream", None))
     st_a, ops, totals = aggregate(trace.k_dur, rk, trace.r_op, trace.counters, idx, trace.n_ops)
     return dict(enclose_status=st_e, range_of_kernel=rk, n_op_enclosing=nop, match_status=st_m,
                 ncu_idx=idx, match_kind=kind, summary=summ, aggregate_status=st_a, ops=ops, totals=totals)

@@ -50,7 +50,7 @@ class Ranges(ctypes.Structure):
 
 
 class Ncu(ctypes.Structure):
-    _fields_ = [("name_id", _vp), ("counters", _vp), ("n", ctypes.c_int64)]
+    _fields_ = [("name_id", _vp), ("counters", _vp), ("n", ctypes.c_int64), ("stream", _vp)]
 
 
 class Dedup(ctypes.Structure):
@@ -215,6 +215,7 @@ class DeviceTrace:
     counters: object
     class_of_layer: object = None   # host (numpy / list) tables
     rep_of_class: object = None
+    ncu_stream: object = None       # stream of each ncu row (per-stream replay runs), or None
 
     @property
     def K(self):
@@ -244,7 +245,7 @@ def to_device(trace, device: int = 0, pin: bool = False) -> DeviceTrace:
     return DeviceTrace(d(trace.k_stream), d(trace.k_start), d(trace.k_dur), d(trace.k_name), d(trace.k_layer),
                        d(trace.r_stream), d(trace.r_start), d(trace.r_end), d(trace.r_depth), d(trace.r_op),
                        int(trace.n_ops), d(trace.ncu_name), d(trace.counters), trace.class_of_layer,
-                       trace.rep_of_class)
+                       trace.rep_of_class, d(getattr(trace, "ncu_stream", None)))
 
 
 class Context:
@@ -297,7 +298,7 @@ class Context:
         import torch
         dv = self.device
         return Ncu(_ptr(tr.ncu_name, torch.uint32, "ncu_name", dv), _ptr(tr.counters, torch.float32, "counters", dv),
-                   tr.M)
+                   tr.M, _ptr(tr.ncu_stream, torch.uint8, "ncu_stream", dv))
 
     # -- calls
     def enclose(self, tr: DeviceTrace, out_range=None, out_nop=None, need_nop: bool = True):

@@ -223,6 +223,19 @@ __global__ void k_dedup_broadcast(const uint32_t *__restrict__ sll, const uint32
 }
 
 // ------------------------------------------------------------------ host
+// (name, stream) as one key, name << 8 | stream, for per-stream ordinals; a
+// name id of 2^24 or more cannot be packed and is an invalid argument.
+__global__ void k_stream_keys(const uint32_t *__restrict__ name, const uint8_t *__restrict__ stream, int64_t n,
+                              uint32_t *__restrict__ key, DevStatus *st) {
+    int bad = 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const uint32_t x = name[i];
+        bad |= x >> 24 != 0;
+        key[i] = (x << 8) | stream[i];
+    }
+    if (bad) set_err(st, ERR_INVALID);
+}
+
 __global__ void k_iota(uint32_t *dst, int64_t n) {
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         dst[i] = (uint32_t)i;
@@ -259,7 +272,10 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     }
     const int64_t NL = dedup_on ? (dd->n_layers > 0 ? dd->n_layers : 1) : 1;
     const int64_t NX = std::max(K, M);
+    const bool per_stream = ncu->stream != nullptr;
+    if (per_stream && M > 0 && !ncu->name_id) return OPATTR_E_INVALID_ARG;
     Need nd;
+    if (per_stream) nd.add<uint32_t>(K).add<uint32_t>(M);        // (name, stream) keys
     nd.add<int32_t>(NL);
     for (int i = 0; i < 5; ++i) nd.add<uint32_t>(K);                 // flag, pos, rk, lk, keys
     for (int i = 0; i < 3; ++i) nd.add<uint32_t>(NX);                // sort buffers
@@ -284,6 +300,20 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
         return OPATTR_E_OOM;
     if (dedup_on && dd->n_layers > 0)
         cudaMemcpyAsync(d_rep, rep_layer.data(), sizeof(int32_t) * dd->n_layers, cudaMemcpyHostToDevice, c.stream);
+    // the matching key: the name id, or (name, stream) when the rows carry streams
+    const uint32_t *kname = kern->name_id, *nname = ncu->name_id;
+    if (per_stream) {
+        uint32_t *kkey = a.take<uint32_t>(K), *nkey = a.take<uint32_t>(M);
+        if ((K > 0 && !kkey) || (M > 0 && !nkey)) return OPATTR_E_OOM;
+        if (K > 0)
+            launch(c, "stream_keys", k_stream_keys, dim3(grid_for(K, 256, REDUCE_GRID)), dim3(256), 0, kern->name_id,
+                   kern->stream, K, kkey, c.d_status);
+        if (M > 0)
+            launch(c, "stream_keys", k_stream_keys, dim3(grid_for(M, 256, REDUCE_GRID)), dim3(256), 0, ncu->name_id,
+                   ncu->stream, M, nkey, c.d_status);
+        kname = kkey;
+        nname = nkey;
+    }
 
     const unsigned gK = grid_for(K, 256, REDUCE_GRID);
     check_kernel_order(c, kern->stream, kern->start_ns, K);
@@ -293,7 +323,7 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     const bool try_identity = !dedup_on && K == M && K > 0;
     if (try_identity)
         launch(c, "match_identity", k_match_identity, dim3(grid_for(K, 256 * 16, REDUCE_GRID)), dim3(256), 0,
-               kern->name_id, ncu->name_id, K, out_idx,
+               kname, nname, K, out_idx,
                out_kind, c.d_status);
     if ((st = read_status(c))) return st;
     if (c.h_status->err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
@@ -331,7 +361,7 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     bool direct_done = false;
     if (dedup_on && nrep == M && nrep > 0) {
         launch(c, "match_identity_list", k_match_identity_list, dim3(grid_for(nrep, 256, REDUCE_GRID)), dim3(256), 0,
-               (const uint32_t *)rk, kern->name_id, ncu->name_id, nrep, out_idx, out_kind, c.d_status);
+               (const uint32_t *)rk, kname, nname, nrep, out_idx, out_kind, c.d_status);
         if ((st = read_status(c))) return st;
         direct_done = !(c.h_status->flags & F_NAMES_DIFFER);
         if (direct_done) S.fast_path = 1;
@@ -340,13 +370,13 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     if (!direct_done && (nrep > 0 || M > 0)) {
         cudaMemsetAsync(dsm, 0, sizeof(unsigned long long), c.stream);
         if (nrep > 0) {
-            launch(c, "gather_names", k_gather_u32, dim3(grid_for(nrep, 256, REDUCE_GRID)), dim3(256), 0, kern->name_id,
+            launch(c, "gather_names", k_gather_u32, dim3(grid_for(nrep, 256, REDUCE_GRID)), dim3(256), 0, kname,
                    (const uint32_t *)rk, nrep, k0);
             launch(c, "max_name", k_max_u32, dim3(grid_for(nrep, 256, 4096)), dim3(256), 0, (const uint32_t *)k0, nrep,
                    dsm);
         }
         if (M > 0) {
-            cudaMemcpyAsync(n0, ncu->name_id, sizeof(uint32_t) * M, cudaMemcpyDeviceToDevice, c.stream);
+            cudaMemcpyAsync(n0, nname, sizeof(uint32_t) * M, cudaMemcpyDeviceToDevice, c.stream);
             launch(c, "max_name", k_max_u32, dim3(grid_for(M, 256, 4096)), dim3(256), 0, (const uint32_t *)n0, M, dsm);
         }
         unsigned long long hmax = 0;
@@ -383,7 +413,7 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
                                        &sll, &slj);
             launch(c, "dedup_broadcast", k_dedup_broadcast, dim3(grid_for(nlk, 256, REDUCE_GRID)), dim3(256), 0,
                    (const uint32_t *)sll, (const uint32_t *)slj, (const uint32_t *)lk, nlk, (const int32_t *)d_rep,
-                   kern->name_id, out_idx, out_kind, c.d_status);
+                   kname, out_idx, out_kind, c.d_status);
         }
     }
     if ((st = read_status(c))) return st;

@@ -37,6 +37,7 @@ extern "C" opattr_status opattr_match_noalloc(const opattr_kernels *kernels, con
                                               void *cuda_stream) {
     if (!kernels || !ncu) return OPATTR_E_INVALID_ARG;
     if ((int)mismatch < 0 || (int)mismatch > 2) return OPATTR_E_INVALID_ARG;
+    if (ncu->stream) return OPATTR_E_INVALID_ARG;
     if (kernels->n < 0 || ncu->n < 0 || kernels->n > OPATTR_MATCH_NOALLOC_MAX || ncu->n > OPATTR_MATCH_NOALLOC_MAX)
         return OPATTR_E_INVALID_ARG;
     int dev = 0;

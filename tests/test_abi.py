@@ -36,7 +36,7 @@ def test_struct_layouts_match_header():
     # pointer-sized fields then int64 n; sizes follow the C layout on LP64
     assert ctypes.sizeof(opa.Kernels) == 6 * 8
     assert ctypes.sizeof(opa.Ranges) == 6 * 8
-    assert ctypes.sizeof(opa.Ncu) == 3 * 8
+    assert ctypes.sizeof(opa.Ncu) == 4 * 8
     assert ctypes.sizeof(opa.Dedup) == 2 * 8 + 2 * 4
     assert ctypes.sizeof(opa.Config) == 4 + 4 + 4 + 4 + 8
     assert ctypes.sizeof(opa.MatchSummary) == 8 * 8 + 2 * 4

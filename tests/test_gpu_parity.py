@@ -338,3 +338,72 @@ def test_adversarial_sampled(opa):
         np.testing.assert_array_equal(g["ops"][k], ops[k])
     assert_close(g["ops"]["agg"], ops["agg"], what="agg")
     assert g["totals"]["attributed_ns"] == tot["attributed_ns"] and g["totals"]["total_ns"] == tot["total_ns"]
+
+
+@pytest.mark.parametrize("name,order", [("gpt2", None), ("gpt2", "reversed"), ("large2m", None)])
+def test_per_stream_runs(opa, name, order):
+    """ncu rows as per-stream replay runs, tagged with their stream: ordinals
+    per (name, stream), against the oracle; every kernel gets its own row."""
+    t = tracegen.generate("large", n_kernels=2_000_000) if name == "large2m" else tracegen.generate(name)
+    streams = np.unique(t.k_stream)
+    u = tracegen.per_stream_runs(t, None if order is None else streams[::-1])
+    g = gpu_run(u)
+    assert_parity(g, oracle.run(u, enclose_mode="indexed"))
+    assert (g["match_kind"] == 1).all()
+    np.testing.assert_array_equal(u.counters[g["ncu_idx"]], t.counters)
+
+
+@pytest.mark.parametrize("seed", range(0, 40, 3))
+def test_per_stream_small_random(opa, seed):
+    """Random traces with rows as per-stream runs, some rows dropped so the
+    mismatch modes see per-(name, stream) count differences."""
+    t = tracegen.small_random(seed, n_streams=1 + seed % 4, n_events=10 + (seed * 7) % 90, max_depth=1 + seed % 7,
+                              n_names=2 + seed % 5)
+    if t.M != t.K:
+        pytest.skip("needs one row per kernel")
+    u = tracegen.per_stream_runs(t)
+    if seed % 2 and u.M > 2:
+        keep = np.ones(u.M, bool)
+        keep[[0, u.M // 2]] = False
+        u.ncu_name, u.counters, u.ncu_stream = u.ncu_name[keep], u.counters[keep], u.ncu_stream[keep]
+    mode = ["skip_name", "prefix"][seed % 2]
+    assert_parity(gpu_run(u, mode=mode), oracle.run(u, mode=mode, enclose_mode="brute"))
+
+
+def test_per_stream_name_limit(opa):
+    """With stream-tagged rows a name id must fit in 24 bits."""
+    t = tracegen.per_stream_runs(tracegen.generate("tiny"))
+    t.k_name = t.k_name.copy()
+    t.k_name[5] = 1 << 24
+    ctx = opa.Context(0)
+    with pytest.raises(opa.OpattrError) as ei:
+        ctx.match(opa.to_device(t))
+    assert ei.value.status == opa.E_INVALID_ARG
+    ctx.close()
+
+
+def test_launch_time_query(opa):
+    """Algorithm 2 queries at the host launch timestamp, which precedes the
+    GPU start by a variable lag: the enclosure takes those times as its query
+    points (kernels then out of time order) while matching keeps GPU order."""
+    import torch
+    t = tracegen.generate("gpt2")
+    rng = np.random.default_rng(3)
+    launch = t.k_start - rng.integers(0, 4000, t.K)
+    st, want_rk, want_nop = oracle.enclose(t.k_stream, launch, t.r_stream, t.r_start, t.r_end, t.r_depth, t.r_op,
+                                           mode="indexed")
+    assert st == oracle.OK
+    ctx = opa.Context(0)
+    tr = opa.to_device(t)
+    tq = opa.to_device(t)
+    tq.k_start = torch.from_numpy(launch).cuda()
+    st, rk, nop = ctx.enclose(tq)
+    np.testing.assert_array_equal(rk.cpu().numpy(), want_rk)
+    np.testing.assert_array_equal(nop.cpu().numpy(), want_nop)
+    st, idx, kind, _ = ctx.match(tr)
+    st, ops, tot = ctx.aggregate(tr, rk, idx)
+    o = oracle.aggregate(t.k_dur, want_rk, t.r_op, t.counters, idx.cpu().numpy(), t.n_ops)
+    for k in ("kernel_count", "total_duration_ns", "matched_count"):
+        np.testing.assert_array_equal(ops[k].cpu().numpy(), o[1][k])
+    assert_close(ops["agg"].cpu().numpy(), o[1]["agg"], what="agg")
+    ctx.close()

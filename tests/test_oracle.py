@@ -100,6 +100,43 @@ def test_worked_permuted(golden, mode):
     assert idx.tolist() == np.array(g["expect"][mode]["ncu_idx"])[kp].tolist()
 
 
+@pytest.mark.parametrize("brute", [False, True])
+def test_per_stream_ordinals(brute):
+    # Limitations paragraph (Sec. 6): Nsight Compute replays a multi-stream
+    # workload one stream per run, so its rows come as per-stream runs and
+    # the k-th launch of a name must be counted per (name, stream).
+    # Launches in time order: t0 A on s0, t1 A on s1, t2 A on s0, t3 B on s1.
+    # Rows: the s0 run (A, A), then the s1 run (A, B).
+    ks = np.array([0, 1, 0, 1], np.uint8)
+    kt = np.array([0, 1, 2, 3], np.int64)
+    kn = np.array([7, 7, 7, 9], np.uint32)
+    nn = np.array([7, 7, 7, 9], np.uint32)
+    ns = np.array([0, 0, 1, 1], np.uint8)
+    st, idx, kind, summ = oracle.match(ks, kt, kn, nn, ncu_stream=ns, brute=brute)
+    assert st == oracle.OK and idx.tolist() == [0, 2, 1, 3] and kind.tolist() == [1, 1, 1, 1]
+    # the per-name reading pairs the rows with the wrong launches
+    st, idx, kind, summ = oracle.match(ks, kt, kn, nn, brute=brute)
+    assert idx.tolist() == [0, 1, 2, 3]
+    # a run missing one launch: skip-name drops only that (name, stream)
+    st, idx, kind, summ = oracle.match(ks, kt, kn, nn[[0, 2, 3]], ncu_stream=ns[[0, 2, 3]], brute=brute)
+    assert st == oracle.W_COUNT_MISMATCH and idx.tolist() == [-1, 1, -1, 2]
+    assert summ["names_mismatched"] == 1 and summ["count_unmatched"] == 2
+    # names must fit beside the stream in one 32-bit key
+    st, _, _, _ = oracle.match(ks, kt, np.array([7, 7, 1 << 24, 9], np.uint32), nn, ncu_stream=ns, brute=brute)
+    assert st == oracle.E_INVALID_ARG
+
+
+def test_per_stream_runs_generator():
+    # tracegen.per_stream_runs regroups one-row-per-kernel traces into runs:
+    # with per-stream ordinals every kernel gets its own row back
+    t = tracegen.generate("gpt2")
+    u = tracegen.per_stream_runs(t)
+    st, idx, kind, summ = oracle.match(u.k_stream, u.k_start, u.k_name, u.ncu_name, ncu_stream=u.ncu_stream)
+    assert st == oracle.OK and (kind == 1).all()
+    assert np.array_equal(u.counters[idx], t.counters)
+    assert np.array_equal(u.ncu_stream[idx], u.k_stream)
+
+
 def test_table8_rules():
     # Table 8: SUM for #1 #2 #3 #11 #15 #19, MAX for #18 #20, DW-mean for the rest
     sums, maxes = {1, 2, 3, 11, 15, 19}, {18, 20}

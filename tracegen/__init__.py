@@ -139,6 +139,7 @@ class Trace:
     class_of_layer: np.ndarray | None = None   # i32[n_layers]
     rep_of_class: np.ndarray | None = None     # i32[n_classes]
     config: dict = field(default_factory=dict)
+    ncu_stream: np.ndarray | None = None       # u8[M] stream of each ncu row (per-stream replay runs)
 
     @property
     def K(self) -> int:
@@ -257,3 +258,21 @@ def small_random(seed: int, n_streams: int = 2, n_events: int = 40, t_max: int =
         r_op=np.array(ro, np.uint32)[rp] if R else np.zeros(0, np.uint32),
         n_ops=next_op, ncu_name=ncu_name, counters=counters,
         config=dict(seed=seed, small=True))
+
+
+def per_stream_runs(trace: Trace, stream_order=None) -> Trace:
+    """The same trace with its ncu rows as Nsight Compute gives them when it
+    replays one stream per run: the rows of each stream in launch order, the
+    runs one after another (streams ascending, or in `stream_order`), every
+    row tagged with its stream.  Needs one row per kernel in kernel time
+    order (the generator's default)."""
+    import dataclasses
+    K = trace.K
+    if trace.M != K:
+        raise ValueError("per_stream_runs needs one ncu row per kernel")
+    ks = trace.k_stream.astype(np.int64)
+    rank = np.arange(K) if stream_order is None else np.argsort(np.asarray(stream_order))[ks]
+    # kernels are in time order, so a stable sort by stream keeps each run in launch order
+    order = np.argsort(ks if stream_order is None else rank, kind="stable")
+    return dataclasses.replace(trace, ncu_name=trace.ncu_name[order].copy(), counters=trace.counters[order].copy(),
+                               ncu_stream=trace.k_stream[order].copy())
