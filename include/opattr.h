@@ -213,8 +213,11 @@ opattr_status opattr_enclose(opattr_ctx *ctx, const opattr_kernels *kernels, con
  * row of kernel k or -1; match_kind[k] = 0 none, 1 direct, 2 broadcast.
  * Ordinals are taken over replayed kernels in time order and over rows in
  * array order, per name -- or per (name, stream) when ncu->stream is given:
- * then a kernel's "name" everywhere below (counts, ordinals, mismatch modes,
- * the duplicate-layer name check) is the pair.  `dedup` (host) may be NULL;
+ * then a kernel's "name" in counts, ordinals and mismatch modes is the pair,
+ * while the duplicate-layer check of Sec. 3.7 still compares plain names (a
+ * class's representative layer may run on another stream).  When the two
+ * sides, each partitioned stably by stream, carry the same keys position by
+ * position, the pairing is read off directly.  `dedup` (host) may be NULL;
  * deduplication also needs kernels->layer_id and cfg.dedup = 1.
  * Reads kernels->stream, start_ns, name_id (and layer_id), ncu->name_id (and
  * ncu->stream).

@@ -60,7 +60,7 @@ def _lib():
             lib.orc_validate_ranges_brute.argtypes = [i64, vp, vp, vp, vp]
             lib.orc_validate_ranges_indexed.argtypes = [i64, vp, vp, vp, vp]
             lib.orc_enclose.argtypes = [ctypes.c_int, i64, vp, vp, i64, vp, vp, vp, vp, vp, vp, vp]
-            lib.orc_match.argtypes = [ctypes.c_int, i64, vp, vp, vp, vp, i64, vp, ctypes.c_int, i32, vp,
+            lib.orc_match.argtypes = [ctypes.c_int, i64, vp, vp, vp, vp, vp, i64, vp, ctypes.c_int, i32, vp,
                                       i32, vp, ctypes.c_int, vp, vp, vp]
             lib.orc_aggregate.argtypes = [i64, vp, vp, i64, vp, i64, vp, vp, i64, vp, vp, vp, vp, vp, vp]
             lib.orc_agg_rule.argtypes = [ctypes.c_int]
@@ -134,9 +134,12 @@ def match(k_stream, k_start, k_name, ncu_name, k_layer=None, class_of_layer=None
     With ncu_stream (the stream of each ncu row, from per-stream replay runs),
     Algorithm 1's key is the pair (name, stream) rather than the name: kernels
     and rows are keyed name * 256 + stream (names below 2^24), and everything
-    the algorithm does with names it does with those keys."""
+    the algorithm does with names it does with those keys.  The dedup
+    broadcast (Sec. 3.7) still compares plain names: a layer and its class's
+    representative may run on different streams."""
     lib = _lib()
     ks, kt, kn = _c(k_stream, np.uint8), _c(k_start, np.int64), _c(k_name, np.uint32)
+    kname_plain = kn
     kl = _c(k_layer, np.int32)
     nn = _c(ncu_name, np.uint32)
     if ncu_stream is not None and len(nn) > 0:
@@ -153,7 +156,7 @@ def match(k_stream, k_start, k_name, ncu_name, k_layer=None, class_of_layer=None
     out_i = np.full(K, -1, np.int32)
     out_k = np.zeros(K, np.uint8)
     summ = np.zeros(len(SUMMARY_FIELDS), np.int64)
-    st = lib.orc_match(int(brute), K, _p(ks), _p(kt), _p(kn), _p(kl), M, _p(nn), int(bool(dedup)),
+    st = lib.orc_match(int(brute), K, _p(ks), _p(kt), _p(kn), _p(kname_plain), _p(kl), M, _p(nn), int(bool(dedup)),
                        n_layers, _p(col), n_classes, _p(roc), MODES[mode], _p(out_i), _p(out_k), _p(summ))
     return st, out_i, out_k, dict(zip(SUMMARY_FIELDS, (int(x) for x in summ)))
 

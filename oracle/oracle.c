@@ -357,11 +357,16 @@ static int check_dedup(int64_t K, const int32_t *layer, int32_t n_layers, const 
 
 /* Matching.  mode: 0 skip-name, 1 prefix (Algorithm 1 as printed), 2 error.
  * dedup_on: 1 when layer deduplication applies (k_layer and tables given).
+ * k_name is the matching key (the kernel name, or the (name, stream) key
+ * with per-stream rows); k_layer_name is the kernel name itself, which the
+ * broadcast of Sec. 3.7 compares between a layer and its class's
+ * representative -- the two may run on different streams.
  * brute: 1 computes ordinals by rescanning all earlier records (definition
  * written out, O(K^2 + M^2)); 0 runs Algorithm 1's single pass with per-name
  * counters. */
 int orc_match(int brute, int64_t K, const uint8_t *k_stream, const int64_t *k_start, const uint32_t *k_name,
-              const int32_t *k_layer, int64_t M, const uint32_t *ncu_name, int dedup_on, int32_t n_layers,
+              const uint32_t *k_layer_name, const int32_t *k_layer, int64_t M, const uint32_t *ncu_name,
+              int dedup_on, int32_t n_layers,
               const int32_t *class_of_layer, int32_t n_classes, const int32_t *rep_of_class, int mode,
               int32_t *out_idx, uint8_t *out_kind, int64_t *summary) {
     if (mode < 0 || mode > 2) return ORC_E_INVALID_ARG;
@@ -470,7 +475,7 @@ int orc_match(int brute, int64_t K, const uint8_t *k_stream, const int64_t *k_st
                 int32_t rep = rep_of_class[class_of_layer[k_layer[k]]];
                 int64_t p = pos[k];
                 int64_t src = p < lay_cnt[rep] ? lay_kern[rep][p] : -1;
-                if (src >= 0 && k_name[src] == k_name[k] && out_idx[src] >= 0) {
+                if (src >= 0 && k_layer_name[src] == k_layer_name[k] && out_idx[src] >= 0) {
                     out_idx[k] = out_idx[src]; out_kind[k] = 2; summary[3]++;
                 } else {
                     summary[7]++;

@@ -34,6 +34,7 @@ struct AggIn {
     const int32_t *ncu_idx;
     const float *counters;
     int64_t n_ops;
+    unsigned *ctr;              // next chunk of the ops pass, zeroed before it
     opattr_op_aggregates out;
 };
 
@@ -473,9 +474,11 @@ __global__ void __launch_bounds__(SL_THREADS) k_agg_sort_long(const uint32_t *__
 // time, orders them by segment length (longest first) and walks them in
 // AG_CHUNK / 32 rounds, so that the threads of a round walk segments of
 // similar length; warps share nothing and never wait for each other.  The
-// grid is what stays resident and takes the chunks in order, so the kernels
-// and outputs the GPU works on at any moment form one window that stays in
-// L2.  Segments are walked in ascending kernel index: a short one is checked
+// grid is what stays resident; warps draw the chunks in increasing order
+// from one counter, so the ops in flight at any moment are one narrow band
+// of op ids whatever each warp's pace (a fixed chunk-to-warp assignment lets
+// fast and slow warps drift apart and widens the band), and with op ids in
+// range order the kernels and outputs of that band stay in L2.  Segments are walked in ascending kernel index: a short one is checked
 // and, in the rare case the fill left it out of order, insertion-sorted in
 // place by its thread; long ones were sorted by k_agg_sort_long.  While a
 // kernel is added, the counter rows and durations of the next two arrive in
@@ -483,7 +486,7 @@ __global__ void __launch_bounds__(SL_THREADS) k_agg_sort_long(const uint32_t *__
 // row indices loaded a step earlier still.
 constexpr int AG_THREADS = 128;
 constexpr int AG_WARPS = AG_THREADS / 32;
-constexpr int AG_CHUNK = 128;                   // op ids per warp and chunk
+constexpr int AG_CHUNK = 64;                    // op ids per warp and chunk
 constexpr int AG_LBUCKETS = 32;
 
 // An op whose fast sums saw a null or infinite value: the segment again, in
@@ -519,10 +522,13 @@ __global__ void __launch_bounds__(AG_THREADS) k_agg_ops(const uint32_t *__restri
     uint32_t *lcount = lcount_s[threadIdx.x / 32];
     uint8_t *order = order_s[threadIdx.x / 32];
     const unsigned lane = lane_id();
-    const int64_t nwarps = (int64_t)gridDim.x * AG_WARPS;
     int bad = 0;
-    for (int64_t o0 = ((int64_t)blockIdx.x * AG_WARPS + threadIdx.x / 32) * AG_CHUNK; o0 < A.n_ops;
-         o0 += nwarps * AG_CHUNK) {
+    auto next_chunk = [&]() -> int64_t {
+        unsigned v = 0;
+        if (lane == 0) v = atomicAdd(A.ctr, 1u);
+        return (int64_t)__shfl_sync(0xffffffffu, v, 0) * AG_CHUNK;
+    };
+    for (int64_t o0 = next_chunk(); o0 < A.n_ops; o0 = next_chunk()) {
         const int nchunk = A.n_ops - o0 < AG_CHUNK ? (int)(A.n_ops - o0) : AG_CHUNK;
         // lengths of the chunk's ops, counting sort by length (descending, capped)
         constexpr int PER = AG_CHUNK / 32;
@@ -644,7 +650,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
 
     Need nd;
     nd.add<uint32_t>(O + 1).add<uint32_t>(O + 1).add<uint32_t>(O + 1).add<uint32_t>(K).add<uint32_t>(K);
-    nd.add<uint32_t>(O + 1).add<unsigned>(1);
+    nd.add<uint32_t>(O + 1).add<unsigned>(1).add<unsigned>(1);
     nd.add<uint32_t>(scan_scratch_elems(O + 1));
     opattr_status st = ensure_arena(c, nd.bytes + 4096);
     if (st) return st;
@@ -653,6 +659,8 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     uint32_t *cnt = a.take<uint32_t>(O + 1), *off = a.take<uint32_t>(O + 1), *cur = a.take<uint32_t>(O + 1);
     uint32_t *list = a.take<uint32_t>(K), *tmp = a.take<uint32_t>(K), *longs = a.take<uint32_t>(O + 1);
     unsigned *nlong = a.take<unsigned>(1);
+    unsigned *ctr = a.take<unsigned>(1);
+    cudaMemsetAsync(ctr, 0, sizeof(unsigned), c.stream);
     uint32_t *part = a.take<uint32_t>(scan_scratch_elems(O + 1));
     if (!cnt || !off || !cur || !list || !tmp || !longs || !nlong || !part) return OPATTR_E_OOM;
     cudaMemsetAsync(cnt, 0, sizeof(uint32_t) * (O + 1), c.stream);
@@ -666,6 +674,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     in.ncu_idx = nidx;
     in.counters = ncu->counters;
     in.n_ops = O;
+    in.ctr = ctr;
     in.out = *out;
     if (O > 0) {
         scan_exclusive_u32(c, cnt, off, O + 1, part, nullptr);

@@ -5,7 +5,9 @@
 // names of the ncu rows in array order, launch i pairs with row i and no
 // ordinal is computed: one pass compares the two name arrays and writes the
 // identity.  Exports in time order with ncu replaying the same launches hit
-// this path.
+// this path.  With per-stream rows (the rows of each stream in launch order,
+// streams one after another) the same test runs on the replayed kernels and
+// the rows each partitioned stably by stream.
 //
 // General path.  Ordinals come from stable radix sorts: replayed kernels in
 // time order sorted by name give o(k) = position - start of the name's run;
@@ -56,6 +58,45 @@ __global__ void k_match_identity_list(const uint32_t *__restrict__ rk, const uin
         if (out_kind) out_kind[k] = 1;
     }
     if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_flag(st, F_NAMES_DIFFER);
+}
+
+// Per-stream rows.  Replayed kernel j (kernel rk[j], or j when rk is null)
+// sits at position dest[j] of the replayed kernels partitioned stably by
+// stream; the row at that position of the rows partitioned the same way is
+// pn[dest[j]].  The pairing holds when name and stream agree everywhere;
+// name ids must also fit in 24 bits, as (name, stream) keys require.
+__global__ void k_match_stream_pairs(const uint32_t *__restrict__ rk, const uint32_t *__restrict__ dest,
+                                     const uint32_t *__restrict__ pn, const uint32_t *__restrict__ kname,
+                                     const uint8_t *__restrict__ kstream, const uint32_t *__restrict__ nname,
+                                     const uint8_t *__restrict__ nstream, int64_t n, int32_t *__restrict__ out_idx,
+                                     uint8_t *__restrict__ out_kind, DevStatus *st) {
+    int bad = 0, wide = 0;
+    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n; j += (int64_t)gridDim.x * blockDim.x) {
+        const uint32_t k = rk ? rk[j] : (uint32_t)j;
+        const uint32_t r = pn[dest[j]];
+        const uint32_t x = kname[k], y = nname[r];
+        wide |= (x | y) >> 24 != 0;
+        bad |= x != y || kstream[k] != nstream[r];
+        out_idx[k] = (int32_t)r;
+        if (out_kind) out_kind[k] = 1;
+    }
+    if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_flag(st, F_NAMES_DIFFER);
+    if (__any_sync(0xffffffffu, wide) && lane_id() == 0) set_err(st, ERR_INVALID);
+}
+
+// Name ids of every kernel below 2^24 (per-stream rows with layer classes,
+// where the pairing above sees the replayed kernels only).
+__global__ void k_check_names24(const uint32_t *__restrict__ name, int64_t n, DevStatus *st) {
+    uint32_t acc = 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        acc |= name[i];
+    if (__any_sync(0xffffffffu, acc >> 24 != 0) && lane_id() == 0) set_err(st, ERR_INVALID);
+}
+
+__global__ void k_gather_u8(const uint8_t *__restrict__ src, const uint32_t *__restrict__ idx, int64_t n,
+                            uint8_t *__restrict__ dst) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        dst[i] = src[idx[i]];
 }
 
 __global__ void k_fill_match(int32_t *out_idx, uint8_t *out_kind, int64_t n) {
@@ -142,53 +183,106 @@ __device__ __forceinline__ int64_t upper_bound_u32(const uint32_t *a, int64_t n,
     return lo;
 }
 
-// The ordinal join.  i runs over replayed kernels sorted by (name, time).
-//   skn / skj: sorted names, and the time rank j of each (rk[j] = kernel)
-//   snn / snj: ncu names sorted, and the row index of each
-__global__ void k_ordinal_join(const uint32_t *__restrict__ skn, const uint32_t *__restrict__ skj,
-                               const uint32_t *__restrict__ rk, int64_t nrep, const uint32_t *__restrict__ snn,
-                               const uint32_t *__restrict__ snj, int64_t M, int mode, int32_t *__restrict__ out_idx,
-                               uint8_t *__restrict__ out_kind, DevStatus *st) {
-    unsigned long long direct = 0, unmatched = 0, names_bad = 0;
-    int err = 0;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nrep; i += (int64_t)gridDim.x * blockDim.x) {
-        uint32_t name = skn[i];
-        bool head = i == 0 || skn[i - 1] != name;
-        int64_t lo = head ? i : lower_bound_u32(skn, nrep, name);
-        int64_t ck = upper_bound_u32(skn, nrep, name) - lo;
-        int64_t b = lower_bound_u32(snn, M, name);
-        int64_t cq = upper_bound_u32(snn, M, name) - b;
-        int64_t o = i - lo;
-        bool ok = mode == OPATTR_MISMATCH_SKIP_NAME ? (ck == cq) : (o < cq);
-        if (mode == OPATTR_MISMATCH_ERROR && ck != cq) err = 1;
-        int32_t idx = ok && o < cq ? (int32_t)snj[b + o] : -1;
-        uint32_t k = rk[skj[i]];
-        out_idx[k] = idx;
-        if (out_kind) out_kind[k] = idx >= 0 ? 1 : 0;
-        direct += idx >= 0;
-        unmatched += idx < 0;
-        names_bad += head && ck != cq;
+// Runs of equal keys in a sorted array.  flag[i] = 1 at each run's first
+// element; after an exclusive scan pos[i] counts the runs that start before
+// i, so element i lies in run pos[i] + head(i) - 1 and start[pos[i]] = i at
+// each head.
+__device__ __forceinline__ bool run_head(const uint32_t *a, int64_t i) { return i == 0 || a[i - 1] != a[i]; }
+
+__global__ void k_run_heads(const uint32_t *__restrict__ a, int64_t n, uint32_t *__restrict__ flag) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        flag[i] = run_head(a, i);
+}
+__global__ void k_run_starts(const uint32_t *__restrict__ a, const uint32_t *__restrict__ pos, int64_t n,
+                             uint32_t *__restrict__ start) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        if (run_head(a, i)) start[pos[i]] = (uint32_t)i;
+}
+
+// First run r in [0, nr) whose key a[start[r]] is >= x.
+__device__ __forceinline__ int64_t lower_bound_runs(const uint32_t *a, const uint32_t *start, int64_t nr, uint32_t x) {
+    int64_t lo = 0, hi = nr;
+    while (lo < hi) {
+        int64_t m = (lo + hi) >> 1;
+        if (a[start[m]] < x) lo = m + 1; else hi = m;
+    }
+    return lo;
+}
+
+// Per kernel name run u (replayed kernels sorted by (name, time)): the ncu
+// rows of the same name, as the first position b[u] in the sorted rows and
+// their count cq[u].  Runs whose kernel and row counts differ are counted
+// (and are an error in the error mode).
+__global__ void k_run_pair(const uint32_t *__restrict__ skn, const uint32_t *__restrict__ ustart,
+                           const uint32_t *__restrict__ n_urun, int64_t nrep, const uint32_t *__restrict__ snn,
+                           const uint32_t *__restrict__ vstart, const uint32_t *__restrict__ n_vrun, int64_t M,
+                           int mode, uint32_t *__restrict__ b_of, uint32_t *__restrict__ cq_of, DevStatus *st) {
+    const int64_t U = *n_urun, V = *n_vrun;
+    unsigned long long names_bad = 0;
+    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < U; u += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t lo = ustart[u], hi = u + 1 < U ? ustart[u + 1] : nrep;
+        const uint32_t name = skn[lo];
+        const int64_t v = lower_bound_runs(snn, vstart, V, name);
+        const bool found = v < V && snn[vstart[v]] == name;
+        const int64_t b = found ? vstart[v] : 0;
+        const int64_t cq = found ? (v + 1 < V ? vstart[v + 1] : M) - b : 0;
+        b_of[u] = (uint32_t)b;
+        cq_of[u] = (uint32_t)cq;
+        names_bad += hi - lo != cq;
     }
     __shared__ unsigned long long red[33];
-    if (__any_sync(0xffffffffu, err) && lane_id() == 0) set_err(st, ERR_COUNT);
-    block_add_u64(direct, &st->cnt[C_DIRECT], red);
-    block_add_u64(unmatched, &st->cnt[C_COUNT_UNMATCHED], red);
+    if (__any_sync(0xffffffffu, names_bad != 0) && lane_id() == 0 && mode == OPATTR_MISMATCH_ERROR)
+        set_err(st, ERR_COUNT);
     block_add_u64(names_bad, &st->cnt[C_NAMES_MISMATCH], red);
 }
 
-// Names that have ncu rows but no replayed kernel at all.
-__global__ void k_ncu_only_names(const uint32_t *__restrict__ snn, int64_t M, const uint32_t *__restrict__ skn,
-                                 int64_t nrep, int mode, DevStatus *st) {
+// Names that have ncu rows but no replayed kernel at all (one thread per
+// ncu name run).
+__global__ void k_ncu_only_names(const uint32_t *__restrict__ snn, const uint32_t *__restrict__ vstart,
+                                 const uint32_t *__restrict__ n_vrun, const uint32_t *__restrict__ skn,
+                                 const uint32_t *__restrict__ ustart, const uint32_t *__restrict__ n_urun, int mode,
+                                 DevStatus *st) {
+    const int64_t U = *n_urun, V = *n_vrun;
     unsigned long long bad = 0;
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < M; i += (int64_t)gridDim.x * blockDim.x) {
-        uint32_t name = snn[i];
-        if (i > 0 && snn[i - 1] == name) continue;
-        int64_t lo = lower_bound_u32(skn, nrep, name);
-        bad += lo == nrep || skn[lo] != name;
+    for (int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < V; v += (int64_t)gridDim.x * blockDim.x) {
+        const uint32_t name = snn[vstart[v]];
+        const int64_t u = lower_bound_runs(skn, ustart, U, name);
+        bad += u == U || skn[ustart[u]] != name;
     }
     __shared__ unsigned long long red[33];
     if (__any_sync(0xffffffffu, bad != 0) && lane_id() == 0 && mode == OPATTR_MISMATCH_ERROR) set_err(st, ERR_COUNT);
     block_add_u64(bad, &st->cnt[C_NAMES_MISMATCH], red);
+}
+
+// The ordinal join.  i runs over replayed kernels sorted by (name, time):
+//   skn / skj: sorted names, and the time rank j of each (rk[j] = kernel)
+//   kpos / ustart / b_of / cq_of: the run tables of skn
+//   snj: the row index of each ncu row in name-sorted order
+// Kernel i is the o-th of its name with o = i - ustart[run]; its row is the
+// o-th row of the name, subject to the mismatch mode.
+__global__ void k_ordinal_join(const uint32_t *__restrict__ skn, const uint32_t *__restrict__ skj,
+                               const uint32_t *__restrict__ kpos, const uint32_t *__restrict__ ustart,
+                               const uint32_t *__restrict__ n_urun, const uint32_t *__restrict__ b_of,
+                               const uint32_t *__restrict__ cq_of, const uint32_t *__restrict__ rk, int64_t nrep,
+                               const uint32_t *__restrict__ snj, int mode, int32_t *__restrict__ out_idx,
+                               uint8_t *__restrict__ out_kind, DevStatus *st) {
+    const int64_t U = *n_urun;
+    unsigned long long direct = 0, unmatched = 0;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nrep; i += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t u = (int64_t)kpos[i] + run_head(skn, i) - 1;
+        const int64_t lo = ustart[u], hi = u + 1 < U ? ustart[u + 1] : nrep;
+        const int64_t cq = cq_of[u], o = i - lo;
+        const bool ok = mode == OPATTR_MISMATCH_SKIP_NAME ? (hi - lo == cq) : (o < cq);
+        const int32_t idx = ok && o < cq ? (int32_t)snj[b_of[u] + o] : -1;
+        const uint32_t k = rk[skj[i]];
+        out_idx[k] = idx;
+        if (out_kind) out_kind[k] = idx >= 0 ? 1 : 0;
+        direct += idx >= 0;
+        unmatched += idx < 0;
+    }
+    __shared__ unsigned long long red[33];
+    block_add_u64(direct, &st->cnt[C_DIRECT], red);
+    block_add_u64(unmatched, &st->cnt[C_COUNT_UNMATCHED], red);
 }
 
 // Broadcast.  i runs over layer-tagged kernels sorted by (layer, time).
@@ -248,6 +342,28 @@ static opattr_status read_u64(Ctx &c, const unsigned long long *d, unsigned long
     return OPATTR_OK;
 }
 
+// The stream-partitioned pairing over n replayed kernels (list rk, or the
+// kernel array itself when rk is null) and the n rows.  Scratch: kst (n
+// bytes), dest (n), nb (n bytes), nv0 / nv1 (n).
+static void stream_pairs(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu, const uint32_t *rk, int64_t n,
+                         uint8_t *kst, uint32_t *dest, uint8_t *nb, uint32_t *nv0, uint32_t *nv1, uint32_t *hist,
+                         uint32_t *part, int32_t *out_idx, uint8_t *out_kind) {
+    const uint8_t *keys = kern->stream;
+    if (rk) {
+        launch(c, "gather_streams", k_gather_u8, dim3(grid_for(n, 256, REDUCE_GRID)), dim3(256), 0, kern->stream, rk,
+               n, kst);
+        keys = kst;
+    }
+    radix_rank<uint8_t>(c, keys, n, 0, hist, part, dest);
+    // one 8-bit pass: the row streams are only read
+    uint8_t *ko;
+    uint32_t *pn;
+    radix_sort_pairs<uint8_t>(c, const_cast<uint8_t *>(ncu->stream), nv0, nb, nv1, n, 8, true, hist, part, &ko, &pn);
+    launch(c, "match_stream_pairs", k_match_stream_pairs, dim3(grid_for(n, 256, REDUCE_GRID)), dim3(256), 0, rk,
+           (const uint32_t *)dest, (const uint32_t *)pn, kern->name_id, kern->stream, ncu->name_id, ncu->stream, n,
+           out_idx, out_kind, c.d_status);
+}
+
 opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu, const opattr_dedup *dd,
                        int32_t *out_idx, uint8_t *out_kind, opattr_match_summary *sum) {
     const int64_t K = kern->n, M = ncu->n;
@@ -280,8 +396,8 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     for (int i = 0; i < 5; ++i) nd.add<uint32_t>(K);                 // flag, pos, rk, lk, keys
     for (int i = 0; i < 3; ++i) nd.add<uint32_t>(NX);                // sort buffers
     for (int i = 0; i < 4; ++i) nd.add<uint32_t>(M);                 // ncu sort
-    nd.add<uint32_t>(radix_hist_elems(NX)).add<uint32_t>(scan_scratch_elems(std::max(radix_hist_elems(NX), K)));
-    nd.add<unsigned long long>(2);
+    nd.add<uint32_t>(radix_hist_elems(NX)).add<uint32_t>(scan_scratch_elems(std::max(radix_hist_elems(NX), NX)));
+    nd.add<unsigned long long>(4);
     size_t need = nd.bytes + kernel_order_scratch(K) + 4096;
     opattr_status st = ensure_arena(c, need);
     if (st) return st;
@@ -293,26 +409,21 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     uint32_t *s0 = a.take<uint32_t>(NX), *s1 = a.take<uint32_t>(NX), *s2 = a.take<uint32_t>(NX);
     uint32_t *n0 = a.take<uint32_t>(M), *n1 = a.take<uint32_t>(M), *n2 = a.take<uint32_t>(M), *n3 = a.take<uint32_t>(M);
     uint32_t *hist = a.take<uint32_t>(radix_hist_elems(NX));
-    uint32_t *part = a.take<uint32_t>(scan_scratch_elems(std::max(radix_hist_elems(NX), K)));
-    unsigned long long *dsm = a.take<unsigned long long>(2);
+    uint32_t *part = a.take<uint32_t>(scan_scratch_elems(std::max(radix_hist_elems(NX), NX)));
+    unsigned long long *dsm = a.take<unsigned long long>(4);
     if (!d_rep || !flag || !pos || !rk || !lk || !k0 || !s0 || !s1 || !s2 || !n0 || !n1 || !n2 || !n3 || !hist ||
         !part || !dsm)
         return OPATTR_E_OOM;
     if (dedup_on && dd->n_layers > 0)
         cudaMemcpyAsync(d_rep, rep_layer.data(), sizeof(int32_t) * dd->n_layers, cudaMemcpyHostToDevice, c.stream);
-    // the matching key: the name id, or (name, stream) when the rows carry streams
+    // the matching key: the name id, or (name, stream) when the rows carry
+    // streams (built only if the general path runs)
     const uint32_t *kname = kern->name_id, *nname = ncu->name_id;
+    uint32_t *kkey = nullptr, *nkey = nullptr;
     if (per_stream) {
-        uint32_t *kkey = a.take<uint32_t>(K), *nkey = a.take<uint32_t>(M);
+        kkey = a.take<uint32_t>(K);
+        nkey = a.take<uint32_t>(M);
         if ((K > 0 && !kkey) || (M > 0 && !nkey)) return OPATTR_E_OOM;
-        if (K > 0)
-            launch(c, "stream_keys", k_stream_keys, dim3(grid_for(K, 256, REDUCE_GRID)), dim3(256), 0, kern->name_id,
-                   kern->stream, K, kkey, c.d_status);
-        if (M > 0)
-            launch(c, "stream_keys", k_stream_keys, dim3(grid_for(M, 256, REDUCE_GRID)), dim3(256), 0, ncu->name_id,
-                   ncu->stream, M, nkey, c.d_status);
-        kname = kkey;
-        nname = nkey;
     }
 
     const unsigned gK = grid_for(K, 256, REDUCE_GRID);
@@ -320,23 +431,34 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     if (dedup_on && K > 0)
         launch(c, "check_layers", k_check_layers, dim3(gK), dim3(256), 0, kern->layer_id, K, dd->n_layers,
                (const int32_t *)d_rep, c.d_status);
-    const bool try_identity = !dedup_on && K == M && K > 0;
+    if (per_stream && dedup_on && K > 0)
+        launch(c, "check_names24", k_check_names24, dim3(grid_for(K, 256 * 8, REDUCE_GRID)), dim3(256), 0,
+               kern->name_id, K, c.d_status);
+    // Speculative fast paths, taking the kernel array to be in time order
+    // (confirmed or refuted by the order check in the same batch).
+    const bool try_identity = !dedup_on && !per_stream && K == M && K > 0;
+    const bool try_streams = !dedup_on && per_stream && K == M && K > 0;
     if (try_identity)
         launch(c, "match_identity", k_match_identity, dim3(grid_for(K, 256 * 16, REDUCE_GRID)), dim3(256), 0,
                kname, nname, K, out_idx,
                out_kind, c.d_status);
+    if (try_streams)
+        stream_pairs(c, kern, ncu, nullptr, K, reinterpret_cast<uint8_t *>(k0), s0, reinterpret_cast<uint8_t *>(n2),
+                     n0, n1, hist, part, out_idx, out_kind);
     if ((st = read_status(c))) return st;
     if (c.h_status->err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
     const bool k_sorted = !(c.h_status->flags & F_K_UNSORTED);
     opattr_match_summary S{};
     S.kernels = K;
     S.replayed = dedup_on ? (int64_t)c.h_status->cnt[C_REPLAYED] : K;
-    if (try_identity && k_sorted && !(c.h_status->flags & F_NAMES_DIFFER)) {
+    if ((try_identity || try_streams) && k_sorted && !(c.h_status->flags & F_NAMES_DIFFER)) {
         S.direct = K;
         S.fast_path = 1;
         if (sum) *sum = S;
         return OPATTR_OK;
     }
+    // the speculative verdicts are spent: later checks start from clear flags
+    cudaMemsetAsync(&c.d_status->flags, 0, sizeof(unsigned), c.stream);
 
     // ---- general path
     if (K > 0) launch(c, "fill_match", k_fill_match, dim3(gK), dim3(256), 0, out_idx, out_kind, K);
@@ -359,15 +481,31 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
         else launch(c, "iota", k_iota, dim3(gK), dim3(256), 0, rk, K);
     }
     bool direct_done = false;
-    if (dedup_on && nrep == M && nrep > 0) {
-        launch(c, "match_identity_list", k_match_identity_list, dim3(grid_for(nrep, 256, REDUCE_GRID)), dim3(256), 0,
-               (const uint32_t *)rk, kname, nname, nrep, out_idx, out_kind, c.d_status);
+    const bool retry_streams = per_stream && (dedup_on || korder) && nrep == M && nrep > 0;
+    if ((dedup_on && !per_stream && nrep == M && nrep > 0) || retry_streams) {
+        if (retry_streams)
+            stream_pairs(c, kern, ncu, rk, nrep, reinterpret_cast<uint8_t *>(k0), s0, reinterpret_cast<uint8_t *>(n2),
+                         n0, n1, hist, part, out_idx, out_kind);
+        else
+            launch(c, "match_identity_list", k_match_identity_list, dim3(grid_for(nrep, 256, REDUCE_GRID)),
+                   dim3(256), 0, (const uint32_t *)rk, kname, nname, nrep, out_idx, out_kind, c.d_status);
         if ((st = read_status(c))) return st;
+        if (c.h_status->err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
         direct_done = !(c.h_status->flags & F_NAMES_DIFFER);
         if (direct_done) S.fast_path = 1;
         else launch(c, "fill_match", k_fill_match, dim3(gK), dim3(256), 0, out_idx, out_kind, K);
     }
     if (!direct_done && (nrep > 0 || M > 0)) {
+        if (per_stream) {
+            if (K > 0)
+                launch(c, "stream_keys", k_stream_keys, dim3(grid_for(K, 256, REDUCE_GRID)), dim3(256), 0,
+                       kern->name_id, kern->stream, K, kkey, c.d_status);
+            if (M > 0)
+                launch(c, "stream_keys", k_stream_keys, dim3(grid_for(M, 256, REDUCE_GRID)), dim3(256), 0,
+                       ncu->name_id, ncu->stream, M, nkey, c.d_status);
+            kname = kkey;
+            nname = nkey;
+        }
         cudaMemsetAsync(dsm, 0, sizeof(unsigned long long), c.stream);
         if (nrep > 0) {
             launch(c, "gather_names", k_gather_u32, dim3(grid_for(nrep, 256, REDUCE_GRID)), dim3(256), 0, kname,
@@ -385,13 +523,41 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
         uint32_t *skn = nullptr, *skj = nullptr, *snn = n0, *snj = n1;
         if (nrep > 0) radix_sort_pairs<uint32_t>(c, k0, s0, s1, s2, nrep, bits, true, hist, part, &skn, &skj);
         if (M > 0) radix_sort_pairs<uint32_t>(c, n0, n1, n2, n3, M, bits, true, hist, part, &snn, &snj);
+        // run tables of both sorted name arrays (pos / start pairs in the
+        // buffers the sorts left free)
+        uint32_t *kfree0 = skn == k0 ? s1 : k0, *kfree1 = skn == k0 ? s2 : s0;
+        uint32_t *nfree0 = snn == n0 ? n2 : n0, *nfree1 = snn == n0 ? n3 : n1;
+        uint32_t *kpos = flag, *ustart = pos, *b_of = kfree0, *cq_of = kfree1, *vpos = nfree0, *vstart = nfree1;
+        uint32_t *n_urun = reinterpret_cast<uint32_t *>(dsm + 2), *n_vrun = reinterpret_cast<uint32_t *>(dsm + 3);
+        if (nrep > 0) {
+            launch(c, "run_heads", k_run_heads, dim3(grid_for(nrep, 256, REDUCE_GRID)), dim3(256), 0,
+                   (const uint32_t *)skn, nrep, kpos);
+        }
+        scan_exclusive_u32(c, kpos, kpos, nrep, part, n_urun);
         if (nrep > 0)
+            launch(c, "run_starts", k_run_starts, dim3(grid_for(nrep, 256, REDUCE_GRID)), dim3(256), 0,
+                   (const uint32_t *)skn, (const uint32_t *)kpos, nrep, ustart);
+        if (M > 0)
+            launch(c, "run_heads", k_run_heads, dim3(grid_for(M, 256, REDUCE_GRID)), dim3(256), 0,
+                   (const uint32_t *)snn, M, vpos);
+        scan_exclusive_u32(c, vpos, vpos, M, part, n_vrun);
+        if (M > 0)
+            launch(c, "run_starts", k_run_starts, dim3(grid_for(M, 256, REDUCE_GRID)), dim3(256), 0,
+                   (const uint32_t *)snn, (const uint32_t *)vpos, M, vstart);
+        if (nrep > 0) {
+            launch(c, "run_pair", k_run_pair, dim3(grid_for(nrep, 256, REDUCE_GRID)), dim3(256), 0,
+                   (const uint32_t *)skn, (const uint32_t *)ustart, (const uint32_t *)n_urun, nrep,
+                   (const uint32_t *)snn, (const uint32_t *)vstart, (const uint32_t *)n_vrun, M, mode, b_of, cq_of,
+                   c.d_status);
             launch(c, "ordinal_join", k_ordinal_join, dim3(grid_for(nrep, 256, REDUCE_GRID)), dim3(256), 0,
-                   (const uint32_t *)skn, (const uint32_t *)skj, (const uint32_t *)rk, nrep, (const uint32_t *)snn,
-                   (const uint32_t *)snj, M, mode, out_idx, out_kind, c.d_status);
+                   (const uint32_t *)skn, (const uint32_t *)skj, (const uint32_t *)kpos, (const uint32_t *)ustart,
+                   (const uint32_t *)n_urun, (const uint32_t *)b_of, (const uint32_t *)cq_of, (const uint32_t *)rk,
+                   nrep, (const uint32_t *)snj, mode, out_idx, out_kind, c.d_status);
+        }
         if (M > 0)
             launch(c, "ncu_only_names", k_ncu_only_names, dim3(grid_for(M, 256, REDUCE_GRID)), dim3(256), 0,
-                   (const uint32_t *)snn, M, (const uint32_t *)skn, nrep, mode, c.d_status);
+                   (const uint32_t *)snn, (const uint32_t *)vstart, (const uint32_t *)n_vrun, (const uint32_t *)skn,
+                   (const uint32_t *)ustart, (const uint32_t *)n_urun, mode, c.d_status);
     }
     if (dedup_on && K > 0) {
         // positions within layers: layer-tagged kernels in time order, sorted by layer
@@ -413,11 +579,12 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
                                        &sll, &slj);
             launch(c, "dedup_broadcast", k_dedup_broadcast, dim3(grid_for(nlk, 256, REDUCE_GRID)), dim3(256), 0,
                    (const uint32_t *)sll, (const uint32_t *)slj, (const uint32_t *)lk, nlk, (const int32_t *)d_rep,
-                   kname, out_idx, out_kind, c.d_status);
+                   kern->name_id, out_idx, out_kind, c.d_status);   // plain names: a class may span streams
         }
     }
     if ((st = read_status(c))) return st;
     const DevStatus &H = *c.h_status;
+    if (H.err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
     if (H.err & ERR_COUNT) return OPATTR_E_COUNT_MISMATCH;
     S.direct = direct_done ? nrep : (int64_t)H.cnt[C_DIRECT];
     S.broadcast = (int64_t)H.cnt[C_BROADCAST];

@@ -36,6 +36,12 @@ template <typename K>
 void radix_sort_pairs(Ctx &c, K *k0, uint32_t *v0, K *k1, uint32_t *v1, int64_t n, int bits, bool iota,
                       uint32_t *hist, uint32_t *partials, K **kout, uint32_t **vout);
 
+// One stable counting pass on key bits [shift, shift + 8) that moves
+// nothing: dest[i] receives the position element i would take.  hist /
+// partials as for radix_sort_pairs.
+template <typename K>
+void radix_rank(Ctx &c, const K *keys, int64_t n, int shift, uint32_t *hist, uint32_t *partials, uint32_t *dest);
+
 // Number of bits needed to represent v (0 for v == 0).
 inline int bits_for(uint64_t v) {
     int b = 0;

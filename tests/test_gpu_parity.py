@@ -350,7 +350,37 @@ def test_per_stream_runs(opa, name, order):
     g = gpu_run(u)
     assert_parity(g, oracle.run(u, enclose_mode="indexed"))
     assert (g["match_kind"] == 1).all()
+    assert g["summary"]["fast_path"] == 1
     np.testing.assert_array_equal(u.counters[g["ncu_idx"]], t.counters)
+
+
+@pytest.mark.parametrize("name,shuffle", [("dedup", False), ("gpt2", True), ("dedup", True), ("gpt2_dedup", False)])
+def test_per_stream_partition_paths(opa, name, shuffle):
+    """Per-stream rows with layer classes (the rows are the replayed kernels,
+    gathered by stream) and with kernel arrays out of time order: the
+    stream-partitioned pairing gives the oracle's answer."""
+    t = tracegen.generate(name, shuffle=shuffle)
+    u = tracegen.per_stream_runs(t)
+    g = gpu_run(u)
+    assert_parity(g, oracle.run(u, enclose_mode="indexed"))
+    assert g["summary"]["fast_path"] == 1
+    assert g["summary"]["unmatched"] == 0
+
+
+@pytest.mark.parametrize("mode", ["skip_name", "prefix", "error"])
+def test_per_stream_swapped_rows(opa, mode):
+    """Two rows of different names swapped inside one stream's run: the
+    stream-partitioned pairing no longer holds and the general ordinal join
+    decides, name by name."""
+    t = tracegen.generate("gpt2")
+    u = tracegen.per_stream_runs(t)
+    s0 = np.nonzero(u.ncu_stream == u.ncu_stream[0])[0]
+    j = s0[1 + np.nonzero(u.ncu_name[s0[1:]] != u.ncu_name[s0[0]])[0][0]]
+    for a in (u.ncu_name, u.counters):
+        a[[s0[0], j]] = a[[j, s0[0]]]
+    g = gpu_run(u, mode=mode)
+    assert_parity(g, oracle.run(u, mode=mode, enclose_mode="indexed"))
+    assert g["summary"]["fast_path"] == 0
 
 
 @pytest.mark.parametrize("seed", range(0, 40, 3))

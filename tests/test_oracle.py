@@ -137,6 +137,26 @@ def test_per_stream_runs_generator():
     assert np.array_equal(u.ncu_stream[idx], u.k_stream)
 
 
+@pytest.mark.parametrize("name,shuffle", [("dedup", False), ("gpt2", True), ("dedup", True)])
+def test_per_stream_runs_generator_dedup_shuffled(name, shuffle):
+    # with layer classes the rows are the replayed kernels only, and with
+    # shuffled kernel arrays the rows still follow kernel time order: per-
+    # stream ordinals give every replayed kernel the row the time-ordered
+    # join gave it
+    t = tracegen.generate(name, shuffle=shuffle)
+    u = tracegen.per_stream_runs(t)
+    dd = bool(t.config.get("dedup")) and t.k_layer is not None
+    args = dict(k_layer=t.k_layer, class_of_layer=t.class_of_layer, rep_of_class=t.rep_of_class, dedup=dd)
+    st0, idx0, kind0, _ = oracle.match(t.k_stream, t.k_start, t.k_name, t.ncu_name, **args)
+    st1, idx1, kind1, _ = oracle.match(u.k_stream, u.k_start, u.k_name, u.ncu_name, ncu_stream=u.ncu_stream, **args)
+    assert st0 == oracle.OK and st1 == oracle.OK
+    assert np.array_equal(kind0, kind1)
+    m = idx0 >= 0
+    assert np.array_equal(idx1 >= 0, m)
+    assert np.array_equal(u.counters[idx1[m]], t.counters[idx0[m]])
+    assert np.array_equal(u.ncu_stream[idx1[kind1 == 1]], u.k_stream[kind1 == 1])
+
+
 def test_table8_rules():
     # Table 8: SUM for #1 #2 #3 #11 #15 #19, MAX for #18 #20, DW-mean for the rest
     sums, maxes = {1, 2, 3, 11, 15, 19}, {18, 20}

@@ -264,15 +264,25 @@ def per_stream_runs(trace: Trace, stream_order=None) -> Trace:
     """The same trace with its ncu rows as Nsight Compute gives them when it
     replays one stream per run: the rows of each stream in launch order, the
     runs one after another (streams ascending, or in `stream_order`), every
-    row tagged with its stream.  Needs one row per kernel in kernel time
-    order (the generator's default)."""
+    row tagged with its stream.  Needs one row per replayed kernel in kernel
+    time order (the generator's default): every kernel, or with layer classes
+    the kernels outside layers and in each class's representative layer."""
     import dataclasses
-    K = trace.K
-    if trace.M != K:
-        raise ValueError("per_stream_runs needs one ncu row per kernel")
-    ks = trace.k_stream.astype(np.int64)
-    rank = np.arange(K) if stream_order is None else np.argsort(np.asarray(stream_order))[ks]
-    # kernels are in time order, so a stable sort by stream keeps each run in launch order
-    order = np.argsort(ks if stream_order is None else rank, kind="stable")
+    tk = np.lexsort((trace.k_stream.astype(np.int64), trace.k_start))        # kernels in time order
+    replayed = np.ones(trace.K, bool)
+    if trace.k_layer is not None and trace.class_of_layer is not None and trace.M != trace.K:
+        layer = trace.k_layer[tk]
+        rep = trace.rep_of_class[trace.class_of_layer[np.maximum(layer, 0)]]
+        replayed = (layer < 0) | (rep == layer)
+    row_stream = trace.k_stream[tk][replayed].astype(np.int64)
+    if row_stream.shape[0] != trace.M:
+        raise ValueError("per_stream_runs needs one ncu row per replayed kernel")
+    key = row_stream
+    if stream_order is not None:
+        pos = np.full(256, 256, np.int64)                   # streams not listed go last
+        pos[np.asarray(stream_order, np.int64)] = np.arange(len(stream_order))
+        key = pos[row_stream]
+    # rows are in time order, so a stable sort by stream keeps each run in launch order
+    order = np.argsort(key, kind="stable")
     return dataclasses.replace(trace, ncu_name=trace.ncu_name[order].copy(), counters=trace.counters[order].copy(),
-                               ncu_stream=trace.k_stream[order].copy())
+                               ncu_stream=row_stream[order].astype(np.uint8))
