@@ -41,6 +41,8 @@ KERNEL_BYTES = {
     "check_kernel_order": lambda K, R, M, O: 9 * K,
     "check_ranges": lambda K, R, M, O: 18 * R,
     "level_gather": lambda K, R, M, O: 44 * R,
+    "level_place": lambda K, R, M, O: 42 * R,
+    "match_stream_pairs": lambda K, R, M, O: 18 * K,
     "validate_levels": lambda K, R, M, O: 22 * R,
     "window_table": lambda K, R, M, O: 0,
 }

@@ -108,6 +108,105 @@ __global__ void k_level_gather(const int64_t *__restrict__ start, const int64_t 
     }
 }
 
+// The same partition in one counting pass when at most 256 levels are
+// present: range i's digit is its compact level id (levels numbered in
+// (stream, depth) order, so a stable partition by compact id is the stable
+// sort by level key), and k_level_place writes each range's level-list
+// entry in place of the key sort and the gather.
+struct LevelDigit {
+    const uint8_t *stream, *depth;
+    const uint8_t *cmap;        // [LEVELS] compact id of each present level
+    const uint32_t *perm;       // NULL = array order
+    __device__ __forceinline__ unsigned operator()(int64_t i) const {
+        const uint32_t r = perm ? perm[i] : (uint32_t)i;
+        return cmap[stream[r] * 32u + depth[r]];
+    }
+};
+// The placing pass: the digit-rank of the tile's ranges gives each its
+// place in the tile sorted by compact level; the range is staged there in
+// shared memory, then each level's run of the tile goes out to consecutive
+// addresses (one coalesced write per run instead of one scattered write per
+// range).  Same tiles as digit_offsets.
+struct PlaceSmem {
+    int64_t s[RADIX_TILE];
+    int64_t e[RADIX_TILE];
+    uint32_t info[RADIX_TILE];
+    uint8_t dig[RADIX_TILE];
+    uint32_t wcnt[(RADIX_THREADS / 32) * RADIX_BINS];
+    uint32_t dstart[RADIX_BINS];
+    uint32_t gbase[RADIX_BINS];
+    uint32_t wbuf[33];
+};
+__global__ void __launch_bounds__(RADIX_THREADS) k_level_place(LevelDigit digit, const int64_t *__restrict__ start,
+                                                               const int64_t *__restrict__ end,
+                                                               const uint32_t *__restrict__ op, int64_t n,
+                                                               const uint32_t *__restrict__ offs, int64_t ntiles,
+                                                               int64_t *__restrict__ ls, int64_t *__restrict__ le,
+                                                               uint32_t *__restrict__ li) {
+    extern __shared__ __align__(16) unsigned char place_raw[];
+    PlaceSmem &S = *reinterpret_cast<PlaceSmem *>(place_raw);
+    const unsigned w = threadIdx.x >> 5, lane = lane_id();
+    for (int i = threadIdx.x; i < (RADIX_THREADS / 32) * RADIX_BINS; i += RADIX_THREADS) S.wcnt[i] = 0;
+    __syncthreads();
+    const int64_t tile0 = (int64_t)blockIdx.x * RADIX_TILE;
+    const int64_t base = tile0 + w * (RADIX_TILE / 8);
+    unsigned dg[RADIX_ITEMS];
+    uint32_t rank[RADIX_ITEMS];
+    const unsigned lt = lanemask_lt();
+#pragma unroll
+    for (int it = 0; it < RADIX_ITEMS; ++it) {
+        const int64_t i = base + it * 32 + lane;
+        const unsigned d = i < n ? digit(i) : (unsigned)RADIX_BINS;
+        const unsigned peers = __match_any_sync(0xffffffffu, d);
+        const unsigned before = d < RADIX_BINS ? S.wcnt[w * RADIX_BINS + d] : 0u;
+        __syncwarp();
+        if (d < RADIX_BINS && (peers & lt) == 0) S.wcnt[w * RADIX_BINS + d] = before + __popc(peers);
+        __syncwarp();
+        rank[it] = before + __popc(peers & lt);
+        dg[it] = d;
+    }
+    __syncthreads();
+    uint32_t tot;
+    {
+        // RADIX_THREADS == RADIX_BINS: thread d owns digit d
+        const unsigned d = threadIdx.x;
+        uint32_t sum = 0;
+#pragma unroll
+        for (int q = 0; q < RADIX_THREADS / 32; ++q) {
+            const uint32_t x = S.wcnt[q * RADIX_BINS + d];
+            S.wcnt[q * RADIX_BINS + d] = sum;
+            sum += x;
+        }
+        tot = sum;
+    }
+    const uint32_t ds = block_exclusive_scan<uint32_t>(tot, S.wbuf, (uint32_t *)nullptr);
+    S.dstart[threadIdx.x] = ds;
+    S.gbase[threadIdx.x] = offs[(int64_t)threadIdx.x * ntiles + blockIdx.x];
+    __syncthreads();
+#pragma unroll
+    for (int it = 0; it < RADIX_ITEMS; ++it) {
+        const int64_t i = base + it * 32 + lane;
+        const unsigned d = dg[it];
+        if (d < RADIX_BINS) {
+            const uint32_t p = S.dstart[d] + S.wcnt[w * RADIX_BINS + d] + rank[it];
+            const uint32_t r = digit.perm ? digit.perm[i] : (uint32_t)i;
+            S.s[p] = start[r];
+            S.e[p] = end[r];
+            S.info[p] = r | (kind_of(op[r]) << 30);
+            S.dig[p] = (uint8_t)d;
+        }
+    }
+    __syncthreads();
+    const int cnt = (int)(n - tile0 < RADIX_TILE ? n - tile0 : RADIX_TILE);
+    for (int j = threadIdx.x; j < cnt; j += RADIX_THREADS) {
+        const unsigned d = S.dig[j];
+        const int64_t o = (int64_t)S.gbase[d] + (j - S.dstart[d]);
+        ls[o] = S.s[j];
+        le[o] = S.e[j];
+        li[o] = S.info[j];
+    }
+}
+
 // Laminar checks over level positions: adjacent pairs of a level, and the
 // parent of every range at depth > 0 (the last range of level (s, d-1) that
 // starts no later; it must end no earlier).
@@ -140,25 +239,52 @@ __global__ void k_validate_levels(const uint8_t *__restrict__ stream, const uint
 // ------------------------------------------------------------------ window table
 // P[t * nl + l] = (last position p of level l with lvl_start[p] <= b_t) - level
 // start, or -1; b_t = start of the time-ordered kernel t*ENC_TILE for
-// t < nt, and of the last kernel for t = nt.
+// t < nt, and of the last kernel for t = nt.  The b_t do not decrease, so
+// one thread takes WT_CHUNK consecutive tiles of one level: a binary search
+// for the first, then an exponential search forward from the previous
+// answer for each next one (cost logarithmic in the entries passed, however
+// unevenly a level's ranges fall between tiles).  Neighbouring threads take
+// neighbouring levels, so the rows of P are written together.
+constexpr int WT_CHUNK = 16;
+__device__ __forceinline__ long long tile_bound(const int64_t *k_start, const uint32_t *korder, int64_t K, int64_t nt,
+                                                int64_t t) {
+    const int64_t pos = t < nt ? t * ENC_TILE : K - 1;
+    return k_start[korder ? korder[pos] : pos];
+}
 __global__ void k_window_table(const int64_t *__restrict__ ls, const uint32_t *__restrict__ lvl_off,
                                const uint16_t *__restrict__ level_of_compact, int nl,
                                const int64_t *__restrict__ k_start, const uint32_t *__restrict__ korder, int64_t K,
                                int64_t nt, int32_t *__restrict__ P) {
-    const int64_t total = (nt + 1) * nl;
+    const int64_t nchunk = (nt + 1 + WT_CHUNK - 1) / WT_CHUNK;
+    const int64_t total = nchunk * nl;
     for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < total; q += (int64_t)gridDim.x * blockDim.x) {
-        int64_t t = q / nl;
-        int l = (int)(q - t * nl);
-        int64_t pos = t < nt ? t * ENC_TILE : K - 1;
-        long long b = k_start[korder ? korder[pos] : pos];
-        uint32_t L = level_of_compact[l];
-        int64_t lo = lvl_off[L], hi = lvl_off[L + 1];
-        int64_t x = lo, y = hi;
-        while (x < y) {
-            int64_t m = (x + y) >> 1;
-            if (ls[m] <= b) x = m + 1; else y = m;
+        const int64_t ch = q / nl;
+        const int l = (int)(q - ch * nl);
+        const uint32_t L = level_of_compact[l];
+        const int64_t lo = lvl_off[L], hi = lvl_off[L + 1];
+        const int64_t t0 = ch * WT_CHUNK, t1 = t0 + WT_CHUNK < nt + 1 ? t0 + WT_CHUNK : nt + 1;
+        int64_t x = lo;                       // first position with start > b (for the current tile)
+        for (int64_t t = t0; t < t1; ++t) {
+            const long long b = tile_bound(k_start, korder, K, nt, t);
+            int64_t a2 = x, z = x;
+            if (t > t0) {
+                int64_t step = 1;
+                while (z < hi && ls[z] <= b) {
+                    a2 = z + 1;
+                    z += step;
+                    step <<= 1;
+                }
+                if (z > hi) z = hi;
+            } else {
+                z = hi;
+            }
+            while (a2 < z) {                  // first position in [a2, z) with start > b, else z
+                const int64_t m = (a2 + z) >> 1;
+                if (ls[m] <= b) a2 = m + 1; else z = m;
+            }
+            x = a2;
+            P[t * nl + l] = (int32_t)(x - lo - 1);
         }
-        P[q] = (int32_t)(x - lo - 1);
     }
 }
 
@@ -315,8 +441,9 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
         constexpr int RD = 8;                     // depths whose positions stay in registers
         int cur_s = -1, nd = 0, a0 = 0;
         int pr[RD];                               // window position + 1 (0 none, -1 not searched yet)
+        int wo[RD], wc[RD];                       // window offset and length of each depth (current stream)
 #pragma unroll
-        for (int d = 0; d < RD; ++d) pr[d] = -1;
+        for (int d = 0; d < RD; ++d) pr[d] = -1, wo[d] = 0, wc[d] = 0;
         // The last walk's answer holds for a later kernel of the stream while
         // no range of a depth the walk looked at starts in between and every
         // range it found still contains the kernel: the walk would visit the
@@ -336,10 +463,38 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
                 nd = A.ndepth[s];
                 a0 = S.sbase[s];
 #pragma unroll
-                for (int d = 0; d < RD; ++d) pr[d] = -1;
+                for (int d = 0; d < RD; ++d) {
+                    pr[d] = -1;
+                    wo[d] = d < nd ? S.act_off[a0 + d] : 0;
+                    wc[d] = d < nd ? S.act_cnt[a0 + d] : 0;
+                }
                 reuse_below = 0;
             }
             if (!(T < reuse_below && T <= reuse_upto)) {
+                // every depth's candidate first (independent lookups, in
+                // flight together), then the walk over them in registers
+                uint32_t cs[RD], ce[RD], ci[RD], cn[RD];
+#pragma unroll
+                for (int d = 0; d < RD; ++d) {
+                    const int c = wc[d], o = wo[d];
+                    int p;                          // last window position with start <= T, or -1
+                    if (pr[d] < 0) {
+                        int x = o, y = o + c;
+                        while (x < y) {
+                            const int m = (x + y) >> 1;
+                            if (S.ws[m] <= T) x = m + 1; else y = m;
+                        }
+                        p = x - o - 1;
+                    } else {
+                        p = pr[d] - 1;
+                        while (p + 1 < c && S.ws[o + p + 1] <= T) ++p;
+                    }
+                    pr[d] = p + 1;
+                    cn[d] = p + 1 < c ? S.ws[o + p + 1] : 0xFFFFFFFFu;
+                    cs[d] = p >= 0 ? 1u : 0u;
+                    ce[d] = p >= 0 ? S.we[o + p] : 0u;
+                    ci[d] = p >= 0 ? S.wi[o + p] : 0u;
+                }
                 ans = -1;
                 nop = 0;
                 bool alive = true;
@@ -347,30 +502,14 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
 #pragma unroll
                 for (int d = 0; d < RD; ++d) {
                     if (alive && d < nd) {
-                        const int c = S.act_cnt[a0 + d], o = S.act_off[a0 + d];
-                        int p;                          // last window position with start <= T, or -1
-                        if (pr[d] < 0) {
-                            int x = o, y = o + c;
-                            while (x < y) {
-                                const int m = (x + y) >> 1;
-                                if (S.ws[m] <= T) x = m + 1; else y = m;
-                            }
-                            p = x - o - 1;
-                        } else {
-                            p = pr[d] - 1;
-                            while (p + 1 < c && S.ws[o + p + 1] <= T) ++p;
-                        }
-                        pr[d] = p + 1;
-                        if (p + 1 < c) next_start = min(next_start, S.ws[o + p + 1]);
-                        if (p < 0 || S.we[o + p] < T) {
+                        next_start = min(next_start, cn[d]);
+                        if (!cs[d] || ce[d] < T) {
                             alive = false;
                         } else {
-                            const uint32_t e = S.we[o + p];
-                            min_end = min(min_end, e);
-                            const uint32_t info = S.wi[o + p];
-                            const uint32_t kind = info >> 30;
+                            min_end = min(min_end, ce[d]);
+                            const uint32_t kind = ci[d] >> 30;
                             if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
-                            else if (kind == KIND_OP) { ans = (int32_t)(info & 0x3FFFFFFFu); nop++; }
+                            else if (kind == KIND_OP) { ans = (int32_t)(ci[d] & 0x3FFFFFFFu); nop++; }
                         }
                     }
                 }
@@ -459,7 +598,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     const int64_t part_n = std::max<int64_t>(scan_scratch_elems(radix_hist_elems(R)), scan_scratch_elems(LEVELS + 1));
     nd.add<uint32_t>(radix_hist_elems(R)).add<uint32_t>(part_n);
     nd.add<int64_t>(R).add<int64_t>(R).add<uint32_t>(R);
-    nd.add<uint16_t>(LEVELS).add<uint16_t>(256).add<uint8_t>(256);
+    nd.add<uint16_t>(LEVELS).add<uint16_t>(256).add<uint8_t>(256).add<uint8_t>(LEVELS);
     nd.add<int32_t>((nt + 1) * (int64_t)LEVELS);
     size_t need = nd.bytes + kernel_order_scratch(K) + 4096;
     opattr_status st = ensure_arena(c, need);
@@ -511,6 +650,8 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
         ndep[s] = (uint8_t)n;
     }
     const int nl = (int)level_of_compact.size();
+    std::vector<uint8_t> cmap(LEVELS, 0);
+    for (int l = 0; l < nl && l < 256; ++l) cmap[level_of_compact[l]] = (uint8_t)l;
 
     uint64_t *rk0 = a.take<uint64_t>(R), *rk1 = a.take<uint64_t>(R);
     uint32_t *rv0 = a.take<uint32_t>(R), *rv1 = a.take<uint32_t>(R);
@@ -520,13 +661,15 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     uint16_t *d_loc = a.take<uint16_t>(LEVELS);
     uint16_t *d_cbase = a.take<uint16_t>(256);
     uint8_t *d_ndep = a.take<uint8_t>(256);
+    uint8_t *d_cmap = a.take<uint8_t>(LEVELS);
     int32_t *P = a.take<int32_t>((nt + 1) * (int64_t)(nl > 0 ? nl : 1));
-    if (!rk0 || !rk1 || !rv0 || !rv1 || !hist || !ls || !le || !li || !d_loc || !d_cbase || !d_ndep || !P)
+    if (!rk0 || !rk1 || !rv0 || !rv1 || !hist || !ls || !le || !li || !d_loc || !d_cbase || !d_ndep || !d_cmap || !P)
         return OPATTR_E_OOM;
     cudaMemcpyAsync(d_loc, level_of_compact.data(), sizeof(uint16_t) * (nl > 0 ? nl : 1), cudaMemcpyHostToDevice,
                     c.stream);
     cudaMemcpyAsync(d_cbase, cbase.data(), sizeof(uint16_t) * 256, cudaMemcpyHostToDevice, c.stream);
     cudaMemcpyAsync(d_ndep, ndep.data(), 256, cudaMemcpyHostToDevice, c.stream);
+    if (nl <= 256) cudaMemcpyAsync(d_cmap, cmap.data(), LEVELS, cudaMemcpyHostToDevice, c.stream);
 
     // ---- kernel time order
     uint32_t *korder = nullptr;
@@ -559,16 +702,30 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
                    rmin, kfree);
             radix_sort_pairs<uint64_t>(c, kfree, vo, ko, vfree, R, bits, false, hist, part, &ko, &perm);
         }
-        // stable partition by level key (13 bits)
-        uint32_t *lk0 = reinterpret_cast<uint32_t *>(rk0), *lk1 = reinterpret_cast<uint32_t *>(rk1);
-        uint32_t *va = perm ? perm : rv0;
-        uint32_t *vb = perm == rv0 ? rv1 : (perm == rv1 ? rv0 : rv1);
-        launch(c, "level_keys", k_level_keys, dim3(g), dim3(256), 0, rng->stream, rng->depth, (const uint32_t *)perm, R,
-               lk0);
-        uint32_t *ko32, *lperm;
-        radix_sort_pairs<uint32_t>(c, lk0, va, lk1, vb, R, 13, perm == nullptr, hist, part, &ko32, &lperm);
-        launch(c, "level_gather", k_level_gather, dim3(g), dim3(256), 0, rng->start_ns, rng->end_ns, rng->op_id,
-               (const uint32_t *)lperm, R, ls, le, li);
+        if (nl <= 256) {
+            // stable partition by compact level id, ranges written in place
+            const LevelDigit dg{rng->stream, rng->depth, d_cmap, perm};
+            digit_offsets(c, dg, R, hist, part);
+            static unsigned place_attr = 0;
+            if (c.device < 32 && !(place_attr & (1u << c.device))) {
+                cudaFuncSetAttribute(k_level_place, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(PlaceSmem));
+                place_attr |= 1u << c.device;
+            }
+            const int64_t ntiles = (R + RADIX_TILE - 1) / RADIX_TILE;
+            launch(c, "level_place", k_level_place, dim3((unsigned)ntiles), dim3(RADIX_THREADS), sizeof(PlaceSmem), dg,
+                   rng->start_ns, rng->end_ns, rng->op_id, R, (const uint32_t *)hist, ntiles, ls, le, li);
+        } else {
+            // stable partition by level key (13 bits)
+            uint32_t *lk0 = reinterpret_cast<uint32_t *>(rk0), *lk1 = reinterpret_cast<uint32_t *>(rk1);
+            uint32_t *va = perm ? perm : rv0;
+            uint32_t *vb = perm == rv0 ? rv1 : (perm == rv1 ? rv0 : rv1);
+            launch(c, "level_keys", k_level_keys, dim3(g), dim3(256), 0, rng->stream, rng->depth,
+                   (const uint32_t *)perm, R, lk0);
+            uint32_t *ko32, *lperm;
+            radix_sort_pairs<uint32_t>(c, lk0, va, lk1, vb, R, 13, perm == nullptr, hist, part, &ko32, &lperm);
+            launch(c, "level_gather", k_level_gather, dim3(g), dim3(256), 0, rng->start_ns, rng->end_ns, rng->op_id,
+                   (const uint32_t *)lperm, R, ls, le, li);
+        }
         launch(c, "validate_levels", k_validate_levels, dim3(grid_for(R, 256, 65535)), dim3(256), 0, rng->stream,
                rng->depth, (const int64_t *)ls, (const int64_t *)le, (const uint32_t *)li, (const uint32_t *)lvl_off,
                R, c.d_status);
@@ -576,7 +733,8 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
             launch(c, "fill_unattributed", k_fill_unattributed, dim3(grid_for(K, 256, 65535)), dim3(256), 0, out_range,
                    out_nop, K);
         if (K > 0 && nl > 0) {
-            launch(c, "window_table", k_window_table, dim3(grid_for((nt + 1) * nl, 256, 65535)), dim3(256), 0,
+            launch(c, "window_table", k_window_table,
+                   dim3(grid_for((nt + 1 + WT_CHUNK - 1) / WT_CHUNK * nl, 256, 65535)), dim3(256), 0,
                    (const int64_t *)ls, (const uint32_t *)lvl_off, (const uint16_t *)d_loc, nl, kern->start_ns,
                    (const uint32_t *)korder, K, nt, P);
             EncArgs A;

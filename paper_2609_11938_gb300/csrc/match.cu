@@ -61,28 +61,34 @@ __global__ void k_match_identity_list(const uint32_t *__restrict__ rk, const uin
 }
 
 // Per-stream rows.  Replayed kernel j (kernel rk[j], or j when rk is null)
-// sits at position dest[j] of the replayed kernels partitioned stably by
-// stream; the row at that position of the rows partitioned the same way is
-// pn[dest[j]].  The pairing holds when name and stream agree everywhere;
-// name ids must also fit in 24 bits, as (name, stream) keys require.
-__global__ void k_match_stream_pairs(const uint32_t *__restrict__ rk, const uint32_t *__restrict__ dest,
-                                     const uint32_t *__restrict__ pn, const uint32_t *__restrict__ kname,
-                                     const uint8_t *__restrict__ kstream, const uint32_t *__restrict__ nname,
-                                     const uint8_t *__restrict__ nstream, int64_t n, int32_t *__restrict__ out_idx,
-                                     uint8_t *__restrict__ out_kind, DevStatus *st) {
-    int bad = 0, wide = 0;
-    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n; j += (int64_t)gridDim.x * blockDim.x) {
+// takes position dest of the replayed kernels partitioned stably by stream;
+// the row at that position of the rows partitioned the same way is pn[dest].
+// The pairing holds when name and stream agree everywhere; name ids must
+// also fit in 24 bits, as (name, stream) keys require.
+struct StreamDigit {
+    const uint32_t *rk;
+    const uint8_t *stream;
+    __device__ __forceinline__ unsigned operator()(int64_t j) const { return stream[rk ? rk[j] : (uint32_t)j]; }
+};
+struct StreamPairs {
+    const uint32_t *rk, *pn, *kname, *nname;
+    const uint8_t *kstream, *nstream;
+    int32_t *out_idx;
+    uint8_t *out_kind;
+    DevStatus *st;
+    __device__ __forceinline__ unsigned operator()(int64_t j, uint32_t dest) const {
         const uint32_t k = rk ? rk[j] : (uint32_t)j;
-        const uint32_t r = pn[dest[j]];
+        const uint32_t r = pn[dest];
         const uint32_t x = kname[k], y = nname[r];
-        wide |= (x | y) >> 24 != 0;
-        bad |= x != y || kstream[k] != nstream[r];
         out_idx[k] = (int32_t)r;
         if (out_kind) out_kind[k] = 1;
+        return (x != y || kstream[k] != nstream[r] ? 1u : 0u) | ((x | y) >> 24 != 0 ? 2u : 0u);
     }
-    if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_flag(st, F_NAMES_DIFFER);
-    if (__any_sync(0xffffffffu, wide) && lane_id() == 0) set_err(st, ERR_INVALID);
-}
+    __device__ __forceinline__ void done(unsigned bits) const {
+        if (__any_sync(0xffffffffu, bits & 1u) && lane_id() == 0) set_flag(st, F_NAMES_DIFFER);
+        if (__any_sync(0xffffffffu, bits & 2u) && lane_id() == 0) set_err(st, ERR_INVALID);
+    }
+};
 
 // Name ids of every kernel below 2^24 (per-stream rows with layer classes,
 // where the pairing above sees the replayed kernels only).
@@ -91,12 +97,6 @@ __global__ void k_check_names24(const uint32_t *__restrict__ name, int64_t n, De
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         acc |= name[i];
     if (__any_sync(0xffffffffu, acc >> 24 != 0) && lane_id() == 0) set_err(st, ERR_INVALID);
-}
-
-__global__ void k_gather_u8(const uint8_t *__restrict__ src, const uint32_t *__restrict__ idx, int64_t n,
-                            uint8_t *__restrict__ dst) {
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
-        dst[i] = src[idx[i]];
 }
 
 __global__ void k_fill_match(int32_t *out_idx, uint8_t *out_kind, int64_t n) {
@@ -343,25 +343,21 @@ static opattr_status read_u64(Ctx &c, const unsigned long long *d, unsigned long
 }
 
 // The stream-partitioned pairing over n replayed kernels (list rk, or the
-// kernel array itself when rk is null) and the n rows.  Scratch: kst (n
-// bytes), dest (n), nb (n bytes), nv0 / nv1 (n).
+// kernel array itself when rk is null) and the n rows.  Scratch: nb (n
+// bytes), nv0 / nv1 (n).
 static void stream_pairs(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu, const uint32_t *rk, int64_t n,
-                         uint8_t *kst, uint32_t *dest, uint8_t *nb, uint32_t *nv0, uint32_t *nv1, uint32_t *hist,
-                         uint32_t *part, int32_t *out_idx, uint8_t *out_kind) {
-    const uint8_t *keys = kern->stream;
-    if (rk) {
-        launch(c, "gather_streams", k_gather_u8, dim3(grid_for(n, 256, REDUCE_GRID)), dim3(256), 0, kern->stream, rk,
-               n, kst);
-        keys = kst;
-    }
-    radix_rank<uint8_t>(c, keys, n, 0, hist, part, dest);
-    // one 8-bit pass: the row streams are only read
+                         uint8_t *nb, uint32_t *nv0, uint32_t *nv1, uint32_t *hist, uint32_t *part, int32_t *out_idx,
+                         uint8_t *out_kind) {
+    // rows: one 8-bit radix pass (it only reads the row streams)
     uint8_t *ko;
     uint32_t *pn;
     radix_sort_pairs<uint8_t>(c, const_cast<uint8_t *>(ncu->stream), nv0, nb, nv1, n, 8, true, hist, part, &ko, &pn);
-    launch(c, "match_stream_pairs", k_match_stream_pairs, dim3(grid_for(n, 256, REDUCE_GRID)), dim3(256), 0, rk,
-           (const uint32_t *)dest, (const uint32_t *)pn, kern->name_id, kern->stream, ncu->name_id, ncu->stream, n,
-           out_idx, out_kind, c.d_status);
+    // kernels: ranked by stream, each paired in the same pass
+    const StreamDigit dg{rk, kern->stream};
+    digit_offsets(c, dg, n, hist, part);
+    const StreamPairs ep{rk, pn, kern->name_id, ncu->name_id, kern->stream, ncu->stream, out_idx, out_kind,
+                         c.d_status};
+    digit_rank(c, "match_stream_pairs", dg, n, hist, ep);
 }
 
 opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu, const opattr_dedup *dd,
@@ -443,8 +439,8 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
                kname, nname, K, out_idx,
                out_kind, c.d_status);
     if (try_streams)
-        stream_pairs(c, kern, ncu, nullptr, K, reinterpret_cast<uint8_t *>(k0), s0, reinterpret_cast<uint8_t *>(n2),
-                     n0, n1, hist, part, out_idx, out_kind);
+        stream_pairs(c, kern, ncu, nullptr, K, reinterpret_cast<uint8_t *>(n2), n0, n1, hist, part, out_idx,
+                     out_kind);
     if ((st = read_status(c))) return st;
     if (c.h_status->err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
     const bool k_sorted = !(c.h_status->flags & F_K_UNSORTED);
@@ -484,8 +480,8 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     const bool retry_streams = per_stream && (dedup_on || korder) && nrep == M && nrep > 0;
     if ((dedup_on && !per_stream && nrep == M && nrep > 0) || retry_streams) {
         if (retry_streams)
-            stream_pairs(c, kern, ncu, rk, nrep, reinterpret_cast<uint8_t *>(k0), s0, reinterpret_cast<uint8_t *>(n2),
-                         n0, n1, hist, part, out_idx, out_kind);
+            stream_pairs(c, kern, ncu, rk, nrep, reinterpret_cast<uint8_t *>(n2), n0, n1, hist, part, out_idx,
+                         out_kind);
         else
             launch(c, "match_identity_list", k_match_identity_list, dim3(grid_for(nrep, 256, REDUCE_GRID)),
                    dim3(256), 0, (const uint32_t *)rk, kname, nname, nrep, out_idx, out_kind, c.d_status);

@@ -195,68 +195,6 @@ __global__ void __launch_bounds__(RADIX_THREADS) k_radix_downsweep(const K *__re
     }
 }
 
-// The stable destination of every key, written in input order: dest[i] is
-// where a stable sort on this digit would put element i.  The same ranking
-// as the scatter above, without moving the keys.
-template <typename K>
-__global__ void __launch_bounds__(RADIX_THREADS) k_radix_rank(const K *__restrict__ kin, int64_t n, int shift,
-                                                              const uint32_t *__restrict__ offs, int64_t ntiles,
-                                                              uint32_t *__restrict__ dest) {
-    __shared__ uint32_t wcnt[(RADIX_THREADS / 32) * RADIX_BINS];
-    __shared__ uint32_t gbase[RADIX_BINS];
-    const unsigned w = threadIdx.x >> 5, lane = lane_id();
-    for (int i = threadIdx.x; i < (RADIX_THREADS / 32) * RADIX_BINS; i += RADIX_THREADS) wcnt[i] = 0;
-    __syncthreads();
-    const int64_t base = (int64_t)blockIdx.x * RADIX_TILE + w * (RADIX_TILE / 8);
-    unsigned dig[RADIX_ITEMS];
-    uint32_t rank[RADIX_ITEMS];
-    const unsigned lt = lanemask_lt();
-#pragma unroll
-    for (int it = 0; it < RADIX_ITEMS; ++it) {
-        int64_t i = base + it * 32 + lane;
-        unsigned d = i < n ? digit_of(kin[i], shift) : RADIX_BINS;
-        unsigned peers = __match_any_sync(0xffffffffu, d);
-        unsigned before = d < RADIX_BINS ? wcnt[w * RADIX_BINS + d] : 0u;
-        __syncwarp();
-        if (d < RADIX_BINS && (peers & lt) == 0) wcnt[w * RADIX_BINS + d] = before + __popc(peers);
-        __syncwarp();
-        rank[it] = before + __popc(peers & lt);
-        dig[it] = d;
-    }
-    __syncthreads();
-    // RADIX_THREADS == RADIX_BINS: thread d turns digit d's per-warp counts
-    // into exclusive prefixes and fetches the digit's global start
-    {
-        const unsigned d = threadIdx.x;
-        uint32_t s = 0;
-#pragma unroll
-        for (int q = 0; q < RADIX_THREADS / 32; ++q) {
-            uint32_t x = wcnt[q * RADIX_BINS + d];
-            wcnt[q * RADIX_BINS + d] = s;
-            s += x;
-        }
-        gbase[d] = offs[(int64_t)d * ntiles + blockIdx.x];
-    }
-    __syncthreads();
-#pragma unroll
-    for (int it = 0; it < RADIX_ITEMS; ++it) {
-        int64_t i = base + it * 32 + lane;
-        if (i < n) dest[i] = gbase[dig[it]] + wcnt[w * RADIX_BINS + dig[it]] + rank[it];
-    }
-}
-
-template <typename K>
-void radix_rank(Ctx &c, const K *keys, int64_t n, int shift, uint32_t *hist, uint32_t *partials, uint32_t *dest) {
-    if (n <= 0) return;
-    const int64_t ntiles = (n + RADIX_TILE - 1) / RADIX_TILE;
-    launch(c, "radix_upsweep", k_radix_upsweep<K>, dim3((unsigned)ntiles), dim3(RADIX_THREADS), 0, keys, n, shift,
-           hist, ntiles);
-    scan_exclusive_u32(c, hist, hist, ntiles * RADIX_BINS, partials, nullptr);
-    launch(c, "radix_rank", k_radix_rank<K>, dim3((unsigned)ntiles), dim3(RADIX_THREADS), 0, keys, n, shift,
-           (const uint32_t *)hist, ntiles, dest);
-}
-template void radix_rank<uint8_t>(Ctx &, const uint8_t *, int64_t, int, uint32_t *, uint32_t *, uint32_t *);
-
 template <typename K>
 static size_t downsweep_smem() {
     return (size_t)RADIX_TILE * (sizeof(K) + 4) + ((RADIX_THREADS / 32) * RADIX_BINS + 2 * RADIX_BINS + 33) * 4;

@@ -36,11 +36,105 @@ template <typename K>
 void radix_sort_pairs(Ctx &c, K *k0, uint32_t *v0, K *k1, uint32_t *v1, int64_t n, int bits, bool iota,
                       uint32_t *hist, uint32_t *partials, K **kout, uint32_t **vout);
 
-// One stable counting pass on key bits [shift, shift + 8) that moves
-// nothing: dest[i] receives the position element i would take.  hist /
-// partials as for radix_sort_pairs.
-template <typename K>
-void radix_rank(Ctx &c, const K *keys, int64_t n, int shift, uint32_t *hist, uint32_t *partials, uint32_t *dest);
+// ------------------------------------------------------------------ digit passes
+// One stable counting pass whose 8-bit digit comes from a functor:
+// digit(i) in [0, RADIX_BINS) for element i < n, or RADIX_BINS to leave the
+// element out.  digit_offsets counts digits per tile of RADIX_TILE elements
+// (digit-major matrix in `hist`, radix_hist_elems(n) entries) and scans the
+// matrix; digit_rank then hands every counted element to epi(i, dest), where
+// dest is the position a stable sort by digit would give it, without moving
+// anything itself.  epi returns problem bits; epi.done(bits) runs in every
+// thread at the end (for warp votes).  Same tiles and ranking as the radix
+// sort: warps own consecutive 512-element runs, ranked 32 at a time with
+// __match_any_sync peer groups.
+template <typename DigitFn>
+__global__ void __launch_bounds__(RADIX_THREADS) k_digit_hist(DigitFn digit, int64_t n, uint32_t *__restrict__ hist,
+                                                              int64_t ntiles) {
+    __shared__ uint32_t h[RADIX_THREADS / 32][RADIX_BINS];
+    const unsigned w = threadIdx.x >> 5;
+    for (int i = threadIdx.x; i < (RADIX_THREADS / 32) * RADIX_BINS; i += RADIX_THREADS) (&h[0][0])[i] = 0;
+    __syncthreads();
+    const int64_t base = (int64_t)blockIdx.x * RADIX_TILE + w * (RADIX_TILE / 8);
+#pragma unroll 4
+    for (int it = 0; it < RADIX_ITEMS; ++it) {
+        const int64_t i = base + it * 32 + lane_id();
+        const unsigned d = i < n ? digit(i) : (unsigned)RADIX_BINS;
+        if (d < RADIX_BINS) atomicAdd(&h[w][d], 1u);
+    }
+    __syncthreads();
+    for (int d = threadIdx.x; d < RADIX_BINS; d += RADIX_THREADS) {
+        uint32_t s = 0;
+#pragma unroll
+        for (int q = 0; q < RADIX_THREADS / 32; ++q) s += h[q][d];
+        hist[(int64_t)d * ntiles + blockIdx.x] = s;
+    }
+}
+
+template <typename DigitFn, typename Epi>
+__global__ void __launch_bounds__(RADIX_THREADS) k_digit_rank(DigitFn digit, int64_t n,
+                                                              const uint32_t *__restrict__ offs, int64_t ntiles,
+                                                              Epi epi) {
+    __shared__ uint32_t wcnt[(RADIX_THREADS / 32) * RADIX_BINS];
+    __shared__ uint32_t gbase[RADIX_BINS];
+    const unsigned w = threadIdx.x >> 5, lane = lane_id();
+    for (int i = threadIdx.x; i < (RADIX_THREADS / 32) * RADIX_BINS; i += RADIX_THREADS) wcnt[i] = 0;
+    __syncthreads();
+    const int64_t base = (int64_t)blockIdx.x * RADIX_TILE + w * (RADIX_TILE / 8);
+    unsigned dig[RADIX_ITEMS];
+    uint32_t rank[RADIX_ITEMS];
+    const unsigned lt = lanemask_lt();
+#pragma unroll
+    for (int it = 0; it < RADIX_ITEMS; ++it) {
+        const int64_t i = base + it * 32 + lane;
+        const unsigned d = i < n ? digit(i) : (unsigned)RADIX_BINS;
+        const unsigned peers = __match_any_sync(0xffffffffu, d);
+        const unsigned before = d < RADIX_BINS ? wcnt[w * RADIX_BINS + d] : 0u;
+        __syncwarp();
+        if (d < RADIX_BINS && (peers & lt) == 0) wcnt[w * RADIX_BINS + d] = before + __popc(peers);
+        __syncwarp();
+        rank[it] = before + __popc(peers & lt);
+        dig[it] = d;
+    }
+    __syncthreads();
+    // RADIX_THREADS == RADIX_BINS: thread d turns digit d's per-warp counts
+    // into exclusive prefixes and fetches the digit's global start
+    {
+        const unsigned d = threadIdx.x;
+        uint32_t s = 0;
+#pragma unroll
+        for (int q = 0; q < RADIX_THREADS / 32; ++q) {
+            const uint32_t x = wcnt[q * RADIX_BINS + d];
+            wcnt[q * RADIX_BINS + d] = s;
+            s += x;
+        }
+        gbase[d] = offs[(int64_t)d * ntiles + blockIdx.x];
+    }
+    __syncthreads();
+    unsigned bits = 0;
+#pragma unroll
+    for (int it = 0; it < RADIX_ITEMS; ++it) {
+        const int64_t i = base + it * 32 + lane;
+        if (dig[it] < RADIX_BINS) bits |= epi(i, gbase[dig[it]] + wcnt[w * RADIX_BINS + dig[it]] + rank[it]);
+    }
+    epi.done(bits);
+}
+
+template <typename DigitFn>
+void digit_offsets(Ctx &c, DigitFn digit, int64_t n, uint32_t *hist, uint32_t *partials) {
+    if (n <= 0) return;
+    const int64_t ntiles = (n + RADIX_TILE - 1) / RADIX_TILE;
+    launch(c, "digit_hist", k_digit_hist<DigitFn>, dim3((unsigned)ntiles), dim3(RADIX_THREADS), 0, digit, n, hist,
+           ntiles);
+    scan_exclusive_u32(c, hist, hist, ntiles * RADIX_BINS, partials, nullptr);
+}
+
+template <typename DigitFn, typename Epi>
+void digit_rank(Ctx &c, const char *name, DigitFn digit, int64_t n, const uint32_t *hist, Epi epi) {
+    if (n <= 0) return;
+    const int64_t ntiles = (n + RADIX_TILE - 1) / RADIX_TILE;
+    launch(c, name, k_digit_rank<DigitFn, Epi>, dim3((unsigned)ntiles), dim3(RADIX_THREADS), 0, digit, n, hist,
+           ntiles, epi);
+}
 
 // Number of bits needed to represent v (0 for v == 0).
 inline int bits_for(uint64_t v) {
