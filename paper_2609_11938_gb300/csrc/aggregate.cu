@@ -358,18 +358,23 @@ __global__ void k_agg_fill(const int32_t *__restrict__ rok, const uint32_t *__re
     const unsigned lane = lane_id();
     const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / 32;
     const int64_t nwarps = (int64_t)gridDim.x * blockDim.x / 32;
+    // op id of a kernel's range, or none
+    auto key_of = [&](int32_t r) -> unsigned {
+        if (r < 0 || r >= R) return 0xFFFFFFFFu;
+        const uint32_t op = r_op[r];
+        return (int64_t)op < n_ops ? op : 0xFFFFFFFFu;
+    };
     for (int64_t k0 = warp * run; k0 < K; k0 += nwarps * run) {
         const int64_t k1 = k0 + run < K ? k0 + run : K;
-        int32_t r_next = k0 + lane < k1 ? rok[k0 + lane] : -1;
+        // ranges loaded two groups ahead, op ids one group ahead, so each
+        // step waits only on its own atomic
+        unsigned key_next = key_of(k0 + lane < k1 ? rok[k0 + lane] : -1);
+        int32_t r_next = k0 + 32 + lane < k1 ? rok[k0 + 32 + lane] : -1;
         for (int64_t kb = k0; kb < k1; kb += 32) {
             const int64_t k = kb + lane;
-            const int32_t r = r_next;
-            r_next = k + 32 < k1 ? rok[k + 32] : -1;           // the next group's ranges, loaded early
-            unsigned key = 0xFFFFFFFFu;
-            if (r >= 0 && r < R) {
-                const uint32_t op = r_op[r];
-                if ((int64_t)op < n_ops) key = op;
-            }
+            const unsigned key = key_next;
+            key_next = key_of(r_next);
+            r_next = k + 64 < k1 ? rok[k + 64] : -1;
             const unsigned peers = __match_any_sync(0xffffffffu, key);
             const int leader = __ffs(peers) - 1;
             unsigned base = 0;
