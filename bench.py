@@ -87,6 +87,42 @@ def recorded_traffic(kernel, workload, kernels):
     return None
 
 
+def recorded_tiers(trace, seed, share=0.5):
+    """The trace with the maps the attribution tiers read, as a capture would
+    record them (the benchmark's input; parity tests use tracegen.with_tiers).
+    Correlation map: for a random half of the launches the entry (name, number
+    of earlier launches of that name in time order, operator), the operator
+    being the last operator range pushed on the launch's stream before it
+    started (the dispatch that launched it), or a random one for launches
+    outside every range; entries in random order.  Fusion map as in
+    tracegen.with_tiers."""
+    import dataclasses
+
+    import numpy as np
+
+    import tracegen
+    rng = np.random.default_rng(seed)
+    t = tracegen.with_tiers(trace, seed=seed, p_corr=0.0, p_stray=0.0)
+    K = trace.K
+    order = np.lexsort((np.arange(K), trace.k_stream.astype(np.int64), trace.k_start))
+    names = trace.k_name[order].astype(np.int64)
+    by_name = np.argsort(names, kind="stable")
+    first = np.searchsorted(names[by_name], names[by_name], side="left")
+    inv = np.empty(K, np.int64)
+    inv[order[by_name]] = np.arange(K) - first
+    op = rng.integers(0, max(int(trace.n_ops), 1), K)
+    is_op = trace.r_op < trace.n_ops
+    for s in np.unique(trace.k_stream):
+        rs = np.nonzero((trace.r_stream == s) & is_op)[0]
+        rs = rs[np.argsort(trace.r_start[rs], kind="stable")]
+        ks = np.nonzero(trace.k_stream == s)[0]
+        p = np.searchsorted(trace.r_start[rs], trace.k_start[ks], side="right") - 1
+        op[ks[p >= 0]] = trace.r_op[rs[p[p >= 0]]]
+    pick = rng.permutation(np.nonzero(rng.random(K) < share)[0])
+    return dataclasses.replace(t, corr_name=trace.k_name[pick].astype(np.uint32),
+                               corr_inv=inv[pick].astype(np.uint32), corr_op=op[pick].astype(np.uint32))
+
+
 def load_peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -224,6 +260,9 @@ def main():
     ap.add_argument("--oracle-kernels", type=int, default=1_000_000)
     ap.add_argument("--per-stream-ncu", action="store_true",
                     help="ncu rows as per-stream replay runs, matched per (name, stream)")
+    ap.add_argument("--tiers", action="store_true",
+                    help="attribution tiers of Fig. 2 in the step: a correlation map recorded for half of the "
+                         "launches, fusion entries for a tenth of the names, aggregation by each kernel's operator")
     ap.add_argument("--launch-lag", type=int, default=0,
                     help="enclosure queries at start - U[0, LAG) ns (host launch times)")
     ap.add_argument("--kernels", type=int, default=0,
@@ -290,6 +329,8 @@ def main():
     trace = tracegen.generate(cfg, shuffle=args.shuffle)
     if args.per_stream_ncu:
         trace = tracegen.per_stream_runs(trace)
+    if args.tiers:
+        trace = recorded_tiers(trace, seed=cfg["seed"])
     K, R, M, O = trace.K, trace.R, trace.M, trace.n_ops
     use_dedup = bool(cfg.get("dedup")) and trace.k_layer is not None
     tr = opa.to_device(trace, dev)
@@ -305,6 +346,22 @@ def main():
     idx = torch.empty(K, dtype=torch.int32, device=f"cuda:{dev}")
     kind = torch.empty(K, dtype=torch.uint8, device=f"cuda:{dev}")
     ops = ctx.alloc_ops(O)
+    tiers_out = None
+    if args.tiers:
+        tiers_out = dict(op=torch.empty(K, dtype=torch.int32, device=f"cuda:{dev}"),
+                         tier=torch.empty(K, dtype=torch.uint8, device=f"cuda:{dev}"),
+                         fused_with=torch.empty(K, dtype=torch.int32, device=f"cuda:{dev}"),
+                         is_fused=torch.empty(K, dtype=torch.uint8, device=f"cuda:{dev}"))
+
+    def join():
+        ctx.enclose(tq, rk, nop)
+        if tiers_out is not None:
+            ctx.attribute(tr, rk, nop, out=tiers_out)
+        ctx.match(tr, dedup=use_dedup, out_idx=idx, out_kind=kind)
+        if tiers_out is not None:
+            ctx.aggregate(tr, None, idx, ops, op_of_kernel=tiers_out["op"])
+        else:
+            ctx.aggregate(tr, rk, idx, ops)
     in_bytes = sum(x.numel() * x.element_size() for x in (tr.k_stream, tr.k_start, tr.k_dur, tr.k_name,
                                                            tr.r_stream, tr.r_start, tr.r_end, tr.r_depth, tr.r_op,
                                                            tr.ncu_name, tr.counters))
@@ -316,9 +373,7 @@ def main():
         if flush is not None:
             with torch.cuda.stream(stream):
                 flush.fill_(1.0)
-        ctx.enclose(tq, rk, nop)
-        ctx.match(tr, dedup=use_dedup, out_idx=idx, out_kind=kind)
-        ctx.aggregate(tr, rk, idx, ops)
+        join()
 
     def sync():
         stream.synchronize()
@@ -355,7 +410,8 @@ def main():
     # H2D of every input array, the three calls, D2H of every output
     host = {name: torch.from_numpy(getattr(trace, name)).pin_memory()
             for name in ("k_stream", "k_start", "k_dur", "k_name", "r_stream", "r_start", "r_end", "r_depth",
-                         "r_op", "ncu_name", "counters")}
+                         "r_op", "ncu_name", "counters") + (("corr_name", "corr_inv", "corr_op", "fusion_op",
+                                                             "fusion_len") if args.tiers else ())}
     if trace.k_layer is not None:
         host["k_layer"] = torch.from_numpy(trace.k_layer).pin_memory()
     if tq is not tr:
@@ -374,9 +430,7 @@ def main():
                 getattr(tr, name).copy_(v, non_blocking=True)
             if tq is not tr:
                 tq.k_start.copy_(launch_host, non_blocking=True)
-        ctx.enclose(tq, rk, nop)
-        ctx.match(tr, dedup=use_dedup, out_idx=idx, out_kind=kind)
-        ctx.aggregate(tr, rk, idx, ops)
+        join()
         with torch.cuda.stream(stream):
             out_host["rk"].copy_(rk, non_blocking=True)
             out_host["idx"].copy_(idx, non_blocking=True)
@@ -423,7 +477,7 @@ def main():
         "config": {"workload": f"{args.config}: {WORKLOADS[args.config]}" + (
                        f" [scaled to {K} kernels]" if args.kernels else ""), "kernels": K, "ranges": R,
                    "ncu_rows": M, "ops": O, "shuffled": bool(args.shuffle), "per_stream_ncu": bool(args.per_stream_ncu),
-                   "launch_lag_ns": args.launch_lag, "parallelism": f"replicas x{world}",
+                   "launch_lag_ns": args.launch_lag, "tiers": bool(args.tiers), "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2 (129 MB)" if flush is None else "L2 flushed before every step"},
         "roofline": {"bound": "hbm", "kernel": dname, "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": (achieved / peak) if achieved else None, "peak_kind": f"{peak_kind} copy bandwidth",

@@ -2,7 +2,8 @@
  * opattr.h -- C ABI of the GPU trace join behind hardware-attributed operator
  * profiling ("Hardware-Attributed Operator Profiling for PyTorch").
  *
- * The join has three calls, in this order:
+ * The join has three calls, in this order (a fourth, opattr_attribute,
+ * applies the attribution tiers of Fig. 2 between the first and the last):
  *   opattr_enclose   -- Algorithm 2 (Sec. 3.5): each kernel record gets the
  *                       innermost enclosing operator range on its stream.
  *   opattr_match     -- Algorithm 1 (Sec. 3.3): the i-th launch of a kernel
@@ -177,7 +178,7 @@ typedef struct {
 /* Host-side totals of opattr_aggregate (Fig. 3 coverage). */
 typedef struct {
     int64_t total_ns;              /* sum of all kernel durations */
-    int64_t attributed_ns;         /* kernels with range_of_kernel >= 0 */
+    int64_t attributed_ns;         /* attributed kernels: range_of_kernel >= 0, or an operator */
     int64_t unattributed_ns;       /* total_ns - attributed_ns */
     int64_t kernels;
     int64_t attributed_kernels;
@@ -185,6 +186,65 @@ typedef struct {
     double attributed_frac;        /* attributed_ns / total_ns, NaN if total_ns == 0 */
     double unattributed_frac;
 } opattr_totals;
+
+/* ---- Attribution tiers (Fig. 2, Sec. 3.4, Sec. 3.6) ----
+ * Each kernel goes to the first tier that has an operator for it:
+ *   HIGH      the torch.profiler correlation map (Sec. 3.4): an entry for the
+ *             kernel's (name, invocation index), where the invocation index
+ *             is the kernel's rank among all kernels of its name in time
+ *             order (0 = first launch);
+ *   NVTX      the innermost enclosing operator range (opattr_enclose);
+ *   INDUCTOR  the Inductor fusion map (Sec. 3.6): an operator for the
+ *             kernel's name;
+ * and is unattributed otherwise.  The fusion map also enriches kernels of
+ * the first two tiers: fused_with names the fused list's operator, and a
+ * kernel is marked fused when its list holds several operators (or, for the
+ * NVTX tier, when the walk collected several operator ranges). */
+#define OPATTR_OP_NONE 0xFFFFFFFFu        /* no operator (same value as OPATTR_OP_STRUCTURAL) */
+typedef enum {
+    OPATTR_TIER_NONE = 0,
+    OPATTR_TIER_HIGH = 1,
+    OPATTR_TIER_NVTX = 2,
+    OPATTR_TIER_INDUCTOR = 3
+} opattr_tier;
+
+/* torch.profiler correlation map (Phase 1 of the capture), device arrays in
+ * any order:
+ *   name_id     u32[n]  kernel-name id
+ *   invocation  u32[n]  invocation index of that name
+ *   op_id       u32[n]  operator the launch belongs to, < n_ops
+ * A (name, invocation) pair that names an existing launch must appear once;
+ * entries that name no launch (unknown name, index past the name's launch
+ * count) are ignored. */
+typedef struct {
+    const uint32_t *name_id;
+    const uint32_t *invocation;
+    const uint32_t *op_id;
+    int64_t n;
+} opattr_corr;
+
+/* Inductor fusion map (Sec. 3.6), device arrays indexed by kernel-name id:
+ *   op_of_name  u32[n_names]  operator standing for the name's fused
+ *                             operator list (< n_ops), or OPATTR_OP_NONE
+ *   list_len    u8[n_names]   operators in that list (the "Original ATen"
+ *                             comment), or NULL for 1
+ * Names >= n_names have no entry. */
+typedef struct {
+    const uint32_t *op_of_name;
+    const uint8_t *list_len;
+    int64_t n_names;
+} opattr_fusion;
+
+/* Host-side result of opattr_attribute. */
+typedef struct {
+    int64_t kernels;
+    int64_t high;                  /* kernels per tier */
+    int64_t nvtx;
+    int64_t inductor;
+    int64_t none;
+    int64_t fused;                 /* kernels marked fused */
+    int64_t corr_used;             /* correlation entries that named a launch */
+} opattr_attr_summary;
 
 /* Create a context on `device` that orders its work on `cuda_stream` (a
  * cudaStream_t; NULL = the legacy default stream).  `cfg` may be NULL for
@@ -240,20 +300,51 @@ opattr_status opattr_match(opattr_ctx *ctx, const opattr_kernels *kernels, const
  * empty set or a zero total weight.  Floating-point results are within 1e-9
  * relative of an fp64 evaluation (float-float accumulation, see the design
  * notes).  Every op id in [0, n_ops) is written.
- * Reads kernels->dur_ns (and start_ns, stream for the fast path), range
- * start_ns and op_id, ncu->counters.
- *   range_of_kernel    i32[kernels->n]  device, values in [-1, ranges->n)
+ * Reads kernels->dur_ns, ranges->op_id, ncu->counters.
+ *   range_of_kernel    i32[kernels->n]  device, values in [-1, ranges->n);
+ *                                       or NULL: then ranges->op_id holds
+ *                                       one operator per kernel
+ *                                       (ranges->n == kernels->n), and
+ *                                       OPATTR_OP_NONE marks unattributed
+ *                                       kernels (opattr_attribute's output)
  *   ncu_idx_of_kernel  i32[kernels->n]  device, values in [-1, ncu->n)
  *   dev_out            host struct of device pointers, see above
  *   host_totals        host, may be NULL
  * Errors: OPATTR_E_INVALID_ARG (index out of range, attributed range that is
- * not an operator below n_ops, negative duration, infinite counter, counters
- * not 16-byte aligned),
+ * not an operator below n_ops, an operator >= n_ops other than
+ * OPATTR_OP_NONE, negative duration, infinite counter, counters not 16-byte
+ * aligned),
  * OPATTR_E_OOM, OPATTR_E_CUDA. */
 opattr_status opattr_aggregate(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,
                                const int32_t *range_of_kernel, const opattr_ncu *ncu,
                                const int32_t *ncu_idx_of_kernel, uint32_t n_ops,
                                const opattr_op_aggregates *dev_out, opattr_totals *host_totals);
+
+/* The attribution tiers of Fig. 2 for every kernel (see above).
+ *   range_of_kernel  i32[kernels->n]  device, opattr_enclose's result
+ *   n_op_enclosing   u8[kernels->n]   device, opattr_enclose's count, or NULL
+ *   corr             host struct of device arrays, or NULL (no HIGH tier)
+ *   fusion           host struct of device arrays, or NULL (no INDUCTOR tier)
+ *   op_of_kernel     u32[kernels->n]  device, required: the kernel's operator
+ *                                     or OPATTR_OP_NONE
+ *   tier             u8[kernels->n]   device, may be NULL: opattr_tier
+ *   fused_with       u32[kernels->n]  device, may be NULL: the fusion map's
+ *                                     operator for the kernel's name, or
+ *                                     OPATTR_OP_NONE
+ *   is_fused         u8[kernels->n]   device, may be NULL: 1 if the kernel's
+ *                                     fused list has several operators, or
+ *                                     (NVTX tier) n_op_enclosing > 1
+ *   host_summary     host, may be NULL
+ * Reads kernels->stream, start_ns, name_id and ranges->op_id.  op_of_kernel
+ * feeds opattr_aggregate with range_of_kernel NULL.
+ * Errors: OPATTR_E_INVALID_ARG (range index out of [-1, ranges->n), an NVTX
+ * range that is not an operator below n_ops, a correlation or fusion
+ * operator >= n_ops, a repeated (name, invocation) pair that names a
+ * launch), OPATTR_E_OOM, OPATTR_E_CUDA. */
+opattr_status opattr_attribute(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,
+                               const int32_t *range_of_kernel, const uint8_t *n_op_enclosing, const opattr_corr *corr,
+                               const opattr_fusion *fusion, uint32_t n_ops, uint32_t *op_of_kernel, uint8_t *tier,
+                               uint32_t *fused_with, uint8_t *is_fused, opattr_attr_summary *host_summary);
 
 /* Free the context and its scratch.  NULL is ignored. */
 void opattr_destroy(opattr_ctx *ctx);

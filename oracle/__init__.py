@@ -64,6 +64,8 @@ def _lib():
                                       i32, vp, ctypes.c_int, vp, vp, vp]
             lib.orc_aggregate.argtypes = [i64, vp, vp, i64, vp, i64, vp, vp, i64, vp, vp, vp, vp, vp, vp]
             lib.orc_agg_rule.argtypes = [ctypes.c_int]
+            lib.orc_attribute.argtypes = [ctypes.c_int, i64, vp, vp, vp, vp, vp, i64, vp, ctypes.c_uint32, i64, vp,
+                                          vp, vp, i64, vp, vp, vp, vp, vp, vp, vp]
             _lib_handle = lib
         return _lib_handle
 
@@ -81,7 +83,7 @@ class use_library:
         self._saved = _lib_handle
         lib = ctypes.CDLL(self.path)
         for name in ("orc_validate_ranges_brute", "orc_validate_ranges_indexed", "orc_enclose", "orc_match",
-                     "orc_aggregate", "orc_agg_rule"):
+                     "orc_aggregate", "orc_agg_rule", "orc_attribute"):
             getattr(lib, name).argtypes = getattr(self._saved, name).argtypes
         _lib_handle = lib
         return self
@@ -184,6 +186,71 @@ def aggregate(k_dur, range_of_kernel, r_op, counters, ncu_idx, n_ops: int):
                   kernels=int(tot[3]), attributed_kernels=int(tot[4]), matched_kernels=int(tot[5]),
                   attributed_frac=float(fr[0]), unattributed_frac=float(fr[1]))
     return st, ops, totals
+
+
+OP_NONE = 0xFFFFFFFF
+TIER_NONE, TIER_HIGH, TIER_NVTX, TIER_INDUCTOR = 0, 1, 2, 3
+ATTR_SUMMARY_FIELDS = ("kernels", "high", "nvtx", "inductor", "none", "fused", "corr_used")
+
+
+def attribute(k_stream, k_start, k_name, range_of_kernel, n_op_enclosing, r_op, n_ops: int, corr=None, fusion=None,
+              brute: bool = False):
+    """The attribution tiers of Fig. 2.  corr = (name, invocation, op) arrays
+    of the torch.profiler correlation map or None; fusion = (op_of_name,
+    list_len or None) of the Inductor fusion map or None.
+    Returns (status, op_of_kernel u32[K], tier u8[K], fused_with u32[K],
+    is_fused u8[K], summary dict)."""
+    lib = _lib()
+    ks, kt, kn = _c(k_stream, np.uint8), _c(k_start, np.int64), _c(k_name, np.uint32)
+    rk, ro = _c(range_of_kernel, np.int32), _c(r_op, np.uint32)
+    nop = _c(n_op_enclosing, np.uint8)
+    K = len(kt)
+    cn = ci = co = None
+    if corr is not None:
+        cn, ci, co = (_c(a, np.uint32) for a in corr)
+    fo = fl = None
+    if fusion is not None:
+        fo = _c(fusion[0], np.uint32)
+        fl = _c(fusion[1], np.uint8) if fusion[1] is not None else None
+    NC = 0 if cn is None else len(cn)
+    NF = 0 if fo is None else len(fo)
+    op = np.full(K, OP_NONE, np.uint32)
+    tier = np.zeros(K, np.uint8)
+    fw = np.full(K, OP_NONE, np.uint32)
+    fz = np.zeros(K, np.uint8)
+    summ = np.zeros(len(ATTR_SUMMARY_FIELDS), np.int64)
+    st = lib.orc_attribute(int(brute), K, _p(ks), _p(kt), _p(kn), _p(rk), _p(nop), len(ro), _p(ro),
+                           ctypes.c_uint32(n_ops), NC, _p(cn), _p(ci), _p(co), NF, _p(fo), _p(fl), _p(op), _p(tier),
+                           _p(fw), _p(fz), _p(summ))
+    return st, op, tier, fw, fz, dict(zip(ATTR_SUMMARY_FIELDS, (int(x) for x in summ)))
+
+
+def aggregate_by_op(k_dur, op_of_kernel, counters, ncu_idx, n_ops: int):
+    """aggregate() with each kernel's operator given directly (OP_NONE =
+    unattributed): every kernel with an operator is its own one-kernel "range"."""
+    op = _c(op_of_kernel, np.uint32)
+    rk = np.where(op != OP_NONE, np.arange(len(op)), -1).astype(np.int32)
+    return aggregate(k_dur, rk, op, counters, ncu_idx, n_ops)
+
+
+def run_tiers(trace, mode: str = "skip_name", enclose_mode: str = "indexed", dedup: bool | None = None,
+              brute: bool = False, use_corr: bool = True, use_fusion: bool = True):
+    """The join with the attribution tiers: enclose, attribute, match, aggregate by operator."""
+    st_e, rk, nop = enclose(trace.k_stream, trace.k_start, trace.r_stream, trace.r_start, trace.r_end,
+                            trace.r_depth, trace.r_op, mode=enclose_mode)
+    corr = (trace.corr_name, trace.corr_inv, trace.corr_op) if use_corr and trace.corr_name is not None else None
+    fusion = (trace.fusion_op, trace.fusion_len) if use_fusion and trace.fusion_op is not None else None
+    st_t, op, tier, fw, fz, tsum = attribute(trace.k_stream, trace.k_start, trace.k_name, rk, nop, trace.r_op,
+                                             trace.n_ops, corr, fusion, brute=brute)
+    if dedup is None:
+        dedup = bool(trace.config.get("dedup")) and trace.k_layer is not None
+    st_m, idx, kind, summ = match(trace.k_stream, trace.k_start, trace.k_name, trace.ncu_name, trace.k_layer,
+                                  trace.class_of_layer, trace.rep_of_class, mode=mode, dedup=dedup,
+                                  ncu_stream=getattr(trace, "ncu_stream", None))
+    st_a, ops, totals = aggregate_by_op(trace.k_dur, op, trace.counters, idx, trace.n_ops)
+    return dict(enclose_status=st_e, range_of_kernel=rk, n_op_enclosing=nop, attribute_status=st_t,
+                op_of_kernel=op, tier=tier, fused_with=fw, is_fused=fz, tier_summary=tsum, match_status=st_m,
+                ncu_idx=idx, match_kind=kind, summary=summ, aggregate_status=st_a, ops=ops, totals=totals)
 
 
 def run(trace, mode: str = "skip_name", enclose_mode: str = "indexed", dedup: bool | None = None):

@@ -569,3 +569,122 @@ int orc_aggregate(int64_t K, const int64_t *k_dur, const int32_t *range_of_kerne
     free(num); free(den); free(mx); free(seen);
     return ORC_OK;
 }
+
+/* ------------------------------------------------------------------ attribution tiers
+ * Fig. 2, tried per kernel in this order:
+ *   HIGH      the torch.profiler correlation map (Sec. 3.4) holds an entry for
+ *             the kernel's (name, invocation index); the invocation index is
+ *             the number of earlier kernels (time order) with the same name;
+ *   NVTX      the kernel has an enclosing operator range (Algorithm 2's
+ *             result, range_of_kernel >= 0);
+ *   INDUCTOR  the Inductor fusion map (Sec. 3.6) names an operator for the
+ *             kernel's name;
+ *   otherwise the kernel is unattributed.
+ * The fusion map enriches every tier: fused_with = the name's fusion
+ * operator; is_fused = its operator list is longer than one, or (NVTX tier)
+ * the walk collected more than one operator range.
+ * A map entry that names a launch must be the only entry for that pair; map
+ * entries naming no launch are ignored.
+ * brute: invocation indices by rescanning every earlier kernel, map lookups
+ * by scanning the whole map; otherwise per-name counters and a sorted map.
+ * summary: [0] kernels [1] high [2] nvtx [3] inductor [4] none [5] fused
+ *          [6] map entries that named a launch */
+#define ATTR_SUMMARY_N 7
+#define OP_NONE 0xFFFFFFFFu
+enum { TIER_NONE = 0, TIER_HIGH = 1, TIER_NVTX = 2, TIER_INDUCTOR = 3 };
+
+typedef struct { const uint32_t *name, *inv; } corrkey_t;
+static int cmp_corr(int64_t a, int64_t b, const void *ctx) {
+    const corrkey_t *c = (const corrkey_t *)ctx;
+    if (c->name[a] != c->name[b]) return c->name[a] < c->name[b] ? -1 : 1;
+    if (c->inv[a] != c->inv[b]) return c->inv[a] < c->inv[b] ? -1 : 1;
+    return 0;
+}
+
+int orc_attribute(int brute, int64_t K, const uint8_t *k_stream, const int64_t *k_start, const uint32_t *k_name,
+                  const int32_t *rok, const uint8_t *nop, int64_t R, const uint32_t *r_op, uint32_t n_ops,
+                  int64_t NM, const uint32_t *c_name, const uint32_t *c_inv, const uint32_t *c_op, int64_t NF,
+                  const uint32_t *f_op, const uint8_t *f_len, uint32_t *op_of_kernel, uint8_t *tier,
+                  uint32_t *fused_with, uint8_t *is_fused, int64_t *summary) {
+    memset(summary, 0, sizeof(int64_t) * ATTR_SUMMARY_N);
+    summary[0] = K;
+    for (int64_t k = 0; k < K; ++k) {
+        if (rok[k] < -1 || rok[k] >= R) return ORC_E_INVALID_ARG;
+        if (rok[k] >= 0 && r_op[rok[k]] >= n_ops) return ORC_E_INVALID_ARG;
+    }
+    for (int64_t e = 0; e < NM; ++e) if (c_op[e] >= n_ops) return ORC_E_INVALID_ARG;
+    for (int64_t n = 0; n < NF; ++n) if (f_op[n] != OP_NONE && f_op[n] >= n_ops) return ORC_E_INVALID_ARG;
+
+    int st = ORC_OK;
+    int64_t *order = (int64_t *)malloc(sizeof(int64_t) * (K ? K : 1));
+    uint32_t *inv = (uint32_t *)malloc(sizeof(uint32_t) * (K ? K : 1));
+    int64_t *cix = (int64_t *)malloc(sizeof(int64_t) * (NM ? NM : 1));
+    int64_t *cnt = NULL;
+    dict_t D = { NULL, 0 };
+    if (!order || !inv || !cix) { st = ORC_E_OOM; goto done; }
+    for (int64_t k = 0; k < K; ++k) order[k] = k;
+    korder_t ko = { k_start, k_stream };
+    if ((st = stable_sort_idx(order, K, cmp_time, &ko))) goto done;
+
+    /* invocation index of every kernel */
+    if (brute) {
+        for (int64_t a = 0; a < K; ++a) {
+            uint32_t c = 0;
+            for (int64_t b = 0; b < a; ++b) c += k_name[order[b]] == k_name[order[a]];
+            inv[order[a]] = c;
+        }
+    } else {
+        if ((st = dict_build(&D, k_name, K, k_name, 0))) goto done;
+        cnt = (int64_t *)calloc(D.n ? D.n : 1, sizeof(int64_t));
+        if (!cnt) { st = ORC_E_OOM; goto done; }
+        for (int64_t a = 0; a < K; ++a) {
+            int64_t k = order[a];
+            inv[k] = (uint32_t)cnt[dict_find(&D, k_name[k])]++;
+        }
+    }
+    /* the map, sorted by (name, invocation) unless scanned whole */
+    for (int64_t e = 0; e < NM; ++e) cix[e] = e;
+    corrkey_t ck = { c_name, c_inv };
+    if (!brute && (st = stable_sort_idx(cix, NM, cmp_corr, &ck))) goto done;
+
+    for (int64_t k = 0; k < K; ++k) {
+        /* HIGH: entries for (name, invocation index) */
+        int64_t hits = 0, hit = -1;
+        if (brute) {
+            for (int64_t e = 0; e < NM; ++e)
+                if (c_name[e] == k_name[k] && c_inv[e] == inv[k]) { hits++; hit = e; }
+        } else {
+            int64_t lo = 0, hi = NM;          /* first entry >= (name, inv) */
+            while (lo < hi) {
+                int64_t m = lo + (hi - lo) / 2, e = cix[m];
+                if (c_name[e] < k_name[k] || (c_name[e] == k_name[k] && c_inv[e] < inv[k])) lo = m + 1; else hi = m;
+            }
+            for (int64_t m = lo; m < NM && c_name[cix[m]] == k_name[k] && c_inv[cix[m]] == inv[k]; ++m) {
+                hits++;
+                hit = cix[m];
+            }
+        }
+        if (hits > 1) { st = ORC_E_INVALID_ARG; goto done; }
+        summary[6] += hits;
+        const uint32_t fo = (int64_t)k_name[k] < NF ? f_op[k_name[k]] : OP_NONE;
+        const unsigned fl = ((int64_t)k_name[k] < NF && f_len) ? f_len[k_name[k]] : 1u;
+        uint32_t op = OP_NONE;
+        uint8_t t = TIER_NONE;
+        if (hits == 1) { op = c_op[hit]; t = TIER_HIGH; }
+        else if (rok[k] >= 0) { op = r_op[rok[k]]; t = TIER_NVTX; }
+        else if (fo != OP_NONE) { op = fo; t = TIER_INDUCTOR; }
+        const int fused = (fo != OP_NONE && fl > 1) || (t == TIER_NVTX && nop && nop[k] > 1);
+        op_of_kernel[k] = op;
+        tier[k] = t;
+        fused_with[k] = fo;
+        is_fused[k] = (uint8_t)fused;
+        summary[1] += t == TIER_HIGH;
+        summary[2] += t == TIER_NVTX;
+        summary[3] += t == TIER_INDUCTOR;
+        summary[4] += t == TIER_NONE;
+        summary[5] += fused;
+    }
+done:
+    free(order); free(inv); free(cix); free(cnt); free(D.name);
+    return st;
+}

@@ -33,6 +33,8 @@ E_CUDA, E_OOM, E_TIMEOUT, E_STATE = -5, -6, -7, -8
 OP_STRUCTURAL = 0xFFFFFFFF
 OP_NONOP = 0xFFFFFFFE
 N_COUNTERS = 20
+OP_NONE = 0xFFFFFFFF
+TIER_NONE, TIER_HIGH, TIER_NVTX, TIER_INDUCTOR = 0, 1, 2, 3
 MATCH_NOALLOC_MAX = 65536
 MISMATCH = {"skip_name": 0, "prefix": 1, "error": 2}
 
@@ -72,6 +74,21 @@ class MatchSummary(ctypes.Structure):
         return {f: int(getattr(self, f)) for f, _ in self._fields_ if f != "reserved"}
 
 
+class Corr(ctypes.Structure):
+    _fields_ = [("name_id", _vp), ("invocation", _vp), ("op_id", _vp), ("n", ctypes.c_int64)]
+
+
+class Fusion(ctypes.Structure):
+    _fields_ = [("op_of_name", _vp), ("list_len", _vp), ("n_names", ctypes.c_int64)]
+
+
+class AttrSummary(ctypes.Structure):
+    _fields_ = [(f, ctypes.c_int64) for f in ("kernels", "high", "nvtx", "inductor", "none", "fused", "corr_used")]
+
+    def as_dict(self) -> dict:
+        return {f: int(getattr(self, f)) for f, _ in self._fields_}
+
+
 class OpAggregates(ctypes.Structure):
     _fields_ = [("kernel_count", _vp), ("total_duration_ns", _vp), ("matched_count", _vp), ("agg", _vp)]
 
@@ -109,6 +126,8 @@ def library():
             lib.opattr_match.argtypes = [_vp, P(Kernels), P(Ncu), P(Dedup), _vp, _vp, P(MatchSummary)]
             lib.opattr_aggregate.argtypes = [_vp, P(Kernels), P(Ranges), _vp, P(Ncu), _vp, ctypes.c_uint32,
                                              P(OpAggregates), P(Totals)]
+            lib.opattr_attribute.argtypes = [_vp, P(Kernels), P(Ranges), _vp, _vp, P(Corr), P(Fusion),
+                                             ctypes.c_uint32, _vp, _vp, _vp, _vp, P(AttrSummary)]
             lib.opattr_destroy.argtypes = [_vp]
             lib.opattr_destroy.restype = None
             lib.opattr_status_string.argtypes = [ctypes.c_int]
@@ -122,8 +141,8 @@ def library():
             lib.opattr_launch_count.restype = ctypes.c_int64
             lib.opattr_match_noalloc.argtypes = [P(Kernels), P(Ncu), ctypes.c_int, _vp, _vp, P(MatchSummary), _vp]
             lib.opattr_match_noalloc.restype = ctypes.c_int
-            for f in ("opattr_create", "opattr_enclose", "opattr_match", "opattr_aggregate", "opattr_set_timing",
-                      "opattr_timing_report"):
+            for f in ("opattr_create", "opattr_enclose", "opattr_match", "opattr_aggregate", "opattr_attribute",
+                      "opattr_set_timing", "opattr_timing_report"):
                 getattr(lib, f).restype = ctypes.c_int
             _lib = lib
         return _lib
@@ -166,6 +185,16 @@ def opattr_aggregate(handle, kernels: Kernels, ranges: Ranges, rok_ptr: int, ncu
     return library().opattr_aggregate(handle, ctypes.byref(kernels), ctypes.byref(ranges), _vp(rok_ptr),
                                       ctypes.byref(ncu), _vp(idx_ptr), ctypes.c_uint32(n_ops), ctypes.byref(out),
                                       ctypes.byref(totals))
+
+
+def opattr_attribute(handle, kernels: Kernels, ranges: Ranges, rok_ptr: int, nop_ptr: int | None,
+                     corr: Corr | None, fusion: Fusion | None, n_ops: int, op_ptr: int, tier_ptr: int | None,
+                     fused_with_ptr: int | None, is_fused_ptr: int | None, summary: AttrSummary) -> int:
+    return library().opattr_attribute(handle, ctypes.byref(kernels), ctypes.byref(ranges), _vp(rok_ptr),
+                                      _vp(nop_ptr or 0), ctypes.byref(corr) if corr is not None else None,
+                                      ctypes.byref(fusion) if fusion is not None else None, ctypes.c_uint32(n_ops),
+                                      _vp(op_ptr), _vp(tier_ptr or 0), _vp(fused_with_ptr or 0),
+                                      _vp(is_fused_ptr or 0), ctypes.byref(summary))
 
 
 def opattr_match_noalloc(kernels: Kernels, ncu: Ncu, mismatch: str, idx_ptr: int, kind_ptr: int | None,
@@ -216,6 +245,11 @@ class DeviceTrace:
     class_of_layer: object = None   # host (numpy / list) tables
     rep_of_class: object = None
     ncu_stream: object = None       # stream of each ncu row (per-stream replay runs), or None
+    corr_name: object = None        # torch.profiler correlation map (HIGH tier), or None
+    corr_inv: object = None
+    corr_op: object = None
+    fusion_op: object = None        # Inductor fusion map per name id (INDUCTOR tier), or None
+    fusion_len: object = None
 
     @property
     def K(self):
@@ -245,7 +279,9 @@ def to_device(trace, device: int = 0, pin: bool = False) -> DeviceTrace:
     return DeviceTrace(d(trace.k_stream), d(trace.k_start), d(trace.k_dur), d(trace.k_name), d(trace.k_layer),
                        d(trace.r_stream), d(trace.r_start), d(trace.r_end), d(trace.r_depth), d(trace.r_op),
                        int(trace.n_ops), d(trace.ncu_name), d(trace.counters), trace.class_of_layer,
-                       trace.rep_of_class, d(getattr(trace, "ncu_stream", None)))
+                       trace.rep_of_class, d(getattr(trace, "ncu_stream", None)), d(getattr(trace, "corr_name", None)),
+                       d(getattr(trace, "corr_inv", None)), d(getattr(trace, "corr_op", None)),
+                       d(getattr(trace, "fusion_op", None)), d(getattr(trace, "fusion_len", None)))
 
 
 class Context:
@@ -348,7 +384,39 @@ class Context:
                     matched_count=torch.empty(n_ops, dtype=torch.int64, device=dev),
                     agg=torch.empty((N_COUNTERS, n_ops), dtype=torch.float64, device=dev))
 
-    def aggregate(self, tr: DeviceTrace, range_of_kernel, ncu_idx, ops=None):
+    def attribute(self, tr: DeviceTrace, range_of_kernel, n_op_enclosing=None, use_corr: bool = True,
+                  use_fusion: bool = True, out=None):
+        """The attribution tiers of Fig. 2: returns (status, op_of_kernel, tier, fused_with, is_fused, summary)."""
+        import torch
+        dv = self.device
+        dev = f"cuda:{dv}"
+        if out is None:
+            out = dict(op=torch.empty(tr.K, dtype=torch.int32, device=dev),
+                       tier=torch.empty(tr.K, dtype=torch.uint8, device=dev),
+                       fused_with=torch.empty(tr.K, dtype=torch.int32, device=dev),
+                       is_fused=torch.empty(tr.K, dtype=torch.uint8, device=dev))
+        corr = fusion = None
+        if use_corr and tr.corr_name is not None:
+            corr = Corr(_ptr(tr.corr_name, torch.uint32, "corr_name", dv), _ptr(tr.corr_inv, torch.uint32, "corr_inv", dv),
+                        _ptr(tr.corr_op, torch.uint32, "corr_op", dv), int(tr.corr_name.shape[0]))
+        if use_fusion and tr.fusion_op is not None:
+            fusion = Fusion(_ptr(tr.fusion_op, torch.uint32, "fusion_op", dv),
+                            _ptr(tr.fusion_len, torch.uint8, "fusion_len", dv), int(tr.fusion_op.shape[0]))
+        summ = AttrSummary()
+        st = opattr_attribute(self.handle, self.kernels(tr), self.ranges(tr),
+                              _ptr(range_of_kernel, torch.int32, "range_of_kernel", dv),
+                              _ptr(n_op_enclosing, torch.uint8, "n_op_enclosing", dv) if n_op_enclosing is not None
+                              else None, corr, fusion, tr.n_ops, _ptr(out["op"], torch.uint32, "op_of_kernel", dv),
+                              _ptr(out["tier"], torch.uint8, "tier", dv),
+                              _ptr(out["fused_with"], torch.uint32, "fused_with", dv),
+                              _ptr(out["is_fused"], torch.uint8, "is_fused", dv), summ)
+        if st < 0:
+            raise OpattrError(st, "opattr_attribute")
+        return st, out["op"], out["tier"], out["fused_with"], out["is_fused"], summ.as_dict()
+
+    def aggregate(self, tr: DeviceTrace, range_of_kernel, ncu_idx, ops=None, op_of_kernel=None):
+        """Eq. (1) per operator.  With op_of_kernel (opattr_attribute's output)
+        in place of range_of_kernel, each kernel's operator is taken from it."""
         import torch
         if ops is None:
             ops = self.alloc_ops(tr.n_ops)
@@ -358,8 +426,13 @@ class Context:
                            _ptr(ops["matched_count"], torch.int64, "matched_count", dv),
                            _ptr(ops["agg"], torch.float64, "agg", dv))
         tot = Totals()
-        st = opattr_aggregate(self.handle, self.kernels(tr), self.ranges(tr),
-                              _ptr(range_of_kernel, torch.int32, "range_of_kernel", dv), self.ncu(tr),
+        if op_of_kernel is not None:
+            rng = Ranges(None, None, None, None, _ptr(op_of_kernel, torch.uint32, "op_of_kernel", dv), tr.K)
+            rok_ptr = None
+        else:
+            rng = self.ranges(tr)
+            rok_ptr = _ptr(range_of_kernel, torch.int32, "range_of_kernel", dv)
+        st = opattr_aggregate(self.handle, self.kernels(tr), rng, rok_ptr, self.ncu(tr),
                               _ptr(ncu_idx, torch.int32, "ncu_idx_of_kernel", dv), tr.n_ops, out, tot)
         if st < 0:
             raise OpattrError(st, "opattr_aggregate")

@@ -286,6 +286,12 @@ struct AccF {
     }
 };
 
+// The range of kernel k; without range_of_kernel, r_op holds one operator
+// per kernel and the kernel is its own "range" when it has one.
+__device__ __forceinline__ int32_t range_of(const int32_t *rok, const uint32_t *r_op, int64_t k) {
+    return rok ? rok[k] : (r_op[k] != OPATTR_OP_NONE ? (int32_t)k : -1);
+}
+
 // ------------------------------------------------------------------ count
 // Per kernel: duration >= 0, range index in [-1, R), an attributed range is an
 // operator below n_ops, row index in [-1, M).  Totals: all / attributed time,
@@ -307,7 +313,7 @@ __global__ void k_agg_count(const int64_t *__restrict__ dur, const int32_t *__re
             const int64_t k = k0 + u * stride;
             const bool in = k < K;
             d[u] = in ? dur[k] : 0;
-            r[u] = in ? rok[k] : -1;
+            r[u] = in ? range_of(rok, r_op, k) : -1;
             j[u] = in ? nidx[k] : -1;
         }
 #pragma unroll
@@ -368,13 +374,13 @@ __global__ void k_agg_fill(const int32_t *__restrict__ rok, const uint32_t *__re
         const int64_t k1 = k0 + run < K ? k0 + run : K;
         // ranges loaded two groups ahead, op ids one group ahead, so each
         // step waits only on its own atomic
-        unsigned key_next = key_of(k0 + lane < k1 ? rok[k0 + lane] : -1);
-        int32_t r_next = k0 + 32 + lane < k1 ? rok[k0 + 32 + lane] : -1;
+        unsigned key_next = key_of(k0 + lane < k1 ? range_of(rok, r_op, k0 + lane) : -1);
+        int32_t r_next = k0 + 32 + lane < k1 ? range_of(rok, r_op, k0 + 32 + lane) : -1;
         for (int64_t kb = k0; kb < k1; kb += 32) {
             const int64_t k = kb + lane;
             const unsigned key = key_next;
             key_next = key_of(r_next);
-            r_next = k + 64 < k1 ? rok[k + 64] : -1;
+            r_next = k + 64 < k1 ? range_of(rok, r_op, k + 64) : -1;
             const unsigned peers = __match_any_sync(0xffffffffu, key);
             const int leader = __ffs(peers) - 1;
             unsigned base = 0;
@@ -395,6 +401,10 @@ constexpr int SL_THREADS = 256;
 constexpr int SL_SMEM = 8192;
 constexpr uint32_t AG_SHORT_MAX = 64;           // segments up to this length: sorted by one warp; longer: one block
 
+constexpr uint32_t AG_HUGE = 256;               // longer segments: split into pieces over several warps
+constexpr uint32_t AG_PIECE = 1024;              // kernels of a huge op per warp of the pieces pass
+
+// Ops with segments longer than `limit`, listed (in no particular order).
 __global__ void k_agg_long_list(const uint32_t *__restrict__ off, int64_t n_ops, uint32_t limit,
                                 uint32_t *__restrict__ longs, unsigned *__restrict__ nlong) {
     for (int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o - threadIdx.x < n_ops;
@@ -571,6 +581,7 @@ __global__ void __launch_bounds__(AG_THREADS) k_agg_ops(const uint32_t *__restri
             const int64_t o = o0 + order[i];
             const uint32_t s0 = off[o], len = off[o + 1] - s0;
             uint32_t *seg = list + s0;
+            if (len > AG_HUGE) continue;                 // a huge op: k_agg_long_ops writes it
             if (len <= AG_SHORT_MAX) {                   // ascending unless the fill met the op in two runs
                 bool up = true;
                 for (uint32_t t = 1; t < len; ++t) up &= seg[t - 1] < seg[t];
@@ -629,6 +640,150 @@ __global__ void __launch_bounds__(AG_THREADS) k_agg_ops(const uint32_t *__restri
 }
 
 // ------------------------------------------------------------------ host
+// ------------------------------------------------------------------ long ops
+// Ops whose segments are longer than AG_HUGE (listed by k_agg_long_list,
+// sorted by k_agg_sort_long) are split into pieces of AG_PIECE kernels, so an
+// operator with a very long segment (an Inductor fusion-map operator gathers
+// every unattributed launch of its kernel name) is spread over many warps
+// instead of holding one thread for its whole length.  Each lane adds a
+// contiguous run of a piece in ascending kernel index with the careful
+// accumulator; partials are combined by fixed trees of pairwise float-float
+// additions (lane l takes lane l + 16, then l + 8, ...; a piece's partials in
+// piece order), so results are reproducible, with an error bound of the
+// longest run plus the pairwise steps.
+__device__ __forceinline__ ff ff_pair_add(ff a, ff b) {
+    const ff t = two_sum(a.hi, b.hi);
+    return ff{t.hi, __fadd_rn(t.lo, __fadd_rn(a.lo, b.lo))};
+}
+__device__ __forceinline__ ff shfl_down_ff(ff v, int d) {
+    return ff{__shfl_down_sync(0xffffffffu, v.hi, d), __shfl_down_sync(0xffffffffu, v.lo, d)};
+}
+__device__ __forceinline__ void acc_merge_down(Acc &a, int d) {
+    const bool take = (int)lane_id() < d;
+    const int kc = __shfl_down_sync(0xffffffffu, a.kc, d), mc = __shfl_down_sync(0xffffffffu, a.mc, d);
+    const long long ds = __shfl_down_sync(0xffffffffu, a.dsum, d), da = __shfl_down_sync(0xffffffffu, a.dall, d);
+    const unsigned seen = __shfl_down_sync(0xffffffffu, a.seen, d);
+    const int bad = __shfl_down_sync(0xffffffffu, a.bad, d);
+    if (take) {
+        a.kc += kc; a.mc += mc; a.dsum += ds; a.dall += da; a.seen |= seen; a.bad |= bad;
+    }
+#pragma unroll
+    for (int i = 0; i < N_SUM; ++i) {
+        const ff x = shfl_down_ff(a.s[i], d);
+        if (take) a.s[i] = ff_pair_add(a.s[i], x);
+    }
+#pragma unroll
+    for (int i = 0; i < N_DW; ++i) {
+        const ff x = shfl_down_ff(a.w[i], d);
+        const long long nw = __shfl_down_sync(0xffffffffu, a.nanw[i], d);
+        if (take) {
+            a.w[i] = ff_pair_add(a.w[i], x);
+            a.nanw[i] += nw;
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < N_MAX; ++i) {
+        const float x = __shfl_down_sync(0xffffffffu, a.mx[i], d);
+        if (take) a.mx[i] = fmaxf(a.mx[i], x);
+    }
+}
+// a += b, the same pairwise steps as acc_merge_down
+__device__ __forceinline__ void acc_merge(Acc &a, const Acc &b) {
+    a.kc += b.kc; a.mc += b.mc; a.dsum += b.dsum; a.dall += b.dall; a.seen |= b.seen; a.bad |= b.bad;
+#pragma unroll
+    for (int i = 0; i < N_SUM; ++i) a.s[i] = ff_pair_add(a.s[i], b.s[i]);
+#pragma unroll
+    for (int i = 0; i < N_DW; ++i) {
+        a.w[i] = ff_pair_add(a.w[i], b.w[i]);
+        a.nanw[i] += b.nanw[i];
+    }
+#pragma unroll
+    for (int i = 0; i < N_MAX; ++i) a.mx[i] = fmaxf(a.mx[i], b.mx[i]);
+}
+
+// Piece offsets of the listed long ops, one block: poff[j] = pieces of the
+// ops listed before j (an op longer than AG_HUGE has ceil(len / AG_PIECE)
+// pieces, a shorter one none); poff[nlong] = all pieces.
+__global__ void __launch_bounds__(1024) k_agg_piece_offsets(const uint32_t *__restrict__ off,
+                                                            const uint32_t *__restrict__ longs,
+                                                            const unsigned *__restrict__ nlong,
+                                                            uint32_t *__restrict__ poff) {
+    __shared__ uint32_t wbuf[33];
+    const int64_t n = *nlong;
+    uint32_t carry = 0;
+    for (int64_t b = 0; b < n; b += 1024) {
+        const int64_t j = b + threadIdx.x;
+        uint32_t np = 0;
+        if (j < n) {
+            const uint32_t o = longs[j], len = off[o + 1] - off[o];
+            np = len > AG_HUGE ? (len + AG_PIECE - 1) / AG_PIECE : 0u;
+        }
+        uint32_t tot;
+        const uint32_t ex = block_exclusive_scan<uint32_t>(np, wbuf, &tot);
+        if (j < n) poff[j] = carry + ex;
+        carry += tot;
+    }
+    if (threadIdx.x == 0) poff[n] = carry;
+}
+
+// Pieces: one warp per AG_PIECE kernels of a huge op (lane l adds AG_PIECE /
+// 32 consecutive kernels), the warp's 32 partials merged by the fixed tree,
+// the piece's partial stored at its index.
+__global__ void k_agg_pieces(const uint32_t *__restrict__ off, const uint32_t *__restrict__ list,
+                             const uint32_t *__restrict__ longs, const unsigned *__restrict__ nlong,
+                             const uint32_t *__restrict__ poff, AggIn A, Acc *__restrict__ part) {
+    const int64_t n = *nlong;
+    const int64_t P = poff[n];
+    const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const unsigned lane = lane_id();
+    for (int64_t p = warp; p < P; p += nwarps) {
+        int64_t lo = 0, hi = n;                   // the listed op: last j with poff[j] <= p
+        while (hi - lo > 1) {
+            const int64_t m = (lo + hi) >> 1;
+            if ((int64_t)poff[m] <= p) lo = m; else hi = m;
+        }
+        const uint32_t o = longs[lo];
+        const uint32_t s0 = off[o], len = off[o + 1] - s0;
+        const uint32_t b0 = (uint32_t)(p - poff[lo]) * AG_PIECE;
+        const uint32_t b1 = b0 + AG_PIECE < len ? b0 + AG_PIECE : len;
+        const uint32_t per = AG_PIECE / 32;
+        const uint32_t l0 = min(b0 + lane * per, b1), l1 = min(l0 + per, b1);
+        Acc acc;
+        acc.init();
+        for (uint32_t t = l0; t < l1; ++t) acc.add(A, list[s0 + t]);
+#pragma unroll 1
+        for (int d = 16; d > 0; d >>= 1) acc_merge_down(acc, d);
+        if (lane == 0) part[p] = acc;
+    }
+}
+
+// Finish: one warp per huge op merges its pieces' partials (lane l takes
+// pieces l, l + 32, ... in order, then the fixed tree) and writes the record.
+__global__ void k_agg_long_ops(const uint32_t *__restrict__ longs, const unsigned *__restrict__ nlong,
+                               const uint32_t *__restrict__ poff, const Acc *__restrict__ part, AggIn A,
+                               DevStatus *st) {
+    const int64_t n = *nlong;
+    const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+    const unsigned lane = lane_id();
+    int bad = 0;
+    for (int64_t q = warp; q < n; q += nwarps) {
+        if (poff[q + 1] == poff[q]) continue;   // not huge: the ops pass writes it
+        const uint32_t o = longs[q];
+        Acc acc;
+        acc.init();
+        for (uint32_t p = poff[q] + lane; p < poff[q + 1]; p += 32) acc_merge(acc, part[p]);
+#pragma unroll 1
+        for (int d = 16; d > 0; d >>= 1) acc_merge_down(acc, d);
+        if (lane == 0) {
+            acc.write(A, o);
+            bad |= acc.bad;
+        }
+    }
+    if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_err(st, ERR_INVALID);
+}
+
 // Blocks of the ops pass: what stays resident, fewer for few ops.
 static unsigned ops_grid(Ctx &c, int64_t O) {
     int sms = 0, per_sm = 0;
@@ -646,7 +801,8 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     const int64_t K = kern->n, R = rng->n, M = ncu->n, O = n_ops;
     if (K < 0 || R < 0 || M < 0 || K >= (1ll << 31) || R >= (1ll << 31) || M >= (1ll << 31) || !out)
         return OPATTR_E_INVALID_ARG;
-    if (K > 0 && (!kern->dur_ns || !rok || !nidx)) return OPATTR_E_INVALID_ARG;
+    if (K > 0 && (!kern->dur_ns || !nidx)) return OPATTR_E_INVALID_ARG;
+    if (K > 0 && !rok && R != K) return OPATTR_E_INVALID_ARG;     // one operator per kernel in rng->op_id
     if (R > 0 && !rng->op_id) return OPATTR_E_INVALID_ARG;
     if (M > 0 && !ncu->counters) return OPATTR_E_INVALID_ARG;
     if (O > 0 && (!out->kernel_count || !out->total_duration_ns || !out->matched_count || !out->agg))
@@ -656,6 +812,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     Need nd;
     nd.add<uint32_t>(O + 1).add<uint32_t>(O + 1).add<uint32_t>(O + 1).add<uint32_t>(K).add<uint32_t>(K);
     nd.add<uint32_t>(O + 1).add<unsigned>(1).add<unsigned>(1);
+    nd.add<uint32_t>(O + 1).add<Acc>(K / AG_PIECE + (K / (AG_SHORT_MAX + 1)) + 1);   // pieces per op, partials
     nd.add<uint32_t>(scan_scratch_elems(O + 1));
     opattr_status st = ensure_arena(c, nd.bytes + 4096);
     if (st) return st;
@@ -665,6 +822,9 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     uint32_t *list = a.take<uint32_t>(K), *tmp = a.take<uint32_t>(K), *longs = a.take<uint32_t>(O + 1);
     unsigned *nlong = a.take<unsigned>(1);
     unsigned *ctr = a.take<unsigned>(1);
+    uint32_t *npc = a.take<uint32_t>(O + 1);
+    Acc *partials = a.take<Acc>(K / AG_PIECE + (K / (AG_SHORT_MAX + 1)) + 1);
+    if (!npc || !partials) return OPATTR_E_OOM;
     cudaMemsetAsync(ctr, 0, sizeof(unsigned), c.stream);
     uint32_t *part = a.take<uint32_t>(scan_scratch_elems(O + 1));
     if (!cnt || !off || !cur || !list || !tmp || !longs || !nlong || !part) return OPATTR_E_OOM;
@@ -693,12 +853,19 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
             launch(c, "agg_fill", k_agg_fill, dim3(grid_for(K, 256 / 32 * run, 65535)), dim3(256), 0, rok,
                    rng->op_id, K, R, O, (const uint32_t *)off, cur, list, run);
         }
-        launch(c, "agg_long_list", k_agg_long_list, dim3(grid_for(O, 256, 4096)), dim3(256), 0, (const uint32_t *)off,
-               O, AG_SHORT_MAX, longs, nlong);
+        launch(c, "agg_long_list", k_agg_long_list, dim3(grid_for(O, 256, 4096)), dim3(256), 0,
+               (const uint32_t *)off, O, AG_SHORT_MAX, longs, nlong);
+        launch(c, "agg_piece_offsets", k_agg_piece_offsets, dim3(1), dim3(1024), 0, (const uint32_t *)off,
+               (const uint32_t *)longs, (const unsigned *)nlong, npc);
         int sms = 0;
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
         launch(c, "agg_sort_long", k_agg_sort_long, dim3(2 * std::max(1, sms)), dim3(SL_THREADS), 0, (const uint32_t *)off,
                (const uint32_t *)longs, (const unsigned *)nlong, list, tmp);
+        launch(c, "agg_pieces", k_agg_pieces, dim3(4 * std::max(1, sms)), dim3(256), 0, (const uint32_t *)off,
+               (const uint32_t *)list, (const uint32_t *)longs, (const unsigned *)nlong, (const uint32_t *)npc, in,
+               partials);
+        launch(c, "agg_long_ops", k_agg_long_ops, dim3(std::max(1, sms)), dim3(256), 0, (const uint32_t *)longs,
+               (const unsigned *)nlong, (const uint32_t *)npc, (const Acc *)partials, in, c.d_status);
         launch(c, "agg_ops", k_agg_ops, dim3(ops_grid(c, O)), dim3(AG_THREADS), 0,
                (const uint32_t *)off, list, in, c.d_status);
     }

@@ -1,5 +1,5 @@
 // api.cu -- the C ABI of libopattr: context life cycle, scratch arena, status
-// block, launch timing, and the three calls of the join.
+// block, launch timing, and the calls of the join.
 #include <stdlib.h>
 
 #include <algorithm>
@@ -16,6 +16,11 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
 opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_ranges *rng, const int32_t *rok,
                            const opattr_ncu *ncu, const int32_t *nidx, uint32_t n_ops,
                            const opattr_op_aggregates *out, opattr_totals *tot_out);
+
+opattr_status do_attribute(Ctx &c, const opattr_kernels *kern, const opattr_ranges *rng, const int32_t *rok,
+                           const uint8_t *nop, const opattr_corr *corr, const opattr_fusion *fusion,
+                           uint32_t n_ops, uint32_t *op_of_kernel, uint8_t *tier, uint32_t *fused_with,
+                           uint8_t *is_fused, opattr_attr_summary *sum);
 
 opattr_status cuda_status(Ctx &c, cudaError_t e) {
     if (e == cudaSuccess) e = c.last_error;
@@ -214,6 +219,19 @@ opattr_status opattr_aggregate(opattr_ctx *ctx, const opattr_kernels *kernels, c
     if (!g.ok) return OPATTR_E_CUDA;
     return finish(c, do_aggregate(c, kernels, ranges, range_of_kernel, ncu, ncu_idx_of_kernel, n_ops, dev_out,
                                   host_totals));
+}
+
+opattr_status opattr_attribute(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,
+                               const int32_t *range_of_kernel, const uint8_t *n_op_enclosing, const opattr_corr *corr,
+                               const opattr_fusion *fusion, uint32_t n_ops, uint32_t *op_of_kernel, uint8_t *tier,
+                               uint32_t *fused_with, uint8_t *is_fused, opattr_attr_summary *host_summary) {
+    if (!ctx || !kernels || !ranges) return OPATTR_E_INVALID_ARG;
+    Ctx &c = ctx->c;
+    if (c.broken) return OPATTR_E_STATE;
+    DeviceGuard g(c.device);
+    if (!g.ok) return OPATTR_E_CUDA;
+    return finish(c, do_attribute(c, kernels, ranges, range_of_kernel, n_op_enclosing, corr, fusion, n_ops,
+                                  op_of_kernel, tier, fused_with, is_fused, host_summary));
 }
 
 void opattr_destroy(opattr_ctx *ctx) {

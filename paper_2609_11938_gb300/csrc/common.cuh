@@ -46,7 +46,12 @@ enum CountSlot {
     C_MATCHED_K,
     C_AGG_SEEN,
     C_UNMATCHED,
-    C_NSLOTS = 16
+    C_TIER_HIGH,
+    C_TIER_NVTX,
+    C_TIER_INDUCTOR,
+    C_FUSED,
+    C_CORR_USED,
+    C_NSLOTS = 24
 };
 enum MinMaxSlot { MM_KSTART_MIN = 0, MM_KSTART_MAX, MM_RSTART_MIN, MM_REND_MAX, MM_NSLOTS = 8 };
 

@@ -32,6 +32,43 @@ def gpu_run(trace, mode: str = "skip_name", dedup: bool | None = None, ctx=None)
             ctx.close()
 
 
+def gpu_run_tiers(trace, mode: str = "skip_name", dedup: bool | None = None, use_corr: bool = True,
+                  use_fusion: bool = True, ctx=None):
+    """enclose, attribute (Fig. 2 tiers), match, aggregate by operator on the GPU."""
+    import torch
+
+    import paper_2609_11938_gb300 as opa
+    own = ctx is None
+    if own:
+        ctx = opa.Context(0, mismatch=mode)
+    try:
+        tr = opa.to_device(trace)
+        if dedup is None:
+            dedup = bool(trace.config.get("dedup")) and trace.k_layer is not None
+        st_e, rk, nop = ctx.enclose(tr)
+        st_t, op, tier, fw, fz, tsum = ctx.attribute(tr, rk, nop, use_corr=use_corr, use_fusion=use_fusion)
+        st_m, idx, kind, summ = ctx.match(tr, dedup=dedup)
+        st_a, ops, tot = ctx.aggregate(tr, None, idx, op_of_kernel=op)
+        torch.cuda.synchronize()
+        u32 = lambda x: x.cpu().numpy().view(np.uint32)
+        return dict(enclose_status=st_e, range_of_kernel=rk.cpu().numpy(), n_op_enclosing=nop.cpu().numpy(),
+                    attribute_status=st_t, op_of_kernel=u32(op), tier=tier.cpu().numpy(), fused_with=u32(fw),
+                    is_fused=fz.cpu().numpy(), tier_summary=tsum, match_status=st_m, ncu_idx=idx.cpu().numpy(),
+                    match_kind=kind.cpu().numpy(), summary=summ, aggregate_status=st_a,
+                    ops={k: v.cpu().numpy() for k, v in ops.items()}, totals=tot)
+    finally:
+        if own:
+            ctx.close()
+
+
+def assert_parity_tiers(g, o):
+    assert g["attribute_status"] == o["attribute_status"]
+    for k in ("op_of_kernel", "tier", "fused_with", "is_fused"):
+        np.testing.assert_array_equal(g[k], o[k], err_msg=k)
+    assert g["tier_summary"] == o["tier_summary"], (g["tier_summary"], o["tier_summary"])
+    assert_parity(g, o)
+
+
 def assert_close(got, want, rtol=RTOL, what=""):
     got = np.asarray(got, np.float64)
     want = np.asarray(want, np.float64)

@@ -42,6 +42,9 @@ def test_struct_layouts_match_header():
     assert ctypes.sizeof(opa.MatchSummary) == 8 * 8 + 2 * 4
     assert ctypes.sizeof(opa.OpAggregates) == 4 * 8
     assert ctypes.sizeof(opa.Totals) == 6 * 8 + 2 * 8
+    assert ctypes.sizeof(opa.Corr) == 4 * 8
+    assert ctypes.sizeof(opa.Fusion) == 3 * 8
+    assert ctypes.sizeof(opa.AttrSummary) == 7 * 8
 
 
 def test_status_strings_without_gpu():

@@ -9,7 +9,7 @@ import pytest
 
 import oracle
 import tracegen
-from gpu_util import RTOL, assert_close, assert_parity, gpu_run
+from gpu_util import RTOL, assert_close, assert_parity, assert_parity_tiers, gpu_run, gpu_run_tiers
 
 pytestmark = pytest.mark.gpu
 GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
@@ -279,7 +279,7 @@ def test_aggregate_segment_lengths(opa, nan_frac):
     """Ops whose kernels are walked by selection (<= 48), after an in-place
     sort (49 .. 16384) and in list order (above), with kernels scattered over
     the array, duplicate op ids and null counters: against the oracle."""
-    seg_lens = [1, 2, 48, 49, 300, 5000, 16384, 16385, 40000]
+    seg_lens = [1, 2, 48, 49, 64, 65, 100, 256, 257, 300, 1024, 1025, 5000, 16384, 16385, 40000]
     t, rk, idx = _agg_inputs(7, 200_000, seg_lens, 20_000, nan_frac)
     o = oracle.aggregate(t.k_dur, rk, t.r_op, t.counters, idx, t.n_ops)
     _check_aggregate(_gpu_aggregate(opa, t, rk, idx), o)
@@ -437,3 +437,72 @@ def test_launch_time_query(opa):
         np.testing.assert_array_equal(ops[k].cpu().numpy(), o[1][k])
     assert_close(ops["agg"].cpu().numpy(), o[1]["agg"], what="agg")
     ctx.close()
+
+
+# ---------------------------------------------------------------- attribution tiers (Fig. 2)
+
+def test_tiers_worked(opa):
+    """The hand-derived tiers example (tests/golden/tiers.json) through the C ABI."""
+    import torch
+    g = json.load(open(os.path.join(GOLDEN, "tiers.json")))
+    k = g["kernels"]
+    dev = "cuda:0"
+    t = lambda a, dt: torch.tensor(np.array(a, dt), device=dev)
+    K = len(k["start"])
+    tr = opa.DeviceTrace(t(k["stream"], np.uint8), t(k["start"], np.int64), t([1] * K, np.int64),
+                         t(k["name"], np.int32), None, None, t([0] * 3, np.int64), t([0] * 3, np.int64), None,
+                         t(g["r_op"], np.int32), g["n_ops"], t([], np.int32), None,
+                         corr_name=t(g["corr"]["name"], np.int32), corr_inv=t(g["corr"]["invocation"], np.int32),
+                         corr_op=t(g["corr"]["op"], np.int32),
+                         fusion_op=t(np.array(g["fusion"]["op_of_name"], np.uint32).view(np.int32), np.int32),
+                         fusion_len=t(g["fusion"]["list_len"], np.uint8))
+    ctx = opa.Context(0)
+    st, op, tier, fw, fz, summ = ctx.attribute(tr, t(k["range_of_kernel"], np.int32), t(k["n_op_enclosing"], np.uint8))
+    e = g["expect"]
+    assert st == 0
+    assert op.cpu().numpy().view(np.uint32).tolist() == e["op_of_kernel"]
+    assert tier.cpu().numpy().tolist() == e["tier"]
+    assert fw.cpu().numpy().view(np.uint32).tolist() == e["fused_with"]
+    assert fz.cpu().numpy().tolist() == e["is_fused"]
+    assert summ == e["summary"]
+    # a repeated pair that names a launch is rejected; the context stays usable
+    tr.corr_name = t(g["corr"]["name"] + [1], np.int32)
+    tr.corr_inv = t(g["corr"]["invocation"] + [2], np.int32)
+    tr.corr_op = t(g["corr"]["op"] + [3], np.int32)
+    with pytest.raises(opa.OpattrError) as ei:
+        ctx.attribute(tr, t(k["range_of_kernel"], np.int32), t(k["n_op_enclosing"], np.uint8))
+    assert ei.value.status == opa.E_INVALID_ARG
+    tr.corr_op = t(g["corr"]["op"] + [g["n_ops"]], np.int32)
+    tr.corr_name = t(g["corr"]["name"] + [1], np.int32)
+    tr.corr_inv = t(g["corr"]["invocation"] + [7], np.int32)       # names no launch, but its operator is invalid
+    with pytest.raises(opa.OpattrError) as ei:
+        ctx.attribute(tr, t(k["range_of_kernel"], np.int32), t(k["n_op_enclosing"], np.uint8))
+    assert ei.value.status == opa.E_INVALID_ARG
+    ctx.close()
+
+
+@pytest.mark.parametrize("name,shuffle,p_corr", [("tiny", False, 0.5), ("gpt2", False, 0.5), ("gpt2", True, 0.5),
+                                                ("gpt2_dedup", False, 1.0), ("dedup", False, 0.3),
+                                                ("dedup", True, 0.0)])
+def test_tiers_configs(opa, name, shuffle, p_corr):
+    """The tiers on the generator's configurations (kernels in and out of time
+    order), against the oracle on every output, aggregation by operator included."""
+    t = tracegen.with_tiers(tracegen.generate(name, shuffle=shuffle), p_corr=p_corr)
+    assert_parity_tiers(gpu_run_tiers(t), oracle.run_tiers(t))
+
+
+@pytest.mark.parametrize("seed", range(0, 80, 3))
+def test_tiers_small_random(opa, seed):
+    t = tracegen.small_random(seed, n_streams=1 + seed % 4, n_events=10 + (seed * 7) % 90, max_depth=1 + seed % 7,
+                              n_names=2 + seed % 5)
+    u = tracegen.with_tiers(t, seed=seed, p_corr=[0.0, 0.3, 0.7, 1.0][seed % 4], p_fused=[0.0, 0.4, 1.0][seed % 3])
+    use_corr, use_fusion = seed % 5 != 1, seed % 7 != 2
+    assert_parity_tiers(gpu_run_tiers(u, use_corr=use_corr, use_fusion=use_fusion),
+                        oracle.run_tiers(u, use_corr=use_corr, use_fusion=use_fusion, enclose_mode="brute", brute=True))
+
+
+def test_tiers_large(opa):
+    """The 20 M-kernel trace with a correlation map for half of the launches and
+    fusion entries for a tenth of the names, against the indexed oracle."""
+    t = tracegen.with_tiers(tracegen.generate("large"))
+    assert_parity_tiers(gpu_run_tiers(t), oracle.run_tiers(t))

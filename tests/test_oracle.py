@@ -431,6 +431,99 @@ def test_config_invariants(name):
         assert res["summary"]["replayed"] == t.M
 
 
+# ---------------------------------------------------------------- attribution tiers (Fig. 2)
+
+def _tiers_args(g):
+    k = g["kernels"]
+    kern = (np.array(k["stream"], np.uint8), np.array(k["start"], np.int64), np.array(k["name"], np.uint32),
+            np.array(k["range_of_kernel"], np.int32), np.array(k["n_op_enclosing"], np.uint8))
+    corr = tuple(np.array(g["corr"][f], np.uint32) for f in ("name", "invocation", "op"))
+    fusion = (np.array(g["fusion"]["op_of_name"], np.uint32), np.array(g["fusion"]["list_len"], np.uint8))
+    return kern, np.array(g["r_op"], np.uint32), g["n_ops"], corr, fusion
+
+
+@pytest.mark.parametrize("brute", [True, False])
+def test_tiers_worked(golden, brute):
+    g = golden("tiers.json")
+    (ks, kt, kn, rk, nop), r_op, n_ops, corr, fusion = _tiers_args(g)
+    st, op, tier, fw, fz, summ = oracle.attribute(ks, kt, kn, rk, nop, r_op, n_ops, corr, fusion, brute=brute)
+    e = g["expect"]
+    assert st == oracle.OK
+    assert op.tolist() == e["op_of_kernel"]
+    assert tier.tolist() == e["tier"]
+    assert fw.tolist() == e["fused_with"]
+    assert fz.tolist() == e["is_fused"]
+    assert summ == e["summary"]
+
+
+def test_tiers_rejects(golden):
+    g = golden("tiers.json")
+    (ks, kt, kn, rk, nop), r_op, n_ops, corr, fusion = _tiers_args(g)
+    # a repeated pair that names a launch (B, 2 -> k6)
+    dup = tuple(np.append(a, v).astype(np.uint32) for a, v in zip(corr, (1, 2, 3)))
+    assert oracle.attribute(ks, kt, kn, rk, nop, r_op, n_ops, dup, fusion)[0] == oracle.E_INVALID_ARG
+    big = (corr[0], corr[1], np.where(np.arange(len(corr[2])) == 4, n_ops, corr[2]).astype(np.uint32))
+    assert oracle.attribute(ks, kt, kn, rk, nop, r_op, n_ops, big, fusion)[0] == oracle.E_INVALID_ARG
+    fbig = (np.array([n_ops, 15, 16, 16], np.uint32), fusion[1])
+    assert oracle.attribute(ks, kt, kn, rk, nop, r_op, n_ops, corr, fbig)[0] == oracle.E_INVALID_ARG
+    rbad = rk.copy(); rbad[1] = len(r_op)
+    assert oracle.attribute(ks, kt, kn, rbad, nop, r_op, n_ops, corr, fusion)[0] == oracle.E_INVALID_ARG
+    nonop = np.array([10, oracle.NONOP, 12], np.uint32)                 # an attributed range must be an operator
+    assert oracle.attribute(ks, kt, kn, rk, nop, nonop, n_ops, corr, fusion)[0] == oracle.E_INVALID_ARG
+
+
+@pytest.mark.parametrize("seed", range(0, 60, 4))
+def test_tiers_brute_vs_indexed(seed):
+    # invocation indices by rescanning every earlier kernel and map lookups by
+    # scanning the whole map, against per-name counters and the sorted map
+    t = tracegen.small_random(seed, n_streams=1 + seed % 4, n_events=10 + (seed * 7) % 90, max_depth=1 + seed % 7,
+                              n_names=2 + seed % 5)
+    u = tracegen.with_tiers(t, seed=seed, p_corr=[0.0, 0.3, 0.7, 1.0][seed % 4], p_fused=0.4)
+    a = oracle.run_tiers(u, enclose_mode="brute", brute=True)
+    b = oracle.run_tiers(u, enclose_mode="indexed", brute=False)
+    assert a["attribute_status"] == b["attribute_status"] == oracle.OK
+    for k in ("op_of_kernel", "tier", "fused_with", "is_fused"):
+        assert np.array_equal(a[k], b[k]), k
+    assert a["tier_summary"] == b["tier_summary"]
+
+
+@pytest.mark.parametrize("name", ["tiny", "gpt2", "dedup"])
+def test_tiers_reduce_to_enclosure(name):
+    # without either map every kernel takes its enclosing operator (NVTX) or
+    # none, and aggregating by operator equals aggregating by range
+    t = tracegen.generate(name)
+    r = oracle.run(t)
+    q = oracle.run_tiers(t, use_corr=False, use_fusion=False)
+    rk = r["range_of_kernel"]
+    want = np.where(rk >= 0, t.r_op[np.maximum(rk, 0)], oracle.OP_NONE).astype(np.uint32)
+    assert np.array_equal(q["op_of_kernel"], want)
+    assert np.array_equal(q["tier"], np.where(rk >= 0, oracle.TIER_NVTX, oracle.TIER_NONE))
+    assert np.array_equal(q["is_fused"], (r["n_op_enclosing"] > 1).astype(np.uint8))
+    for k in ("kernel_count", "total_duration_ns", "matched_count"):
+        assert np.array_equal(q["ops"][k], r["ops"][k])
+    assert np.array_equal(np.isnan(q["ops"]["agg"]), np.isnan(r["ops"]["agg"]))
+    m = ~np.isnan(r["ops"]["agg"])
+    assert np.array_equal(q["ops"]["agg"][m], r["ops"]["agg"][m])
+    assert q["totals"] == r["totals"]
+
+
+@pytest.mark.parametrize("name", ["tiny", "gpt2"])
+def test_tiers_full_map(name):
+    # a map entry for every launch: every kernel is HIGH, and its operator is
+    # the entry for (its name, the number of earlier launches of that name)
+    t = tracegen.with_tiers(tracegen.generate(name), p_corr=1.0, p_stray=0.0)
+    q = oracle.run_tiers(t)
+    assert (q["tier"] == oracle.TIER_HIGH).all()
+    order = np.lexsort((np.arange(t.K), t.k_stream.astype(np.int64), t.k_start))
+    seen = {}
+    lookup = {(int(n), int(i)): int(o) for n, i, o in zip(t.corr_name, t.corr_inv, t.corr_op)}
+    for k in order[:2000]:
+        n = int(t.k_name[k])
+        i = seen.get(n, 0)
+        seen[n] = i + 1
+        assert q["op_of_kernel"][k] == lookup[(n, i)]
+
+
 # ---------------------------------------------------------------- the pins catch planted mistakes
 
 MUTATIONS = [
@@ -450,6 +543,15 @@ MUTATIONS = [
     ("SUM and DW swapped for counter #1", "    AGG_SUM, AGG_SUM, AGG_SUM,                  /* 1 gpu time",
      "    AGG_DW, AGG_SUM, AGG_SUM,                  /* 1 gpu time"),
     ("attributed time counts every kernel", "att += d; natt++;", "natt++;"),
+    ("invocation index over array order", "int64_t k = order[a];\n            inv[k] = ",
+     "int64_t k = a;\n            inv[k] = "),
+    ("NVTX before HIGH", "if (hits == 1) { op = c_op[hit]; t = TIER_HIGH; }\n        else if (rok[k] >= 0)",
+     "if (rok[k] >= 0 && 0) { }\n        else if (rok[k] >= 0) { op = r_op[rok[k]]; t = TIER_NVTX; }\n"
+     "        else if (hits == 1) { op = c_op[hit]; t = TIER_HIGH; }\n        else if (0)"),
+    ("fusion overrides NVTX", "else if (rok[k] >= 0) { op = r_op[rok[k]]; t = TIER_NVTX; }\n        else if (fo != OP_NONE)",
+     "else if (fo != OP_NONE) { op = fo; t = TIER_INDUCTOR; }\n        else if (rok[k] >= 0) { op = r_op[rok[k]]; t = TIER_NVTX; }\n        else if (0)"),
+    ("fused list length ignored", "(fo != OP_NONE && fl > 1)", "(fo != OP_NONE)"),
+    ("walk count marks every tier fused", "(t == TIER_NVTX && nop && nop[k] > 1)", "(nop && nop[k] > 1)"),
 ]
 
 
@@ -462,7 +564,8 @@ def _all_pins(golden):
                      (test_worked_match_and_aggregate, ("prefix", True)),
                      (test_worked_permuted, ("skip_name",)), (test_worked_permuted, ("prefix",)),
                      (test_dedup_mini, (False,)), (test_table8_rules, ()), (test_single_kernel_operator, ()),
-                     (test_walk_cases, ()), (test_fig4_order_not_time, ())]:
+                     (test_walk_cases, ()), (test_fig4_order_not_time, ()), (test_tiers_worked, (True,)),
+                     (test_tiers_worked, (False,))]:
         try:
             if fn in (test_table8_rules, test_walk_cases):
                 fn()

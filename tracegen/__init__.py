@@ -140,6 +140,11 @@ class Trace:
     rep_of_class: np.ndarray | None = None     # i32[n_classes]
     config: dict = field(default_factory=dict)
     ncu_stream: np.ndarray | None = None       # u8[M] stream of each ncu row (per-stream replay runs)
+    corr_name: np.ndarray | None = None        # u32[C] torch.profiler correlation map: kernel name,
+    corr_inv: np.ndarray | None = None         # u32[C]   invocation index of that name,
+    corr_op: np.ndarray | None = None          # u32[C]   operator (HIGH tier)
+    fusion_op: np.ndarray | None = None        # u32[n_names] Inductor fusion map: operator per name or OP_NONE
+    fusion_len: np.ndarray | None = None       # u8[n_names]  operators in the fused list
 
     @property
     def K(self) -> int:
@@ -286,3 +291,58 @@ def per_stream_runs(trace: Trace, stream_order=None) -> Trace:
     order = np.argsort(key, kind="stable")
     return dataclasses.replace(trace, ncu_name=trace.ncu_name[order].copy(), counters=trace.counters[order].copy(),
                                ncu_stream=row_stream[order].astype(np.uint8))
+
+
+OP_NONE = 0xFFFFFFFF
+
+
+def with_tiers(trace: Trace, seed: int = 7, p_corr: float = 0.5, p_fused: float = 0.1, p_stray: float = 0.01,
+               p_unfused_list: float = 0.3, min_count: int = 0) -> Trace:
+    """The same trace with a torch.profiler correlation map and an Inductor
+    fusion map, as the attribution tiers of Fig. 2 read them.
+
+    Correlation map: for a random share p_corr of every name's invocation
+    indices 0 .. count-1 an entry (name, index, operator).  Op ids follow range
+    order in time, and a name's launches spread over the trace, so the
+    operator of index i of a name launched c times is drawn near the same
+    fraction of the op ids, floor((i + U[0,1)) / c * n_ops): map operators stay
+    local in time, as dispatches are (the closer the more launches a name
+    has; with min_count only names launched at least that often get entries).
+    Plus stray entries (a share p_stray
+    each) that name no launch: indices at or past the name's count, and names
+    that never ran, with uniform operators.  Entries come in random order.  Fusion map: per name id, with
+    probability p_fused an operator drawn uniformly, else OP_NONE; list lengths
+    1-4 (1 with probability p_unfused_list)."""
+    import dataclasses
+    rng = np.random.default_rng(seed)
+    K, O = trace.K, max(int(trace.n_ops), 1)
+    names = trace.k_name.astype(np.int64)
+    n_names = int(names.max()) + 1 if K else 0
+    count = np.bincount(names, minlength=n_names) if K else np.zeros(0, np.int64)
+    present = np.nonzero(count)[0]
+    pair_name = np.repeat(present, count[present])
+    starts = np.repeat(np.cumsum(count[present]) - count[present], count[present])
+    pair_inv = np.arange(len(pair_name)) - starts
+    keep = (rng.random(len(pair_name)) < p_corr) & (count[pair_name] >= min_count)
+    cn, ci = pair_name[keep], pair_inv[keep]
+    n_stray = int(p_stray * len(cn)) + (1 if K else 0)
+    if len(present):
+        sn = rng.choice(present, n_stray)
+        si = count[sn] + rng.integers(0, 3, n_stray)                 # past the name's launches
+        un = n_names + rng.integers(0, 100, n_stray)                  # names that never ran
+        ui = rng.integers(0, 3, n_stray)
+        cn = np.concatenate([cn, sn, un])
+        ci = np.concatenate([ci, si, ui])
+    n_named = int(keep.sum())
+    frac = (ci[:n_named] + rng.random(n_named)) / np.maximum(count[cn[:n_named]], 1)
+    co = np.concatenate([np.minimum((frac * O).astype(np.int64), O - 1), rng.integers(0, O, len(cn) - n_named)])
+    perm = rng.permutation(len(cn))
+    cn, ci, co = cn[perm], ci[perm], co[perm]
+    if trace.n_ops == 0:
+        cn, ci, co = cn[:0], ci[:0], co[:0]
+    fo = np.where(rng.random(n_names) < p_fused, rng.integers(0, O, n_names), OP_NONE) if trace.n_ops > 0 \
+        else np.full(n_names, OP_NONE)
+    fl = np.where(rng.random(n_names) < p_unfused_list, 1, rng.integers(2, 5, n_names))
+    return dataclasses.replace(trace, corr_name=cn.astype(np.uint32), corr_inv=ci.astype(np.uint32),
+                               corr_op=co.astype(np.uint32), fusion_op=fo.astype(np.uint32),
+                               fusion_len=fl.astype(np.uint8))
