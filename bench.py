@@ -263,6 +263,8 @@ def main():
     ap.add_argument("--tiers", action="store_true",
                     help="attribution tiers of Fig. 2 in the step: a correlation map recorded for half of the "
                          "launches, fusion entries for a tenth of the names, aggregation by each kernel's operator")
+    ap.add_argument("--rollup", type=int, default=0,
+                    help="also roll the operator records up to this many operator classes in each step")
     ap.add_argument("--launch-lag", type=int, default=0,
                     help="enclosure queries at start - U[0, LAG) ns (host launch times)")
     ap.add_argument("--kernels", type=int, default=0,
@@ -353,6 +355,12 @@ def main():
                          fused_with=torch.empty(K, dtype=torch.int32, device=f"cuda:{dev}"),
                          is_fused=torch.empty(K, dtype=torch.uint8, device=f"cuda:{dev}"))
 
+    rollup_out = class_of_op = None
+    if args.rollup:
+        class_of_op = torch.from_numpy(tracegen.op_classes(trace, n_classes=args.rollup).view(np.int32)).to(
+            f"cuda:{dev}")
+        rollup_out = ctx.alloc_ops(args.rollup)
+
     def join():
         ctx.enclose(tq, rk, nop)
         if tiers_out is not None:
@@ -362,6 +370,9 @@ def main():
             ctx.aggregate(tr, None, idx, ops, op_of_kernel=tiers_out["op"])
         else:
             ctx.aggregate(tr, rk, idx, ops)
+        if rollup_out is not None:
+            ctx.rollup(tr, rk, idx, class_of_op, args.rollup, out=rollup_out,
+                       op_of_kernel=tiers_out["op"] if tiers_out is not None else None)
     in_bytes = sum(x.numel() * x.element_size() for x in (tr.k_stream, tr.k_start, tr.k_dur, tr.k_name,
                                                            tr.r_stream, tr.r_start, tr.r_end, tr.r_depth, tr.r_op,
                                                            tr.ncu_name, tr.counters))
@@ -477,7 +488,8 @@ def main():
         "config": {"workload": f"{args.config}: {WORKLOADS[args.config]}" + (
                        f" [scaled to {K} kernels]" if args.kernels else ""), "kernels": K, "ranges": R,
                    "ncu_rows": M, "ops": O, "shuffled": bool(args.shuffle), "per_stream_ncu": bool(args.per_stream_ncu),
-                   "launch_lag_ns": args.launch_lag, "tiers": bool(args.tiers), "parallelism": f"replicas x{world}",
+                   "launch_lag_ns": args.launch_lag, "tiers": bool(args.tiers), "rollup_classes": args.rollup,
+                   "parallelism": f"replicas x{world}",
                    "l2": "inputs larger than L2 (129 MB)" if flush is None else "L2 flushed before every step"},
         "roofline": {"bound": "hbm", "kernel": dname, "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": (achieved / peak) if achieved else None, "peak_kind": f"{peak_kind} copy bandwidth",

@@ -346,6 +346,26 @@ opattr_status opattr_attribute(opattr_ctx *ctx, const opattr_kernels *kernels, c
                                const opattr_fusion *fusion, uint32_t n_ops, uint32_t *op_of_kernel, uint8_t *tier,
                                uint32_t *fused_with, uint8_t *is_fused, opattr_attr_summary *host_summary);
 
+/* Class roll-up: the records of opattr_aggregate per operator class instead
+ * of per operator (the per-class breakdowns of the case studies, where every
+ * dispatch aten::mm_N counts towards aten::mm).  class_of_op maps each op id
+ * to a class below n_classes, or OPATTR_OP_NONE to leave the op out.  Per
+ * class: kernel count, duration, matched count and the 20 counters by Table
+ * 8's rules over all kernels of the class's operators -- Eq. (1) at class
+ * granularity, so a class's duration-weighted mean weighs every kernel, not
+ * every operator.  Every class in [0, n_classes) is written (empty classes
+ * get zero counts and NaN counters).
+ *   kernels, ranges, range_of_kernel, ncu, ncu_idx_of_kernel, n_ops: as for
+ *                      opattr_aggregate (range_of_kernel may be NULL there too)
+ *   class_of_op        u32[n_ops]  device
+ *   dev_out            host struct of device pointers, n_classes entries
+ * Errors: OPATTR_E_INVALID_ARG (as opattr_aggregate, a class >= n_classes
+ * other than OPATTR_OP_NONE, n_classes > 2^24), OPATTR_E_OOM, OPATTR_E_CUDA. */
+opattr_status opattr_rollup(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,
+                            const int32_t *range_of_kernel, const opattr_ncu *ncu, const int32_t *ncu_idx_of_kernel,
+                            uint32_t n_ops, const uint32_t *class_of_op, uint32_t n_classes,
+                            const opattr_op_aggregates *dev_out);
+
 /* Free the context and its scratch.  NULL is ignored. */
 void opattr_destroy(opattr_ctx *ctx);
 

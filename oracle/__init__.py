@@ -233,6 +233,17 @@ def aggregate_by_op(k_dur, op_of_kernel, counters, ncu_idx, n_ops: int):
     return aggregate(k_dur, rk, op, counters, ncu_idx, n_ops)
 
 
+def rollup(k_dur, op_of_kernel, counters, ncu_idx, class_of_op, n_classes: int):
+    """aggregate() per operator class: each kernel's operator mapped through
+    class_of_op (OP_NONE leaves it out)."""
+    op = _c(op_of_kernel, np.uint32).astype(np.int64)
+    cm = _c(class_of_op, np.uint32)
+    has = op != OP_NONE
+    cls = np.full(len(op), OP_NONE, np.uint32)
+    cls[has] = cm[op[has]]
+    return aggregate_by_op(k_dur, cls, counters, ncu_idx, n_classes)
+
+
 def run_tiers(trace, mode: str = "skip_name", enclose_mode: str = "indexed", dedup: bool | None = None,
               brute: bool = False, use_corr: bool = True, use_fusion: bool = True):
     """The join with the attribution tiers: enclose, attribute, match, aggregate by operator."""

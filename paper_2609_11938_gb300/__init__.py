@@ -128,6 +128,8 @@ def library():
                                              P(OpAggregates), P(Totals)]
             lib.opattr_attribute.argtypes = [_vp, P(Kernels), P(Ranges), _vp, _vp, P(Corr), P(Fusion),
                                              ctypes.c_uint32, _vp, _vp, _vp, _vp, P(AttrSummary)]
+            lib.opattr_rollup.argtypes = [_vp, P(Kernels), P(Ranges), _vp, P(Ncu), _vp, ctypes.c_uint32, _vp,
+                                          ctypes.c_uint32, P(OpAggregates)]
             lib.opattr_destroy.argtypes = [_vp]
             lib.opattr_destroy.restype = None
             lib.opattr_status_string.argtypes = [ctypes.c_int]
@@ -142,7 +144,7 @@ def library():
             lib.opattr_match_noalloc.argtypes = [P(Kernels), P(Ncu), ctypes.c_int, _vp, _vp, P(MatchSummary), _vp]
             lib.opattr_match_noalloc.restype = ctypes.c_int
             for f in ("opattr_create", "opattr_enclose", "opattr_match", "opattr_aggregate", "opattr_attribute",
-                      "opattr_set_timing", "opattr_timing_report"):
+                      "opattr_rollup", "opattr_set_timing", "opattr_timing_report"):
                 getattr(lib, f).restype = ctypes.c_int
             _lib = lib
         return _lib
@@ -195,6 +197,13 @@ def opattr_attribute(handle, kernels: Kernels, ranges: Ranges, rok_ptr: int, nop
                                       ctypes.byref(fusion) if fusion is not None else None, ctypes.c_uint32(n_ops),
                                       _vp(op_ptr), _vp(tier_ptr or 0), _vp(fused_with_ptr or 0),
                                       _vp(is_fused_ptr or 0), ctypes.byref(summary))
+
+
+def opattr_rollup(handle, kernels: Kernels, ranges: Ranges, rok_ptr: int | None, ncu: Ncu, idx_ptr: int, n_ops: int,
+                  class_ptr: int, n_classes: int, out: OpAggregates) -> int:
+    return library().opattr_rollup(handle, ctypes.byref(kernels), ctypes.byref(ranges), _vp(rok_ptr or 0),
+                                   ctypes.byref(ncu), _vp(idx_ptr), ctypes.c_uint32(n_ops), _vp(class_ptr),
+                                   ctypes.c_uint32(n_classes), ctypes.byref(out))
 
 
 def opattr_match_noalloc(kernels: Kernels, ncu: Ncu, mismatch: str, idx_ptr: int, kind_ptr: int | None,
@@ -437,6 +446,30 @@ class Context:
         if st < 0:
             raise OpattrError(st, "opattr_aggregate")
         return st, ops, tot.as_dict()
+
+    def rollup(self, tr: DeviceTrace, range_of_kernel, ncu_idx, class_of_op, n_classes: int, out=None,
+               op_of_kernel=None):
+        """Per-class records (opattr_rollup); class_of_op: int32/uint32 device tensor of n_ops entries."""
+        import torch
+        if out is None:
+            out = self.alloc_ops(n_classes)
+        dv = self.device
+        o = OpAggregates(_ptr(out["kernel_count"], torch.int64, "kernel_count", dv),
+                         _ptr(out["total_duration_ns"], torch.int64, "total_duration_ns", dv),
+                         _ptr(out["matched_count"], torch.int64, "matched_count", dv),
+                         _ptr(out["agg"], torch.float64, "agg", dv))
+        if op_of_kernel is not None:
+            rng = Ranges(None, None, None, None, _ptr(op_of_kernel, torch.uint32, "op_of_kernel", dv), tr.K)
+            rok_ptr = None
+        else:
+            rng = self.ranges(tr)
+            rok_ptr = _ptr(range_of_kernel, torch.int32, "range_of_kernel", dv)
+        st = opattr_rollup(self.handle, self.kernels(tr), rng, rok_ptr, self.ncu(tr),
+                           _ptr(ncu_idx, torch.int32, "ncu_idx_of_kernel", dv), tr.n_ops,
+                           _ptr(class_of_op, torch.uint32, "class_of_op", dv), n_classes, o)
+        if st < 0:
+            raise OpattrError(st, "opattr_rollup")
+        return st, out
 
     def run(self, tr: DeviceTrace, dedup: bool | None = None):
         """enclose + match + aggregate on device-resident inputs."""

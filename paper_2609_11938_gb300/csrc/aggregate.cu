@@ -702,11 +702,11 @@ __device__ __forceinline__ void acc_merge(Acc &a, const Acc &b) {
 }
 
 // Piece offsets of the listed long ops, one block: poff[j] = pieces of the
-// ops listed before j (an op longer than AG_HUGE has ceil(len / AG_PIECE)
+// ops listed before j (an op longer than `huge` has ceil(len / AG_PIECE)
 // pieces, a shorter one none); poff[nlong] = all pieces.
 __global__ void __launch_bounds__(1024) k_agg_piece_offsets(const uint32_t *__restrict__ off,
                                                             const uint32_t *__restrict__ longs,
-                                                            const unsigned *__restrict__ nlong,
+                                                            const unsigned *__restrict__ nlong, uint32_t huge,
                                                             uint32_t *__restrict__ poff) {
     __shared__ uint32_t wbuf[33];
     const int64_t n = *nlong;
@@ -716,7 +716,7 @@ __global__ void __launch_bounds__(1024) k_agg_piece_offsets(const uint32_t *__re
         uint32_t np = 0;
         if (j < n) {
             const uint32_t o = longs[j], len = off[o + 1] - off[o];
-            np = len > AG_HUGE ? (len + AG_PIECE - 1) / AG_PIECE : 0u;
+            np = len > huge ? (len + AG_PIECE - 1) / AG_PIECE : 0u;
         }
         uint32_t tot;
         const uint32_t ex = block_exclusive_scan<uint32_t>(np, wbuf, &tot);
@@ -724,6 +724,38 @@ __global__ void __launch_bounds__(1024) k_agg_piece_offsets(const uint32_t *__re
         carry += tot;
     }
     if (threadIdx.x == 0) poff[n] = carry;
+}
+
+// A lane's run of a piece with the fast accumulator: returns false when a
+// null or infinite value took part (the caller redoes the run carefully),
+// else the run's partial in careful form (every counter non-null).
+__device__ __forceinline__ bool piece_fast(const AggIn &A, const uint32_t *seg, uint32_t l0, uint32_t l1, Acc &out) {
+    AccF f;
+    f.init();
+#pragma unroll 4
+    for (uint32_t t = l0; t < l1; ++t) {
+        const uint32_t k = seg[t];
+        const int32_t j = A.ncu_idx[k];
+        f.accumulate(A.dur[k], j >= 0, reinterpret_cast<const float4 *>(A.counters + (int64_t)(j >= 0 ? j : 0) * NC));
+    }
+    if (!f.clean()) return false;
+    out.kc = (int)(l1 - l0);
+    out.mc = f.mc;
+    out.dsum = f.dsum;
+    out.dall = f.dall;
+#pragma unroll
+    for (int i = 0; i < N_SUM; ++i) out.s[i] = f.s[i];
+#pragma unroll
+    for (int i = 0; i < N_DW; ++i) {
+        out.w[i] = f.w[i];
+        out.nanw[i] = 0;
+    }
+#pragma unroll
+    for (int i = 0; i < N_MAX; ++i) out.mx[i] = f.mx[i];
+    out.seen = f.mc > 0 ? ALL_COUNTERS : 0u;
+    out.bad = 0;
+    out.terms = 0;
+    return true;
 }
 
 // Pieces: one warp per AG_PIECE kernels of a huge op (lane l adds AG_PIECE /
@@ -750,38 +782,48 @@ __global__ void k_agg_pieces(const uint32_t *__restrict__ off, const uint32_t *_
         const uint32_t per = AG_PIECE / 32;
         const uint32_t l0 = min(b0 + lane * per, b1), l1 = min(l0 + per, b1);
         Acc acc;
-        acc.init();
-        for (uint32_t t = l0; t < l1; ++t) acc.add(A, list[s0 + t]);
+        if (!piece_fast(A, list + s0, l0, l1, acc)) {     // a null or infinite value: redo with null handling
+            acc.init();
+            for (uint32_t t = l0; t < l1; ++t) acc.add(A, list[s0 + t]);
+        }
 #pragma unroll 1
         for (int d = 16; d > 0; d >>= 1) acc_merge_down(acc, d);
         if (lane == 0) part[p] = acc;
     }
 }
 
-// Finish: one warp per huge op merges its pieces' partials (lane l takes
-// pieces l, l + 32, ... in order, then the fixed tree) and writes the record.
-__global__ void k_agg_long_ops(const uint32_t *__restrict__ longs, const unsigned *__restrict__ nlong,
-                               const uint32_t *__restrict__ poff, const Acc *__restrict__ part, AggIn A,
-                               DevStatus *st) {
+// Finish: one block per huge op merges its pieces' partials -- thread t takes
+// pieces t, t + FIN_THREADS, ... in order, then each warp's fixed tree, then
+// thread 0 takes the warps' partials in warp order -- and writes the record.
+constexpr int FIN_THREADS = 256;
+__global__ void __launch_bounds__(FIN_THREADS) k_agg_long_ops(const uint32_t *__restrict__ longs,
+                                                              const unsigned *__restrict__ nlong,
+                                                              const uint32_t *__restrict__ poff,
+                                                              const Acc *__restrict__ part, int write_empty, AggIn A,
+                                                              DevStatus *st) {
+    __shared__ Acc wpart[FIN_THREADS / 32];
     const int64_t n = *nlong;
-    const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-    const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-    const unsigned lane = lane_id();
+    const unsigned lane = lane_id(), w = threadIdx.x >> 5;
     int bad = 0;
-    for (int64_t q = warp; q < n; q += nwarps) {
-        if (poff[q + 1] == poff[q]) continue;   // not huge: the ops pass writes it
+    for (int64_t q = blockIdx.x; q < n; q += gridDim.x) {
+        if (poff[q + 1] == poff[q] && !write_empty) continue;   // not huge: the ops pass writes it
         const uint32_t o = longs[q];
         Acc acc;
         acc.init();
-        for (uint32_t p = poff[q] + lane; p < poff[q + 1]; p += 32) acc_merge(acc, part[p]);
+        for (uint32_t p = poff[q] + threadIdx.x; p < poff[q + 1]; p += FIN_THREADS) acc_merge(acc, part[p]);
 #pragma unroll 1
         for (int d = 16; d > 0; d >>= 1) acc_merge_down(acc, d);
-        if (lane == 0) {
-            acc.write(A, o);
-            bad |= acc.bad;
+        if (lane == 0) wpart[w] = acc;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            Acc total = wpart[0];
+            for (int v = 1; v < FIN_THREADS / 32; ++v) acc_merge(total, wpart[v]);
+            total.write(A, o);
+            bad |= total.bad;
         }
+        __syncthreads();
     }
-    if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_err(st, ERR_INVALID);
+    if (bad) set_err(st, ERR_INVALID);
 }
 
 // Blocks of the ops pass: what stays resident, fewer for few ops.
@@ -856,7 +898,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
         launch(c, "agg_long_list", k_agg_long_list, dim3(grid_for(O, 256, 4096)), dim3(256), 0,
                (const uint32_t *)off, O, AG_SHORT_MAX, longs, nlong);
         launch(c, "agg_piece_offsets", k_agg_piece_offsets, dim3(1), dim3(1024), 0, (const uint32_t *)off,
-               (const uint32_t *)longs, (const unsigned *)nlong, npc);
+               (const uint32_t *)longs, (const unsigned *)nlong, AG_HUGE, npc);
         int sms = 0;
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
         launch(c, "agg_sort_long", k_agg_sort_long, dim3(2 * std::max(1, sms)), dim3(SL_THREADS), 0, (const uint32_t *)off,
@@ -864,8 +906,9 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
         launch(c, "agg_pieces", k_agg_pieces, dim3(4 * std::max(1, sms)), dim3(256), 0, (const uint32_t *)off,
                (const uint32_t *)list, (const uint32_t *)longs, (const unsigned *)nlong, (const uint32_t *)npc, in,
                partials);
-        launch(c, "agg_long_ops", k_agg_long_ops, dim3(std::max(1, sms)), dim3(256), 0, (const uint32_t *)longs,
-               (const unsigned *)nlong, (const uint32_t *)npc, (const Acc *)partials, in, c.d_status);
+        launch(c, "agg_long_ops", k_agg_long_ops, dim3(2 * std::max(1, sms)), dim3(FIN_THREADS), 0,
+               (const uint32_t *)longs,
+               (const unsigned *)nlong, (const uint32_t *)npc, (const Acc *)partials, 0, in, c.d_status);
         launch(c, "agg_ops", k_agg_ops, dim3(ops_grid(c, O)), dim3(AG_THREADS), 0,
                (const uint32_t *)off, list, in, c.d_status);
     }
@@ -882,6 +925,142 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     T.attributed_frac = T.total_ns > 0 ? (double)T.attributed_ns / (double)T.total_ns : qnan;
     T.unattributed_frac = T.total_ns > 0 ? (double)T.unattributed_ns / (double)T.total_ns : qnan;
     if (tot_out) *tot_out = T;
+    return OPATTR_OK;
+}
+
+}  // namespace opattr
+
+namespace opattr {
+
+// ------------------------------------------------------------------ class roll-up
+// The per-operator records of Eq. (1) rolled up to operator classes (the
+// per-class breakdown of the case studies): every attributed kernel whose
+// operator has a class is aggregated with the other kernels of that class.
+// Few, large groups: a stable radix sort of the kernels by class key (kernel
+// index order kept within a class) replaces the fill and the segment sort,
+// and every class is accumulated by pieces.
+__global__ void k_class_check(const uint32_t *__restrict__ class_of_op, int64_t n_ops, uint32_t n_classes,
+                              DevStatus *st) {
+    int bad = 0;
+    for (int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < n_ops; o += (int64_t)gridDim.x * blockDim.x) {
+        const uint32_t c = class_of_op[o];
+        bad |= c >= n_classes && c != OPATTR_OP_NONE;
+    }
+    if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_err(st, ERR_INVALID);
+}
+// key = class of the kernel's operator, n_classes when it has none; counts
+// per class (in a block histogram in shared memory when there are at most
+// CK_SMEM classes, flushed once per block; else one global atomic per class
+// and warp).
+constexpr int CK_SMEM = 4096;
+__global__ void k_class_keys(const int32_t *__restrict__ rok, const uint32_t *__restrict__ r_op, int64_t K, int64_t R,
+                             int64_t n_ops, const uint32_t *__restrict__ class_of_op, uint32_t n_classes,
+                             uint32_t *__restrict__ key, uint32_t *__restrict__ cnt) {
+    __shared__ uint32_t h[CK_SMEM];
+    const bool local = n_classes <= (uint32_t)CK_SMEM;
+    if (local)
+        for (uint32_t i = threadIdx.x; i < n_classes; i += blockDim.x) h[i] = 0;
+    __syncthreads();
+    uint32_t *dst = local ? h : cnt;
+    for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k - threadIdx.x < K;
+         k += (int64_t)gridDim.x * blockDim.x) {
+        uint32_t c = n_classes;
+        if (k < K) {
+            const int32_t r = range_of(rok, r_op, k);
+            if (r >= 0 && r < R) {
+                const uint32_t op = r_op[r];
+                if ((int64_t)op < n_ops) {
+                    const uint32_t x = class_of_op[op];
+                    if (x < n_classes) c = x;
+                }
+            }
+            key[k] = c;
+        }
+        const unsigned peers = __match_any_sync(0xffffffffu, c);
+        if (k < K && c < n_classes && (peers & lanemask_lt()) == 0) atomicAdd(&dst[c], (unsigned)__popc(peers));
+    }
+    if (local) {
+        __syncthreads();
+        for (uint32_t i = threadIdx.x; i < n_classes; i += blockDim.x)
+            if (h[i]) atomicAdd(&cnt[i], h[i]);
+    }
+}
+__global__ void k_iota_u32(uint32_t *dst, int64_t n, unsigned *count) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        dst[i] = (uint32_t)i;
+    if (blockIdx.x == 0 && threadIdx.x == 0) *count = (unsigned)n;
+}
+
+opattr_status do_rollup(Ctx &c, const opattr_kernels *kern, const opattr_ranges *rng, const int32_t *rok,
+                        const opattr_ncu *ncu, const int32_t *nidx, uint32_t n_ops, const uint32_t *class_of_op,
+                        uint32_t n_classes, const opattr_op_aggregates *out) {
+    const int64_t K = kern->n, R = rng->n, M = ncu->n, O = n_ops, C = n_classes;
+    if (K < 0 || R < 0 || M < 0 || K >= (1ll << 31) || R >= (1ll << 31) || M >= (1ll << 31) || !out)
+        return OPATTR_E_INVALID_ARG;
+    if (C > (1 << 24)) return OPATTR_E_INVALID_ARG;
+    if (K > 0 && (!kern->dur_ns || !nidx)) return OPATTR_E_INVALID_ARG;
+    if (K > 0 && !rok && R != K) return OPATTR_E_INVALID_ARG;
+    if (R > 0 && !rng->op_id) return OPATTR_E_INVALID_ARG;
+    if (O > 0 && !class_of_op) return OPATTR_E_INVALID_ARG;
+    if (M > 0 && !ncu->counters) return OPATTR_E_INVALID_ARG;
+    if (C > 0 && (!out->kernel_count || !out->total_duration_ns || !out->matched_count || !out->agg))
+        return OPATTR_E_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(ncu->counters) & 15) != 0) return OPATTR_E_INVALID_ARG;
+
+    const int64_t maxp = K / AG_PIECE + C + 1;
+    Need nd;
+    for (int i = 0; i < 4; ++i) nd.add<uint32_t>(K);
+    nd.add<uint32_t>(radix_hist_elems(K)).add<uint32_t>(scan_scratch_elems(std::max(radix_hist_elems(K), C + 2)));
+    nd.add<uint32_t>(C + 2).add<uint32_t>(C + 2).add<uint32_t>(C + 1).add<uint32_t>(C + 1).add<unsigned>(1);
+    nd.add<Acc>(maxp);
+    opattr_status st = ensure_arena(c, nd.bytes + 4096);
+    if (st) return st;
+    Arena a(c);
+    if ((st = reset_status(c))) return st;
+    uint32_t *k0 = a.take<uint32_t>(K), *v0 = a.take<uint32_t>(K), *k1 = a.take<uint32_t>(K), *v1 = a.take<uint32_t>(K);
+    uint32_t *hist = a.take<uint32_t>(radix_hist_elems(K));
+    uint32_t *part = a.take<uint32_t>(scan_scratch_elems(std::max(radix_hist_elems(K), C + 2)));
+    uint32_t *cnt = a.take<uint32_t>(C + 2), *off = a.take<uint32_t>(C + 2);
+    uint32_t *cls = a.take<uint32_t>(C + 1), *poff = a.take<uint32_t>(C + 1);
+    unsigned *ncls = a.take<unsigned>(1);
+    Acc *partials = a.take<Acc>(maxp);
+    if (!k0 || !v0 || !k1 || !v1 || !hist || !part || !cnt || !off || !cls || !poff || !ncls || !partials)
+        return OPATTR_E_OOM;
+    if (O > 0)
+        launch(c, "class_check", k_class_check, dim3(grid_for(O, 256, REDUCE_GRID)), dim3(256), 0, class_of_op, O,
+               n_classes, c.d_status);
+    cudaMemsetAsync(cnt, 0, sizeof(uint32_t) * (C + 2), c.stream);
+    uint32_t *list = nullptr;
+    if (K > 0) {
+        launch(c, "class_keys", k_class_keys, dim3(grid_for(K, 256, REDUCE_GRID)), dim3(256), 0, rok, rng->op_id, K, R,
+               O, class_of_op, n_classes, k0, cnt);
+        uint32_t *ko;
+        radix_sort_pairs<uint32_t>(c, k0, v0, k1, v1, K, bits_for((uint64_t)C), true, hist, part, &ko, &list);
+    }
+    scan_exclusive_u32(c, cnt, off, C + 1, part, nullptr);           // off[C] = kernels with a class
+    if (C > 0) {
+        AggIn in;
+        in.dur = kern->dur_ns;
+        in.ncu_idx = nidx;
+        in.counters = ncu->counters;
+        in.n_ops = C;
+        in.ctr = nullptr;
+        in.out = *out;
+        int sms = 0;
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
+        launch(c, "class_iota", k_iota_u32, dim3(grid_for(C, 256, 4096)), dim3(256), 0, cls, C, ncls);
+        launch(c, "agg_piece_offsets", k_agg_piece_offsets, dim3(1), dim3(1024), 0, (const uint32_t *)off,
+               (const uint32_t *)cls, (const unsigned *)ncls, 0u, poff);
+        if (K > 0)
+            launch(c, "agg_pieces", k_agg_pieces, dim3(4 * std::max(1, sms)), dim3(256), 0, (const uint32_t *)off,
+                   (const uint32_t *)list, (const uint32_t *)cls, (const unsigned *)ncls, (const uint32_t *)poff, in,
+                   partials);
+        launch(c, "class_records", k_agg_long_ops, dim3(2 * std::max(1, sms)), dim3(FIN_THREADS), 0,
+               (const uint32_t *)cls,
+               (const unsigned *)ncls, (const uint32_t *)poff, (const Acc *)partials, 1, in, c.d_status);
+    }
+    if ((st = read_status(c))) return st;
+    if (c.h_status->err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
     return OPATTR_OK;
 }
 

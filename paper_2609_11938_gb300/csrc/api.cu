@@ -22,6 +22,10 @@ opattr_status do_attribute(Ctx &c, const opattr_kernels *kern, const opattr_rang
                            uint32_t n_ops, uint32_t *op_of_kernel, uint8_t *tier, uint32_t *fused_with,
                            uint8_t *is_fused, opattr_attr_summary *sum);
 
+opattr_status do_rollup(Ctx &c, const opattr_kernels *kern, const opattr_ranges *rng, const int32_t *rok,
+                        const opattr_ncu *ncu, const int32_t *nidx, uint32_t n_ops, const uint32_t *class_of_op,
+                        uint32_t n_classes, const opattr_op_aggregates *out);
+
 opattr_status cuda_status(Ctx &c, cudaError_t e) {
     if (e == cudaSuccess) e = c.last_error;
     if (e == cudaSuccess) return OPATTR_OK;
@@ -232,6 +236,19 @@ opattr_status opattr_attribute(opattr_ctx *ctx, const opattr_kernels *kernels, c
     if (!g.ok) return OPATTR_E_CUDA;
     return finish(c, do_attribute(c, kernels, ranges, range_of_kernel, n_op_enclosing, corr, fusion, n_ops,
                                   op_of_kernel, tier, fused_with, is_fused, host_summary));
+}
+
+opattr_status opattr_rollup(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,
+                            const int32_t *range_of_kernel, const opattr_ncu *ncu, const int32_t *ncu_idx_of_kernel,
+                            uint32_t n_ops, const uint32_t *class_of_op, uint32_t n_classes,
+                            const opattr_op_aggregates *dev_out) {
+    if (!ctx || !kernels || !ranges || !ncu) return OPATTR_E_INVALID_ARG;
+    Ctx &c = ctx->c;
+    if (c.broken) return OPATTR_E_STATE;
+    DeviceGuard g(c.device);
+    if (!g.ok) return OPATTR_E_CUDA;
+    return finish(c, do_rollup(c, kernels, ranges, range_of_kernel, ncu, ncu_idx_of_kernel, n_ops, class_of_op,
+                               n_classes, dev_out));
 }
 
 void opattr_destroy(opattr_ctx *ctx) {

@@ -506,3 +506,63 @@ def test_tiers_large(opa):
     fusion entries for a tenth of the names, against the indexed oracle."""
     t = tracegen.with_tiers(tracegen.generate("large"))
     assert_parity_tiers(gpu_run_tiers(t), oracle.run_tiers(t))
+
+
+# ---------------------------------------------------------------- class roll-up
+
+def _rollup_case(opa, t, C, seed=3, tiers=False):
+    import torch
+    cm = tracegen.op_classes(t, n_classes=C, seed=seed)
+    ctx = opa.Context(0)
+    tr = opa.to_device(t)
+    st, rk, nop = ctx.enclose(tr)
+    st, idx, kind, summ = ctx.match(tr)
+    dcm = torch.from_numpy(cm.view(np.int32)).cuda()
+    if tiers:
+        st, op, tier, fw, fz, ts = ctx.attribute(tr, rk, nop)
+        st, cr = ctx.rollup(tr, None, idx, dcm, C, op_of_kernel=op)
+        op_h = op.cpu().numpy().view(np.uint32)
+    else:
+        st, cr = ctx.rollup(tr, rk, idx, dcm, C)
+        rk_h = rk.cpu().numpy()
+        op_h = np.where(rk_h >= 0, t.r_op[np.maximum(rk_h, 0)], oracle.OP_NONE).astype(np.uint32)
+    torch.cuda.synchronize()
+    g = {k: v.cpu().numpy() for k, v in cr.items()}
+    ctx.close()
+    o_st, o, _ = oracle.rollup(t.k_dur, op_h, t.counters, idx.cpu().numpy(), cm, C)
+    assert st == o_st == 0
+    for k in ("kernel_count", "total_duration_ns", "matched_count"):
+        np.testing.assert_array_equal(g[k], o[k], err_msg=k)
+    assert_close(g["agg"], o["agg"], what="rollup agg")
+
+
+@pytest.mark.parametrize("name,C", [("tiny", 5), ("gpt2", 64), ("dedup", 300), ("gpt2", 1)])
+def test_rollup_configs(opa, name, C):
+    """Per-class records against the oracle's aggregation by class (empty and
+    left-out classes included)."""
+    _rollup_case(opa, tracegen.generate(name), C)
+
+
+def test_rollup_tiers(opa):
+    """Roll-up of the tiered attribution (operators given per kernel)."""
+    _rollup_case(opa, tracegen.with_tiers(tracegen.generate("gpt2")), 40, tiers=True)
+
+
+def test_rollup_large(opa):
+    """The 20 M-kernel trace rolled up to 64 classes."""
+    _rollup_case(opa, tracegen.generate("large"), 64)
+
+
+def test_rollup_rejects(opa):
+    import torch
+    t = tracegen.generate("tiny")
+    ctx = opa.Context(0)
+    tr = opa.to_device(t)
+    st, rk, nop = ctx.enclose(tr)
+    st, idx, kind, summ = ctx.match(tr)
+    cm = np.zeros(t.n_ops, np.uint32)
+    cm[3] = 7
+    with pytest.raises(opa.OpattrError) as ei:
+        ctx.rollup(tr, rk, idx, torch.from_numpy(cm.view(np.int32)).cuda(), 7)
+    assert ei.value.status == opa.E_INVALID_ARG
+    ctx.close()

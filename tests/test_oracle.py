@@ -524,6 +524,61 @@ def test_tiers_full_map(name):
         assert q["op_of_kernel"][k] == lookup[(n, i)]
 
 
+# ---------------------------------------------------------------- class roll-up
+
+@pytest.mark.parametrize("name", ["tiny", "gpt2", "dedup"])
+def test_rollup_from_operator_records(name):
+    # the class records follow from the operator records and the operators'
+    # matched durations alone: counts and durations add up, SUM counters add
+    # up, MAX counters take the maximum, and a duration-weighted mean is the
+    # mean of its operators' means weighted by their matched duration (no
+    # null counters in these traces)
+    t = tracegen.generate(name)
+    r = oracle.run(t)
+    rk, idx = r["range_of_kernel"], r["ncu_idx"]
+    op = np.where(rk >= 0, t.r_op[np.maximum(rk, 0)], oracle.OP_NONE).astype(np.uint32)
+    C = 9
+    cm = tracegen.op_classes(t, n_classes=C, seed=3)
+    st, cr, _ = oracle.rollup(t.k_dur, op, t.counters, idx, cm, C)
+    assert st == oracle.OK
+    ops = r["ops"]
+    has = cm != oracle.OP_NONE
+    cl = cm[has].astype(np.int64)
+    for k in ("kernel_count", "total_duration_ns", "matched_count"):
+        assert np.array_equal(cr[k], np.bincount(cl, ops[k][has], minlength=C).astype(np.int64))
+    att = (op != oracle.OP_NONE) & (idx >= 0)
+    wop = np.bincount(op[att].astype(np.int64), t.k_dur[att].astype(np.float64), minlength=t.n_ops)
+    rules = oracle.agg_rules()
+    for c in range(NC):
+        v = ops["agg"][c][has]
+        ok = ~np.isnan(v)
+        if rules[c] == oracle.SUM:
+            want = np.bincount(cl[ok], v[ok], minlength=C)
+        elif rules[c] == oracle.MAX:
+            want = np.full(C, -np.inf)
+            np.maximum.at(want, cl[ok], v[ok])
+        else:
+            w = wop[has][ok]
+            want = np.bincount(cl[ok], v[ok] * w, minlength=C) / np.bincount(cl[ok], w, minlength=C)
+        got = cr["agg"][c]
+        m = np.bincount(cl[ok], minlength=C) > 0
+        assert np.all(np.isnan(got[~m]))
+        np.testing.assert_allclose(got[m], want[m], rtol=1e-12, err_msg=f"counter {c}")
+
+
+def test_rollup_one_class_per_op():
+    # classes equal to operators: the roll-up is the operator aggregation
+    t = tracegen.generate("tiny")
+    r = oracle.run(t)
+    rk = r["range_of_kernel"]
+    op = np.where(rk >= 0, t.r_op[np.maximum(rk, 0)], oracle.OP_NONE).astype(np.uint32)
+    st, cr, _ = oracle.rollup(t.k_dur, op, t.counters, r["ncu_idx"], np.arange(t.n_ops, dtype=np.uint32), t.n_ops)
+    assert st == oracle.OK
+    for k in ("kernel_count", "total_duration_ns", "matched_count"):
+        assert np.array_equal(cr[k], r["ops"][k])
+    assert np.array_equal(np.isnan(cr["agg"]), np.isnan(r["ops"]["agg"]))
+
+
 # ---------------------------------------------------------------- the pins catch planted mistakes
 
 MUTATIONS = [

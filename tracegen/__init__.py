@@ -346,3 +346,14 @@ def with_tiers(trace: Trace, seed: int = 7, p_corr: float = 0.5, p_fused: float 
     return dataclasses.replace(trace, corr_name=cn.astype(np.uint32), corr_inv=ci.astype(np.uint32),
                                corr_op=co.astype(np.uint32), fusion_op=fo.astype(np.uint32),
                                fusion_len=fl.astype(np.uint8))
+
+
+def op_classes(trace: Trace, n_classes: int = 64, seed: int = 11, p_none: float = 0.02) -> np.ndarray:
+    """An operator class per op id (the aten:: name that dispatches share), for
+    class roll-ups: classes drawn Zipf(1.1)-distributed over n_classes, a share
+    p_none of the ops left out (OP_NONE)."""
+    rng = np.random.default_rng(seed)
+    w = 1.0 / np.arange(1, n_classes + 1) ** 1.1
+    cls = rng.choice(n_classes, size=int(trace.n_ops), p=w / w.sum()).astype(np.int64)
+    cls[rng.random(int(trace.n_ops)) < p_none] = OP_NONE
+    return cls.astype(np.uint32)
