@@ -366,6 +366,47 @@ opattr_status opattr_rollup(opattr_ctx *ctx, const opattr_kernels *kernels, cons
                             uint32_t n_ops, const uint32_t *class_of_op, uint32_t n_classes,
                             const opattr_op_aggregates *dev_out);
 
+/* ---- profile.json (App. A.4 schema) ----
+ * A host-side writer over the join's outputs: one entry per attributed
+ * operator with its kernels (name, attribution tier and confidence,
+ * duration, stream, the 20 raw counters of its ncu row) and its aggregated
+ * record, then the unattributed kernels.  Counter fields carry the profile
+ * names of Table 8; NaN is written as null.  Every array here is HOST memory
+ * (copy the device outputs back first). */
+typedef struct {
+    const char *model_name;            /* capture_metadata fields, NULL = omitted */
+    const char *device_name;
+    const char *compile_mode;
+    const char *capture_timestamp_utc;
+    int32_t include_kernels;           /* 0: operators without per-kernel records (large traces) */
+} opattr_profile_meta;
+
+typedef struct {
+    const char *const *kernel_name;    /* [n_kernel_names] by name id, NULL = "kernel_<id>" */
+    int64_t n_kernel_names;
+    const char *const *op_name;        /* [n_ops] canonical operator name (aten::mm), NULL = "op_<id>" */
+    const int64_t *op_call_index;      /* [n_ops] dispatch ordinal (operator_id = name_index), NULL = op id */
+} opattr_profile_names;
+
+/* Writes the document to `path`.
+ *   kernels          host struct of HOST arrays: stream, dur_ns, name_id, n
+ *   op_of_kernel     u32[kernels->n]  operator of each kernel or OPATTR_OP_NONE
+ *   tier             u8[kernels->n]   opattr_tier, or NULL (NVTX for attributed kernels)
+ *   is_fused         u8[kernels->n]   or NULL
+ *   fused_with       u32[kernels->n]  or NULL (operator of the kernel's fused list)
+ *   ncu_idx_of_kernel i32[kernels->n] row of each kernel or -1
+ *   counters         f32[n_rows * 20] the ncu rows
+ *   ops              host struct of HOST arrays, n_ops entries (opattr_aggregate's output)
+ *   bytes_written    may be NULL
+ * Errors: OPATTR_E_INVALID_ARG (NULL required array, an operator >= n_ops,
+ * a row index out of range, the file cannot be written). */
+opattr_status opattr_write_profile(const char *path, const opattr_profile_meta *meta,
+                                   const opattr_profile_names *names, const opattr_kernels *kernels,
+                                   const uint32_t *op_of_kernel, const uint8_t *tier, const uint8_t *is_fused,
+                                   const uint32_t *fused_with, const int32_t *ncu_idx_of_kernel, const float *counters,
+                                   int64_t n_rows, uint32_t n_ops, const opattr_op_aggregates *ops,
+                                   int64_t *bytes_written);
+
 /* Free the context and its scratch.  NULL is ignored. */
 void opattr_destroy(opattr_ctx *ctx);
 

@@ -89,6 +89,16 @@ class AttrSummary(ctypes.Structure):
         return {f: int(getattr(self, f)) for f, _ in self._fields_}
 
 
+class ProfileMeta(ctypes.Structure):
+    _fields_ = [("model_name", ctypes.c_char_p), ("device_name", ctypes.c_char_p), ("compile_mode", ctypes.c_char_p),
+                ("capture_timestamp_utc", ctypes.c_char_p), ("include_kernels", ctypes.c_int32)]
+
+
+class ProfileNames(ctypes.Structure):
+    _fields_ = [("kernel_name", _vp), ("n_kernel_names", ctypes.c_int64), ("op_name", _vp),
+                ("op_call_index", _vp)]
+
+
 class OpAggregates(ctypes.Structure):
     _fields_ = [("kernel_count", _vp), ("total_duration_ns", _vp), ("matched_count", _vp), ("agg", _vp)]
 
@@ -130,6 +140,10 @@ def library():
                                              ctypes.c_uint32, _vp, _vp, _vp, _vp, P(AttrSummary)]
             lib.opattr_rollup.argtypes = [_vp, P(Kernels), P(Ranges), _vp, P(Ncu), _vp, ctypes.c_uint32, _vp,
                                           ctypes.c_uint32, P(OpAggregates)]
+            lib.opattr_write_profile.argtypes = [ctypes.c_char_p, P(ProfileMeta), P(ProfileNames), P(Kernels), _vp,
+                                                 _vp, _vp, _vp, _vp, _vp, ctypes.c_int64, ctypes.c_uint32,
+                                                 P(OpAggregates), P(ctypes.c_int64)]
+            lib.opattr_write_profile.restype = ctypes.c_int
             lib.opattr_destroy.argtypes = [_vp]
             lib.opattr_destroy.restype = None
             lib.opattr_status_string.argtypes = [ctypes.c_int]
@@ -204,6 +218,52 @@ def opattr_rollup(handle, kernels: Kernels, ranges: Ranges, rok_ptr: int | None,
     return library().opattr_rollup(handle, ctypes.byref(kernels), ctypes.byref(ranges), _vp(rok_ptr or 0),
                                    ctypes.byref(ncu), _vp(idx_ptr), ctypes.c_uint32(n_ops), _vp(class_ptr),
                                    ctypes.c_uint32(n_classes), ctypes.byref(out))
+
+
+def write_profile(path: str, k_stream, k_dur, k_name, op_of_kernel, ncu_idx, counters, ops: dict, tier=None,
+                  is_fused=None, fused_with=None, kernel_names=None, op_names=None, op_call_index=None,
+                  meta: dict | None = None, include_kernels: bool = True) -> int:
+    """profile.json (App. A.4) from HOST (numpy) arrays: opattr_write_profile.
+    Returns the number of bytes written; raises OpattrError on failure."""
+    import numpy as np
+    c = lambda a, dt: None if a is None else np.ascontiguousarray(a).view(dt) if np.asarray(a).dtype.itemsize == \
+        np.dtype(dt).itemsize else np.ascontiguousarray(a, dtype=dt)
+    ks, kd, kn = c(k_stream, np.uint8), c(k_dur, np.int64), c(k_name, np.uint32)
+    op, ni = c(op_of_kernel, np.uint32), c(ncu_idx, np.int32)
+    cn = np.ascontiguousarray(counters, dtype=np.float32)
+    tr, fz, fw = c(tier, np.uint8), c(is_fused, np.uint8), c(fused_with, np.uint32)
+    kc, td, mc = (np.ascontiguousarray(ops[k], dtype=np.int64) for k in ("kernel_count", "total_duration_ns",
+                                                                         "matched_count"))
+    agg = np.ascontiguousarray(ops["agg"], dtype=np.float64)
+    p = lambda a: None if a is None else a.ctypes.data
+    K = len(kd)
+    kern = Kernels(p(ks), None, p(kd), p(kn), None, K)
+    out = OpAggregates(p(kc), p(td), p(mc), p(agg))
+    keep = []
+    names = ProfileNames(None, 0, None, None)
+    if kernel_names is not None:
+        arr = (ctypes.c_char_p * len(kernel_names))(*[s.encode() for s in kernel_names])
+        keep.append(arr)
+        names.kernel_name, names.n_kernel_names = ctypes.cast(arr, _vp), len(kernel_names)
+    if op_names is not None:
+        arr = (ctypes.c_char_p * len(op_names))(*[s.encode() for s in op_names])
+        keep.append(arr)
+        names.op_name = ctypes.cast(arr, _vp)
+    ci = c(op_call_index, np.int64)
+    if ci is not None:
+        names.op_call_index = p(ci)
+    m = meta or {}
+    pm = ProfileMeta(*[(m.get(k).encode() if m.get(k) is not None else None)
+                       for k in ("model_name", "device_name", "compile_mode", "capture_timestamp_utc")],
+                     int(bool(include_kernels)))
+    nbytes = ctypes.c_int64(0)
+    st = library().opattr_write_profile(str(path).encode(), ctypes.byref(pm), ctypes.byref(names), ctypes.byref(kern),
+                                        p(op), p(tr), p(fz), p(fw), p(ni), p(cn), cn.shape[0] if cn.ndim == 2 else
+                                        cn.size // N_COUNTERS, int(len(kc)), ctypes.byref(out), ctypes.byref(nbytes))
+    del keep
+    if st != OK:
+        raise OpattrError(st, "opattr_write_profile")
+    return int(nbytes.value)
 
 
 def opattr_match_noalloc(kernels: Kernels, ncu: Ncu, mismatch: str, idx_ptr: int, kind_ptr: int | None,

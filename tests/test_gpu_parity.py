@@ -566,3 +566,29 @@ def test_rollup_rejects(opa):
         ctx.rollup(tr, rk, idx, torch.from_numpy(cm.view(np.int32)).cuda(), 7)
     assert ei.value.status == opa.E_INVALID_ARG
     ctx.close()
+
+
+# ---------------------------------------------------------------- profile.json
+
+def test_profile_from_gpu(opa, tmp_path):
+    """profile.json written from the GPU join's outputs against the one written
+    from the oracle's: the same operators, kernels and tiers; aggregated
+    counters within 1e-9."""
+    t = tracegen.with_tiers(tracegen.generate("gpt2"))
+    g = gpu_run_tiers(t)
+    o = oracle.run_tiers(t)
+    docs = []
+    for r, tag in ((g, "gpu"), (o, "oracle")):
+        path = tmp_path / f"{tag}.json"
+        opa.write_profile(path, t.k_stream, t.k_dur, t.k_name, r["op_of_kernel"], r["ncu_idx"], t.counters, r["ops"],
+                          tier=r["tier"], is_fused=r["is_fused"], fused_with=r["fused_with"])
+        docs.append(json.load(open(path)))
+    a, b = docs
+    assert len(a["operators"]) == len(b["operators"]) and a["unattributed_kernels"] == b["unattributed_kernels"]
+    for x, y in zip(a["operators"], b["operators"]):
+        assert {k: v for k, v in x.items() if k != "aggregated"} == {k: v for k, v in y.items() if k != "aggregated"}
+        for k, v in x["aggregated"].items():
+            w = y["aggregated"][k]
+            assert (v is None) == (w is None), k
+            if v is not None:
+                assert abs(v - w) <= RTOL * abs(w), (k, v, w)
