@@ -461,7 +461,10 @@ def main():
 
     # ---- roofline of the dominant kernel (CUDA events around each launch)
     peak, peak_kind = load_peaks()
-    dom = max(report.items(), key=lambda kv: kv[1][0])
+    # the dominant kernel among those with algorithmic bytes (a search-bound
+    # helper such as the window table has none, so no memory roofline)
+    known = {k: v for k, v in report.items() if k in KERNEL_BYTES and KERNEL_BYTES[k](K, R, M, O) > 0}
+    dom = max((known or report).items(), key=lambda kv: kv[1][0])
     dname, (dms, dcount) = dom
     dbytes = KERNEL_BYTES.get(dname, lambda *a: 0)(K, R, M, O)
     avg_s = dms / 1e3 / max(dcount, 1)
