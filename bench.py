@@ -35,6 +35,7 @@ PATH_BYTES = dict(kernel=29, range=22, ncu=84, op=184)
 KERNEL_BYTES = {
     "agg_ops": lambda K, R, M, O: 96 * K + 188 * O,
     "enclose": lambda K, R, M, O: 14 * K + 20 * R,
+    "enclose_wide": lambda K, R, M, O: 14 * K + 20 * R,
     "agg_fill": lambda K, R, M, O: 12 * K,
     "agg_count": lambda K, R, M, O: 20 * K + 4 * O,
     "match_identity": lambda K, R, M, O: 13 * K,

@@ -291,12 +291,18 @@ struct AccF {
 __device__ __forceinline__ int32_t range_of(const int32_t *rok, const uint32_t *r_op, int64_t k) {
     return rok ? rok[k] : (r_op[k] != OPATTR_OP_NONE ? (int32_t)k : -1);
 }
+template <bool DIRECT>           // DIRECT: one operator per kernel (no range_of_kernel)
+__device__ __forceinline__ int32_t range_of_t(const int32_t *rok, const uint32_t *r_op, int64_t k) {
+    if (DIRECT) return r_op[k] != OPATTR_OP_NONE ? (int32_t)k : -1;
+    return rok[k];
+}
 
 // ------------------------------------------------------------------ count
 // Per kernel: duration >= 0, range index in [-1, R), an attributed range is an
 // operator below n_ops, row index in [-1, M).  Totals: all / attributed time,
 // attributed and matched kernel counts; cnt[op] += 1 per attributed kernel
 // (one atomic per distinct op id of a warp).
+template <bool DIRECT>
 __global__ void k_agg_count(const int64_t *__restrict__ dur, const int32_t *__restrict__ rok,
                             const int32_t *__restrict__ nidx, const uint32_t *__restrict__ r_op, int64_t K, int64_t R,
                             int64_t M, int64_t n_ops, uint32_t *__restrict__ cnt, DevStatus *st) {
@@ -313,7 +319,7 @@ __global__ void k_agg_count(const int64_t *__restrict__ dur, const int32_t *__re
             const int64_t k = k0 + u * stride;
             const bool in = k < K;
             d[u] = in ? dur[k] : 0;
-            r[u] = in ? range_of(rok, r_op, k) : -1;
+            r[u] = in ? range_of_t<DIRECT>(rok, r_op, k) : -1;
             j[u] = in ? nidx[k] : -1;
         }
 #pragma unroll
@@ -358,6 +364,7 @@ __global__ void k_agg_count(const int64_t *__restrict__ dur, const int32_t *__re
 // the few segments that do not.
 constexpr int AF_RUN = 2048;
 
+template <bool DIRECT>
 __global__ void k_agg_fill(const int32_t *__restrict__ rok, const uint32_t *__restrict__ r_op, int64_t K, int64_t R,
                            int64_t n_ops, const uint32_t *__restrict__ off, uint32_t *__restrict__ cur,
                            uint32_t *__restrict__ list, int64_t run) {
@@ -374,13 +381,13 @@ __global__ void k_agg_fill(const int32_t *__restrict__ rok, const uint32_t *__re
         const int64_t k1 = k0 + run < K ? k0 + run : K;
         // ranges loaded two groups ahead, op ids one group ahead, so each
         // step waits only on its own atomic
-        unsigned key_next = key_of(k0 + lane < k1 ? range_of(rok, r_op, k0 + lane) : -1);
-        int32_t r_next = k0 + 32 + lane < k1 ? range_of(rok, r_op, k0 + 32 + lane) : -1;
+        unsigned key_next = key_of(k0 + lane < k1 ? range_of_t<DIRECT>(rok, r_op, k0 + lane) : -1);
+        int32_t r_next = k0 + 32 + lane < k1 ? range_of_t<DIRECT>(rok, r_op, k0 + 32 + lane) : -1;
         for (int64_t kb = k0; kb < k1; kb += 32) {
             const int64_t k = kb + lane;
             const unsigned key = key_next;
             key_next = key_of(r_next);
-            r_next = k + 64 < k1 ? range_of(rok, r_op, k + 64) : -1;
+            r_next = k + 64 < k1 ? range_of_t<DIRECT>(rok, r_op, k + 64) : -1;
             const unsigned peers = __match_any_sync(0xffffffffu, key);
             const int leader = __ffs(peers) - 1;
             unsigned base = 0;
@@ -874,7 +881,8 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     cudaMemsetAsync(cur, 0, sizeof(uint32_t) * (O + 1), c.stream);
     cudaMemsetAsync(nlong, 0, sizeof(unsigned), c.stream);
     if (K > 0)
-        launch(c, "agg_count", k_agg_count, dim3(grid_for(K, 256 * 4, REDUCE_GRID)), dim3(256), 0, kern->dur_ns, rok,
+        launch(c, "agg_count", rok ? k_agg_count<false> : k_agg_count<true>, dim3(grid_for(K, 256 * 4, REDUCE_GRID)),
+               dim3(256), 0, kern->dur_ns, rok,
                nidx, rng->op_id, K, R, M, O, cnt, c.d_status);
     AggIn in;
     in.dur = kern->dur_ns;
@@ -892,7 +900,8 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
             cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
             const int64_t warps = (int64_t)std::max(1, sms) * 64;
             const int64_t run = std::min<int64_t>(AF_RUN, std::max<int64_t>(32, ((K + warps - 1) / warps + 31) / 32 * 32));
-            launch(c, "agg_fill", k_agg_fill, dim3(grid_for(K, 256 / 32 * run, 65535)), dim3(256), 0, rok,
+            launch(c, "agg_fill", rok ? k_agg_fill<false> : k_agg_fill<true>, dim3(grid_for(K, 256 / 32 * run, 65535)),
+                   dim3(256), 0, rok,
                    rng->op_id, K, R, O, (const uint32_t *)off, cur, list, run);
         }
         launch(c, "agg_long_list", k_agg_long_list, dim3(grid_for(O, 256, 4096)), dim3(256), 0,

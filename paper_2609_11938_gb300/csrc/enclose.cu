@@ -26,8 +26,12 @@ namespace opattr {
 constexpr int LEVELS = N_LEVELS;
 constexpr int ENC_THREADS = 256;
 constexpr int ENC_TILE = 2048;          // kernels per tile
-constexpr int ENC_WIN_CAP = 3072;       // staged range entries per tile
-constexpr int ENC_ACT_CAP = 2048;       // active (stream, depth) levels per tile
+// Shared-memory capacities: staged range entries and active (stream, depth)
+// levels per tile.  With few levels a compact layout (and 64 registers)
+// keeps four blocks per SM; a tile that outgrows it is deferred to the wide
+// layout, which handles any tile (overflowing ones by global searches).
+constexpr int ENC_WIN_SMALL = 1024, ENC_ACT_SMALL = 256;
+constexpr int ENC_WIN_WIDE = 3072, ENC_ACT_WIDE = 2048;
 constexpr int ENC_CHUNK = ENC_TILE / ENC_THREADS;   // consecutive same-stream kernels per thread
 constexpr uint32_t KIND_OP = 0, KIND_NONOP = 1, KIND_STRUCT = 2;
 
@@ -305,15 +309,20 @@ struct EncArgs {
     const uint8_t *ndepth;      // [256] levels of a stream (depths 0 .. n-1)
     int32_t *out_range;
     uint8_t *out_nop;
+    const uint32_t *tiles;      // tiles to process (deferred ones), or NULL for 0 .. nt-1
+    const unsigned *ntiles;     // their count (device), with `tiles`
+    uint32_t *deferred;         // compact-layout pass: tiles handed to the wide pass
+    unsigned *ndeferred;
 };
 
+template <int WIN, int ACT>
 struct EncSmem {
-    uint32_t ws[ENC_WIN_CAP];       // staged start, relative to tile base (+1, clamped)
-    uint32_t we[ENC_WIN_CAP];       // staged end, same encoding
-    uint32_t wi[ENC_WIN_CAP];       // staged lvl_info
-    uint16_t act_off[ENC_ACT_CAP];  // window offset of an active level
-    uint16_t act_cnt[ENC_ACT_CAP];  // window length
-    int32_t act_gpos[ENC_ACT_CAP];  // global level position of the window's first entry (-1 none)
+    uint32_t ws[WIN];               // staged start, relative to tile base (+1, clamped)
+    uint32_t we[WIN];               // staged end, same encoding
+    uint32_t wi[WIN];               // staged lvl_info
+    uint16_t act_off[ACT];          // window offset of an active level
+    uint16_t act_cnt[ACT];          // window length
+    int32_t act_gpos[ACT];          // global level position of the window's first entry (-1 none)
     uint16_t sbase[256];            // first active slot of a present stream
     uint32_t kt[ENC_TILE];          // the tile's kernel times, relative to the tile base (+1, clamped)
     uint8_t ks[ENC_TILE];           // the tile's kernel streams
@@ -331,10 +340,10 @@ __device__ __forceinline__ uint32_t rel32(long long x, long long base) {
     return v <= 0 ? 0u : (v >= 0xFFFFFFFFll ? 0xFFFFFFFFu : (uint32_t)v);
 }
 
-__global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    EncSmem &S = *reinterpret_cast<EncSmem *>(smem_raw);
-    const int64_t t = blockIdx.x;
+// One tile.  DEFER: a tile that outgrows the layout is handed on (its index
+// appended to A.deferred) instead of taking the global-search path.
+template <int WIN, int ACT, bool DEFER>
+__device__ __forceinline__ void enclose_tile(const EncArgs &A, EncSmem<WIN, ACT> &S, const int64_t t) {
     const int64_t pos0 = t * ENC_TILE;
     const int64_t cnt = A.K - pos0 < ENC_TILE ? A.K - pos0 : ENC_TILE;
     if (threadIdx.x < 8) S.present[threadIdx.x] = 0;
@@ -372,15 +381,15 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
         unsigned n = ((S.present[s >> 5] >> (s & 31)) & 1u) ? A.ndepth[s] : 0u;
         unsigned tot;
         unsigned off = block_exclusive_scan<unsigned>(n, S.wbuf, &tot);
-        S.sbase[s] = (uint16_t)(off < ENC_ACT_CAP ? off : ENC_ACT_CAP);
+        S.sbase[s] = (uint16_t)(off < ACT ? off : ACT);
         if (threadIdx.x == 0) S.nact = (int)tot;
-        if (tot <= ENC_ACT_CAP && n) {
+        if (tot <= ACT && n) {
             const unsigned cb = A.cbase[s];
             for (unsigned d = 0; d < n; ++d) S.act_off[off + d] = (uint16_t)(cb + d);   // compact level, for now
         }
         __syncthreads();
         // window bounds of every active level, one thread per level
-        if (tot <= ENC_ACT_CAP) {
+        if (tot <= ACT) {
             for (unsigned a = threadIdx.x; a < tot; a += ENC_THREADS) {
                 const int l = S.act_off[a];
                 const int32_t lo = A.P[t * A.nl + l], hi = A.P[(t + 1) * A.nl + l];
@@ -395,7 +404,7 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
     __syncthreads();
     // span of the tile: its last kernel (time order) minus its first
     const long long tlast = A.k_start[A.korder ? A.korder[pos0 + cnt - 1] : pos0 + cnt - 1];
-    int slow = S.nact > ENC_ACT_CAP || (tlast - tbase) >= 0xFFFFFFF0ll;
+    int slow = S.nact > ACT || (tlast - tbase) >= 0xFFFFFFF0ll;
     if (!slow) {
         // window offsets: exclusive scan of counts over active slots
         unsigned carry = 0;
@@ -409,7 +418,7 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
         }
         if (threadIdx.x == 0) S.nwin = (int)carry;
         __syncthreads();
-        slow = S.nwin > ENC_WIN_CAP;
+        slow = S.nwin > WIN;
     }
     if (!slow) {
         // stage the windows: one thread per staged entry (its level found by a
@@ -536,6 +545,10 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
         }
         return;
     }
+    if (DEFER) {                           // the wide pass takes this tile
+        if (threadIdx.x == 0) A.deferred[atomicAdd(A.ndeferred, 1u)] = (uint32_t)t;
+        return;
+    }
     // slow tile: search the global level lists inside the window bounds
     for (int j = threadIdx.x; j < cnt; j += ENC_THREADS) {
         const int64_t p = pos0 + j;
@@ -563,6 +576,27 @@ __global__ void __launch_bounds__(ENC_THREADS) k_enclose(EncArgs A) {
         }
         A.out_range[k] = ans;
         if (A.out_nop) A.out_nop[k] = (uint8_t)nop;
+    }
+}
+
+using EncSmemSmall = EncSmem<ENC_WIN_SMALL, ENC_ACT_SMALL>;
+using EncSmemWide = EncSmem<ENC_WIN_WIDE, ENC_ACT_WIDE>;
+
+// Compact layout, one tile per block, four blocks per SM; tiles that outgrow
+// it are deferred to k_enclose_wide.
+__global__ void __launch_bounds__(ENC_THREADS, 4) k_enclose(EncArgs A) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    enclose_tile<ENC_WIN_SMALL, ENC_ACT_SMALL, true>(A, *reinterpret_cast<EncSmemSmall *>(smem_raw), blockIdx.x);
+}
+
+// Wide layout: every tile (A.tiles NULL) or the deferred ones.
+__global__ void __launch_bounds__(ENC_THREADS) k_enclose_wide(EncArgs A) {
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    EncSmemWide &S = *reinterpret_cast<EncSmemWide *>(smem_raw);
+    const int64_t n = A.tiles ? (int64_t)*A.ntiles : A.nt;
+    for (int64_t i = blockIdx.x; i < n; i += gridDim.x) {
+        enclose_tile<ENC_WIN_WIDE, ENC_ACT_WIDE, false>(A, S, A.tiles ? (int64_t)A.tiles[i] : i);
+        __syncthreads();                   // the next tile reuses the shared memory
     }
 }
 
@@ -599,7 +633,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     nd.add<uint32_t>(radix_hist_elems(R)).add<uint32_t>(part_n);
     nd.add<int64_t>(R).add<int64_t>(R).add<uint32_t>(R);
     nd.add<uint16_t>(LEVELS).add<uint16_t>(256).add<uint8_t>(256).add<uint8_t>(LEVELS);
-    nd.add<int32_t>((nt + 1) * (int64_t)LEVELS);
+    nd.add<int32_t>((nt + 1) * (int64_t)LEVELS).add<uint32_t>(nt).add<unsigned>(1);
     size_t need = nd.bytes + kernel_order_scratch(K) + 4096;
     opattr_status st = ensure_arena(c, need);
     if (st) return st;
@@ -662,6 +696,9 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     uint16_t *d_cbase = a.take<uint16_t>(256);
     uint8_t *d_ndep = a.take<uint8_t>(256);
     uint8_t *d_cmap = a.take<uint8_t>(LEVELS);
+    uint32_t *deferred = a.take<uint32_t>(nt);
+    unsigned *ndeferred = a.take<unsigned>(1);
+    if (!deferred || !ndeferred) return OPATTR_E_OOM;
     int32_t *P = a.take<int32_t>((nt + 1) * (int64_t)(nl > 0 ? nl : 1));
     if (!rk0 || !rk1 || !rv0 || !rv1 || !hist || !ls || !le || !li || !d_loc || !d_cbase || !d_ndep || !d_cmap || !P)
         return OPATTR_E_OOM;
@@ -756,10 +793,29 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
             A.out_nop = out_nop;
             static unsigned attr_done = 0;
             if (c.device < 32 && !(attr_done & (1u << c.device))) {
-                cudaFuncSetAttribute(k_enclose, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(EncSmem));
+                cudaFuncSetAttribute(k_enclose, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(EncSmemSmall));
+                cudaFuncSetAttribute(k_enclose_wide, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)sizeof(EncSmemWide));
                 attr_done |= 1u << c.device;
             }
-            launch(c, "enclose", k_enclose, dim3((unsigned)nt), dim3(ENC_THREADS), sizeof(EncSmem), A);
+            A.tiles = nullptr;
+            A.ntiles = nullptr;
+            A.deferred = deferred;
+            A.ndeferred = ndeferred;
+            if (nl <= ENC_ACT_SMALL) {
+                // compact layout first; the tiles it defers go through the wide one
+                cudaMemsetAsync(ndeferred, 0, sizeof(unsigned), c.stream);
+                launch(c, "enclose", k_enclose, dim3((unsigned)nt), dim3(ENC_THREADS), sizeof(EncSmemSmall), A);
+                A.tiles = deferred;
+                A.ntiles = ndeferred;
+                int sms = 0;
+                cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
+                launch(c, "enclose_wide", k_enclose_wide, dim3((unsigned)std::min<int64_t>(nt, 3 * std::max(1, sms))),
+                       dim3(ENC_THREADS), sizeof(EncSmemWide), A);
+            } else {
+                launch(c, "enclose_wide", k_enclose_wide, dim3((unsigned)nt), dim3(ENC_THREADS), sizeof(EncSmemWide),
+                       A);
+            }
         }
         if ((st = read_status(c))) return st;
         if ((st = status_from_err(c.h_status->err))) return st;

@@ -592,3 +592,16 @@ def test_profile_from_gpu(opa, tmp_path):
             assert (v is None) == (w is None), k
             if v is not None:
                 assert abs(v - w) <= RTOL * abs(w), (k, v, w)
+
+
+@pytest.mark.parametrize("kids,p_kernel", [(1.2, 0.3), (2.0, 0.55), (3.0, 0.7)])
+def test_enclose_dense_ranges(opa, kids, p_kernel):
+    """Range-dense traces (about one range per kernel and fewer): tiles whose
+    range windows outgrow the compact shared-memory layout are deferred to the
+    wide layout, some or all of them; the result is the oracle's."""
+    t = tracegen.generate("large", n_kernels=200_000, n_streams=2, max_depth=8, kids_mean=kids,
+                          p_kernel_child=p_kernel, uncovered_frac=0.0)
+    g = gpu_run(t)
+    o = oracle.run(t, enclose_mode="indexed")
+    np.testing.assert_array_equal(g["range_of_kernel"], o["range_of_kernel"])
+    np.testing.assert_array_equal(g["n_op_enclosing"], o["n_op_enclosing"])
