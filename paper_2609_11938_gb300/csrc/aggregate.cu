@@ -410,6 +410,7 @@ constexpr uint32_t AG_SHORT_MAX = 64;           // segments up to this length: s
 
 constexpr uint32_t AG_HUGE = 256;               // longer segments: split into pieces over several warps
 constexpr uint32_t AG_PIECE = 1024;              // kernels of a huge op per warp of the pieces pass
+constexpr uint32_t AG_BLOCK_SORT_MAX = 4096;     // longer huge segments: placed by a counting pass, not sorted
 
 // Ops with segments longer than `limit`, listed (in no particular order).
 __global__ void k_agg_long_list(const uint32_t *__restrict__ off, int64_t n_ops, uint32_t limit,
@@ -442,12 +443,13 @@ __device__ void bitonic_smem(uint32_t *a, int n2) {     // n2 a power of two; th
 
 __global__ void __launch_bounds__(SL_THREADS) k_agg_sort_long(const uint32_t *__restrict__ off,
                                                               const uint32_t *__restrict__ longs,
-                                                              const unsigned *__restrict__ nlong, uint32_t *list,
-                                                              uint32_t *tmp) {
+                                                              const unsigned *__restrict__ nlong, uint32_t min_len,
+                                                              uint32_t max_len, uint32_t *list, uint32_t *tmp) {
     __shared__ uint32_t a[SL_SMEM];
     const unsigned n_long = *nlong;
     for (unsigned li = blockIdx.x; li < n_long; li += gridDim.x) {
         const uint32_t o = longs[li], s0 = off[o], len = off[o + 1] - s0;
+        if (len < min_len || len > max_len) continue;      // uniform per block
         uint32_t *seg = list + s0, *alt = tmp + s0;
         // runs of SL_SMEM (the whole segment if it fits)
         for (uint32_t r0 = 0; r0 < len; r0 += SL_SMEM) {
@@ -506,7 +508,7 @@ __global__ void __launch_bounds__(SL_THREADS) k_agg_sort_long(const uint32_t *__
 // kernel is added, the counter rows and durations of the next two arrive in
 // per-thread shared-memory slots by asynchronous copy (cp.async), with their
 // row indices loaded a step earlier still.
-constexpr int AG_THREADS = 128;
+constexpr int AG_THREADS = 128;                // five blocks per SM (96 registers, a few spilled)
 constexpr int AG_WARPS = AG_THREADS / 32;
 constexpr int AG_CHUNK = 64;                    // op ids per warp and chunk
 constexpr int AG_LBUCKETS = 32;
@@ -534,7 +536,7 @@ __device__ __forceinline__ void cp_async_wait() {
     asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-__global__ void __launch_bounds__(AG_THREADS) k_agg_ops(const uint32_t *__restrict__ off, uint32_t *__restrict__ list,
+__global__ void __launch_bounds__(AG_THREADS, 5) k_agg_ops(const uint32_t *__restrict__ off, uint32_t *__restrict__ list,
                                                           AggIn A, DevStatus *st) {
     __shared__ uint32_t lcount_s[AG_WARPS][AG_LBUCKETS];
     __shared__ uint8_t order_s[AG_WARPS][AG_CHUNK];
@@ -711,26 +713,89 @@ __device__ __forceinline__ void acc_merge(Acc &a, const Acc &b) {
 // Piece offsets of the listed long ops, one block: poff[j] = pieces of the
 // ops listed before j (an op longer than `huge` has ceil(len / AG_PIECE)
 // pieces, a shorter one none); poff[nlong] = all pieces.
+// info (may be NULL) receives {listed ops, pieces, longest huge op, kernels
+// in huge ops, huge ops}; hop (with info) the huge ops in list order.
 __global__ void __launch_bounds__(1024) k_agg_piece_offsets(const uint32_t *__restrict__ off,
                                                             const uint32_t *__restrict__ longs,
                                                             const unsigned *__restrict__ nlong, uint32_t huge,
-                                                            uint32_t *__restrict__ poff) {
+                                                            uint32_t *__restrict__ poff, uint32_t *__restrict__ info,
+                                                            uint32_t *__restrict__ hop) {
     __shared__ uint32_t wbuf[33];
     const int64_t n = *nlong;
-    uint32_t carry = 0;
+    uint32_t carry = 0, longest = 0, kern = 0, hcarry = 0;
     for (int64_t b = 0; b < n; b += 1024) {
         const int64_t j = b + threadIdx.x;
-        uint32_t np = 0;
+        uint32_t np = 0, o = 0;
         if (j < n) {
-            const uint32_t o = longs[j], len = off[o + 1] - off[o];
+            o = longs[j];
+            const uint32_t len = off[o + 1] - off[o];
             np = len > huge ? (len + AG_PIECE - 1) / AG_PIECE : 0u;
+            if (np) {
+                longest = len > longest ? len : longest;
+                kern += len;
+            }
         }
         uint32_t tot;
         const uint32_t ex = block_exclusive_scan<uint32_t>(np, wbuf, &tot);
         if (j < n) poff[j] = carry + ex;
         carry += tot;
+        if (info) {
+            uint32_t htot;
+            const uint32_t hx = block_exclusive_scan<uint32_t>(np ? 1u : 0u, wbuf, &htot);
+            if (np) hop[hcarry + hx] = o;
+            hcarry += htot;
+        }
     }
     if (threadIdx.x == 0) poff[n] = carry;
+    if (info) {
+        const uint32_t ksum = block_sum<uint32_t>(kern, wbuf);
+        __shared__ uint32_t lmax;
+        if (threadIdx.x == 0) lmax = 0;
+        __syncthreads();
+        atomicMax(&lmax, longest);
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            info[0] = (uint32_t)n;
+            info[1] = carry;
+            info[2] = lmax;
+            info[3] = ksum;
+            info[4] = hcarry;
+        }
+    }
+}
+
+// Huge ops' segments in ascending kernel index without sorting: with at most
+// 256 huge ops, one counting pass over all kernels in index order, the digit
+// being the index of the kernel's op among the huge ops, writes each such
+// kernel to its op's segment at its rank among the op's kernels.
+struct HugeDigit {
+    const int32_t *rok;
+    const uint32_t *r_op;
+    int64_t R, n_ops;
+    const uint32_t *hidx;        // [n_ops] index of a huge op among the huge ops, else 0xFFFFFFFF
+    __device__ __forceinline__ unsigned operator()(int64_t k) const {
+        const int32_t r = range_of(rok, r_op, k);
+        if (r < 0 || r >= R) return RADIX_BINS;
+        const uint32_t op = r_op[r];
+        if ((int64_t)op >= n_ops) return RADIX_BINS;
+        const uint32_t j = hidx[op];
+        return j < RADIX_BINS ? j : (unsigned)RADIX_BINS;
+    }
+};
+struct HugePlace {
+    const uint32_t *hist;        // scanned digit-major histogram: hist[j * ntiles] = start of digit j
+    int64_t ntiles;
+    const uint32_t *hop, *off;   // the huge ops; the segment offsets
+    uint32_t *list;
+    __device__ __forceinline__ unsigned operator()(int64_t k, uint32_t dest, unsigned j) const {
+        list[off[hop[j]] + (dest - hist[(int64_t)j * ntiles])] = (uint32_t)k;
+        return 0u;
+    }
+    __device__ __forceinline__ void done(unsigned) const {}
+};
+__global__ void k_huge_index(const uint32_t *__restrict__ hop, int64_t n_huge, uint32_t *__restrict__ hidx) {
+    for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < n_huge; c += (int64_t)gridDim.x * blockDim.x)
+        hidx[hop[c]] = (uint32_t)c;
 }
 
 // A lane's run of a piece with the fast accumulator: returns false when a
@@ -862,7 +927,9 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     nd.add<uint32_t>(O + 1).add<uint32_t>(O + 1).add<uint32_t>(O + 1).add<uint32_t>(K).add<uint32_t>(K);
     nd.add<uint32_t>(O + 1).add<unsigned>(1).add<unsigned>(1);
     nd.add<uint32_t>(O + 1).add<Acc>(K / AG_PIECE + (K / (AG_SHORT_MAX + 1)) + 1);   // pieces per op, partials
-    nd.add<uint32_t>(scan_scratch_elems(O + 1));
+    nd.add<uint32_t>(scan_scratch_elems(std::max<int64_t>(O + 1, radix_hist_elems(K))));
+    nd.add<uint32_t>(O + 1).add<uint32_t>(radix_hist_elems(K)).add<uint32_t>(8);   // huge-op index, histogram, info
+    nd.add<uint32_t>(O + 1);                                                         // huge ops
     opattr_status st = ensure_arena(c, nd.bytes + 4096);
     if (st) return st;
     Arena a(c);
@@ -875,7 +942,10 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     Acc *partials = a.take<Acc>(K / AG_PIECE + (K / (AG_SHORT_MAX + 1)) + 1);
     if (!npc || !partials) return OPATTR_E_OOM;
     cudaMemsetAsync(ctr, 0, sizeof(unsigned), c.stream);
-    uint32_t *part = a.take<uint32_t>(scan_scratch_elems(O + 1));
+    uint32_t *part = a.take<uint32_t>(scan_scratch_elems(std::max<int64_t>(O + 1, radix_hist_elems(K))));
+    uint32_t *hidx = a.take<uint32_t>(O + 1), *hhist = a.take<uint32_t>(radix_hist_elems(K));
+    uint32_t *info = a.take<uint32_t>(8), *hop = a.take<uint32_t>(O + 1);
+    if (!hidx || !hhist || !info || !hop) return OPATTR_E_OOM;
     if (!cnt || !off || !cur || !list || !tmp || !longs || !nlong || !part) return OPATTR_E_OOM;
     cudaMemsetAsync(cnt, 0, sizeof(uint32_t) * (O + 1), c.stream);
     cudaMemsetAsync(cur, 0, sizeof(uint32_t) * (O + 1), c.stream);
@@ -907,19 +977,45 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
         launch(c, "agg_long_list", k_agg_long_list, dim3(grid_for(O, 256, 4096)), dim3(256), 0,
                (const uint32_t *)off, O, AG_SHORT_MAX, longs, nlong);
         launch(c, "agg_piece_offsets", k_agg_piece_offsets, dim3(1), dim3(1024), 0, (const uint32_t *)off,
-               (const uint32_t *)longs, (const unsigned *)nlong, AG_HUGE, npc);
+               (const uint32_t *)longs, (const unsigned *)nlong, AG_HUGE, npc, info, hop);
         int sms = 0;
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
-        launch(c, "agg_sort_long", k_agg_sort_long, dim3(2 * std::max(1, sms)), dim3(SL_THREADS), 0, (const uint32_t *)off,
-               (const uint32_t *)longs, (const unsigned *)nlong, list, tmp);
-        launch(c, "agg_pieces", k_agg_pieces, dim3(4 * std::max(1, sms)), dim3(256), 0, (const uint32_t *)off,
-               (const uint32_t *)list, (const uint32_t *)longs, (const unsigned *)nlong, (const uint32_t *)npc, in,
-               partials);
-        launch(c, "agg_long_ops", k_agg_long_ops, dim3(2 * std::max(1, sms)), dim3(FIN_THREADS), 0,
-               (const uint32_t *)longs,
-               (const unsigned *)nlong, (const uint32_t *)npc, (const Acc *)partials, 0, in, c.d_status);
+        // long segments the ops pass walks: sorted first
+        launch(c, "agg_sort_long", k_agg_sort_long, dim3(2 * std::max(1, sms)), dim3(SL_THREADS), 0,
+               (const uint32_t *)off, (const uint32_t *)longs, (const unsigned *)nlong, AG_SHORT_MAX + 1, AG_HUGE,
+               list, tmp);
+        // whether huge ops exist is read while the ops pass runs
+        if (!c.ev_aux && cudaEventCreateWithFlags(&c.ev_aux, cudaEventDisableTiming) != cudaSuccess)
+            return cuda_status(c, cudaGetLastError());
+        cudaMemcpyAsync(c.h_levels, info, 5 * sizeof(uint32_t), cudaMemcpyDeviceToHost, c.stream);
+        cudaEventRecord(c.ev_aux, c.stream);
         launch(c, "agg_ops", k_agg_ops, dim3(ops_grid(c, O)), dim3(AG_THREADS), 0,
                (const uint32_t *)off, list, in, c.d_status);
+        if (cudaEventSynchronize(c.ev_aux) != cudaSuccess) return cuda_status(c, cudaGetLastError());
+        const uint32_t pieces = c.h_levels[1], longest = c.h_levels[2], n_huge = c.h_levels[4];
+        if (pieces > 0) {
+            if (n_huge <= (uint32_t)RADIX_BINS && longest > AG_BLOCK_SORT_MAX && K > 0) {
+                // very long segments: placed in kernel order by one counting pass
+                cudaMemsetAsync(hidx, 0xFF, sizeof(uint32_t) * (O + 1), c.stream);
+                launch(c, "huge_index", k_huge_index, dim3(grid_for(n_huge, 256, 4096)), dim3(256), 0,
+                       (const uint32_t *)hop, (int64_t)n_huge, hidx);
+                const HugeDigit dg{rok, rng->op_id, R, O, hidx};
+                digit_offsets(c, dg, K, hhist, part);
+                const int64_t ntiles = (K + RADIX_TILE - 1) / RADIX_TILE;
+                digit_rank(c, "huge_place", dg, K, hhist,
+                           HugePlace{hhist, ntiles, (const uint32_t *)hop, (const uint32_t *)off, list});
+            } else {
+                launch(c, "agg_sort_long", k_agg_sort_long, dim3(2 * std::max(1, sms)), dim3(SL_THREADS), 0,
+                       (const uint32_t *)off, (const uint32_t *)longs, (const unsigned *)nlong, AG_HUGE + 1,
+                       0xFFFFFFFFu, list, tmp);
+            }
+            launch(c, "agg_pieces", k_agg_pieces, dim3(4 * std::max(1, sms)), dim3(256), 0, (const uint32_t *)off,
+                   (const uint32_t *)list, (const uint32_t *)longs, (const unsigned *)nlong, (const uint32_t *)npc,
+                   in, partials);
+            launch(c, "agg_long_ops", k_agg_long_ops, dim3(2 * std::max(1, sms)), dim3(FIN_THREADS), 0,
+                   (const uint32_t *)longs, (const unsigned *)nlong, (const uint32_t *)npc,
+                   (const Acc *)partials, 0, in, c.d_status);
+        }
     }
     if ((st = read_status(c))) return st;
     if (c.h_status->err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
@@ -1059,7 +1155,7 @@ opattr_status do_rollup(Ctx &c, const opattr_kernels *kern, const opattr_ranges 
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
         launch(c, "class_iota", k_iota_u32, dim3(grid_for(C, 256, 4096)), dim3(256), 0, cls, C, ncls);
         launch(c, "agg_piece_offsets", k_agg_piece_offsets, dim3(1), dim3(1024), 0, (const uint32_t *)off,
-               (const uint32_t *)cls, (const unsigned *)ncls, 0u, poff);
+               (const uint32_t *)cls, (const unsigned *)ncls, 0u, poff, (uint32_t *)nullptr, (uint32_t *)nullptr);
         if (K > 0)
             launch(c, "agg_pieces", k_agg_pieces, dim3(4 * std::max(1, sms)), dim3(256), 0, (const uint32_t *)off,
                    (const uint32_t *)list, (const uint32_t *)cls, (const unsigned *)ncls, (const uint32_t *)poff, in,

@@ -172,6 +172,7 @@ opattr_status opattr_create(opattr_ctx **out, int device, void *cuda_stream, con
         if (c.h_status) cudaFreeHost(c.h_status);
         if (c.h_init) cudaFreeHost(c.h_init);
         if (c.h_levels) cudaFreeHost(c.h_levels);
+        if (c.ev_aux) cudaEventDestroy(c.ev_aux);
         delete x;
         return OPATTR_E_OOM;
     }

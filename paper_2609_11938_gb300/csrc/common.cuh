@@ -84,7 +84,9 @@ struct Ctx {
     DevStatus *d_status = nullptr;
     DevStatus *h_status = nullptr;   // pinned mirror
     DevStatus *h_init = nullptr;     // pinned reset template
-    uint32_t *h_levels = nullptr;    // pinned host copy of the enclosure's level offsets [N_LEVELS + 1]
+    uint32_t *h_levels = nullptr;    // pinned host copy of the enclosure's level offsets [N_LEVELS + 1];
+                                     // the aggregation reuses it for a few values read mid-call
+    cudaEvent_t ev_aux = nullptr;    // marks a mid-call host read (created on first use)
     // launch accounting
     int64_t launches = 0;
     bool timing = false;

@@ -76,7 +76,7 @@ struct StreamPairs {
     int32_t *out_idx;
     uint8_t *out_kind;
     DevStatus *st;
-    __device__ __forceinline__ unsigned operator()(int64_t j, uint32_t dest) const {
+    __device__ __forceinline__ unsigned operator()(int64_t j, uint32_t dest, unsigned) const {
         const uint32_t k = rk ? rk[j] : (uint32_t)j;
         const uint32_t r = pn[dest];
         const uint32_t x = kname[k], y = nname[r];

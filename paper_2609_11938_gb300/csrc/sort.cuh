@@ -41,9 +41,9 @@ void radix_sort_pairs(Ctx &c, K *k0, uint32_t *v0, K *k1, uint32_t *v1, int64_t 
 // digit(i) in [0, RADIX_BINS) for element i < n, or RADIX_BINS to leave the
 // element out.  digit_offsets counts digits per tile of RADIX_TILE elements
 // (digit-major matrix in `hist`, radix_hist_elems(n) entries) and scans the
-// matrix; digit_rank then hands every counted element to epi(i, dest), where
-// dest is the position a stable sort by digit would give it, without moving
-// anything itself.  epi returns problem bits; epi.done(bits) runs in every
+// matrix; digit_rank then hands every counted element to epi(i, dest, digit),
+// where dest is the position a stable sort by digit would give it, without
+// moving anything itself.  epi returns problem bits; epi.done(bits) runs in every
 // thread at the end (for warp votes).  Same tiles and ranking as the radix
 // sort: warps own consecutive 512-element runs, ranked 32 at a time with
 // __match_any_sync peer groups.
@@ -114,7 +114,7 @@ __global__ void __launch_bounds__(RADIX_THREADS) k_digit_rank(DigitFn digit, int
 #pragma unroll
     for (int it = 0; it < RADIX_ITEMS; ++it) {
         const int64_t i = base + it * 32 + lane;
-        if (dig[it] < RADIX_BINS) bits |= epi(i, gbase[dig[it]] + wcnt[w * RADIX_BINS + dig[it]] + rank[it]);
+        if (dig[it] < RADIX_BINS) bits |= epi(i, gbase[dig[it]] + wcnt[w * RADIX_BINS + dig[it]] + rank[it], dig[it]);
     }
     epi.done(bits);
 }
