@@ -166,13 +166,14 @@ opattr_status opattr_create(opattr_ctx **out, int device, void *cuda_stream, con
     fail = fail || cudaMallocHost(&c.h_status, sizeof(DevStatus)) != cudaSuccess;
     fail = fail || cudaMallocHost(&c.h_init, sizeof(DevStatus)) != cudaSuccess;
     fail = fail || cudaMallocHost(&c.h_levels, sizeof(uint32_t) * (N_LEVELS + 1)) != cudaSuccess;
+    fail = fail || cudaMallocHost(&c.h_stage, STAGE_BYTES) != cudaSuccess;
     if (fail) {
         cudaGetLastError();
         if (c.d_status) cudaFree(c.d_status);
         if (c.h_status) cudaFreeHost(c.h_status);
         if (c.h_init) cudaFreeHost(c.h_init);
         if (c.h_levels) cudaFreeHost(c.h_levels);
-        if (c.ev_aux) cudaEventDestroy(c.ev_aux);
+        if (c.h_stage) cudaFreeHost(c.h_stage);
         delete x;
         return OPATTR_E_OOM;
     }

@@ -70,6 +70,7 @@ struct TimingSlot {
 };
 
 constexpr int N_LEVELS = 256 * 32;   // (stream, depth) levels of the enclosure
+constexpr size_t STAGE_BYTES = 32768;  // pinned staging of host-built tables (one copy per call)
 
 struct Ctx {
     int device = 0;
@@ -87,6 +88,7 @@ struct Ctx {
     uint32_t *h_levels = nullptr;    // pinned host copy of the enclosure's level offsets [N_LEVELS + 1];
                                      // the aggregation reuses it for a few values read mid-call
     cudaEvent_t ev_aux = nullptr;    // marks a mid-call host read (created on first use)
+    unsigned char *h_stage = nullptr; // pinned staging for small host-built tables [STAGE_BYTES]
     // launch accounting
     int64_t launches = 0;
     bool timing = false;

@@ -244,11 +244,12 @@ __global__ void k_validate_levels(const uint8_t *__restrict__ stream, const uint
 // P[t * nl + l] = (last position p of level l with lvl_start[p] <= b_t) - level
 // start, or -1; b_t = start of the time-ordered kernel t*ENC_TILE for
 // t < nt, and of the last kernel for t = nt.  The b_t do not decrease, so
-// one thread takes WT_CHUNK consecutive tiles of one level: a binary search
+// one thread takes `chunk` consecutive tiles of one level: a binary search
 // for the first, then an exponential search forward from the previous
 // answer for each next one (cost logarithmic in the entries passed, however
 // unevenly a level's ranges fall between tiles).  Neighbouring threads take
-// neighbouring levels, so the rows of P are written together.
+// neighbouring levels, so the rows of P are written together.  Small tables
+// take chunks of one tile (every search in parallel).
 constexpr int WT_CHUNK = 16;
 __device__ __forceinline__ long long tile_bound(const int64_t *k_start, const uint32_t *korder, int64_t K, int64_t nt,
                                                 int64_t t) {
@@ -258,15 +259,15 @@ __device__ __forceinline__ long long tile_bound(const int64_t *k_start, const ui
 __global__ void k_window_table(const int64_t *__restrict__ ls, const uint32_t *__restrict__ lvl_off,
                                const uint16_t *__restrict__ level_of_compact, int nl,
                                const int64_t *__restrict__ k_start, const uint32_t *__restrict__ korder, int64_t K,
-                               int64_t nt, int32_t *__restrict__ P) {
-    const int64_t nchunk = (nt + 1 + WT_CHUNK - 1) / WT_CHUNK;
+                               int64_t nt, int chunk, int32_t *__restrict__ P) {
+    const int64_t nchunk = (nt + 1 + chunk - 1) / chunk;
     const int64_t total = nchunk * nl;
     for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < total; q += (int64_t)gridDim.x * blockDim.x) {
         const int64_t ch = q / nl;
         const int l = (int)(q - ch * nl);
         const uint32_t L = level_of_compact[l];
         const int64_t lo = lvl_off[L], hi = lvl_off[L + 1];
-        const int64_t t0 = ch * WT_CHUNK, t1 = t0 + WT_CHUNK < nt + 1 ? t0 + WT_CHUNK : nt + 1;
+        const int64_t t0 = ch * chunk, t1 = t0 + chunk < nt + 1 ? t0 + chunk : nt + 1;
         int64_t x = lo;                       // first position with start > b (for the current tile)
         for (int64_t t = t0; t < t1; ++t) {
             const long long b = tile_bound(k_start, korder, K, nt, t);
@@ -632,7 +633,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     const int64_t part_n = std::max<int64_t>(scan_scratch_elems(radix_hist_elems(R)), scan_scratch_elems(LEVELS + 1));
     nd.add<uint32_t>(radix_hist_elems(R)).add<uint32_t>(part_n);
     nd.add<int64_t>(R).add<int64_t>(R).add<uint32_t>(R);
-    nd.add<uint16_t>(LEVELS).add<uint16_t>(256).add<uint8_t>(256).add<uint8_t>(LEVELS);
+    nd.add<unsigned char>(STAGE_BYTES);
     nd.add<int32_t>((nt + 1) * (int64_t)LEVELS).add<uint32_t>(nt).add<unsigned>(1);
     size_t need = nd.bytes + kernel_order_scratch(K) + 4096;
     opattr_status st = ensure_arena(c, need);
@@ -669,22 +670,29 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
         return read_status(c);
     }
 
-    // ---- compact level table (host side, from the level offsets)
+    // ---- compact level tables (host side, from the level offsets), built in
+    // pinned staging and sent with one copy: level of each compact level
+    // (u16 [LEVELS]), first compact level of a stream (u16 [256]), levels of a
+    // stream (u8 [256]), compact id of a level (u8 [LEVELS], at most 256 levels)
+    constexpr size_t ST_LOC = 0, ST_CBASE = ST_LOC + 2 * LEVELS, ST_NDEP = ST_CBASE + 2 * 256,
+                     ST_CMAP = ST_NDEP + 256, ST_END = ST_CMAP + LEVELS;
+    static_assert(ST_END <= STAGE_BYTES, "staging too small");
     const uint32_t *off = c.h_levels;
-    std::vector<uint16_t> level_of_compact;
-    std::vector<uint16_t> cbase(256, 0);
-    std::vector<uint8_t> ndep(256, 0);
+    uint16_t *level_of_compact = reinterpret_cast<uint16_t *>(c.h_stage + ST_LOC);
+    uint16_t *cbase = reinterpret_cast<uint16_t *>(c.h_stage + ST_CBASE);
+    uint8_t *ndep = c.h_stage + ST_NDEP;
+    uint8_t *cmap = c.h_stage + ST_CMAP;
+    int nl = 0;
     for (int s = 0; s < 256; ++s) {
-        cbase[s] = (uint16_t)level_of_compact.size();
+        cbase[s] = (uint16_t)nl;
         int n = 0;
         while (n < 32 && off[s * 32 + n + 1] > off[s * 32 + n]) {
-            level_of_compact.push_back((uint16_t)(s * 32 + n));
+            level_of_compact[nl++] = (uint16_t)(s * 32 + n);
             n++;
         }
         ndep[s] = (uint8_t)n;
     }
-    const int nl = (int)level_of_compact.size();
-    std::vector<uint8_t> cmap(LEVELS, 0);
+    memset(cmap, 0, LEVELS);
     for (int l = 0; l < nl && l < 256; ++l) cmap[level_of_compact[l]] = (uint8_t)l;
 
     uint64_t *rk0 = a.take<uint64_t>(R), *rk1 = a.take<uint64_t>(R);
@@ -692,21 +700,17 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     uint32_t *hist = a.take<uint32_t>(radix_hist_elems(R));
     int64_t *ls = a.take<int64_t>(R), *le = a.take<int64_t>(R);
     uint32_t *li = a.take<uint32_t>(R);
-    uint16_t *d_loc = a.take<uint16_t>(LEVELS);
-    uint16_t *d_cbase = a.take<uint16_t>(256);
-    uint8_t *d_ndep = a.take<uint8_t>(256);
-    uint8_t *d_cmap = a.take<uint8_t>(LEVELS);
+    unsigned char *d_stage = a.take<unsigned char>(ST_END);
+    const uint16_t *d_loc = reinterpret_cast<const uint16_t *>(d_stage + ST_LOC);
+    const uint16_t *d_cbase = reinterpret_cast<const uint16_t *>(d_stage + ST_CBASE);
+    const uint8_t *d_ndep = d_stage + ST_NDEP;
+    const uint8_t *d_cmap = d_stage + ST_CMAP;
     uint32_t *deferred = a.take<uint32_t>(nt);
     unsigned *ndeferred = a.take<unsigned>(1);
     if (!deferred || !ndeferred) return OPATTR_E_OOM;
     int32_t *P = a.take<int32_t>((nt + 1) * (int64_t)(nl > 0 ? nl : 1));
-    if (!rk0 || !rk1 || !rv0 || !rv1 || !hist || !ls || !le || !li || !d_loc || !d_cbase || !d_ndep || !d_cmap || !P)
-        return OPATTR_E_OOM;
-    cudaMemcpyAsync(d_loc, level_of_compact.data(), sizeof(uint16_t) * (nl > 0 ? nl : 1), cudaMemcpyHostToDevice,
-                    c.stream);
-    cudaMemcpyAsync(d_cbase, cbase.data(), sizeof(uint16_t) * 256, cudaMemcpyHostToDevice, c.stream);
-    cudaMemcpyAsync(d_ndep, ndep.data(), 256, cudaMemcpyHostToDevice, c.stream);
-    if (nl <= 256) cudaMemcpyAsync(d_cmap, cmap.data(), LEVELS, cudaMemcpyHostToDevice, c.stream);
+    if (!rk0 || !rk1 || !rv0 || !rv1 || !hist || !ls || !le || !li || !d_stage || !P) return OPATTR_E_OOM;
+    cudaMemcpyAsync(d_stage, c.h_stage, ST_END, cudaMemcpyHostToDevice, c.stream);
 
     // ---- kernel time order
     uint32_t *korder = nullptr;
@@ -770,10 +774,13 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
             launch(c, "fill_unattributed", k_fill_unattributed, dim3(grid_for(K, 256, 65535)), dim3(256), 0, out_range,
                    out_nop, K);
         if (K > 0 && nl > 0) {
+            // chunks of WT_CHUNK tiles once the table is large (searches for
+            // every entry in parallel would then repeat most of their steps)
+            const int wt_chunk = (nt + 1) * (int64_t)nl >= ((int64_t)1 << 22) ? WT_CHUNK : 1;
             launch(c, "window_table", k_window_table,
-                   dim3(grid_for((nt + 1 + WT_CHUNK - 1) / WT_CHUNK * nl, 256, 65535)), dim3(256), 0,
+                   dim3(grid_for((nt + 1 + wt_chunk - 1) / wt_chunk * nl, 256, 65535)), dim3(256), 0,
                    (const int64_t *)ls, (const uint32_t *)lvl_off, (const uint16_t *)d_loc, nl, kern->start_ns,
-                   (const uint32_t *)korder, K, nt, P);
+                   (const uint32_t *)korder, K, nt, wt_chunk, P);
             EncArgs A;
             A.k_stream = kern->stream;
             A.k_start = kern->start_ns;
