@@ -420,6 +420,10 @@ const char *opattr_status_string(opattr_status status);
  * names have been seen; opattr_launch_count returns the number of kernels the
  * context has launched since creation or the last reset. */
 opattr_status opattr_set_timing(opattr_ctx *ctx, int enable);
+/* With timing on, bracket only the launches of the kernel named `kernel` (a
+ * name opattr_timing_report lists); NULL brackets every launch again.  The
+ * name is copied. */
+opattr_status opattr_set_timing_only(opattr_ctx *ctx, const char *kernel);
 int opattr_timing_report(opattr_ctx *ctx, const char **names, double *total_ms, int64_t *launches, int cap);
 void opattr_timing_reset(opattr_ctx *ctx);
 int64_t opattr_launch_count(const opattr_ctx *ctx);

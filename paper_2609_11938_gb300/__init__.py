@@ -149,6 +149,8 @@ def library():
             lib.opattr_status_string.argtypes = [ctypes.c_int]
             lib.opattr_status_string.restype = ctypes.c_char_p
             lib.opattr_set_timing.argtypes = [_vp, ctypes.c_int]
+            lib.opattr_set_timing_only.argtypes = [_vp, ctypes.c_char_p]
+            lib.opattr_set_timing_only.restype = ctypes.c_int
             lib.opattr_timing_report.argtypes = [_vp, P(ctypes.c_char_p), P(ctypes.c_double), P(ctypes.c_int64),
                                                  ctypes.c_int]
             lib.opattr_timing_reset.argtypes = [_vp]
@@ -542,6 +544,10 @@ class Context:
     # -- accounting
     def set_timing(self, on: bool):
         library().opattr_set_timing(self.handle, int(bool(on)))
+
+    def set_timing_only(self, kernel: str | None):
+        """With timing on, bracket only the launches of `kernel` (None: all)."""
+        library().opattr_set_timing_only(self.handle, kernel.encode() if kernel else None)
 
     def timing_report(self) -> dict:
         lib = library()

@@ -297,6 +297,12 @@ opattr_status opattr_set_timing(opattr_ctx *ctx, int enable) {
     return OPATTR_OK;
 }
 
+opattr_status opattr_set_timing_only(opattr_ctx *ctx, const char *kernel) {
+    if (!ctx) return OPATTR_E_INVALID_ARG;
+    ctx->c.timing_only = kernel ? kernel : "";
+    return OPATTR_OK;
+}
+
 int opattr_timing_report(opattr_ctx *ctx, const char **names, double *total_ms, int64_t *launches, int cap) {
     if (!ctx) return 0;
     Ctx &c = ctx->c;

@@ -92,6 +92,7 @@ struct Ctx {
     // launch accounting
     int64_t launches = 0;
     bool timing = false;
+    std::string timing_only;         // with timing on: bracket only this kernel (empty = all)
     std::vector<TimingSlot> slots;
     std::vector<std::pair<int, std::pair<cudaEvent_t, cudaEvent_t>>> pending;
     std::vector<cudaEvent_t> event_pool;
@@ -137,7 +138,8 @@ inline void launch(Ctx &c, const char *name, void (*kern)(KArgs...), dim3 grid, 
     if (grid.x == 0 || grid.y == 0 || grid.z == 0) return;
     cudaEvent_t e0 = nullptr, e1 = nullptr;
     int slot = -1;
-    if (c.timing) {
+    const bool timed = c.timing && (c.timing_only.empty() || c.timing_only == name);
+    if (timed) {
         slot = timing_slot(c, name);
         timing_begin(c, slot, &e0, &e1);
     }
@@ -145,7 +147,7 @@ inline void launch(Ctx &c, const char *name, void (*kern)(KArgs...), dim3 grid, 
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess && c.last_error == cudaSuccess) c.last_error = e;
     c.launches++;
-    if (c.timing) timing_end(c, slot, e0, e1);
+    if (timed) timing_end(c, slot, e0, e1);
 }
 
 inline unsigned grid_for(int64_t n, int per_block, unsigned cap = 1u << 30) {
