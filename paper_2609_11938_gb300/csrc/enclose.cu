@@ -444,23 +444,26 @@ __device__ __forceinline__ void enclose_tile(const EncArgs &A, EncSmem<WIN, ACT>
             256, [&](int j) -> unsigned { return j < cnt ? (unsigned)S.ks[j] : GROUP_NONE; }, &S.wcnt[0][0], 256,
             S.soff, S.klist, S.wbuf);
         // Each thread sweeps ENC_CHUNK consecutive kernels of one stream in
-        // time order.  Per depth it keeps the window position of the last
-        // range starting at or before the current kernel; positions only move
-        // forward, so after one search per depth the sweep advances them by
-        // comparison.
-        constexpr int RD = 8;                     // depths whose positions stay in registers
+        // time order, keeping per depth (the first RD depths, in registers)
+        // the last window range starting at or before the current kernel:
+        // its position, end and info, and the start of the next one.  A depth
+        // is searched once when the stream changes and afterwards moves only
+        // when the next range's start is passed (positions only move
+        // forward), so a kernel usually costs one comparison per depth.
+        // The walk over the depths is redone only when a depth moved or a
+        // range it found has ended; otherwise it would visit the same ranges
+        // with the same results.
+        constexpr int RD = 8;                     // depths whose state stays in registers
+        constexpr uint32_t NONE_T = 0xFFFFFFFFu;
         int cur_s = -1, nd = 0, a0 = 0;
-        int pr[RD];                               // window position + 1 (0 none, -1 not searched yet)
-        int wo[RD], wc[RD];                       // window offset and length of each depth (current stream)
+        int pos[RD];                              // window position of the depth's range, -1 none
+        uint32_t nxt[RD], cend[RD], cinf[RD];     // next start; end and info of the range
 #pragma unroll
-        for (int d = 0; d < RD; ++d) pr[d] = -1, wo[d] = 0, wc[d] = 0;
-        // The last walk's answer holds for a later kernel of the stream while
-        // no range of a depth the walk looked at starts in between and every
-        // range it found still contains the kernel: the walk would visit the
-        // same ranges with the same results.
+        for (int d = 0; d < RD; ++d) pos[d] = -1, nxt[d] = NONE_T, cend[d] = 0, cinf[d] = 0;
         int32_t ans = -1;
         int nop = 0;
-        uint32_t reuse_below = 0, reuse_upto = 0;    // valid for next_start > T and T <= min_end
+        bool redo = true;                         // the walk must be redone
+        uint32_t min_end = 0;                     // earliest end among the ranges the walk went through
         for (int u = 0; u < ENC_CHUNK; ++u) {
             const int idx = threadIdx.x * ENC_CHUNK + u;
             if (idx >= cnt) break;
@@ -474,52 +477,50 @@ __device__ __forceinline__ void enclose_tile(const EncArgs &A, EncSmem<WIN, ACT>
                 a0 = S.sbase[s];
 #pragma unroll
                 for (int d = 0; d < RD; ++d) {
-                    pr[d] = -1;
-                    wo[d] = d < nd ? S.act_off[a0 + d] : 0;
-                    wc[d] = d < nd ? S.act_cnt[a0 + d] : 0;
+                    const int c = d < nd ? S.act_cnt[a0 + d] : 0, o = d < nd ? S.act_off[a0 + d] : 0;
+                    int x = o, y = o + c;         // last window position with start <= T
+                    while (x < y) {
+                        const int m = (x + y) >> 1;
+                        if (S.ws[m] <= T) x = m + 1; else y = m;
+                    }
+                    const int p = x - o - 1;
+                    pos[d] = p;
+                    nxt[d] = p + 1 < c ? S.ws[o + p + 1] : NONE_T;
+                    cend[d] = p >= 0 ? S.we[o + p] : 0u;
+                    cinf[d] = p >= 0 ? S.wi[o + p] : 0u;
                 }
-                reuse_below = 0;
-            }
-            if (!(T < reuse_below && T <= reuse_upto)) {
-                // every depth's candidate first (independent lookups, in
-                // flight together), then the walk over them in registers
-                uint32_t cs[RD], ce[RD], ci[RD], cn[RD];
+                redo = true;
+            } else {
 #pragma unroll
                 for (int d = 0; d < RD; ++d) {
-                    const int c = wc[d], o = wo[d];
-                    int p;                          // last window position with start <= T, or -1
-                    if (pr[d] < 0) {
-                        int x = o, y = o + c;
-                        while (x < y) {
-                            const int m = (x + y) >> 1;
-                            if (S.ws[m] <= T) x = m + 1; else y = m;
-                        }
-                        p = x - o - 1;
-                    } else {
-                        p = pr[d] - 1;
+                    if (nxt[d] <= T) {            // a later range of this depth starts by T
+                        const int c = S.act_cnt[a0 + d], o = S.act_off[a0 + d];
+                        int p = pos[d] + 1;
                         while (p + 1 < c && S.ws[o + p + 1] <= T) ++p;
+                        pos[d] = p;
+                        nxt[d] = p + 1 < c ? S.ws[o + p + 1] : NONE_T;
+                        cend[d] = S.we[o + p];
+                        cinf[d] = S.wi[o + p];
+                        redo = true;
                     }
-                    pr[d] = p + 1;
-                    cn[d] = p + 1 < c ? S.ws[o + p + 1] : 0xFFFFFFFFu;
-                    cs[d] = p >= 0 ? 1u : 0u;
-                    ce[d] = p >= 0 ? S.we[o + p] : 0u;
-                    ci[d] = p >= 0 ? S.wi[o + p] : 0u;
                 }
+                redo = redo || T > min_end;
+            }
+            if (redo) {
                 ans = -1;
                 nop = 0;
                 bool alive = true;
-                uint32_t next_start = 0xFFFFFFFFu, min_end = 0xFFFFFFFFu;
+                min_end = NONE_T;
 #pragma unroll
                 for (int d = 0; d < RD; ++d) {
                     if (alive && d < nd) {
-                        next_start = min(next_start, cn[d]);
-                        if (!cs[d] || ce[d] < T) {
+                        if (pos[d] < 0 || cend[d] < T) {
                             alive = false;
                         } else {
-                            min_end = min(min_end, ce[d]);
-                            const uint32_t kind = ci[d] >> 30;
+                            min_end = min(min_end, cend[d]);
+                            const uint32_t kind = cinf[d] >> 30;
                             if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
-                            else if (kind == KIND_OP) { ans = (int32_t)(ci[d] & 0x3FFFFFFFu); nop++; }
+                            else if (kind == KIND_OP) { ans = (int32_t)(cinf[d] & 0x3FFFFFFFu); nop++; }
                         }
                     }
                 }
@@ -538,8 +539,7 @@ __device__ __forceinline__ void enclose_tile(const EncArgs &A, EncSmem<WIN, ACT>
                     if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
                     else if (kind == KIND_OP) { ans = (int32_t)(info & 0x3FFFFFFFu); nop++; }
                 }
-                reuse_below = deep ? 0u : next_start;
-                reuse_upto = min_end;
+                redo = deep;                      // deep levels are not tracked: search again next time
             }
             A.out_range[k] = ans;
             if (A.out_nop) A.out_nop[k] = (uint8_t)nop;
