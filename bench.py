@@ -36,8 +36,8 @@ KERNEL_BYTES = {
     "agg_ops": lambda K, R, M, O: 96 * K + 188 * O,
     "enclose": lambda K, R, M, O: 14 * K + 20 * R,
     "enclose_wide": lambda K, R, M, O: 14 * K + 20 * R,
-    "agg_fill": lambda K, R, M, O: 12 * K,
-    "agg_count": lambda K, R, M, O: 20 * K + 4 * O,
+    "agg_place": lambda K, R, M, O: 16 * K,
+    "agg_count": lambda K, R, M, O: 24 * K + 4 * O,
     "match_identity": lambda K, R, M, O: 13 * K,
     "check_kernel_order": lambda K, R, M, O: 9 * K,
     "check_ranges": lambda K, R, M, O: 18 * R,

@@ -300,51 +300,68 @@ __device__ __forceinline__ int32_t range_of_t(const int32_t *rok, const uint32_t
 // ------------------------------------------------------------------ count
 // Per kernel: duration >= 0, range index in [-1, R), an attributed range is an
 // operator below n_ops, row index in [-1, M).  Totals: all / attributed time,
-// attributed and matched kernel counts; cnt[op] += 1 per attributed kernel
-// (one atomic per distinct op id of a warp).
+// attributed and matched kernel counts.  Each attributed kernel (valid range
+// and op id) also takes its slot among its op's kernels: one atomic per
+// distinct op id of a warp on cnt[op], whose old value plus the kernel's rank
+// among its warp peers is the slot (rank[k]); cnt ends as the per-op counts.
+// Each warp takes a run of `run` consecutive kernels (a multiple of 32, up to
+// AF_RUN) 32 at a time in index order, so an op whose kernels all lie in one
+// run gets ascending slots; the ops pass sorts the few segments that do not.
+constexpr int AF_RUN = 2048;
+
 template <bool DIRECT>
 __global__ void k_agg_count(const int64_t *__restrict__ dur, const int32_t *__restrict__ rok,
                             const int32_t *__restrict__ nidx, const uint32_t *__restrict__ r_op, int64_t K, int64_t R,
-                            int64_t M, int64_t n_ops, uint32_t *__restrict__ cnt, DevStatus *st) {
-    constexpr int U = 4;                    // kernels per thread per round, loads issued together
+                            int64_t M, int64_t n_ops, uint32_t *__restrict__ cnt, uint32_t *__restrict__ rank,
+                            int64_t run, DevStatus *st) {
+    const unsigned lane = lane_id(), lt = lanemask_lt();
+    const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / 32;
+    const int64_t nwarps = (int64_t)gridDim.x * blockDim.x / 32;
     unsigned long long tot = 0, att = 0, natt = 0, nmatch = 0;
     int bad = 0;
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t k0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k0 - threadIdx.x < K; k0 += stride * U) {
-        long long d[U];
-        int32_t r[U], j[U];
-        uint32_t op[U];
-#pragma unroll
-        for (int u = 0; u < U; ++u) {               // lane-consecutive kernels: coalesced
-            const int64_t k = k0 + u * stride;
-            const bool in = k < K;
-            d[u] = in ? dur[k] : 0;
-            r[u] = in ? range_of_t<DIRECT>(rok, r_op, k) : -1;
-            j[u] = in ? nidx[k] : -1;
-        }
-#pragma unroll
-        for (int u = 0; u < U; ++u) op[u] = (r[u] >= 0 && r[u] < R) ? r_op[r[u]] : 0xFFFFFFFFu;
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int64_t k = k0 + u * stride;
-            bool valid = k < K;
-            if (valid && (d[u] < 0 || r[u] < -1 || r[u] >= R || j[u] < -1 || j[u] >= M ||
-                          (r[u] >= 0 && (int64_t)op[u] >= n_ops))) {
+    auto op_of = [&](int32_t r) -> uint32_t { return (r >= 0 && r < R) ? r_op[r] : 0xFFFFFFFFu; };
+    for (int64_t k0 = warp * run; k0 < K; k0 += nwarps * run) {
+        const int64_t k1 = k0 + run < K ? k0 + run : K;
+        // ranges two groups ahead; op ids, durations and row indices one group
+        // ahead, so each step waits only on its own atomic
+        int64_t k = k0 + lane;
+        int32_t r_c = k < k1 ? range_of_t<DIRECT>(rok, r_op, k) : -1;
+        uint32_t op_c = op_of(r_c);
+        long long d_c = k < k1 ? dur[k] : 0;
+        int32_t j_c = k < k1 ? nidx[k] : -1;
+        int32_t r_n = k + 32 < k1 ? range_of_t<DIRECT>(rok, r_op, k + 32) : -1;
+        for (int64_t kb = k0; kb < k1; kb += 32) {
+            k = kb + lane;
+            const bool in = k < k1;
+            const int32_t r = r_c, j = j_c;
+            const uint32_t op = op_c;
+            const long long d = d_c;
+            r_c = r_n;
+            op_c = op_of(r_n);
+            d_c = k + 32 < k1 ? dur[k + 32] : 0;
+            j_c = k + 32 < k1 ? nidx[k + 32] : -1;
+            r_n = k + 64 < k1 ? range_of_t<DIRECT>(rok, r_op, k + 64) : -1;
+            bool valid = in;
+            if (in && (d < 0 || r < -1 || r >= R || j < -1 || j >= M || (r >= 0 && (int64_t)op >= n_ops))) {
                 bad = 1;
                 valid = false;
             }
             if (valid) {
-                tot += (unsigned long long)d[u];
-                if (r[u] >= 0) {
-                    att += (unsigned long long)d[u];
+                tot += (unsigned long long)d;
+                if (r >= 0) {
+                    att += (unsigned long long)d;
                     natt++;
-                    nmatch += j[u] >= 0;
+                    nmatch += j >= 0;
                 }
             }
-            // counted exactly as k_agg_fill places it: by range and op id alone
-            const unsigned key = (k < K && r[u] >= 0 && r[u] < R && (int64_t)op[u] < n_ops) ? op[u] : 0xFFFFFFFFu;
+            // slotted exactly as k_agg_place places it: by range and op id alone
+            const unsigned key = (in && r >= 0 && r < R && (int64_t)op < n_ops) ? op : 0xFFFFFFFFu;
             const unsigned peers = __match_any_sync(0xffffffffu, key);
-            if (key != 0xFFFFFFFFu && (peers & lanemask_lt()) == 0) atomicAdd(&cnt[key], (unsigned)__popc(peers));
+            const int leader = __ffs(peers) - 1;
+            unsigned base = 0;
+            if (key != 0xFFFFFFFFu && (int)lane == leader) base = atomicAdd(&cnt[key], (unsigned)__popc(peers));
+            base = __shfl_sync(0xffffffffu, base, leader);
+            if (key != 0xFFFFFFFFu) rank[k] = base + __popc(peers & lt);
         }
     }
     __shared__ unsigned long long red[33];
@@ -355,45 +372,28 @@ __global__ void k_agg_count(const int64_t *__restrict__ dur, const int32_t *__re
     block_add_u64(nmatch, &st->cnt[C_MATCHED_K], red);
 }
 
-// ------------------------------------------------------------------ fill
-// list[off[op] + slot] = k for each attributed kernel with a valid range and
-// op id (the kernels k_agg_count counted); slots are taken by atomics on
-// cur[op] (zeroed).  Each warp fills a run of `run` consecutive kernels (a
-// multiple of 32, up to AF_RUN) 32 at a time in index order, so an op whose
-// kernels all lie in one run gets them in ascending order; the ops pass sorts
-// the few segments that do not.
-constexpr int AF_RUN = 2048;
-
+// ------------------------------------------------------------------ place
+// list[off[op] + rank[k]] = k for each kernel k_agg_count slotted.
 template <bool DIRECT>
-__global__ void k_agg_fill(const int32_t *__restrict__ rok, const uint32_t *__restrict__ r_op, int64_t K, int64_t R,
-                           int64_t n_ops, const uint32_t *__restrict__ off, uint32_t *__restrict__ cur,
-                           uint32_t *__restrict__ list, int64_t run) {
-    const unsigned lane = lane_id();
-    const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / 32;
-    const int64_t nwarps = (int64_t)gridDim.x * blockDim.x / 32;
-    // op id of a kernel's range, or none
-    auto key_of = [&](int32_t r) -> unsigned {
-        if (r < 0 || r >= R) return 0xFFFFFFFFu;
-        const uint32_t op = r_op[r];
-        return (int64_t)op < n_ops ? op : 0xFFFFFFFFu;
-    };
-    for (int64_t k0 = warp * run; k0 < K; k0 += nwarps * run) {
-        const int64_t k1 = k0 + run < K ? k0 + run : K;
-        // ranges loaded two groups ahead, op ids one group ahead, so each
-        // step waits only on its own atomic
-        unsigned key_next = key_of(k0 + lane < k1 ? range_of_t<DIRECT>(rok, r_op, k0 + lane) : -1);
-        int32_t r_next = k0 + 32 + lane < k1 ? range_of_t<DIRECT>(rok, r_op, k0 + 32 + lane) : -1;
-        for (int64_t kb = k0; kb < k1; kb += 32) {
-            const int64_t k = kb + lane;
-            const unsigned key = key_next;
-            key_next = key_of(r_next);
-            r_next = k + 64 < k1 ? range_of_t<DIRECT>(rok, r_op, k + 64) : -1;
-            const unsigned peers = __match_any_sync(0xffffffffu, key);
-            const int leader = __ffs(peers) - 1;
-            unsigned base = 0;
-            if (key != 0xFFFFFFFFu && (int)lane == leader) base = atomicAdd(&cur[key], (unsigned)__popc(peers));
-            base = __shfl_sync(0xffffffffu, base, leader);
-            if (key != 0xFFFFFFFFu) list[off[key] + base + __popc(peers & lanemask_lt())] = (uint32_t)k;
+__global__ void k_agg_place(const int32_t *__restrict__ rok, const uint32_t *__restrict__ r_op, int64_t K, int64_t R,
+                            int64_t n_ops, const uint32_t *__restrict__ off, const uint32_t *__restrict__ rank,
+                            uint32_t *__restrict__ list) {
+    constexpr int U = 4;                    // kernels per thread per round, loads issued together
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t k0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k0 < K; k0 += stride * U) {
+        int32_t r[U];
+        uint32_t op[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t k = k0 + u * stride;
+            r[u] = k < K ? range_of_t<DIRECT>(rok, r_op, k) : -1;
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) op[u] = (r[u] >= 0 && r[u] < R) ? r_op[r[u]] : 0xFFFFFFFFu;
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int64_t k = k0 + u * stride;
+            if (r[u] >= 0 && r[u] < R && (int64_t)op[u] < n_ops) list[off[op[u]] + rank[k]] = (uint32_t)k;
         }
     }
 }
@@ -924,7 +924,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     if ((reinterpret_cast<uintptr_t>(ncu->counters) & 15) != 0) return OPATTR_E_INVALID_ARG;
 
     Need nd;
-    nd.add<uint32_t>(O + 1).add<uint32_t>(O + 1).add<uint32_t>(O + 1).add<uint32_t>(K).add<uint32_t>(K);
+    nd.add<uint32_t>(O + 1).add<uint32_t>(O + 1).add<uint32_t>(K).add<uint32_t>(K);
     nd.add<uint32_t>(O + 1).add<unsigned>(1).add<unsigned>(1);
     nd.add<uint32_t>(O + 1).add<Acc>(K / AG_PIECE + (K / (AG_SHORT_MAX + 1)) + 1);   // pieces per op, partials
     nd.add<uint32_t>(scan_scratch_elems(std::max<int64_t>(O + 1, radix_hist_elems(K))));
@@ -934,7 +934,9 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     if (st) return st;
     Arena a(c);
     if ((st = reset_status(c))) return st;
-    uint32_t *cnt = a.take<uint32_t>(O + 1), *off = a.take<uint32_t>(O + 1), *cur = a.take<uint32_t>(O + 1);
+    uint32_t *cnt = a.take<uint32_t>(O + 1), *off = a.take<uint32_t>(O + 1);
+    // tmp holds each kernel's slot among its op's kernels until the list is
+    // placed, then serves the segment sorts
     uint32_t *list = a.take<uint32_t>(K), *tmp = a.take<uint32_t>(K), *longs = a.take<uint32_t>(O + 1);
     unsigned *nlong = a.take<unsigned>(1);
     unsigned *ctr = a.take<unsigned>(1);
@@ -946,14 +948,19 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     uint32_t *hidx = a.take<uint32_t>(O + 1), *hhist = a.take<uint32_t>(radix_hist_elems(K));
     uint32_t *info = a.take<uint32_t>(8), *hop = a.take<uint32_t>(O + 1);
     if (!hidx || !hhist || !info || !hop) return OPATTR_E_OOM;
-    if (!cnt || !off || !cur || !list || !tmp || !longs || !nlong || !part) return OPATTR_E_OOM;
+    if (!cnt || !off || !list || !tmp || !longs || !nlong || !part) return OPATTR_E_OOM;
     cudaMemsetAsync(cnt, 0, sizeof(uint32_t) * (O + 1), c.stream);
-    cudaMemsetAsync(cur, 0, sizeof(uint32_t) * (O + 1), c.stream);
     cudaMemsetAsync(nlong, 0, sizeof(unsigned), c.stream);
+    int sms = 0;
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
+    // runs long enough to keep most segments in one warp, short enough that
+    // small traces still spread over the GPU (64 warps per SM)
+    const int64_t warps = (int64_t)std::max(1, sms) * 64;
+    const int64_t run = std::min<int64_t>(AF_RUN, std::max<int64_t>(32, ((K + warps - 1) / warps + 31) / 32 * 32));
     if (K > 0)
-        launch(c, "agg_count", rok ? k_agg_count<false> : k_agg_count<true>, dim3(grid_for(K, 256 * 4, REDUCE_GRID)),
-               dim3(256), 0, kern->dur_ns, rok,
-               nidx, rng->op_id, K, R, M, O, cnt, c.d_status);
+        launch(c, "agg_count", rok ? k_agg_count<false> : k_agg_count<true>,
+               dim3(grid_for(K, 256 / 32 * run, 65535)), dim3(256), 0, kern->dur_ns, rok, nidx, rng->op_id, K, R, M,
+               O, cnt, tmp, run, c.d_status);
     AggIn in;
     in.dur = kern->dur_ns;
     in.ncu_idx = nidx;
@@ -963,23 +970,14 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     in.out = *out;
     if (O > 0) {
         scan_exclusive_u32(c, cnt, off, O + 1, part, nullptr);
-        if (K > 0) {
-            // runs long enough to keep most segments in one warp, short enough
-            // that small traces still spread over the GPU (64 warps per SM)
-            int sms = 0;
-            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
-            const int64_t warps = (int64_t)std::max(1, sms) * 64;
-            const int64_t run = std::min<int64_t>(AF_RUN, std::max<int64_t>(32, ((K + warps - 1) / warps + 31) / 32 * 32));
-            launch(c, "agg_fill", rok ? k_agg_fill<false> : k_agg_fill<true>, dim3(grid_for(K, 256 / 32 * run, 65535)),
-                   dim3(256), 0, rok,
-                   rng->op_id, K, R, O, (const uint32_t *)off, cur, list, run);
-        }
+        if (K > 0)
+            launch(c, "agg_place", rok ? k_agg_place<false> : k_agg_place<true>,
+                   dim3(grid_for(K, 256 * 4, REDUCE_GRID)), dim3(256), 0, rok, rng->op_id, K, R, O,
+                   (const uint32_t *)off, (const uint32_t *)tmp, list);
         launch(c, "agg_long_list", k_agg_long_list, dim3(grid_for(O, 256, 4096)), dim3(256), 0,
                (const uint32_t *)off, O, AG_SHORT_MAX, longs, nlong);
         launch(c, "agg_piece_offsets", k_agg_piece_offsets, dim3(1), dim3(1024), 0, (const uint32_t *)off,
                (const uint32_t *)longs, (const unsigned *)nlong, AG_HUGE, npc, info, hop);
-        int sms = 0;
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
         // long segments the ops pass walks: sorted first
         launch(c, "agg_sort_long", k_agg_sort_long, dim3(2 * std::max(1, sms)), dim3(SL_THREADS), 0,
                (const uint32_t *)off, (const uint32_t *)longs, (const unsigned *)nlong, AG_SHORT_MAX + 1, AG_HUGE,
