@@ -70,11 +70,49 @@ __global__ void __launch_bounds__(SCAN_THREADS) k_scan_down(const uint32_t *in, 
     }
 }
 
+// Small scans in one block (one launch instead of three): each of the 32
+// warps scans a contiguous run of 1,024 elements in 32 coalesced rounds,
+// carrying the running total in registers; one barrier exchanges the warp
+// totals.  Every element is read and written by the same thread, so the
+// scan may run in place.
+constexpr int64_t SCAN_ONE_BLOCK = 32 * 1024;
+__global__ void __launch_bounds__(1024) k_scan_small(const uint32_t *in, uint32_t *out, int64_t n,
+                                                     uint32_t *total_dev) {
+    __shared__ uint32_t wsum[32];
+    const unsigned w = threadIdx.x >> 5, lane = lane_id();
+    const int64_t b = (int64_t)w * 1024 + lane;
+    uint32_t v[32];
+#pragma unroll
+    for (int r = 0; r < 32; ++r) v[r] = b + r * 32 < n ? in[b + r * 32] : 0u;
+    uint32_t carry = 0;
+#pragma unroll
+    for (int r = 0; r < 32; ++r) {
+        const uint32_t inc = warp_inclusive_scan(v[r]);
+        const uint32_t ex = carry + inc - v[r];
+        carry += __shfl_sync(0xffffffffu, inc, 31);
+        v[r] = ex;
+    }
+    if (lane == 0) wsum[w] = carry;
+    __syncthreads();
+    const uint32_t x = wsum[lane];
+    const uint32_t xs = warp_inclusive_scan(x);
+    const uint32_t base = __shfl_sync(0xffffffffu, xs - x, (int)w);
+    const uint32_t tot = __shfl_sync(0xffffffffu, xs, 31);
+#pragma unroll
+    for (int r = 0; r < 32; ++r)
+        if (b + r * 32 < n) out[b + r * 32] = base + v[r];
+    if (threadIdx.x == 0 && total_dev) *total_dev = tot;
+}
+
 void scan_exclusive_u32(Ctx &c, const uint32_t *in, uint32_t *out, int64_t n, uint32_t *partials,
                         uint32_t *total_dev) {
     int64_t nt = (n + SCAN_TILE - 1) / SCAN_TILE;
     if (n <= 0) {
         if (total_dev) cudaMemsetAsync(total_dev, 0, sizeof(uint32_t), c.stream);
+        return;
+    }
+    if (n <= SCAN_ONE_BLOCK) {
+        launch(c, "scan_small", k_scan_small, dim3(1), dim3(1024), 0, in, out, n, total_dev);
         return;
     }
     launch(c, "scan_reduce", k_scan_reduce, dim3((unsigned)nt), dim3(SCAN_THREADS), 0, in, n, partials);
