@@ -59,17 +59,31 @@ __global__ void __launch_bounds__(RCHK_THREADS) k_check_ranges(const uint8_t *__
     const int64_t base = (int64_t)blockIdx.x * RCHK_THREADS * RCHK_ITEMS;
     long long mn = LLONG_MAX, mx = LLONG_MIN;
     int f = 0;
-    for (int it = 0; it < RCHK_ITEMS; ++it) {
-        int64_t i = base + it * RCHK_THREADS + threadIdx.x;
-        if (i >= n) break;
-        long long s = start[i], e = end[i];
-        unsigned d = depth[i];
-        if (e < s) f |= 1;
-        if (d >= OPATTR_MAX_DEPTH) f |= 2;
-        if (i + 1 < n && start[i + 1] < s) f |= 4;
-        mn = s < mn ? s : mn;
-        mx = e > mx ? e : mx;
-        if (d < OPATTR_MAX_DEPTH) atomicAdd(&h[stream[i] * 32 + d], 1u);
+    constexpr int B = 4;                    // items per batch, loads issued together
+    for (int it0 = 0; it0 < RCHK_ITEMS; it0 += B) {
+        long long sv[B], ev[B], nv[B];
+        unsigned dv[B], stv[B];
+#pragma unroll
+        for (int u = 0; u < B; ++u) {
+            const int64_t i = base + (it0 + u) * RCHK_THREADS + threadIdx.x;
+            const bool in = i < n;
+            sv[u] = in ? start[i] : 0;
+            ev[u] = in ? end[i] : 0;
+            nv[u] = i + 1 < n ? start[i + 1] : LLONG_MAX;
+            dv[u] = in ? depth[i] : 0u;
+            stv[u] = in ? stream[i] : 0u;
+        }
+#pragma unroll
+        for (int u = 0; u < B; ++u) {
+            const int64_t i = base + (it0 + u) * RCHK_THREADS + threadIdx.x;
+            if (i >= n) continue;
+            if (ev[u] < sv[u]) f |= 1;
+            if (dv[u] >= OPATTR_MAX_DEPTH) f |= 2;
+            if (nv[u] < sv[u]) f |= 4;
+            mn = sv[u] < mn ? sv[u] : mn;
+            mx = ev[u] > mx ? ev[u] : mx;
+            if (dv[u] < OPATTR_MAX_DEPTH) atomicAdd(&h[stv[u] * 32 + dv[u]], 1u);
+        }
     }
     if (f) atomicOr(&flags, f);
     atomicMin(&smin, mn);

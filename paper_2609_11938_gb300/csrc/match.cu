@@ -23,12 +23,27 @@
 namespace opattr {
 
 // ------------------------------------------------------------------ fast path
+// Whether the identity pass may use 16-byte accesses (every array aligned).
+static int identity_vec(const void *kname, const void *nname, const void *out_idx, const void *out_kind) {
+    auto al = [](const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; };
+    return al(kname, 16) && al(nname, 16) && al(out_idx, 16) && al(out_kind, 4);
+}
 __global__ void k_match_identity(const uint32_t *__restrict__ kname, const uint32_t *__restrict__ nname, int64_t n,
-                                 int32_t *__restrict__ out_idx, uint8_t *__restrict__ out_kind, DevStatus *st) {
+                                 int32_t *__restrict__ out_idx, uint8_t *__restrict__ out_kind, int vec,
+                                 DevStatus *st) {
     constexpr int U = 4;                    // elements per thread per round, loads issued together
     int bad = 0;
-    for (int64_t base = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * U; base < n;
-         base += (int64_t)gridDim.x * blockDim.x * U) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x * U;
+    for (int64_t base = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * U; base < n; base += stride) {
+        if (vec && base + U <= n) {         // 16-byte loads and stores
+            const uint4 a = *reinterpret_cast<const uint4 *>(kname + base);
+            const uint4 b = *reinterpret_cast<const uint4 *>(nname + base);
+            bad |= (a.x != b.x) | (a.y != b.y) | (a.z != b.z) | (a.w != b.w);
+            const int32_t i0 = (int32_t)base;
+            *reinterpret_cast<int4 *>(out_idx + base) = make_int4(i0, i0 + 1, i0 + 2, i0 + 3);
+            if (out_kind) *reinterpret_cast<uint32_t *>(out_kind + base) = 0x01010101u;
+            continue;
+        }
         uint32_t a[U], b[U];
 #pragma unroll
         for (int u = 0; u < U; ++u) {
@@ -436,8 +451,7 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     const bool try_streams = !dedup_on && per_stream && K == M && K > 0;
     if (try_identity)
         launch(c, "match_identity", k_match_identity, dim3(grid_for(K, 256 * 16, REDUCE_GRID)), dim3(256), 0,
-               kname, nname, K, out_idx,
-               out_kind, c.d_status);
+               kname, nname, K, out_idx, out_kind, identity_vec(kname, nname, out_idx, out_kind), c.d_status);
     if (try_streams)
         stream_pairs(c, kern, ncu, nullptr, K, reinterpret_cast<uint8_t *>(n2), n0, n1, hist, part, out_idx,
                      out_kind);

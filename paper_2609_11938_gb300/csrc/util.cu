@@ -6,10 +6,11 @@ namespace opattr {
 
 constexpr int CHK_THREADS = 256;
 
-// Grid-stride over groups of four consecutive kernels (16-byte loads when
+// Grid-stride over groups of eight consecutive kernels (16-byte loads when
 // the arrays allow), comparing each (start, stream) with its successor; min /
 // max and the order flag are reduced per block and published with one atomic
 // each.
+constexpr int CHK_G = 8;
 __global__ void __launch_bounds__(CHK_THREADS) k_check_kernel_order(const uint8_t *__restrict__ stream,
                                                                     const int64_t *__restrict__ start, int64_t n,
                                                                     int vec, DevStatus *st) {
@@ -17,29 +18,37 @@ __global__ void __launch_bounds__(CHK_THREADS) k_check_kernel_order(const uint8_
     __shared__ int sbad[CHK_THREADS / 32];
     long long mn = LLONG_MAX, mx = LLONG_MIN;
     int unsorted = 0;
-    const int64_t ngroups = (n + 3) / 4;
+    const int64_t ngroups = (n + CHK_G - 1) / CHK_G;
     for (int64_t g = (int64_t)blockIdx.x * CHK_THREADS + threadIdx.x; g < ngroups;
          g += (int64_t)gridDim.x * CHK_THREADS) {
-        const int64_t i0 = g * 4;
-        long long t[5];
-        unsigned s[5];
-        if (vec && i0 + 4 <= n) {
-            const longlong2 a = reinterpret_cast<const longlong2 *>(start)[g * 2];
-            const longlong2 b = reinterpret_cast<const longlong2 *>(start)[g * 2 + 1];
-            const uchar4 q = reinterpret_cast<const uchar4 *>(stream)[g];
-            t[0] = a.x; t[1] = a.y; t[2] = b.x; t[3] = b.y;
-            s[0] = q.x; s[1] = q.y; s[2] = q.z; s[3] = q.w;
-        } else {
+        const int64_t i0 = g * CHK_G;
+        long long t[CHK_G + 1];
+        unsigned s[CHK_G + 1];
+        if (vec && i0 + CHK_G <= n) {
+            const longlong2 *p = reinterpret_cast<const longlong2 *>(start + i0);
+#pragma unroll
+            for (int q = 0; q < CHK_G / 2; ++q) {
+                const longlong2 x = p[q];
+                t[2 * q] = x.x;
+                t[2 * q + 1] = x.y;
+            }
+            const uint2 w = *reinterpret_cast<const uint2 *>(stream + i0);
 #pragma unroll
             for (int u = 0; u < 4; ++u) {
+                s[u] = (w.x >> (8 * u)) & 0xFFu;
+                s[4 + u] = (w.y >> (8 * u)) & 0xFFu;
+            }
+        } else {
+#pragma unroll
+            for (int u = 0; u < CHK_G; ++u) {
                 t[u] = i0 + u < n ? start[i0 + u] : LLONG_MAX;
                 s[u] = i0 + u < n ? stream[i0 + u] : 255u;
             }
         }
-        t[4] = i0 + 4 < n ? start[i0 + 4] : LLONG_MAX;
-        s[4] = i0 + 4 < n ? stream[i0 + 4] : 255u;
+        t[CHK_G] = i0 + CHK_G < n ? start[i0 + CHK_G] : LLONG_MAX;
+        s[CHK_G] = i0 + CHK_G < n ? stream[i0 + CHK_G] : 255u;
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
+        for (int u = 0; u < CHK_G; ++u) {
             if (i0 + u >= n) break;
             mn = t[u] < mn ? t[u] : mn;
             mx = t[u] > mx ? t[u] : mx;
@@ -74,7 +83,7 @@ __global__ void __launch_bounds__(CHK_THREADS) k_check_kernel_order(const uint8_
 
 void check_kernel_order(Ctx &c, const uint8_t *stream, const int64_t *start, int64_t n) {
     if (n <= 0) return;
-    const int vec = ((reinterpret_cast<uintptr_t>(start) & 15) == 0) && ((reinterpret_cast<uintptr_t>(stream) & 3) == 0);
+    const int vec = ((reinterpret_cast<uintptr_t>(start) & 15) == 0) && ((reinterpret_cast<uintptr_t>(stream) & 7) == 0);
     launch(c, "check_kernel_order", k_check_kernel_order, dim3(grid_for(n, CHK_THREADS * 16, REDUCE_GRID)),
            dim3(CHK_THREADS), 0, stream, start, n, vec, c.d_status);
 }
