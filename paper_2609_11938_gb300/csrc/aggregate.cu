@@ -35,6 +35,7 @@ struct AggIn {
     const float *counters;
     int64_t n_ops;
     unsigned *ctr;              // next chunk of the ops pass, zeroed before it
+    const unsigned *nonident;   // nonzero unless ncu_idx[k] == k for every kernel (set by the count pass)
     opattr_op_aggregates out;
 };
 
@@ -300,7 +301,9 @@ __device__ __forceinline__ int32_t range_of_t(const int32_t *rok, const uint32_t
 // ------------------------------------------------------------------ count
 // Per kernel: duration >= 0, range index in [-1, R), an attributed range is an
 // operator below n_ops, row index in [-1, M).  Totals: all / attributed time,
-// attributed and matched kernel counts.  Each attributed kernel (valid range
+// attributed and matched kernel counts.  Whether every kernel's row is its
+// own index (the match of a trace whose ncu rows follow the kernels one for
+// one) is noted, so the ops pass can skip the row-index gather.  Each attributed kernel (valid range
 // and op id) also takes its slot among its op's kernels: one atomic per
 // distinct op id of a warp on cnt[op], whose old value plus the kernel's rank
 // among its warp peers is the slot (rank[k]); cnt ends as the per-op counts.
@@ -310,15 +313,15 @@ __device__ __forceinline__ int32_t range_of_t(const int32_t *rok, const uint32_t
 constexpr int AF_RUN = 2048;
 
 template <bool DIRECT>
-__global__ void k_agg_count(const int64_t *__restrict__ dur, const int32_t *__restrict__ rok,
+__global__ void __launch_bounds__(256, 5) k_agg_count(const int64_t *__restrict__ dur, const int32_t *__restrict__ rok,
                             const int32_t *__restrict__ nidx, const uint32_t *__restrict__ r_op, int64_t K, int64_t R,
                             int64_t M, int64_t n_ops, uint32_t *__restrict__ cnt, uint32_t *__restrict__ rank,
-                            int64_t run, DevStatus *st) {
+                            int64_t run, unsigned *__restrict__ nonident, DevStatus *st) {
     const unsigned lane = lane_id(), lt = lanemask_lt();
     const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / 32;
     const int64_t nwarps = (int64_t)gridDim.x * blockDim.x / 32;
     unsigned long long tot = 0, att = 0, natt = 0, nmatch = 0;
-    int bad = 0;
+    int bad = 0, nid = 0;
     auto op_of = [&](int32_t r) -> uint32_t { return (r >= 0 && r < R) ? r_op[r] : 0xFFFFFFFFu; };
     for (int64_t k0 = warp * run; k0 < K; k0 += nwarps * run) {
         const int64_t k1 = k0 + run < K ? k0 + run : K;
@@ -341,6 +344,7 @@ __global__ void k_agg_count(const int64_t *__restrict__ dur, const int32_t *__re
             d_c = k + 32 < k1 ? dur[k + 32] : 0;
             j_c = k + 32 < k1 ? nidx[k + 32] : -1;
             r_n = k + 64 < k1 ? range_of_t<DIRECT>(rok, r_op, k + 64) : -1;
+            nid |= in && (int64_t)j != k;
             bool valid = in;
             if (in && (d < 0 || r < -1 || r >= R || j < -1 || j >= M || (r >= 0 && (int64_t)op >= n_ops))) {
                 bad = 1;
@@ -366,6 +370,7 @@ __global__ void k_agg_count(const int64_t *__restrict__ dur, const int32_t *__re
     }
     __shared__ unsigned long long red[33];
     if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_err(st, ERR_INVALID);
+    if (__any_sync(0xffffffffu, nid) && lane_id() == 0) atomicOr(nonident, 1u);
     block_add_u64(tot, &st->cnt[C_TOTAL_NS], red);
     block_add_u64(att, &st->cnt[C_ATTR_NS], red);
     block_add_u64(natt, &st->cnt[C_ATTR_K], red);
@@ -547,6 +552,8 @@ __global__ void __launch_bounds__(AG_THREADS, 5) k_agg_ops(const uint32_t *__res
     uint8_t *order = order_s[threadIdx.x / 32];
     const unsigned lane = lane_id();
     int bad = 0;
+    const bool ident = *A.nonident == 0;
+    auto row_of = [&](uint32_t k) -> int32_t { return ident ? (int32_t)k : A.ncu_idx[k]; };
     auto next_chunk = [&]() -> int64_t {
         unsigned v = 0;
         if (lane == 0) v = atomicAdd(A.ctr, 1u);
@@ -621,15 +628,15 @@ __global__ void __launch_bounds__(AG_THREADS, 5) k_agg_ops(const uint32_t *__res
                     cp_async_commit();
                 };
                 const uint32_t k0 = seg[0], k1 = len > 1 ? seg[1] : 0u;
-                const int32_t j0 = A.ncu_idx[k0], j1 = len > 1 ? A.ncu_idx[k1] : -1;
+                const int32_t j0 = row_of(k0), j1 = len > 1 ? row_of(k1) : -1;
                 uint32_t k2 = len > 2 ? seg[2] : 0u;
-                int32_t j2 = len > 2 ? A.ncu_idx[k2] : -1;
+                int32_t j2 = len > 2 ? row_of(k2) : -1;
                 issue(0, k0, j0);
                 issue(1, k1, j1);
                 int32_t js0 = j0, js1 = j1;           // row index of the kernel in each slot
                 for (uint32_t t = 0; t < len; ++t) {
                     const uint32_t k3 = t + 3 < len ? seg[t + 3] : 0u;
-                    const int32_t j3 = t + 3 < len ? A.ncu_idx[k3] : -1;
+                    const int32_t j3 = t + 3 < len ? row_of(k3) : -1;
                     cp_async_wait<1>();
                     const int32_t j = (t & 1) ? js1 : js0;
                     acc.accumulate(durbuf[t & 1][me], j >= 0, rowbuf[t & 1][me]);
@@ -925,7 +932,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
 
     Need nd;
     nd.add<uint32_t>(O + 1).add<uint32_t>(O + 1).add<uint32_t>(K).add<uint32_t>(K);
-    nd.add<uint32_t>(O + 1).add<unsigned>(1).add<unsigned>(1);
+    nd.add<uint32_t>(O + 1).add<unsigned>(1).add<unsigned>(1).add<unsigned>(1);
     nd.add<uint32_t>(O + 1).add<Acc>(K / AG_PIECE + (K / (AG_SHORT_MAX + 1)) + 1);   // pieces per op, partials
     nd.add<uint32_t>(scan_scratch_elems(std::max<int64_t>(O + 1, radix_hist_elems(K))));
     nd.add<uint32_t>(O + 1).add<uint32_t>(radix_hist_elems(K)).add<uint32_t>(8);   // huge-op index, histogram, info
@@ -940,6 +947,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     uint32_t *list = a.take<uint32_t>(K), *tmp = a.take<uint32_t>(K), *longs = a.take<uint32_t>(O + 1);
     unsigned *nlong = a.take<unsigned>(1);
     unsigned *ctr = a.take<unsigned>(1);
+    unsigned *nonident = a.take<unsigned>(1);
     uint32_t *npc = a.take<uint32_t>(O + 1);
     Acc *partials = a.take<Acc>(K / AG_PIECE + (K / (AG_SHORT_MAX + 1)) + 1);
     if (!npc || !partials) return OPATTR_E_OOM;
@@ -948,9 +956,10 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     uint32_t *hidx = a.take<uint32_t>(O + 1), *hhist = a.take<uint32_t>(radix_hist_elems(K));
     uint32_t *info = a.take<uint32_t>(8), *hop = a.take<uint32_t>(O + 1);
     if (!hidx || !hhist || !info || !hop) return OPATTR_E_OOM;
-    if (!cnt || !off || !list || !tmp || !longs || !nlong || !part) return OPATTR_E_OOM;
+    if (!cnt || !off || !list || !tmp || !longs || !nlong || !part || !nonident) return OPATTR_E_OOM;
     cudaMemsetAsync(cnt, 0, sizeof(uint32_t) * (O + 1), c.stream);
     cudaMemsetAsync(nlong, 0, sizeof(unsigned), c.stream);
+    cudaMemsetAsync(nonident, 0, sizeof(unsigned), c.stream);
     int sms = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
     // runs long enough to keep most segments in one warp, short enough that
@@ -960,13 +969,14 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     if (K > 0)
         launch(c, "agg_count", rok ? k_agg_count<false> : k_agg_count<true>,
                dim3(grid_for(K, 256 / 32 * run, 65535)), dim3(256), 0, kern->dur_ns, rok, nidx, rng->op_id, K, R, M,
-               O, cnt, tmp, run, c.d_status);
+               O, cnt, tmp, run, nonident, c.d_status);
     AggIn in;
     in.dur = kern->dur_ns;
     in.ncu_idx = nidx;
     in.counters = ncu->counters;
     in.n_ops = O;
     in.ctr = ctr;
+    in.nonident = nonident;
     in.out = *out;
     if (O > 0) {
         scan_exclusive_u32(c, cnt, off, O + 1, part, nullptr);
@@ -1148,6 +1158,7 @@ opattr_status do_rollup(Ctx &c, const opattr_kernels *kern, const opattr_ranges 
         in.counters = ncu->counters;
         in.n_ops = C;
         in.ctr = nullptr;
+        in.nonident = nullptr;
         in.out = *out;
         int sms = 0;
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);

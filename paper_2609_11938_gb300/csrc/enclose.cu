@@ -141,14 +141,13 @@ struct LevelDigit {
     }
 };
 // The placing pass: the digit-rank of the tile's ranges gives each its
-// place in the tile sorted by compact level; the range is staged there in
-// shared memory, then each level's run of the tile goes out to consecutive
-// addresses (one coalesced write per run instead of one scattered write per
-// range).  Same tiles as digit_offsets.
+// place in the tile sorted by compact level; the range's tile index is
+// staged there in shared memory, then each level's run of the tile goes out
+// to consecutive addresses (one coalesced write per run instead of one
+// scattered write per range), the range fields read back from the tile just
+// loaded (L1 / L2).  Same tiles as digit_offsets.
 struct PlaceSmem {
-    int64_t s[RADIX_TILE];
-    int64_t e[RADIX_TILE];
-    uint32_t info[RADIX_TILE];
+    uint16_t lidx[RADIX_TILE];
     uint8_t dig[RADIX_TILE];
     uint32_t wcnt[(RADIX_THREADS / 32) * RADIX_BINS];
     uint32_t dstart[RADIX_BINS];
@@ -161,8 +160,7 @@ __global__ void __launch_bounds__(RADIX_THREADS) k_level_place(LevelDigit digit,
                                                                const uint32_t *__restrict__ offs, int64_t ntiles,
                                                                int64_t *__restrict__ ls, int64_t *__restrict__ le,
                                                                uint32_t *__restrict__ li) {
-    extern __shared__ __align__(16) unsigned char place_raw[];
-    PlaceSmem &S = *reinterpret_cast<PlaceSmem *>(place_raw);
+    __shared__ PlaceSmem S;
     const unsigned w = threadIdx.x >> 5, lane = lane_id();
     for (int i = threadIdx.x; i < (RADIX_THREADS / 32) * RADIX_BINS; i += RADIX_THREADS) S.wcnt[i] = 0;
     __syncthreads();
@@ -207,21 +205,39 @@ __global__ void __launch_bounds__(RADIX_THREADS) k_level_place(LevelDigit digit,
         const unsigned d = dg[it];
         if (d < RADIX_BINS) {
             const uint32_t p = S.dstart[d] + S.wcnt[w * RADIX_BINS + d] + rank[it];
-            const uint32_t r = digit.perm ? digit.perm[i] : (uint32_t)i;
-            S.s[p] = start[r];
-            S.e[p] = end[r];
-            S.info[p] = r | (kind_of(op[r]) << 30);
+            S.lidx[p] = (uint16_t)(i - tile0);
             S.dig[p] = (uint8_t)d;
         }
     }
     __syncthreads();
     const int cnt = (int)(n - tile0 < RADIX_TILE ? n - tile0 : RADIX_TILE);
-    for (int j = threadIdx.x; j < cnt; j += RADIX_THREADS) {
-        const unsigned d = S.dig[j];
-        const int64_t o = (int64_t)S.gbase[d] + (j - S.dstart[d]);
-        ls[o] = S.s[j];
-        le[o] = S.e[j];
-        li[o] = S.info[j];
+    constexpr int U = 4;                    // entries per thread per round, loads issued together
+    for (int j0 = threadIdx.x; j0 < cnt; j0 += RADIX_THREADS * U) {
+        uint32_t r[U];
+        long long sv[U], ev[U];
+        uint32_t ov[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int j = j0 + u * RADIX_THREADS;
+            const int64_t i = tile0 + (j < cnt ? S.lidx[j] : 0);
+            r[u] = digit.perm ? digit.perm[i] : (uint32_t)i;
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            sv[u] = start[r[u]];
+            ev[u] = end[r[u]];
+            ov[u] = op[r[u]];
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int j = j0 + u * RADIX_THREADS;
+            if (j >= cnt) continue;
+            const unsigned d = S.dig[j];
+            const int64_t o = (int64_t)S.gbase[d] + (j - S.dstart[d]);
+            ls[o] = sv[u];
+            le[o] = ev[u];
+            li[o] = r[u] | (kind_of(ov[u]) << 30);
+        }
     }
 }
 
@@ -761,13 +777,8 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
             // stable partition by compact level id, ranges written in place
             const LevelDigit dg{rng->stream, rng->depth, d_cmap, perm};
             digit_offsets(c, dg, R, hist, part);
-            static unsigned place_attr = 0;
-            if (c.device < 32 && !(place_attr & (1u << c.device))) {
-                cudaFuncSetAttribute(k_level_place, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(PlaceSmem));
-                place_attr |= 1u << c.device;
-            }
             const int64_t ntiles = (R + RADIX_TILE - 1) / RADIX_TILE;
-            launch(c, "level_place", k_level_place, dim3((unsigned)ntiles), dim3(RADIX_THREADS), sizeof(PlaceSmem), dg,
+            launch(c, "level_place", k_level_place, dim3((unsigned)ntiles), dim3(RADIX_THREADS), 0, dg,
                    rng->start_ns, rng->end_ns, rng->op_id, R, (const uint32_t *)hist, ntiles, ls, le, li);
         } else {
             // stable partition by level key (13 bits)

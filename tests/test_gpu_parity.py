@@ -285,6 +285,24 @@ def test_aggregate_segment_lengths(opa, nan_frac):
     _check_aggregate(_gpu_aggregate(opa, t, rk, idx), o)
 
 
+@pytest.mark.parametrize("rows", ["identity", "swapped", "unmatched", "last"])
+def test_aggregate_identity_rows(opa, rows):
+    """Row index k for every kernel k (the ops pass skips the row-index
+    gather) and near misses that must take the gather: two kernels' rows
+    swapped, one kernel without a row, the last kernel's row moved."""
+    t, rk, _ = _agg_inputs(9, 150_000, [3, 64, 65, 300, 5000], 20_000)
+    K = len(rk)
+    idx = np.arange(K, dtype=np.int32)
+    if rows == "swapped":
+        idx[[10, 70_000]] = idx[[70_000, 10]]
+    elif rows == "unmatched":
+        idx[12_345] = -1
+    elif rows == "last":
+        idx[K - 1] = 0
+    o = oracle.aggregate(t.k_dur, rk, t.r_op, t.counters, idx, t.n_ops)
+    _check_aggregate(_gpu_aggregate(opa, t, rk, idx), o)
+
+
 def test_aggregate_reproducible(opa):
     """Two runs give bit-identical records although the fill pass orders each
     op's kernel list by atomics: segments are walked in ascending index."""
