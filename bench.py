@@ -33,6 +33,8 @@ PATH_BYTES = dict(kernel=29, range=22, ncu=84, op=184)
 
 # Per-launch algorithmic bytes of the kernels that can dominate a step.
 KERNEL_BYTES = {
+    # list 4 + duration 8 + row index 4 + counter row 80 per kernel (the row
+    # index is not read when every kernel's row is its own index: 92)
     "agg_ops": lambda K, R, M, O: 96 * K + 188 * O,
     "enclose": lambda K, R, M, O: 14 * K + 20 * R,
     "enclose_wide": lambda K, R, M, O: 14 * K + 20 * R,
@@ -395,6 +397,9 @@ def main():
     for _ in range(args.warmup):
         step()
     sync()
+    # rows matched one for one (the ops pass then skips the row-index gather)
+    if K > 0 and bool((idx == torch.arange(K, dtype=torch.int32, device=idx.device)).all()):
+        KERNEL_BYTES["agg_ops"] = lambda K, R, M, O: 92 * K + 188 * O
     # per-kernel breakdown: a few steps with every launch bracketed by events
     n_brk = max(1, min(args.steps, 10))
     ctx.set_timing(True)

@@ -6,12 +6,13 @@
 // share an op id aggregate together and no order of kernels or ranges is
 // needed.  Three passes over the kernels and one over the ops:
 //   count  validate each kernel, add up the totals, count kernels per op id
+//          and give each kernel its slot among its op's kernels
 //   scan   per-op offsets into one list of attributed kernels
-//   fill   place each attributed kernel in its op's segment
+//   place  put each attributed kernel in its slot of its op's segment
 //   ops    one thread per op id accumulates its segment in ascending kernel
-//          index -- the order the fill left is not used, so results do not
-//          depend on it -- and writes the op's record; ops without kernels
-//          get empty records in the same pass.
+//          index -- the order the count's atomics left is not used, so
+//          results do not depend on it -- and writes the op's record; ops
+//          without kernels get empty records in the same pass.
 // Accumulation is float-float with exact int64 weights (ff.cuh).
 #include <stdlib.h>
 #include <string.h>
@@ -508,7 +509,7 @@ __global__ void __launch_bounds__(SL_THREADS) k_agg_sort_long(const uint32_t *__
 // of op ids whatever each warp's pace (a fixed chunk-to-warp assignment lets
 // fast and slow warps drift apart and widens the band), and with op ids in
 // range order the kernels and outputs of that band stay in L2.  Segments are walked in ascending kernel index: a short one is checked
-// and, in the rare case the fill left it out of order, insertion-sorted in
+// and, in the rare case the placement left it out of order, insertion-sorted in
 // place by its thread; long ones were sorted by k_agg_sort_long.  While a
 // kernel is added, the counter rows and durations of the next two arrive in
 // per-thread shared-memory slots by asynchronous copy (cp.async), with their
@@ -598,7 +599,7 @@ __global__ void __launch_bounds__(AG_THREADS, 5) k_agg_ops(const uint32_t *__res
             const uint32_t s0 = off[o], len = off[o + 1] - s0;
             uint32_t *seg = list + s0;
             if (len > AG_HUGE) continue;                 // a huge op: k_agg_long_ops writes it
-            if (len <= AG_SHORT_MAX) {                   // ascending unless the fill met the op in two runs
+            if (len <= AG_SHORT_MAX) {                   // ascending unless the count met the op in two runs
                 bool up = true;
                 for (uint32_t t = 1; t < len; ++t) up &= seg[t - 1] < seg[t];
                 if (!up) {
@@ -1050,7 +1051,7 @@ namespace opattr {
 // per-class breakdown of the case studies): every attributed kernel whose
 // operator has a class is aggregated with the other kernels of that class.
 // Few, large groups: a stable radix sort of the kernels by class key (kernel
-// index order kept within a class) replaces the fill and the segment sort,
+// index order kept within a class) replaces the placement and the segment sort,
 // and every class is accumulated by pieces.
 __global__ void k_class_check(const uint32_t *__restrict__ class_of_op, int64_t n_ops, uint32_t n_classes,
                               DevStatus *st) {

@@ -304,7 +304,7 @@ def test_aggregate_identity_rows(opa, rows):
 
 
 def test_aggregate_reproducible(opa):
-    """Two runs give bit-identical records although the fill pass orders each
+    """Two runs give bit-identical records although the count pass orders each
     op's kernel list by atomics: segments are walked in ascending index."""
     t, rk, idx = _agg_inputs(8, 300_000, [3000, 700], 40_000)
     ctx = opa.Context(0)
