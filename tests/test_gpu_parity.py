@@ -623,3 +623,70 @@ def test_enclose_dense_ranges(opa, kids, p_kernel):
     o = oracle.run(t, enclose_mode="indexed")
     np.testing.assert_array_equal(g["range_of_kernel"], o["range_of_kernel"])
     np.testing.assert_array_equal(g["n_op_enclosing"], o["n_op_enclosing"])
+
+
+def _nesting_trace(case):
+    """Ranges over several 4,096-range tiles for the laminar checks: stream 0
+    parents each followed by one child (the parent in the child's tile),
+    stream 1 one long parent over 9,000 children (the parent tiles back),
+    stream 3 a child among 6,000 zero-length parents with its start (equal
+    starts across a tile boundary), and per case one defect."""
+    T = 500_000_000
+    st, s, e, d = [], [], [], []
+
+    def add(stream, a, b, depth):
+        st.append(stream); s.append(a); e.append(b); d.append(depth)
+    for i in range(6000):
+        add(0, i * 100, i * 100 + 90, 0)
+        add(0, i * 100 + 10, i * 100 + (95 if case == "past_near_parent" and i == 5000 else 50), 1)
+    add(1, 0, 1_000_000_000, 0)
+    for j in range(9000):
+        add(1, j * 100 + 5, 1_000_000_001 if case == "past_far_parent" and j == 8999 else j * 100 + 55, 1)
+    for q in range(6001):
+        if q == 3000:
+            add(3, T, T + (1 if case == "tie_past_parent" else 0), 1)
+        else:
+            add(3, T, T, 0)
+    if case == "orphan":
+        add(2, 500, 600, 1)
+    order = np.argsort(np.asarray(s, np.int64), kind="stable")
+    r_stream = np.asarray(st, np.uint8)[order]
+    r_start = np.asarray(s, np.int64)[order]
+    r_end = np.asarray(e, np.int64)[order]
+    r_depth = np.asarray(d, np.uint8)[order]
+    R = len(r_start)
+    rng = np.random.default_rng(5)
+    K = 3000
+    k_start = np.sort(rng.integers(0, 1_000_000_100, K)).astype(np.int64)
+    k_start[:5] = T                                   # a few kernels at the tied instant
+    k_start.sort()
+    k_stream = rng.integers(0, 4, K).astype(np.uint8)
+    return tracegen.Trace(k_stream, k_start, np.full(K, 1000, np.int64), np.zeros(K, np.uint32), None,
+                          r_stream, r_start, r_end, r_depth, np.arange(R, dtype=np.uint32), R,
+                          np.zeros(K, np.uint32), np.zeros((K, 20), np.float32))
+
+
+@pytest.mark.parametrize("case", ["valid", "past_near_parent", "past_far_parent", "orphan", "tie_valid",
+                                  "tie_past_parent"])
+def test_nesting_checks_across_tiles(opa, case):
+    """The laminar checks of the level lists -- parent found in the child's
+    tile, in an earlier tile, in a later tile through equal starts, or
+    missing -- give the oracle's status; valid traces give its enclosure."""
+    t = _nesting_trace(case)
+    want = oracle.validate_ranges(t.r_stream, t.r_start, t.r_end, t.r_depth)
+    assert (want == 0) == (case in ("valid", "tie_valid"))
+    ctx = opa.Context(0)
+    try:
+        if want != 0:
+            with pytest.raises(opa.OpattrError) as ei:
+                ctx.enclose(opa.to_device(t))
+            assert ei.value.status == want
+        else:
+            st, rk, nop = ctx.enclose(opa.to_device(t))
+            ost, ork, onop = oracle.enclose(t.k_stream, t.k_start, t.r_stream, t.r_start, t.r_end, t.r_depth,
+                                            t.r_op)
+            assert st == ost == 0
+            np.testing.assert_array_equal(rk.cpu().numpy(), ork)
+            np.testing.assert_array_equal(nop.cpu().numpy(), onop)
+    finally:
+        ctx.close()
