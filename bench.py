@@ -512,7 +512,10 @@ def main():
                    "l2": "inputs larger than L2 (129 MB)" if flush is None else "L2 flushed before every step"},
         "roofline": {"bound": "hbm", "kernel": dname, "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": (achieved / peak) if achieved else None, "peak_kind": f"{peak_kind} copy bandwidth",
-                     "traffic": recorded_traffic(dname, args.config, K), "alg_bytes_per_launch": dbytes,
+                     # recorded on the default options only (the variants change what the kernels move)
+                     "traffic": (recorded_traffic(dname, args.config, K) if not (
+                         args.shuffle or args.per_stream_ncu or args.tiers or args.rollup or args.launch_lag)
+                         else None), "alg_bytes_per_launch": dbytes,
                      "avg_launch_ms": avg_s * 1e3,
                      "launches": dcount},
         "path_roofline": {"alg_bytes_per_step": path_bytes, "achieved_gbs": path_gbs,
