@@ -690,3 +690,15 @@ def test_nesting_checks_across_tiles(opa, case):
             np.testing.assert_array_equal(nop.cpu().numpy(), onop)
     finally:
         ctx.close()
+
+
+@pytest.mark.parametrize("shuffle,per_stream", [(False, False), (True, False), (False, True)])
+def test_max_streams_and_depth(opa, shuffle, per_stream):
+    """Every stream id (0..255) and every depth (0..31): thousands of levels
+    (the radix-sorted level lists and the wide enclosure layout), in time
+    order and permuted, and with per-stream ncu rows: against the oracle."""
+    t = tracegen.generate("adversarial", n_kernels=400_000, n_streams=256, seed=21, shuffle=shuffle)
+    assert len(np.unique(t.r_stream)) == 256 and int(t.r_depth.max()) == 31
+    if per_stream:
+        t = tracegen.per_stream_runs(t)
+    assert_parity(gpu_run(t), oracle.run(t, enclose_mode="indexed"))
