@@ -364,7 +364,15 @@ def main():
             f"cuda:{dev}")
         rollup_out = ctx.alloc_ops(args.rollup)
 
+    join_out = dict(range_of_kernel=rk, n_op_enclosing=nop, ncu_idx=idx, match_kind=kind)
+
     def join():
+        if tq is tr and tiers_out is None:
+            # the whole join in one call (one kernel-order check for both steps)
+            ctx.join(tr, dedup=use_dedup, out=join_out, ops=ops)
+            if rollup_out is not None:
+                ctx.rollup(tr, rk, idx, class_of_op, args.rollup, out=rollup_out)
+            return
         ctx.enclose(tq, rk, nop)
         if tiers_out is not None:
             ctx.attribute(tr, rk, nop, out=tiers_out)
@@ -438,7 +446,7 @@ def main():
     t_max, units = combine_ranks(max(elapsed, 1e-9), K * args.steps, world, rmax, rsum)
 
     # ---- end to end through the C ABI with host buffers (pinned), per step:
-    # H2D of every input array, the three calls, D2H of every output
+    # H2D of every input array, the join, D2H of every output
     host = {name: torch.from_numpy(getattr(trace, name)).pin_memory()
             for name in ("k_stream", "k_start", "k_dur", "k_name", "r_stream", "r_start", "r_end", "r_depth",
                          "r_op", "ncu_name", "counters") + (("corr_name", "corr_inv", "corr_op", "fusion_op",

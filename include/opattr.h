@@ -320,6 +320,21 @@ opattr_status opattr_aggregate(opattr_ctx *ctx, const opattr_kernels *kernels, c
                                const int32_t *ncu_idx_of_kernel, uint32_t n_ops,
                                const opattr_op_aggregates *dev_out, opattr_totals *host_totals);
 
+/* The whole join in one call: opattr_enclose, opattr_match and
+ * opattr_aggregate on the same kernel records, in that order, with the same
+ * arguments and outputs as the three calls (range_of_kernel is written by the
+ * enclosure and read by the aggregation, ncu_idx_of_kernel likewise from the
+ * matching).  The kernel records' time order is verified once for both the
+ * enclosure and the matching.
+ *   n_op_enclosing, match_kind, host_summary, host_totals  may be NULL
+ * Returns the first error of the three steps (later steps are not run), else
+ * the matching's warning if it gave one, else OPATTR_OK. */
+opattr_status opattr_join(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,
+                          const opattr_ncu *ncu, const opattr_dedup *dedup, uint32_t n_ops,
+                          int32_t *range_of_kernel, uint8_t *n_op_enclosing, int32_t *ncu_idx_of_kernel,
+                          uint8_t *match_kind, const opattr_op_aggregates *dev_out,
+                          opattr_match_summary *host_summary, opattr_totals *host_totals);
+
 /* The attribution tiers of Fig. 2 for every kernel (see above).
  *   range_of_kernel  i32[kernels->n]  device, opattr_enclose's result
  *   n_op_enclosing   u8[kernels->n]   device, opattr_enclose's count, or NULL

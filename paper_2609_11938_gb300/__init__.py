@@ -23,7 +23,7 @@ __all__ = [
     "OK", "W_COUNT_MISMATCH", "W_DEDUP_MISMATCH", "E_INVALID_ARG", "E_NOT_NESTED", "E_DEPTH",
     "E_COUNT_MISMATCH", "E_CUDA", "E_OOM", "E_TIMEOUT", "E_STATE", "OP_STRUCTURAL", "OP_NONOP",
     "N_COUNTERS", "OpattrError", "Context", "library", "build",
-    "opattr_create", "opattr_enclose", "opattr_match", "opattr_aggregate", "opattr_destroy",
+    "opattr_create", "opattr_enclose", "opattr_match", "opattr_aggregate", "opattr_join", "opattr_destroy",
     "opattr_status_string", "opattr_match_noalloc", "MATCH_NOALLOC_MAX",
 ]
 
@@ -136,6 +136,8 @@ def library():
             lib.opattr_match.argtypes = [_vp, P(Kernels), P(Ncu), P(Dedup), _vp, _vp, P(MatchSummary)]
             lib.opattr_aggregate.argtypes = [_vp, P(Kernels), P(Ranges), _vp, P(Ncu), _vp, ctypes.c_uint32,
                                              P(OpAggregates), P(Totals)]
+            lib.opattr_join.argtypes = [_vp, P(Kernels), P(Ranges), P(Ncu), P(Dedup), ctypes.c_uint32, _vp, _vp, _vp,
+                                        _vp, P(OpAggregates), P(MatchSummary), P(Totals)]
             lib.opattr_attribute.argtypes = [_vp, P(Kernels), P(Ranges), _vp, _vp, P(Corr), P(Fusion),
                                              ctypes.c_uint32, _vp, _vp, _vp, _vp, P(AttrSummary)]
             lib.opattr_rollup.argtypes = [_vp, P(Kernels), P(Ranges), _vp, P(Ncu), _vp, ctypes.c_uint32, _vp,
@@ -203,6 +205,15 @@ def opattr_aggregate(handle, kernels: Kernels, ranges: Ranges, rok_ptr: int, ncu
     return library().opattr_aggregate(handle, ctypes.byref(kernels), ctypes.byref(ranges), _vp(rok_ptr),
                                       ctypes.byref(ncu), _vp(idx_ptr), ctypes.c_uint32(n_ops), ctypes.byref(out),
                                       ctypes.byref(totals))
+
+
+def opattr_join(handle, kernels: Kernels, ranges: Ranges, ncu: Ncu, dedup: Dedup | None, n_ops: int, rok_ptr: int,
+                nop_ptr: int | None, idx_ptr: int, kind_ptr: int | None, out: OpAggregates, summary: MatchSummary,
+                totals: Totals) -> int:
+    return library().opattr_join(handle, ctypes.byref(kernels), ctypes.byref(ranges), ctypes.byref(ncu),
+                                 ctypes.byref(dedup) if dedup is not None else None, ctypes.c_uint32(n_ops),
+                                 _vp(rok_ptr), _vp(nop_ptr or 0), _vp(idx_ptr), _vp(kind_ptr or 0), ctypes.byref(out),
+                                 ctypes.byref(summary), ctypes.byref(totals))
 
 
 def opattr_attribute(handle, kernels: Kernels, ranges: Ranges, rok_ptr: int, nop_ptr: int | None,
@@ -422,22 +433,26 @@ class Context:
             raise OpattrError(st, "opattr_enclose")
         return st, out_range, out_nop
 
-    def match(self, tr: DeviceTrace, dedup: bool | None = None, out_idx=None, out_kind=None):
+    @staticmethod
+    def _dedup(tr: DeviceTrace, dedup: bool | None):
+        """(Dedup struct or None, the host arrays it points into)."""
         import numpy as np
+        use = (tr.class_of_layer is not None and tr.k_layer is not None) if dedup is None else dedup
+        if not use:
+            return None, None
+        col = np.ascontiguousarray(tr.class_of_layer, dtype=np.int32)
+        roc = np.ascontiguousarray(tr.rep_of_class, dtype=np.int32)
+        return Dedup(col.ctypes.data if col.size else None, roc.ctypes.data if roc.size else None, len(col),
+                     len(roc)), (col, roc)
+
+    def match(self, tr: DeviceTrace, dedup: bool | None = None, out_idx=None, out_kind=None):
         import torch
         dev = f"cuda:{self.device}"
         if out_idx is None:
             out_idx = torch.empty(tr.K, dtype=torch.int32, device=dev)
         if out_kind is None:
             out_kind = torch.empty(tr.K, dtype=torch.uint8, device=dev)
-        dd = None
-        keep = None
-        use = (tr.class_of_layer is not None and tr.k_layer is not None) if dedup is None else dedup
-        if use:
-            col = np.ascontiguousarray(tr.class_of_layer, dtype=np.int32)
-            roc = np.ascontiguousarray(tr.rep_of_class, dtype=np.int32)
-            keep = (col, roc)
-            dd = Dedup(col.ctypes.data if col.size else None, roc.ctypes.data if roc.size else None, len(col), len(roc))
+        dd, keep = self._dedup(tr, dedup)
         summ = MatchSummary()
         st = opattr_match(self.handle, self.kernels(tr), self.ncu(tr), dd,
                           _ptr(out_idx, torch.int32, "ncu_idx_of_kernel", self.device),
@@ -446,6 +461,36 @@ class Context:
         if st < 0:
             raise OpattrError(st, "opattr_match")
         return st, out_idx, out_kind, summ.as_dict()
+
+    def join(self, tr: DeviceTrace, dedup: bool | None = None, out=None, ops=None):
+        """enclose + match + aggregate in one call (opattr_join).  `out` may hold
+        preallocated range_of_kernel / n_op_enclosing / ncu_idx / match_kind
+        tensors; returns (status, out, ops, match summary, totals)."""
+        import torch
+        dev = f"cuda:{self.device}"
+        dv = self.device
+        out = dict(out or {})
+        for k, dt in (("range_of_kernel", torch.int32), ("n_op_enclosing", torch.uint8), ("ncu_idx", torch.int32),
+                      ("match_kind", torch.uint8)):
+            if out.get(k) is None:
+                out[k] = torch.empty(tr.K, dtype=dt, device=dev)
+        if ops is None:
+            ops = self.alloc_ops(tr.n_ops)
+        agg = OpAggregates(_ptr(ops["kernel_count"], torch.int64, "kernel_count", dv),
+                           _ptr(ops["total_duration_ns"], torch.int64, "total_duration_ns", dv),
+                           _ptr(ops["matched_count"], torch.int64, "matched_count", dv),
+                           _ptr(ops["agg"], torch.float64, "agg", dv))
+        dd, keep = self._dedup(tr, dedup)
+        summ, tot = MatchSummary(), Totals()
+        st = opattr_join(self.handle, self.kernels(tr), self.ranges(tr), self.ncu(tr), dd, tr.n_ops,
+                         _ptr(out["range_of_kernel"], torch.int32, "range_of_kernel", dv),
+                         _ptr(out["n_op_enclosing"], torch.uint8, "n_op_enclosing", dv),
+                         _ptr(out["ncu_idx"], torch.int32, "ncu_idx_of_kernel", dv),
+                         _ptr(out["match_kind"], torch.uint8, "match_kind", dv), agg, summ, tot)
+        del keep
+        if st < 0:
+            raise OpattrError(st, "opattr_join")
+        return st, out, ops, summ.as_dict(), tot.as_dict()
 
     def alloc_ops(self, n_ops: int):
         import torch

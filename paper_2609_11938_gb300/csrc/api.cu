@@ -227,6 +227,29 @@ opattr_status opattr_aggregate(opattr_ctx *ctx, const opattr_kernels *kernels, c
                                   host_totals));
 }
 
+opattr_status opattr_join(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,
+                          const opattr_ncu *ncu, const opattr_dedup *dedup, uint32_t n_ops,
+                          int32_t *range_of_kernel, uint8_t *n_op_enclosing, int32_t *ncu_idx_of_kernel,
+                          uint8_t *match_kind, const opattr_op_aggregates *dev_out,
+                          opattr_match_summary *host_summary, opattr_totals *host_totals) {
+    if (!ctx || !kernels || !ranges || !ncu) return OPATTR_E_INVALID_ARG;
+    Ctx &c = ctx->c;
+    if (c.broken) return OPATTR_E_STATE;
+    DeviceGuard g(c.device);
+    if (!g.ok) return OPATTR_E_CUDA;
+    c.enclose_k_sorted = -1;
+    opattr_status st = finish(c, do_enclose(c, kernels, ranges, range_of_kernel, n_op_enclosing));
+    if (st < 0) return st;
+    c.order_from_enclose = true;
+    const opattr_status sm = finish(c, do_match(c, kernels, ncu, dedup, ncu_idx_of_kernel, match_kind, host_summary));
+    c.order_from_enclose = false;
+    if (sm < 0) return sm;
+    st = finish(c, do_aggregate(c, kernels, ranges, range_of_kernel, ncu, ncu_idx_of_kernel, n_ops, dev_out,
+                                host_totals));
+    if (st < 0) return st;
+    return sm;
+}
+
 opattr_status opattr_attribute(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,
                                const int32_t *range_of_kernel, const uint8_t *n_op_enclosing, const opattr_corr *corr,
                                const opattr_fusion *fusion, uint32_t n_ops, uint32_t *op_of_kernel, uint8_t *tier,

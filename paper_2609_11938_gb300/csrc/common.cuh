@@ -89,6 +89,10 @@ struct Ctx {
                                      // the aggregation reuses it for a few values read mid-call
     cudaEvent_t ev_aux = nullptr;    // marks a mid-call host read (created on first use)
     unsigned char *h_stage = nullptr; // pinned staging for small host-built tables [STAGE_BYTES]
+    // kernel time order as the last enclosure found it (-1 unknown, 0 / 1),
+    // and whether the matching may take it instead of checking again (join)
+    int enclose_k_sorted = -1;
+    bool order_from_enclose = false;
     // launch accounting
     int64_t launches = 0;
     bool timing = false;

@@ -689,6 +689,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     if ((st = status_from_err(c.h_status->err))) return st;
     const bool k_sorted = !(c.h_status->flags & F_K_UNSORTED);
     const bool r_sorted = !(c.h_status->flags & F_R_UNSORTED);
+    c.enclose_k_sorted = k_sorted ? 1 : 0;
     const long long rmin = c.h_status->mm[MM_RSTART_MIN], rmax = c.h_status->mm[MM_REND_MAX];
     const long long kmin = c.h_status->mm[MM_KSTART_MIN], kmax = c.h_status->mm[MM_KSTART_MAX];
     if (K > 0 && (kmax - kmin) >= (1ll << 55)) return OPATTR_E_INVALID_ARG;

@@ -438,7 +438,9 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     }
 
     const unsigned gK = grid_for(K, 256, REDUCE_GRID);
-    check_kernel_order(c, kern->stream, kern->start_ns, K);
+    // within a join the enclosure has just verified these records' order
+    const bool known_sorted = c.order_from_enclose && c.enclose_k_sorted == 1;
+    if (!known_sorted) check_kernel_order(c, kern->stream, kern->start_ns, K);
     if (dedup_on && K > 0)
         launch(c, "check_layers", k_check_layers, dim3(gK), dim3(256), 0, kern->layer_id, K, dd->n_layers,
                (const int32_t *)d_rep, c.d_status);
@@ -457,7 +459,7 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
                      out_kind);
     if ((st = read_status(c))) return st;
     if (c.h_status->err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
-    const bool k_sorted = !(c.h_status->flags & F_K_UNSORTED);
+    const bool k_sorted = known_sorted || !(c.h_status->flags & F_K_UNSORTED);
     opattr_match_summary S{};
     S.kernels = K;
     S.replayed = dedup_on ? (int64_t)c.h_status->cnt[C_REPLAYED] : K;

@@ -702,3 +702,65 @@ def test_max_streams_and_depth(opa, shuffle, per_stream):
     if per_stream:
         t = tracegen.per_stream_runs(t)
     assert_parity(gpu_run(t), oracle.run(t, enclose_mode="indexed"))
+
+
+def _join_cases(name):
+    if name == "large1m":
+        return tracegen.generate("large", n_kernels=1_000_000)
+    if name == "gpt2_shuffled":
+        return tracegen.generate("gpt2", shuffle=True)
+    if name == "dedup_per_stream":
+        return tracegen.per_stream_runs(tracegen.generate("dedup"))
+    if name == "gpt2_count_mismatch":
+        t = tracegen.generate("gpt2")
+        keep = np.setdiff1d(np.arange(t.M), np.random.default_rng(7).choice(t.M, 25, replace=False))
+        t.ncu_name, t.counters = t.ncu_name[keep].copy(), t.counters[keep].copy()
+        return t
+    return tracegen.generate(name)
+
+
+@pytest.mark.parametrize("name", ["large1m", "gpt2_shuffled", "dedup", "dedup_per_stream", "gpt2_count_mismatch",
+                                  "tiny"])
+def test_join_matches_three_calls(opa, name):
+    """opattr_join gives the three calls' outputs bit for bit (the order
+    verdict shared between enclosure and matching, sorted or not), their
+    warning, and the oracle's results."""
+    t = _join_cases(name)
+    tr = opa.to_device(t)
+    dd = bool(t.config.get("dedup")) and t.k_layer is not None     # as the oracle decides
+    ctx = opa.Context(0)
+    try:
+        st, out, ops, summ, tot = ctx.join(tr, dedup=dd)
+        e_st, rk, nop = ctx.enclose(tr)
+        m_st, idx, kind, msumm = ctx.match(tr, dedup=dd)
+        a_st, ops3, tot3 = ctx.aggregate(tr, rk, idx)
+    finally:
+        ctx.close()
+    assert st == (m_st if m_st > 0 else a_st)
+    np.testing.assert_array_equal(out["range_of_kernel"].cpu().numpy(), rk.cpu().numpy())
+    np.testing.assert_array_equal(out["n_op_enclosing"].cpu().numpy(), nop.cpu().numpy())
+    np.testing.assert_array_equal(out["ncu_idx"].cpu().numpy(), idx.cpu().numpy())
+    np.testing.assert_array_equal(out["match_kind"].cpu().numpy(), kind.cpu().numpy())
+    for k in ops:
+        assert np.array_equal(ops[k].cpu().numpy().view(np.int64), ops3[k].cpu().numpy().view(np.int64)), k
+    assert summ == msumm and tot == tot3
+    o = oracle.run(t, enclose_mode="indexed")
+    np.testing.assert_array_equal(out["range_of_kernel"].cpu().numpy(), o["range_of_kernel"])
+    np.testing.assert_array_equal(out["ncu_idx"].cpu().numpy(), o["ncu_idx"])
+
+
+def test_join_stops_at_the_first_error(opa):
+    """A nesting error in the enclosure ends the join with that error; the
+    context stays usable."""
+    u = _nesting_trace("orphan")
+    ctx = opa.Context(0)
+    try:
+        with pytest.raises(opa.OpattrError) as ei:
+            ctx.join(opa.to_device(u))
+        assert ei.value.status == opa.E_NOT_NESTED
+        t = tracegen.generate("tiny")
+        st, out, ops, summ, tot = ctx.join(opa.to_device(t))
+        o = oracle.run(t, enclose_mode="brute")
+        np.testing.assert_array_equal(out["range_of_kernel"].cpu().numpy(), o["range_of_kernel"])
+    finally:
+        ctx.close()
