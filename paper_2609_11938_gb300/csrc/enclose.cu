@@ -851,11 +851,18 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
             }
         }
         if ((st = read_status(c))) return st;
+        if (!full_sort && (c.h_status->flags & F_LEVEL_FIXUP)) {
+            // equal starts out of (start, end) order within a level: the
+            // nesting checks above saw a level list out of order, so their
+            // verdict does not count; the pass on fully sorted ranges decides
+            c.h_status->flags &= ~F_LEVEL_FIXUP;
+            c.h_status->err = 0;
+            cudaMemsetAsync(c.d_status, 0, 2 * sizeof(unsigned), c.stream);   // err and flags
+            continue;
+        }
         if ((st = status_from_err(c.h_status->err))) return st;
-        if (!(c.h_status->flags & F_LEVEL_FIXUP)) return OPATTR_OK;
-        if (full_sort) return OPATTR_E_CUDA;      // a full sort leaves no equal-start disorder
-        c.h_status->flags &= ~F_LEVEL_FIXUP;
-        cudaMemsetAsync(&c.d_status->flags, 0, sizeof(unsigned), c.stream);
+        if (c.h_status->flags & F_LEVEL_FIXUP) return OPATTR_E_CUDA;   // a full sort leaves no such disorder
+        return OPATTR_OK;
     }
     return OPATTR_E_CUDA;
 }

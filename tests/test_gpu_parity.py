@@ -764,3 +764,50 @@ def test_join_stops_at_the_first_error(opa):
         np.testing.assert_array_equal(out["range_of_kernel"].cpu().numpy(), o["range_of_kernel"])
     finally:
         ctx.close()
+
+
+def _equal_starts_trace():
+    """Ranges sorted by start whose equal-start pairs at one depth are not in
+    (start, end) order -- a long range listed before a zero-length one at the
+    same instant -- with children below the long ones, over several tiles."""
+    st, s, e, d = [], [], [], []
+    for i in range(3000):
+        a = i * 1000
+        st += [0, 0, 0]
+        s += [a, a, a + 10]
+        e += [a + 500, a, a + 20]
+        d += [0, 0, 1]
+    R = len(s)
+    rng = np.random.default_rng(9)
+    K = 20_000
+    k_start = np.sort(np.concatenate([rng.integers(0, 3_000_000, K - 3000), np.arange(3000) * 1000])).astype(np.int64)
+    K = len(k_start)
+    return tracegen.Trace(np.zeros(K, np.uint8), k_start, np.full(K, 100, np.int64),
+                          rng.integers(0, 50, K).astype(np.uint32), None,
+                          np.asarray(st, np.uint8), np.asarray(s, np.int64), np.asarray(e, np.int64),
+                          np.asarray(d, np.uint8), np.arange(R, dtype=np.uint32), R,
+                          rng.integers(0, 50, K).astype(np.uint32), rng.uniform(0, 100, (K, 20)).astype(np.float32))
+
+
+def test_equal_starts_out_of_order(opa):
+    """The level lists' equal-start fix-up (the enclosure redone on fully
+    sorted ranges), through the enclosure alone and through the join, whose
+    enclosure status is read at the matching's wait: the oracle's results."""
+    t = _equal_starts_trace()
+    t.ncu_name = t.k_name.copy()
+    o = oracle.run(t, enclose_mode="indexed")
+    assert o["enclose_status"] == 0
+    ctx = opa.Context(0)
+    try:
+        tr = opa.to_device(t)
+        st, rk, nop = ctx.enclose(tr)
+        np.testing.assert_array_equal(rk.cpu().numpy(), o["range_of_kernel"])
+        np.testing.assert_array_equal(nop.cpu().numpy(), o["n_op_enclosing"])
+        st, out, ops, summ, tot = ctx.join(tr, dedup=False)
+        np.testing.assert_array_equal(out["range_of_kernel"].cpu().numpy(), o["range_of_kernel"])
+        np.testing.assert_array_equal(out["n_op_enclosing"].cpu().numpy(), o["n_op_enclosing"])
+        np.testing.assert_array_equal(out["ncu_idx"].cpu().numpy(), o["ncu_idx"])
+        for k in ("kernel_count", "total_duration_ns", "matched_count"):
+            np.testing.assert_array_equal(ops[k].cpu().numpy(), o["ops"][k])
+    finally:
+        ctx.close()
