@@ -300,17 +300,18 @@ __device__ __forceinline__ int32_t range_of_t(const int32_t *rok, const uint32_t
 }
 
 // ------------------------------------------------------------------ count
-// Per kernel: duration >= 0, range index in [-1, R), an attributed range is an
-// operator below n_ops, row index in [-1, M).  Totals: all / attributed time,
-// attributed and matched kernel counts.  Whether every kernel's row is its
-// own index (the match of a trace whose ncu rows follow the kernels one for
-// one) is noted, so the ops pass can skip the row-index gather.  Each attributed kernel (valid range
-// and op id) also takes its slot among its op's kernels: one atomic per
-// distinct op id of a warp on cnt[op], whose old value plus the kernel's rank
-// among its warp peers is the slot (rank[k]); cnt ends as the per-op counts.
-// Each warp takes a run of `run` consecutive kernels (a multiple of 32, up to
-// AF_RUN) 32 at a time in index order, so an op whose kernels all lie in one
-// run gets ascending slots; the ops pass sorts the few segments that do not.
+// Per kernel: duration >= 0, range index in [-1, R), an attributed range is
+// an operator below n_ops, row index in [-1, M).  Totals: all / attributed
+// time, attributed and matched kernel counts.  Whether every kernel's row is
+// its own index (the match of a trace whose ncu rows follow the kernels one
+// for one) is noted, so the ops pass can skip the row-index gather.  Each
+// attributed kernel (valid range and op id) also takes its slot among its
+// op's kernels: one atomic per distinct op id of a warp on cnt[op], whose old
+// value plus the kernel's rank among its warp peers is the slot (rank[k]);
+// cnt ends as the per-op counts.  Each warp takes a run of `run` consecutive
+// kernels (a multiple of 32, up to AF_RUN) 32 at a time in index order, so an
+// op whose kernels all lie in one run gets ascending slots; the ops pass
+// sorts the few segments that do not.
 constexpr int AF_RUN = 2048;
 
 template <bool DIRECT>
@@ -508,12 +509,14 @@ __global__ void __launch_bounds__(SL_THREADS) k_agg_sort_long(const uint32_t *__
 // from one counter, so the ops in flight at any moment are one narrow band
 // of op ids whatever each warp's pace (a fixed chunk-to-warp assignment lets
 // fast and slow warps drift apart and widens the band), and with op ids in
-// range order the kernels and outputs of that band stay in L2.  Segments are walked in ascending kernel index: a short one is checked
-// and, in the rare case the placement left it out of order, insertion-sorted in
-// place by its thread; long ones were sorted by k_agg_sort_long.  While a
-// kernel is added, the counter rows and durations of the next two arrive in
-// per-thread shared-memory slots by asynchronous copy (cp.async), with their
-// row indices loaded a step earlier still.
+// range order the kernels and outputs of that band stay in L2.  Segments are
+// walked in ascending kernel index: a short one is checked and, in the rare
+// case the placement left it out of order, insertion-sorted in place by its
+// thread; long ones were sorted by k_agg_sort_long.  While a kernel is
+// added, the counter rows and durations of the next two arrive in per-thread
+// shared-memory slots by asynchronous copy (cp.async), with their row
+// indices loaded a step earlier still (or taken to be the kernel indices
+// when the count pass found every row to be its kernel's own index).
 constexpr int AG_THREADS = 128;                // five blocks per SM (96 registers, a few spilled)
 constexpr int AG_WARPS = AG_THREADS / 32;
 constexpr int AG_CHUNK = 64;                    // op ids per warp and chunk
