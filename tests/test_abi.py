@@ -19,7 +19,8 @@ def declared_functions():
 
 def test_header_declares_the_join():
     names = declared_functions()
-    for f in ("opattr_create", "opattr_enclose", "opattr_match", "opattr_aggregate", "opattr_destroy"):
+    for f in ("opattr_create", "opattr_enclose", "opattr_match", "opattr_aggregate", "opattr_destroy",
+              "opattr_join", "opattr_attribute", "opattr_rollup", "opattr_write_profile", "opattr_match_noalloc"):
         assert f in names
 
 
@@ -60,3 +61,19 @@ def test_create_without_gpu_fails_cleanly():
     import paper_2609_11938_gb300 as opa
     st, h = opa.opattr_create(0)
     assert st in (opa.E_CUDA, opa.E_INVALID_ARG) and not h
+
+
+def test_calls_without_a_context_are_rejected():
+    """Every call checks its context and record structs before touching a
+    device: a NULL context gives OPATTR_E_INVALID_ARG (no GPU needed)."""
+    import paper_2609_11938_gb300 as opa
+    lib = opa.library()
+    k, r, n = opa.Kernels(), opa.Ranges(), opa.Ncu()
+    agg, tot, summ = opa.OpAggregates(), opa.Totals(), opa.MatchSummary()
+    by = ctypes.byref
+    assert lib.opattr_enclose(None, by(k), by(r), None, None) == opa.E_INVALID_ARG
+    assert lib.opattr_match(None, by(k), by(n), None, None, None, by(summ)) == opa.E_INVALID_ARG
+    assert lib.opattr_aggregate(None, by(k), by(r), None, by(n), None, 0, by(agg), by(tot)) == opa.E_INVALID_ARG
+    assert lib.opattr_join(None, by(k), by(r), by(n), None, 0, None, None, None, None, by(agg), by(summ),
+                           by(tot)) == opa.E_INVALID_ARG
+    assert lib.opattr_rollup(None, by(k), by(r), None, by(n), None, 0, None, 0, by(agg)) == opa.E_INVALID_ARG
