@@ -25,7 +25,7 @@ UNIT = "M kernels/s"
 NOMINAL_HBM_GBS = 8000.0
 L2_BYTES = 129 * 2**20
 
-# Algorithmic bytes per unit (the minimum each step must move; see DESIGN.md):
+# Algorithmic bytes per unit (the minimum each step must move):
 #   per kernel: stream 1 + start 8 + dur 8 + name 4 read, range 4 + ncu_idx 4 written
 #   per range: stream 1 + start 8 + end 8 + depth 1 + op 4 read
 #   per ncu row: name 4 + 20 counters x 4 read;  per op: 3 x 8 + 20 x 8 written
@@ -226,28 +226,47 @@ class ClockSampler:
 
 
 # ---------------------------------------------------------------- CPU baseline (the oracle)
-def oracle_sample_config(config_name: str, n_kernels: int):
+def cpu_model() -> str:
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for ln in out.splitlines():
+            if ln.strip().lower().startswith("model name"):
+                return ln.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for ln in f:
+                if ln.lower().startswith(("model name", "cpu part")):
+                    return ln.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
+def time_oracle_full(trace, threads: int):
+    """The CPU oracle (indexed mode) on the whole trace: one thread
+    (oracle.run) or `threads` host threads (oracle.parallel.run_threads, the
+    same functions over streams / names / op blocks).  Returns seconds."""
+    import oracle
+    t0 = time.perf_counter()
+    if threads == 1:
+        res = oracle.run(trace, enclose_mode="indexed")
+    else:
+        from oracle.parallel import run_threads
+        res = run_threads(trace, threads)
+    dt = time.perf_counter() - t0
+    assert res["aggregate_status"] == 0 and res["enclose_status"] == 0
+    return dt
+
+
+def reference_trace(config_name: str, n_kernels: int = 0, shuffle: bool = False):
     import tracegen
     cfg = tracegen.config(config_name)
-    if cfg.get("shape", 0) == 0:
+    if n_kernels and cfg.get("shape", 0) == 0:
         cfg["n_kernels"] = n_kernels
-    return cfg
-
-
-def time_oracle(config_name: str, n_kernels: int = 1_000_000, reps: int = 1):
-    """The CPU oracle (indexed mode, single thread) on a bounded sample of the
-    workload: the same generator parameters with fewer kernels."""
-    import oracle
-    import tracegen
-    t = tracegen.generate(oracle_sample_config(config_name, n_kernels))
-    best = None
-    for _ in range(reps):
-        t0 = time.perf_counter()
-        res = oracle.run(t, enclose_mode="indexed")
-        dt = time.perf_counter() - t0
-        assert res["aggregate_status"] == 0
-        best = dt if best is None else min(best, dt)
-    return t.K, best
+    return tracegen.generate(cfg, shuffle=shuffle)
 
 
 # ---------------------------------------------------------------- main
@@ -260,7 +279,8 @@ def main():
     ap.add_argument("--config", default="large", choices=sorted(WORKLOADS))
     ap.add_argument("--shuffle", action="store_true", help="permute kernel and range arrays (general paths)")
     ap.add_argument("--e2e-steps", type=int, default=5)
-    ap.add_argument("--oracle-kernels", type=int, default=1_000_000)
+    ap.add_argument("--no-oracle-single", dest="oracle_single", action="store_false",
+                    help="skip the single-thread oracle run of the CPU baseline (it takes about 15 s on large)")
     ap.add_argument("--per-stream-ncu", action="store_true",
                     help="ncu rows as per-stream replay runs, matched per (name, stream)")
     ap.add_argument("--tiers", action="store_true",
@@ -278,24 +298,28 @@ def main():
         args.warmup = 3
 
     if args.impl == "reference":
+        # the oracle on the whole workload in all host threads, each step one
+        # full join; rank 0 alone (the other ranks exit without work)
         if rank != 0:
             return
-        n, _ = time_oracle(args.config, args.oracle_kernels, reps=1)       # warm caches
-        times = []
+        trace = reference_trace(args.config, args.kernels, args.shuffle)
+        threads = os.cpu_count() or 1
         for _ in range(args.warmup):
-            time_oracle(args.config, args.oracle_kernels)
-        for _ in range(args.steps):
-            times.append(time_oracle(args.config, args.oracle_kernels)[1])
+            time_oracle_full(trace, threads)
+        times = [time_oracle_full(trace, threads) for _ in range(args.steps)]
         tot = sum(times)
-        value = n * len(times) / tot / 1e6
+        value = trace.K * len(times) / tot / 1e6
+        sample = (f"the whole {args.config} trace ({trace.K} kernels, {trace.R} ranges, {trace.M} ncu rows, "
+                  f"{trace.n_ops} ops) every step; indexed oracle (enclose + match + aggregate) over {threads} "
+                  f"host threads ({cpu_model()})")
         line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
                 "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / len(times),
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-                "data": "synthetic", "config": {"workload": f"{args.config}: {WORKLOADS[args.config]}",
-                                                "sample_kernels": n},
-                "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                                 "sample": f"{n} kernels drawn with the {args.config} generator parameters; "
-                                           f"indexed oracle (enclose + match + aggregate), single thread"},
+                "data": "synthetic", "config": {"workload": f"{args.config}: {WORKLOADS[args.config]}" + (
+                    f" [scaled to {trace.K} kernels]" if args.kernels else ""), "kernels": trace.K,
+                    "same_config": not args.kernels},
+                "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle",
+                                 "sample": sample},
                 "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
         print(json.dumps(line))
         return
@@ -498,7 +522,10 @@ def main():
     path_gbs = path_bytes / step_s / 1e9
     ctx.close()
 
-    n_or, t_or = time_oracle(args.config, args.oracle_kernels)
+    # the oracle on the same whole trace, one thread and all host threads
+    threads = os.cpu_count() or 1
+    t_or1 = time_oracle_full(trace, 1) if args.oracle_single else None
+    t_orn = time_oracle_full(trace, threads)
     line = {
         "metric": METRIC,
         "value": units / t_max / 1e6,
@@ -528,9 +555,11 @@ def main():
                      "launches": dcount},
         "path_roofline": {"alg_bytes_per_step": path_bytes, "achieved_gbs": path_gbs,
                           "frac_of_8tbs": path_gbs / NOMINAL_HBM_GBS, "frac_of_measured": path_gbs / peak},
-        "cpu_baseline": {"value": n_or / t_or / 1e6, "unit": UNIT, "cores": 1, "kind": "oracle",
-                         "sample": f"{n_or} kernels drawn with the {args.config} generator parameters; indexed "
-                                   f"oracle (enclose + match + aggregate), single thread, {t_or:.2f} s"},
+        "cpu_baseline": {"value": K / t_orn / 1e6, "unit": UNIT, "cores": threads, "kind": "oracle",
+                         "sample": f"the whole trace timed on ({K} kernels), {t_orn:.2f} s; indexed oracle (enclose + "
+                                   f"match + aggregate) over {threads} host threads ({cpu_model()})",
+                         "single_thread": ({"value": K / t_or1 / 1e6, "unit": UNIT, "cores": 1,
+                                            "seconds": round(t_or1, 3)} if t_or1 else None)},
         "e2e": {"value": e2e_units / e2e_t / 1e6, "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": launches,

@@ -13,7 +13,7 @@
  *   opattr_aggregate -- Eq. (1) and Sec. 3.8.1: per-operator duration-weighted
  *                       means, sums and maxima of the 20-counter set
  *                       (Table 8), plus attributed / unattributed kernel time
- *                       (Fig. 3).
+ *                       (Fig. 4).
  *
  * Conventions shared by every call
  *  - Record and output arrays are DEVICE pointers owned by the caller, on the
@@ -114,7 +114,7 @@ typedef struct {
  *                          or NaN; 16-byte aligned (read by opattr_aggregate)
  *   stream    u8[n]        stream of the row, or NULL.  Nsight Compute replays
  *                          one stream per run when a workload is multi-stream
- *                          (limitations paragraph of Sec. 6); with the rows of
+ *                          (limitations paragraph of Sec. 5); with the rows of
  *                          those runs tagged here, opattr_match takes ordinals
  *                          per (name, stream) instead of per name, and name ids
  *                          must then be below 2^24.  Rows of one stream keep
@@ -175,7 +175,7 @@ typedef struct {
     double *agg;
 } opattr_op_aggregates;
 
-/* Host-side totals of opattr_aggregate (Fig. 3 coverage). */
+/* Host-side totals of opattr_aggregate (Fig. 4 coverage). */
 typedef struct {
     int64_t total_ns;              /* sum of all kernel durations */
     int64_t attributed_ns;         /* attributed kernels: range_of_kernel >= 0, or an operator */
@@ -452,17 +452,26 @@ int64_t opattr_launch_count(const opattr_ctx *ctx);
  *   Same inputs, outputs, ordering and status codes as opattr_match with
  *   layer deduplication off, on the stream `cuda_stream` of the current
  *   device, with `mismatch` in place of the context's mode.  No context.
- *   All scratch (about 6 MB) lives in one fixed device array inside the
- *   library; every GPU that loads the library holds it until exit.
+ *   All scratch (6 MB) lives in one fixed device array inside the library;
+ *   every GPU that loads the library holds it until exit.  It holds the
+ *   general (sorting) path at the limit below.
  *   kernels->n and ncu->n must each be at most OPATTR_MATCH_NOALLOC_MAX,
  *   else OPATTR_E_INVALID_ARG; per-stream ordinals are not available here
  *   (ncu->stream must be NULL, else OPATTR_E_INVALID_ARG).
- *   The first call on a device looks up the array's device address; make
- *   that first call before any stream capture.
+ *   Every call looks up the array's device address in the CUDA context
+ *   current at the call (a host-side lookup), so a device reset or another
+ *   context between calls is safe.  The first call in a context may also load
+ *   the library's device code (lazy module loading), and that is when the
+ *   array itself comes into being: make one warm-up call per device and
+ *   context outside any region that must not allocate, and before any stream
+ *   capture.  The call synchronises its stream and copies to host memory, so
+ *   it cannot be captured into a CUDA graph.
  *   Calls share the array.  Host threads are serialised inside the call, and
- *   each call finishes its device work before it returns; a caller that lets
- *   other work on the GPU touch the same memory concurrently races.
- *   Allocates nothing: no cudaMalloc, cudaFree or pinned host memory. */
+ *   each call, whatever it returns, finishes its device work before it
+ *   returns; a caller that lets other work on the GPU touch the same memory
+ *   concurrently races.
+ *   Allocates nothing after that first call: no cudaMalloc, cudaFree or
+ *   pinned host memory. */
 #define OPATTR_MATCH_NOALLOC_MAX 65536
 opattr_status opattr_match_noalloc(const opattr_kernels *kernels, const opattr_ncu *ncu,
                                    opattr_mismatch_mode mismatch, int32_t *ncu_idx_of_kernel, uint8_t *match_kind,

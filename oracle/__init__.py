@@ -116,7 +116,12 @@ def validate_ranges(r_stream, r_start, r_end, r_depth, mode: str = "indexed") ->
 
 
 def enclose(k_stream, k_start, r_stream, r_start, r_end, r_depth, r_op, mode: str = "indexed"):
-    """Returns (status, range_of_kernel i32[K], n_op_enclosing u8[K])."""
+    """Returns (status, range_of_kernel i32[K], n_op_enclosing u8[K]).
+
+    mode: "brute" (every range of the kernel's stream tested; all-pairs
+    laminar check), "indexed" (level lists and binary search), or
+    "brute_chain" (the brute per-kernel scan after the indexed laminar check,
+    for kernel samples of traces with millions of ranges)."""
     lib = _lib()
     ks, kt = _c(k_stream, np.uint8), _c(k_start, np.int64)
     rs, rt, re, rd, ro = (_c(r_stream, np.uint8), _c(r_start, np.int64), _c(r_end, np.int64),
@@ -124,7 +129,7 @@ def enclose(k_stream, k_start, r_stream, r_start, r_end, r_depth, r_op, mode: st
     K, R = len(kt), len(rt)
     out_r = np.full(K, -1, np.int32)
     out_n = np.zeros(K, np.uint8)
-    st = lib.orc_enclose(0 if mode == "brute" else 1, K, _p(ks), _p(kt), R, _p(rs), _p(rt), _p(re), _p(rd),
+    st = lib.orc_enclose({"brute": 0, "indexed": 1, "brute_chain": 2}[mode], K, _p(ks), _p(kt), R, _p(rs), _p(rt), _p(re), _p(rd),
                          _p(ro), _p(out_r), _p(out_n))
     return st, out_r, out_n
 

@@ -21,7 +21,7 @@
  *   aggregation  -- Eq. (1) duration-weighted mean, plain sum for additive
  *                   counters, maximum for per-kernel constants (Sec. 3.8.1),
  *                   per counter as Table 8 assigns; total/attributed/
- *                   unattributed kernel time (Sec. 3.2 durations, Fig. 3).
+ *                   unattributed kernel time (Sec. 3.2 durations, Fig. 4).
  *
  * Readings taken where the paper is silent (the same list is kept with the
  * design notes):
@@ -246,7 +246,11 @@ static void walk_chain(const ranges_t *r, const int64_t *chain, int32_t *out_ran
 }
 
 /* Enclosure, brute force: every range of the kernel's stream is tested.
- * mode 0 = brute, 1 = indexed (level lists + binary search). */
+ * mode 0 = brute, 1 = indexed (level lists + binary search), 2 = the brute
+ * chain after the indexed laminar check (the all-pairs check is quadratic in
+ * the ranges; this mode serves kernel samples of traces with millions of
+ * ranges, whose validity the indexed check, itself pinned against the
+ * all-pairs one, decides). */
 int orc_enclose(int mode, int64_t K, const uint8_t *k_stream, const int64_t *k_start,
                 int64_t R, const uint8_t *r_stream, const int64_t *r_start, const int64_t *r_end,
                 const uint8_t *r_depth, const uint32_t *r_op, int32_t *out_range, uint8_t *out_nop) {
@@ -255,7 +259,7 @@ int orc_enclose(int mode, int64_t K, const uint8_t *k_stream, const int64_t *k_s
                        : orc_validate_ranges_indexed(R, r_stream, r_start, r_end, r_depth);
     if (st) return st;
     int64_t chain[MAX_DEPTH];
-    if (mode == 0) {
+    if (mode == 0 || mode == 2) {
         /* per-stream lists of range indices, so the scan visits one stream */
         int64_t *cnt = (int64_t *)calloc(257, sizeof(int64_t));
         int64_t *lst = (int64_t *)malloc(sizeof(int64_t) * (R ? R : 1));

@@ -1,6 +1,6 @@
 // aggregate.cu -- per-operator aggregation, Eq. (1) and Sec. 3.8.1, with the
 // rule of each counter from Table 8, and the attributed / unattributed
-// totals of Fig. 3.
+// totals of Fig. 4.
 //
 // Operators are keyed by op id (op_id[range_of_kernel[k]]), so ranges that
 // share an op id aggregate together and no order of kernels or ranges is

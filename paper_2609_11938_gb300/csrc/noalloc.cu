@@ -19,17 +19,26 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
 }
 using namespace opattr;
 
-// Large enough for OPATTR_MATCH_NOALLOC_MAX kernels and rows (about 4.6 MB of
-// sort buffers) with room to spare.  Every GPU that loads the library holds
-// it until the process exits.
+// Large enough for OPATTR_MATCH_NOALLOC_MAX kernels and rows on the general
+// (sorting) path: 4.8 MB of sort buffers and tables, checked against this size
+// on every call (a request beyond it returns OPATTR_E_OOM, never a stray
+// access).  Every GPU that loads the library holds it until the process exits.
 static constexpr size_t NOALLOC_SCRATCH_BYTES = (size_t)6 << 20;
 static __device__ __align__(256) unsigned char g_match_scratch[NOALLOC_SCRATCH_BYTES];
 
 namespace {
 std::mutex g_lock;                       // one call at a time: every call shares the array
-constexpr int MAX_DEVICES = 64;
-void *g_scratch_addr[MAX_DEVICES];       // device address of g_match_scratch, per device
-}
+
+// Waits for the call's queued work before the lock is released, whatever the
+// call returns, so the next caller never reuses the array under it.
+struct DrainOnExit {
+    cudaStream_t s;
+    ~DrainOnExit() {
+        cudaStreamSynchronize(s);
+        cudaGetLastError();
+    }
+};
+}  // namespace
 
 extern "C" opattr_status opattr_match_noalloc(const opattr_kernels *kernels, const opattr_ncu *ncu,
                                               opattr_mismatch_mode mismatch, int32_t *ncu_idx_of_kernel,
@@ -41,22 +50,21 @@ extern "C" opattr_status opattr_match_noalloc(const opattr_kernels *kernels, con
     if (kernels->n < 0 || ncu->n < 0 || kernels->n > OPATTR_MATCH_NOALLOC_MAX || ncu->n > OPATTR_MATCH_NOALLOC_MAX)
         return OPATTR_E_INVALID_ARG;
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= MAX_DEVICES) {
+    if (cudaGetDevice(&dev) != cudaSuccess) {
         cudaGetLastError();
         return OPATTR_E_CUDA;
     }
     std::lock_guard<std::mutex> guard(g_lock);
-    if (!g_scratch_addr[dev]) {
-        // once per device, with that device current: the array's device
-        // address (the host-side name is only a stand-in for it)
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_match_scratch) != cudaSuccess || !p) {
-            cudaGetLastError();
-            return OPATTR_E_CUDA;
-        }
-        g_scratch_addr[dev] = p;
+    // The array's device address in the CUDA context current now (the
+    // host-side name is only a stand-in for it).  Looked up on every call: an
+    // address kept from an earlier call would belong to a context that a
+    // device reset has destroyed, or to another context of the same device.
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_match_scratch) != cudaSuccess || !p) {
+        cudaGetLastError();
+        return OPATTR_E_CUDA;
     }
-    char *base = static_cast<char *>(g_scratch_addr[dev]);
+    char *base = static_cast<char *>(p);
     // status block first, the arena after it; host mirrors are plain host memory
     DevStatus h_status, h_init;
     memset(&h_init, 0, sizeof h_init);
@@ -77,6 +85,7 @@ extern "C" opattr_status opattr_match_noalloc(const opattr_kernels *kernels, con
     c.arena = base + status_bytes;
     c.arena_cap = NOALLOC_SCRATCH_BYTES - status_bytes;
     c.arena_fixed = true;
+    DrainOnExit drain{c.stream};
     opattr_status st = do_match(c, kernels, ncu, nullptr, ncu_idx_of_kernel, match_kind, host_summary);
     if (c.last_error != cudaSuccess) return OPATTR_E_CUDA;
     return st;

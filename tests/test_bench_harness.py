@@ -72,10 +72,11 @@ def test_two_gloo_ranks_combine():
 def test_reference_arm_runs_on_cpu():
     env = dict(os.environ, CUDA_VISIBLE_DEVICES="")
     out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1",
-                          "--warmup", "3", "--oracle-kernels", "20000"], capture_output=True, text=True, env=env,
+                          "--warmup", "3", "--kernels", "20000"], capture_output=True, text=True, env=env,
                          timeout=600, cwd=ROOT)
     assert out.returncode == 0, out.stderr
     line = json.loads(out.stdout.strip().splitlines()[-1])
     assert line["impl"] == "reference" and line["unit"] == "M kernels/s" and line["value"] > 0
-    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 1
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == (os.cpu_count() or 1)
+    assert line["config"]["kernels"] == 20000 and line["config"]["same_config"] is False
     assert line["e2e"]["h2d_bytes_per_step"] == 0

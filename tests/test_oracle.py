@@ -102,7 +102,7 @@ def test_worked_permuted(golden, mode):
 
 @pytest.mark.parametrize("brute", [False, True])
 def test_per_stream_ordinals(brute):
-    # Limitations paragraph (Sec. 6): Nsight Compute replays a multi-stream
+    # Limitations paragraph (Sec. 5): Nsight Compute replays a multi-stream
     # workload one stream per run, so its rows come as per-stream runs and
     # the k-th launch of a name must be counted per (name, stream).
     # Launches in time order: t0 A on s0, t1 A on s1, t2 A on s0, t3 B on s1.
@@ -164,7 +164,7 @@ def test_table8_rules():
     assert oracle.agg_rules() == want
 
 
-# ---------------------------------------------------------------- dedup, Fig. 4, single kernel
+# ---------------------------------------------------------------- dedup, Fig. 3, single kernel
 
 @pytest.mark.parametrize("brute", [False, True])
 def test_dedup_mini(golden, brute):
@@ -188,8 +188,8 @@ def test_dedup_mini(golden, brute):
     assert summ["dedup_mismatch"] == e["swapped_dedup_mismatch"]
 
 
-def test_fig4_order_not_time(golden):
-    g = golden("fig4.json")
+def test_clock_domain_order_not_time(golden):
+    g = golden("clock_domain.json")
     ns, nc = np.array(g["nsys_t"]), np.array(g["ncu_t"])
     # the figure's failure mode: a nearest-timestamp join sends K_D to K_C's row
     assert int(np.argmin(np.abs(nc - ns[3]))) == g["expect"]["nearest_timestamp_join_of_K_D"]
@@ -278,8 +278,9 @@ def test_enclosure_brute_vs_indexed(seed):
     t = tracegen.small_random(seed, n_streams=1 + seed % 3, n_events=20 + seed % 50, max_depth=1 + seed % 6)
     a = oracle.enclose(t.k_stream, t.k_start, t.r_stream, t.r_start, t.r_end, t.r_depth, t.r_op, mode="brute")
     b = oracle.enclose(t.k_stream, t.k_start, t.r_stream, t.r_start, t.r_end, t.r_depth, t.r_op, mode="indexed")
-    assert a[0] == b[0] == oracle.OK
-    assert a[1].tolist() == b[1].tolist() and a[2].tolist() == b[2].tolist()
+    c = oracle.enclose(t.k_stream, t.k_start, t.r_stream, t.r_start, t.r_end, t.r_depth, t.r_op, mode="brute_chain")
+    assert a[0] == b[0] == c[0] == oracle.OK
+    assert a[1].tolist() == b[1].tolist() == c[1].tolist() and a[2].tolist() == b[2].tolist() == c[2].tolist()
     # the chosen range contains T on the kernel's stream and is an operator
     for k in np.nonzero(a[1] >= 0)[0]:
         r = a[1][k]
@@ -619,7 +620,7 @@ def _all_pins(golden):
                      (test_worked_match_and_aggregate, ("prefix", True)),
                      (test_worked_permuted, ("skip_name",)), (test_worked_permuted, ("prefix",)),
                      (test_dedup_mini, (False,)), (test_table8_rules, ()), (test_single_kernel_operator, ()),
-                     (test_walk_cases, ()), (test_fig4_order_not_time, ()), (test_tiers_worked, (True,)),
+                     (test_walk_cases, ()), (test_clock_domain_order_not_time, ()), (test_tiers_worked, (True,)),
                      (test_tiers_worked, (False,))]:
         try:
             if fn in (test_table8_rules, test_walk_cases):
@@ -643,3 +644,23 @@ def test_pins_catch_mutation(tmp_path, golden, label, old, new):
     with oracle.use_library(str(so)):
         failures = _all_pins(golden)
     assert failures, f"no pin caught the planted mistake: {label}"
+
+
+@pytest.mark.parametrize("name,kw", [("tiny", {}), ("gpt2", {}), ("large", dict(n_kernels=150_000)),
+                                     ("adversarial", dict(n_kernels=150_000))])
+def test_threaded_oracle_equals_single_thread(name, kw):
+    """The CPU baseline's threaded run (streams, names and op blocks split
+    over host threads) gives the single-thread oracle's outputs bit for bit."""
+    from oracle.parallel import run_threads
+    t = tracegen.generate(name, **kw)
+    a = oracle.run(t, enclose_mode="indexed")
+    b = run_threads(t, 5)
+    for k in ("enclose_status", "match_status", "aggregate_status", "summary"):
+        assert a[k] == b[k], k
+    for k in ("range_of_kernel", "n_op_enclosing", "ncu_idx", "match_kind"):
+        np.testing.assert_array_equal(a[k], b[k], err_msg=k)
+    for k in ("kernel_count", "total_duration_ns", "matched_count"):
+        np.testing.assert_array_equal(a["ops"][k], b["ops"][k], err_msg=k)
+    assert np.array_equal(a["ops"]["agg"].view(np.int64), b["ops"]["agg"].view(np.int64))
+    for k, v in a["totals"].items():
+        assert v == b["totals"][k] or (v != v and b["totals"][k] != b["totals"][k]), k
