@@ -37,7 +37,6 @@ KERNEL_BYTES = {
     # index is not read when every kernel's row is its own index: 92)
     "agg_ops": lambda K, R, M, O: 96 * K + 188 * O,
     "enclose": lambda K, R, M, O: 14 * K + 20 * R,
-    "enclose_wide": lambda K, R, M, O: 14 * K + 20 * R,
     "agg_place": lambda K, R, M, O: 16 * K,
     "agg_count": lambda K, R, M, O: 24 * K + 4 * O,
     "match_identity": lambda K, R, M, O: 13 * K,
@@ -47,7 +46,9 @@ KERNEL_BYTES = {
     "level_place": lambda K, R, M, O: 42 * R,
     "match_stream_pairs": lambda K, R, M, O: 18 * K,
     "validate_levels": lambda K, R, M, O: 22 * R,
-    "window_table": lambda K, R, M, O: 0,
+    "stream_place": lambda K, R, M, O: 5 * K,
+    "stream_windows": lambda K, R, M, O: 0,
+    "tile_order": lambda K, R, M, O: 0,
 }
 
 WORKLOADS = {

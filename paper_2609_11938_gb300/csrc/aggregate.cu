@@ -34,6 +34,7 @@ struct AggIn {
     const int64_t *dur;
     const int32_t *ncu_idx;
     const float *counters;
+    int64_t M;                  // ncu rows: a row index at or past M is never read (the count pass reports it)
     int64_t n_ops;
     unsigned *ctr;              // next chunk of the ops pass, zeroed before it
     const unsigned *nonident;   // nonzero unless ncu_idx[k] == k for every kernel (set by the count pass)
@@ -186,7 +187,8 @@ struct Acc {
     __device__ __forceinline__ void add(const AggIn &A, int64_t k) {
         const long long d = A.dur[k];
         const int32_t j = A.ncu_idx[k];
-        accumulate(d, j >= 0, reinterpret_cast<const float4 *>(A.counters + (int64_t)(j >= 0 ? j : 0) * NC));
+        const bool ok = j >= 0 && j < A.M;
+        accumulate(d, ok, reinterpret_cast<const float4 *>(A.counters + (int64_t)(ok ? j : 0) * NC));
     }
 };
 
@@ -271,20 +273,28 @@ struct AccF {
         double *agg = A.out.agg;
         const int64_t n = A.n_ops;
         const double qnan = __longlong_as_double(0x7FF8000000000000ll);
-        const bool any = mc > 0;
+        if (mc == 0) {
+            // no matched kernel: every counter is null; nothing to convert
+#pragma unroll
+            for (int c = 0; c < NC; ++c) agg[(int64_t)c * n + op] = qnan;
+            return;
+        }
 #pragma unroll
         for (int i = 0; i < N_SUM; ++i) {
             ff x = s[i];
             ff_renorm(x);
-            agg[(int64_t)Acc::sum_col(i) * n + op] = any ? ff_to_f64_fast(x) : qnan;
+            agg[(int64_t)Acc::sum_col(i) * n + op] = ff_to_f64_fast(x);
         }
-        const bool wok = any && dall > 0;
-        const ff rcp = ff_recip_i64(wok ? dall : 1);
+        if (dall > 0) {
+            const ff rcp = ff_recip_i64(dall);
 #pragma unroll
-        for (int i = 0; i < N_DW; ++i) agg[(int64_t)Acc::dw_col(i) * n + op] = wok ? ff_mul_to_f64(w[i], rcp) : qnan;
+            for (int i = 0; i < N_DW; ++i) agg[(int64_t)Acc::dw_col(i) * n + op] = ff_mul_to_f64(w[i], rcp);
+        } else {
 #pragma unroll
-        for (int i = 0; i < N_MAX; ++i)
-            agg[(int64_t)Acc::max_col(i) * n + op] = any ? ff_to_f64_fast(ff{mx[i], 0.f}) : qnan;
+            for (int i = 0; i < N_DW; ++i) agg[(int64_t)Acc::dw_col(i) * n + op] = qnan;
+        }
+#pragma unroll
+        for (int i = 0; i < N_MAX; ++i) agg[(int64_t)Acc::max_col(i) * n + op] = f32_to_f64_fast(mx[i]);
     }
 };
 
@@ -504,23 +514,37 @@ __global__ void __launch_bounds__(SL_THREADS) k_agg_sort_long(const uint32_t *__
 // One thread per op id.  Each warp takes AG_CHUNK consecutive op ids at a
 // time, orders them by segment length (longest first) and walks them in
 // AG_CHUNK / 32 rounds, so that the threads of a round walk segments of
-// similar length; warps share nothing and never wait for each other.  The
-// grid is what stays resident; warps draw the chunks in increasing order
-// from one counter, so the ops in flight at any moment are one narrow band
-// of op ids whatever each warp's pace (a fixed chunk-to-warp assignment lets
-// fast and slow warps drift apart and widens the band), and with op ids in
-// range order the kernels and outputs of that band stay in L2.  Segments are
-// walked in ascending kernel index: a short one is checked and, in the rare
-// case the placement left it out of order, insertion-sorted in place by its
-// thread; long ones were sorted by k_agg_sort_long.  While a kernel is
-// added, the counter rows and durations of the next two arrive in per-thread
-// shared-memory slots by asynchronous copy (cp.async), with their row
-// indices loaded a step earlier still (or taken to be the kernel indices
-// when the count pass found every row to be its kernel's own index).
-constexpr int AG_THREADS = 128;                // five blocks per SM (96 registers, a few spilled)
+// similar length and finish together (the record is written by every lane of
+// the round at once); warps share nothing and never wait for each other.
+// The grid is what stays resident; warps draw the chunks in increasing order
+// from one counter (the next chunk is drawn, and its offsets loaded, while
+// the current one runs), so the ops in flight at any moment are one narrow
+// band of op ids whatever each warp's pace, and with op ids in range order
+// the kernels and outputs of that band stay in L2.  The chunk's segments are
+// one contiguous run of the list; when it fits it is first copied to shared
+// memory by coalesced loads, and each thread checks its segments there and,
+// in the rare case the count pass met an op in two runs, sorts them in place,
+// so segments are walked in ascending kernel index (a larger chunk reads the
+// list in place: short segments checked there, long ones sorted before by
+// k_agg_sort_long).  While a kernel is added, the counter rows and durations
+// of the next two arrive in per-thread shared-memory slots by asynchronous
+// copy (cp.async), with their row indices loaded a step earlier still (or
+// taken to be the kernel indices when the count pass found every row to be
+// its kernel's own index).
+constexpr int AG_THREADS = 128;
 constexpr int AG_WARPS = AG_THREADS / 32;
 constexpr int AG_CHUNK = 64;                    // op ids per warp and chunk
 constexpr int AG_LBUCKETS = 32;
+constexpr int AG_STAGE = 1024;                  // list entries of a chunk staged in shared memory
+
+struct OpsWarp {
+    float4 row[2][32][NC / 4];      // two kernels in flight per thread: counter rows
+    long long dur[2][32];           // and durations, by asynchronous copy
+    uint32_t L[AG_STAGE];           // the chunk's list run (when it fits)
+    uint32_t lcount[AG_LBUCKETS];
+    uint8_t order[AG_CHUNK];
+};
+constexpr size_t AG_SMEM = sizeof(OpsWarp) * AG_WARPS;
 
 // An op whose fast sums saw a null or infinite value: the segment again, in
 // the same order, with Acc.  Returns 1 if a value was infinite.
@@ -530,6 +554,20 @@ __device__ __noinline__ int op_careful(const uint32_t *seg, uint32_t len, AggIn 
     for (uint32_t t = 0; t < len; ++t) acc.add(A, seg[t]);
     acc.write(A, o);
     return acc.bad;
+}
+
+// Ascending order of a segment, sorted in place when it is not (insertion
+// sort: the segment is two ascending runs at worst).
+__device__ __forceinline__ void sort_segment(uint32_t *seg, uint32_t len) {
+    bool up = true;
+    for (uint32_t t = 1; t < len; ++t) up &= seg[t - 1] < seg[t];
+    if (up) return;
+    for (uint32_t t = 1; t < len; ++t) {
+        const uint32_t x = seg[t];
+        uint32_t u = t;
+        for (; u > 0 && seg[u - 1] > x; --u) seg[u] = seg[u - 1];
+        seg[u] = x;
+    }
 }
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -545,88 +583,112 @@ __device__ __forceinline__ void cp_async_wait() {
     asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
-__global__ void __launch_bounds__(AG_THREADS, 5) k_agg_ops(const uint32_t *__restrict__ off, uint32_t *__restrict__ list,
+__global__ void __launch_bounds__(AG_THREADS, 5) k_agg_ops(const uint32_t *__restrict__ off, uint32_t *list,
                                                           AggIn A, DevStatus *st) {
-    __shared__ uint32_t lcount_s[AG_WARPS][AG_LBUCKETS];
-    __shared__ uint8_t order_s[AG_WARPS][AG_CHUNK];
-    // two in-flight kernels per thread: counter row and duration, by async copy
-    __shared__ __align__(16) float4 rowbuf[2][AG_THREADS][NC / 4];
-    __shared__ long long durbuf[2][AG_THREADS];
-    uint32_t *lcount = lcount_s[threadIdx.x / 32];
-    uint8_t *order = order_s[threadIdx.x / 32];
+    extern __shared__ __align__(16) unsigned char ag_smem[];
+    OpsWarp &W = reinterpret_cast<OpsWarp *>(ag_smem)[threadIdx.x / 32];
     const unsigned lane = lane_id();
     int bad = 0;
     const bool ident = *A.nonident == 0;
-    auto row_of = [&](uint32_t k) -> int32_t { return ident ? (int32_t)k : A.ncu_idx[k]; };
-    auto next_chunk = [&]() -> int64_t {
+    const float4 *rows = reinterpret_cast<const float4 *>(A.counters);
+    // row index of kernel k, -1 for none (or for an index past the rows)
+    auto row_of = [&](uint32_t k) -> int32_t {
+        const int32_t j = ident ? (int32_t)k : A.ncu_idx[k];
+        return j < A.M ? j : -1;
+    };
+    auto draw = [&]() -> unsigned {
         unsigned v = 0;
         if (lane == 0) v = atomicAdd(A.ctr, 1u);
-        return (int64_t)__shfl_sync(0xffffffffu, v, 0) * AG_CHUNK;
+        return v;
     };
-    for (int64_t o0 = next_chunk(); o0 < A.n_ops; o0 = next_chunk()) {
+    constexpr int PER = AG_CHUNK / 32;
+    // the first chunk's offsets; afterwards the next chunk is drawn and its
+    // offsets loaded while the current one runs
+    int64_t o0 = (int64_t)__shfl_sync(0xffffffffu, draw(), 0) * AG_CHUNK;
+    uint32_t oa[PER], ob[PER];
+#pragma unroll
+    for (int q = 0; q < PER; ++q) {
+        const int64_t o = o0 + q * 32 + lane;
+        oa[q] = o < A.n_ops ? off[o] : 0u;
+        ob[q] = o < A.n_ops ? off[o + 1] : 0u;
+    }
+    while (o0 < A.n_ops) {
+        const unsigned next_raw = draw();           // in flight during this chunk
         const int nchunk = A.n_ops - o0 < AG_CHUNK ? (int)(A.n_ops - o0) : AG_CHUNK;
+        const uint32_t cbase = __shfl_sync(0xffffffffu, oa[0], 0);          // the chunk's list run
+        const uint32_t cend = __shfl_sync(0xffffffffu, ob[(nchunk - 1) >> 5], (nchunk - 1) & 31);
+        const uint32_t ctot = cend - cbase;
+        const bool staged = ctot <= AG_STAGE;
         // lengths of the chunk's ops, counting sort by length (descending, capped)
-        constexpr int PER = AG_CHUNK / 32;
         uint32_t bkt[PER];
-        lcount[lane] = 0;
+        W.lcount[lane] = 0;
         __syncwarp();
 #pragma unroll
         for (int q = 0; q < PER; ++q) {
             const int i = q * 32 + (int)lane;
-            const uint32_t len = i < nchunk ? off[o0 + i + 1] - off[o0 + i] : 0u;
+            const uint32_t len = i < nchunk ? ob[q] - oa[q] : 0u;
             bkt[q] = AG_LBUCKETS - 1 - (len < AG_LBUCKETS - 1 ? len : AG_LBUCKETS - 1);
-            if (i < nchunk) atomicAdd(&lcount[bkt[q]], 1u);
+            if (i < nchunk) atomicAdd(&W.lcount[bkt[q]], 1u);
         }
+        if (staged)
+            for (uint32_t i = lane; i < ctot; i += 32) W.L[i] = list[cbase + i];
         __syncwarp();
         {
-            const unsigned x = lcount[lane];
-            unsigned inc = x;
-#pragma unroll
-            for (int d = 1; d < 32; d <<= 1) {
-                const unsigned y = __shfl_up_sync(0xffffffffu, inc, d);
-                if ((int)lane >= d) inc += y;
-            }
-            lcount[lane] = inc - x;
+            const unsigned x = W.lcount[lane];
+            const unsigned inc = warp_inclusive_scan(x);
+            W.lcount[lane] = inc - x;
         }
         __syncwarp();
 #pragma unroll
         for (int q = 0; q < PER; ++q) {
             const int i = q * 32 + (int)lane;
-            if (i < nchunk) order[atomicAdd(&lcount[bkt[q]], 1u)] = (uint8_t)i;
+            if (i < nchunk) W.order[atomicAdd(&W.lcount[bkt[q]], 1u)] = (uint8_t)i;
+            // each thread puts the segments of its own ops in ascending order
+            const uint32_t len = i < nchunk ? ob[q] - oa[q] : 0u;
+            if (len > 1 && len <= AG_HUGE) {
+                if (staged) sort_segment(W.L + (oa[q] - cbase), len);
+                else if (len <= AG_SHORT_MAX) sort_segment(list + oa[q], len);
+            }
         }
         __syncwarp();
+        // the next chunk's offsets, in flight during the rounds
+        const int64_t o1 = (int64_t)__shfl_sync(0xffffffffu, next_raw, 0) * AG_CHUNK;
+        uint32_t na[PER], nb[PER];
+#pragma unroll
+        for (int q = 0; q < PER; ++q) {
+            const int64_t o = o1 + q * 32 + lane;
+            na[q] = o < A.n_ops ? off[o] : 0u;
+            nb[q] = o < A.n_ops ? off[o + 1] : 0u;
+        }
         for (int g = 0; g * 32 < nchunk; ++g) {
             const int i = g * 32 + (int)lane;
-            if (i >= nchunk) continue;
-            const int64_t o = o0 + order[i];
-            const uint32_t s0 = off[o], len = off[o + 1] - s0;
-            uint32_t *seg = list + s0;
-            if (len > AG_HUGE) continue;                 // a huge op: k_agg_long_ops writes it
-            if (len <= AG_SHORT_MAX) {                   // ascending unless the count met the op in two runs
-                bool up = true;
-                for (uint32_t t = 1; t < len; ++t) up &= seg[t - 1] < seg[t];
-                if (!up) {
-                    for (uint32_t t = 1; t < len; ++t) {
-                        const uint32_t x = seg[t];
-                        uint32_t u = t;
-                        for (; u > 0 && seg[u - 1] > x; --u) seg[u] = seg[u - 1];
-                        seg[u] = x;
-                    }
-                }
+            // offsets of the op each lane walks, from the lane that holds them
+            // (op il sits in register il >> 5 of lane il & 31)
+            const int il = i < nchunk ? W.order[i] : 0;
+            uint32_t sa = 0, sb = 0;
+#pragma unroll
+            for (int q = 0; q < PER; ++q) {
+                const uint32_t xa = __shfl_sync(0xffffffffu, oa[q], il & 31);
+                const uint32_t xb = __shfl_sync(0xffffffffu, ob[q], il & 31);
+                if ((il >> 5) == q) { sa = xa; sb = xb; }
             }
+            if (i >= nchunk) continue;
+            const int64_t o = o0 + il;
+            const uint32_t s0 = sa, len = sb - sa;
+            if (len > AG_HUGE) continue;                 // a huge op: k_agg_long_ops writes it
+            const uint32_t *seg = staged ? W.L + (s0 - cbase) : list + s0;
             AccF acc;
             acc.init();
             if (len > 0) {
                 // kernel t's row and duration land in slot t & 1 while kernel
                 // t - 1 is added; row indices are loaded one step further ahead
-                const unsigned me = threadIdx.x;
                 auto issue = [&](uint32_t t, uint32_t k, int32_t j) {
                     if (t < len) {
-                        cp_async8(&durbuf[t & 1][me], A.dur + k);
+                        cp_async8(&W.dur[t & 1][lane], A.dur + k);
                         if (j >= 0) {
-                            const float4 *src = reinterpret_cast<const float4 *>(A.counters + (int64_t)j * NC);
+                            const float4 *src = rows + (int64_t)j * (NC / 4);
 #pragma unroll
-                            for (int q = 0; q < NC / 4; ++q) cp_async16(&rowbuf[t & 1][me][q], src + q);
+                            for (int c = 0; c < NC / 4; ++c) cp_async16(&W.row[t & 1][lane][c], src + c);
                         }
                     }
                     cp_async_commit();
@@ -643,7 +705,7 @@ __global__ void __launch_bounds__(AG_THREADS, 5) k_agg_ops(const uint32_t *__res
                     const int32_t j3 = t + 3 < len ? row_of(k3) : -1;
                     cp_async_wait<1>();
                     const int32_t j = (t & 1) ? js1 : js0;
-                    acc.accumulate(durbuf[t & 1][me], j >= 0, rowbuf[t & 1][me]);
+                    acc.accumulate(W.dur[t & 1][lane], j >= 0, W.row[t & 1][lane]);
                     issue(t + 2, k2, j2);
                     if (t & 1) js1 = j2; else js0 = j2;
                     k2 = k3;
@@ -655,6 +717,9 @@ __global__ void __launch_bounds__(AG_THREADS, 5) k_agg_ops(const uint32_t *__res
             else bad |= op_careful(seg, len, A, o);
         }
         __syncwarp();
+        o0 = o1;
+#pragma unroll
+        for (int q = 0; q < PER; ++q) { oa[q] = na[q]; ob[q] = nb[q]; }
     }
     if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_err(st, ERR_INVALID);
 }
@@ -819,7 +884,8 @@ __device__ __forceinline__ bool piece_fast(const AggIn &A, const uint32_t *seg, 
     for (uint32_t t = l0; t < l1; ++t) {
         const uint32_t k = seg[t];
         const int32_t j = A.ncu_idx[k];
-        f.accumulate(A.dur[k], j >= 0, reinterpret_cast<const float4 *>(A.counters + (int64_t)(j >= 0 ? j : 0) * NC));
+        const bool ok = j >= 0 && j < A.M;
+        f.accumulate(A.dur[k], ok, reinterpret_cast<const float4 *>(A.counters + (int64_t)(ok ? j : 0) * NC));
     }
     if (!f.clean()) return false;
     out.kc = (int)(l1 - l0);
@@ -913,7 +979,7 @@ __global__ void __launch_bounds__(FIN_THREADS) k_agg_long_ops(const uint32_t *__
 static unsigned ops_grid(Ctx &c, int64_t O) {
     int sms = 0, per_sm = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
-    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_agg_ops, AG_THREADS, 0);
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_agg_ops, AG_THREADS, AG_SMEM);
     cudaGetLastError();
     const int64_t resident = (int64_t)std::max(1, sms) * std::max(1, per_sm);
     const int64_t need = (O + (int64_t)AG_WARPS * AG_CHUNK - 1) / ((int64_t)AG_WARPS * AG_CHUNK);
@@ -978,6 +1044,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     in.dur = kern->dur_ns;
     in.ncu_idx = nidx;
     in.counters = ncu->counters;
+    in.M = M;
     in.n_ops = O;
     in.ctr = ctr;
     in.nonident = nonident;
@@ -1001,7 +1068,12 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
             return cuda_status(c, cudaGetLastError());
         cudaMemcpyAsync(c.h_levels, info, 5 * sizeof(uint32_t), cudaMemcpyDeviceToHost, c.stream);
         cudaEventRecord(c.ev_aux, c.stream);
-        launch(c, "agg_ops", k_agg_ops, dim3(ops_grid(c, O)), dim3(AG_THREADS), 0,
+        static unsigned attr_done = 0;
+        if (c.device < 32 && !(attr_done & (1u << c.device))) {
+            cudaFuncSetAttribute(k_agg_ops, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)AG_SMEM);
+            attr_done |= 1u << c.device;
+        }
+        launch(c, "agg_ops", k_agg_ops, dim3(ops_grid(c, O)), dim3(AG_THREADS), AG_SMEM,
                (const uint32_t *)off, list, in, c.d_status);
         if (cudaEventSynchronize(c.ev_aux) != cudaSuccess) return cuda_status(c, cudaGetLastError());
         const uint32_t pieces = c.h_levels[1], longest = c.h_levels[2], n_huge = c.h_levels[4];
@@ -1160,6 +1232,7 @@ opattr_status do_rollup(Ctx &c, const opattr_kernels *kern, const opattr_ranges 
         in.dur = kern->dur_ns;
         in.ncu_idx = nidx;
         in.counters = ncu->counters;
+        in.M = M;
         in.n_ops = C;
         in.ctr = nullptr;
         in.nonident = nullptr;

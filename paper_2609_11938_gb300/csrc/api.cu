@@ -165,7 +165,7 @@ opattr_status opattr_create(opattr_ctx **out, int device, void *cuda_stream, con
     bool fail = cudaMalloc(&c.d_status, sizeof(DevStatus)) != cudaSuccess;
     fail = fail || cudaMallocHost(&c.h_status, sizeof(DevStatus)) != cudaSuccess;
     fail = fail || cudaMallocHost(&c.h_init, sizeof(DevStatus)) != cudaSuccess;
-    fail = fail || cudaMallocHost(&c.h_levels, sizeof(uint32_t) * (N_LEVELS + 1)) != cudaSuccess;
+    fail = fail || cudaMallocHost(&c.h_levels, sizeof(uint32_t) * (N_LEVELS + 1 + 256)) != cudaSuccess;
     fail = fail || cudaMallocHost(&c.h_stage, STAGE_BYTES) != cudaSuccess;
     if (fail) {
         cudaGetLastError();

@@ -85,7 +85,8 @@ struct Ctx {
     DevStatus *d_status = nullptr;
     DevStatus *h_status = nullptr;   // pinned mirror
     DevStatus *h_init = nullptr;     // pinned reset template
-    uint32_t *h_levels = nullptr;    // pinned host copy of the enclosure's level offsets [N_LEVELS + 1];
+    uint32_t *h_levels = nullptr;    // pinned host copy of the enclosure's level offsets [N_LEVELS + 1] and
+                                     // kernels per stream [256];
                                      // the aggregation reuses it for a few values read mid-call
     cudaEvent_t ev_aux = nullptr;    // marks a mid-call host read (created on first use)
     unsigned char *h_stage = nullptr; // pinned staging for small host-built tables [STAGE_BYTES]
@@ -165,6 +166,20 @@ __device__ __forceinline__ unsigned lane_id() { return threadIdx.x & 31u; }
 __device__ __forceinline__ unsigned lanemask_lt() {
     unsigned m;
     asm volatile("mov.u32 %0, %%lanemask_lt;" : "=r"(m));
+    return m;
+}
+
+// Lanes of the warp whose 8-bit digit equals this lane's, among the lanes
+// with `valid` set: one ballot per digit bit (the rank-by-digit step of a
+// stable multi-split).
+__device__ __forceinline__ unsigned warp_peers8(unsigned d, bool valid) {
+    unsigned m = __ballot_sync(0xffffffffu, valid);
+#pragma unroll
+    for (int b = 0; b < 8; ++b) {
+        const bool bit = (d >> b) & 1u;
+        const unsigned x = __ballot_sync(0xffffffffu, bit);
+        m &= bit ? x : ~x;
+    }
     return m;
 }
 

@@ -7,15 +7,15 @@
 // stream * 32 + depth.  Within a level ranges are disjoint or touching, so
 // "the last range with start <= T" is the only one that can contain T.
 //
-// Kernels are taken in time order, in tiles of ENC_TILE.  A window table
-// P[tile][level] (last level position with start <= the tile's first T) bounds,
-// per level, the ranges a tile can hit; the enclosure kernel stages those
-// windows in shared memory as 32-bit times relative to the tile start and
-// answers each kernel by one search per depth, walking depths outward-in
-// (0, 1, ...) until a depth has no containing range.  The walk state needs no
-// stack: a structural range resets the collection (everything above it is
-// beyond the cut); an operator becomes the innermost answer and counts;
-// a non-op range is passed over.
+// Kernels are answered stream by stream, in tiles of consecutive kernels of
+// one stream (the per-stream tiles section below).  A window table bounds,
+// per tile and depth, the ranges the tile can hit; the enclosure kernel
+// stages those windows in shared memory as 32-bit times relative to the
+// tile's first kernel and sweeps the tile's kernels in time order, walking
+// depths outward-in (0, 1, ...) until a depth has no containing range.  The
+// walk state needs no stack: a structural range resets the collection
+// (everything above it is beyond the cut); an operator becomes the innermost
+// answer and counts; a non-op range is passed over.
 #include <algorithm>
 
 #include "sort.cuh"
@@ -24,15 +24,6 @@
 namespace opattr {
 
 constexpr int LEVELS = N_LEVELS;
-constexpr int ENC_THREADS = 256;
-constexpr int ENC_TILE = 2048;          // kernels per tile
-// Shared-memory capacities: staged range entries and active (stream, depth)
-// levels per tile.  With few levels a compact layout (and 64 registers)
-// keeps four blocks per SM; a tile that outgrows it is deferred to the wide
-// layout, which handles any tile (overflowing ones by global searches).
-constexpr int ENC_WIN_SMALL = 1024, ENC_ACT_SMALL = 256;
-constexpr int ENC_WIN_WIDE = 3072, ENC_ACT_WIDE = 2048;
-constexpr int ENC_CHUNK = ENC_TILE / ENC_THREADS;   // consecutive same-stream kernels per thread
 constexpr uint32_t KIND_OP = 0, KIND_NONOP = 1, KIND_STRUCT = 2;
 
 __device__ __forceinline__ uint32_t kind_of(uint32_t op) {
@@ -169,17 +160,22 @@ __global__ void __launch_bounds__(RADIX_THREADS) k_level_place(LevelDigit digit,
     unsigned dg[RADIX_ITEMS];
     uint32_t rank[RADIX_ITEMS];
     const unsigned lt = lanemask_lt();
+    unsigned peers[RADIX_ITEMS];
 #pragma unroll
-    for (int it = 0; it < RADIX_ITEMS; ++it) {
+    for (int it = 0; it < RADIX_ITEMS; ++it) {        // digits and peer groups first: independent
         const int64_t i = base + it * 32 + lane;
         const unsigned d = i < n ? digit(i) : (unsigned)RADIX_BINS;
-        const unsigned peers = __match_any_sync(0xffffffffu, d);
+        peers[it] = warp_peers8(d, d < RADIX_BINS);
+        dg[it] = d;
+    }
+#pragma unroll
+    for (int it = 0; it < RADIX_ITEMS; ++it) {
+        const unsigned d = dg[it];
         const unsigned before = d < RADIX_BINS ? S.wcnt[w * RADIX_BINS + d] : 0u;
         __syncwarp();
-        if (d < RADIX_BINS && (peers & lt) == 0) S.wcnt[w * RADIX_BINS + d] = before + __popc(peers);
+        if (d < RADIX_BINS && (peers[it] & lt) == 0) S.wcnt[w * RADIX_BINS + d] = before + __popc(peers[it]);
         __syncwarp();
-        rank[it] = before + __popc(peers & lt);
-        dg[it] = d;
+        rank[it] = before + __popc(peers[it] & lt);
     }
     __syncthreads();
     uint32_t tot;
@@ -243,127 +239,173 @@ __global__ void __launch_bounds__(RADIX_THREADS) k_level_place(LevelDigit digit,
 
 // Laminar checks over level positions: adjacent pairs of a level, and the
 // parent of every range at depth > 0 (the last range of level (s, d-1) that
-// starts no later; it must end no earlier).
+// starts no later; it must end no earlier).  A thread takes VL_PER
+// consecutive positions: starts do not decrease along a level, so the parent
+// is searched once and then followed forward.
+constexpr int VL_PER = 8;
 __global__ void k_validate_levels(const uint8_t *__restrict__ stream, const uint8_t *__restrict__ depth,
                                   const int64_t *__restrict__ ls, const int64_t *__restrict__ le,
                                   const uint32_t *__restrict__ li, const uint32_t *__restrict__ lvl_off, int64_t n,
                                   DevStatus *st) {
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-        uint32_t r = li[i] & 0x3FFFFFFFu;
-        uint32_t s = stream[r], d = depth[r];
-        uint32_t L = s * 32 + d;
-        long long a = ls[i], b = le[i];
-        if (i + 1 < (int64_t)lvl_off[L + 1]) {
-            long long a2 = ls[i + 1], b2 = le[i + 1];
-            if (a2 == a && b2 < b) set_flag(st, F_LEVEL_FIXUP);
-            else if (b > a2) set_err(st, ERR_NOT_NESTED);
-        }
-        if (d > 0) {
-            int64_t lo = lvl_off[L - 1], hi = lvl_off[L];
-            int64_t x = lo, y = hi;               // first position with start > a
-            while (x < y) {
-                int64_t m = (x + y) >> 1;
-                if (ls[m] <= a) x = m + 1; else y = m;
+    bool err = false, fix = false;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x * VL_PER;
+    for (int64_t i0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * VL_PER; i0 < n; i0 += stride) {
+        const int64_t i1 = i0 + VL_PER < n ? i0 + VL_PER : n;
+        int64_t lend = -1, plo = 0, phi = 0, pp = 0;
+        uint32_t d = 0;
+        bool have_parent = false;
+        long long a = ls[i0], b = le[i0];
+        for (int64_t i = i0; i < i1; ++i) {
+            if (i >= lend) {                     // the level of position i
+                const uint32_t r = li[i] & 0x3FFFFFFFu;
+                const uint32_t L = (uint32_t)stream[r] * 32u + depth[r];
+                d = depth[r];
+                lend = lvl_off[L + 1];
+                if (d > 0) { plo = lvl_off[L - 1]; phi = lvl_off[L]; }
+                have_parent = false;
             }
-            if (x == lo || le[x - 1] < b) set_err(st, ERR_NOT_NESTED);
-        }
-    }
-}
-
-// ------------------------------------------------------------------ window table
-// P[t * nl + l] = (last position p of level l with lvl_start[p] <= b_t) - level
-// start, or -1; b_t = start of the time-ordered kernel t*ENC_TILE for
-// t < nt, and of the last kernel for t = nt.  The b_t do not decrease, so
-// one thread takes `chunk` consecutive tiles of one level: a binary search
-// for the first, then an exponential search forward from the previous
-// answer for each next one (cost logarithmic in the entries passed, however
-// unevenly a level's ranges fall between tiles).  Neighbouring threads take
-// neighbouring levels, so the rows of P are written together.  Small tables
-// take chunks of one tile (every search in parallel).
-constexpr int WT_CHUNK = 16;
-__device__ __forceinline__ long long tile_bound(const int64_t *k_start, const uint32_t *korder, int64_t K, int64_t nt,
-                                                int64_t t) {
-    const int64_t pos = t < nt ? t * ENC_TILE : K - 1;
-    return k_start[korder ? korder[pos] : pos];
-}
-__global__ void k_window_table(const int64_t *__restrict__ ls, const uint32_t *__restrict__ lvl_off,
-                               const uint16_t *__restrict__ level_of_compact, int nl,
-                               const int64_t *__restrict__ k_start, const uint32_t *__restrict__ korder, int64_t K,
-                               int64_t nt, int chunk, int32_t *__restrict__ P) {
-    const int64_t nchunk = (nt + 1 + chunk - 1) / chunk;
-    const int64_t total = nchunk * nl;
-    for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < total; q += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t ch = q / nl;
-        const int l = (int)(q - ch * nl);
-        const uint32_t L = level_of_compact[l];
-        const int64_t lo = lvl_off[L], hi = lvl_off[L + 1];
-        const int64_t t0 = ch * chunk, t1 = t0 + chunk < nt + 1 ? t0 + chunk : nt + 1;
-        int64_t x = lo;                       // first position with start > b (for the current tile)
-        for (int64_t t = t0; t < t1; ++t) {
-            const long long b = tile_bound(k_start, korder, K, nt, t);
-            int64_t a2 = x, z = x;
-            if (t > t0) {
-                int64_t step = 1;
-                while (z < hi && ls[z] <= b) {
-                    a2 = z + 1;
-                    z += step;
-                    step <<= 1;
+            long long a2 = 0, b2 = 0;
+            if (i + 1 < n) { a2 = ls[i + 1]; b2 = le[i + 1]; }
+            if (i + 1 < lend) {
+                if (a2 == a && b2 < b) fix = true;
+                else if (b > a2) err = true;
+            }
+            if (d > 0) {
+                if (!have_parent) {              // last parent-level position with start <= a
+                    int64_t x = plo, y = phi;
+                    while (x < y) {
+                        const int64_t m = (x + y) >> 1;
+                        if (ls[m] <= a) x = m + 1; else y = m;
+                    }
+                    pp = x - 1;
+                    have_parent = true;
+                } else {
+                    while (pp + 1 < phi && ls[pp + 1] <= a) ++pp;
                 }
-                if (z > hi) z = hi;
-            } else {
-                z = hi;
+                if (pp < plo || le[pp] < b) err = true;
             }
-            while (a2 < z) {                  // first position in [a2, z) with start > b, else z
-                const int64_t m = (a2 + z) >> 1;
-                if (ls[m] <= b) a2 = m + 1; else z = m;
-            }
-            x = a2;
-            P[t * nl + l] = (int32_t)(x - lo - 1);
+            a = a2;
+            b = b2;
         }
+    }
+    if (__any_sync(0xffffffffu, fix) && lane_id() == 0) set_flag(st, F_LEVEL_FIXUP);
+    if (__any_sync(0xffffffffu, err) && lane_id() == 0) set_err(st, ERR_NOT_NESTED);
+}
+
+// ------------------------------------------------------------------ per-stream tiles
+// The enclosure answers kernels stream by stream.  psk holds every kernel
+// index regrouped by stream: a stable partition of the time-ordered kernels,
+// so each stream's kernels are in time order, streams one after another
+// (stream s from koff[s]).  Each stream's run is cut into tiles of EN_TILE
+// kernels; tile r of stream s has the stream-major index u = toff[s] + r.
+// Tiles are launched round-robin over the streams (tile r of every stream
+// before tile r + 1 of any), so the tiles in flight cover one window of time
+// and their gathers of start times and scattered result writes share sectors
+// in L2.
+constexpr int EN_THREADS = 128;
+constexpr int EN_PER = 32;                        // consecutive kernels one thread sweeps
+constexpr int EN_TILE = EN_THREADS * EN_PER;      // kernels of one stream per tile
+constexpr int EN_WIN = 3072;                      // staged range entries per tile
+constexpr int EN_RD = 8;                          // depths whose sweep state stays in registers
+
+// The stream of the kernel at time position i, and its place in psk.
+struct TimeStreamDigit {
+    const uint8_t *stream;
+    const uint32_t *korder;     // time order, NULL = array order
+    __device__ __forceinline__ unsigned operator()(int64_t i) const {
+        return stream[korder ? korder[i] : (uint32_t)i];
+    }
+};
+struct PlaceByStream {
+    const uint32_t *korder;
+    uint32_t *psk;
+    __device__ __forceinline__ unsigned operator()(int64_t i, uint32_t dest, unsigned) const {
+        psk[dest] = korder ? korder[i] : (uint32_t)i;
+        return 0u;
+    }
+    __device__ __forceinline__ void done(unsigned) const {}
+};
+
+// Launch position of every tile: tile u = toff[s] + r goes to
+//   sum over streams q of min(tiles of q, r)  +  #{q < s : tiles of q > r}.
+// tinfo[position] = s | r << 8.
+__global__ void k_tile_order(const uint32_t *__restrict__ toff, int64_t nt, uint32_t *__restrict__ tinfo) {
+    __shared__ uint32_t to[257];
+    for (int i = threadIdx.x; i < 257; i += blockDim.x) to[i] = toff[i];
+    __syncthreads();
+    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < nt; u += (int64_t)gridDim.x * blockDim.x) {
+        int lo = 0, hi = 256;                      // the stream of u: last s with to[s] <= u
+        while (hi - lo > 1) {
+            const int m = (lo + hi) >> 1;
+            if (to[m] <= (uint32_t)u) lo = m; else hi = m;
+        }
+        const uint32_t sid = (uint32_t)lo, r = (uint32_t)u - to[lo];
+        uint32_t p = 0;
+        for (int q = 0; q < 256; ++q) {
+            const uint32_t c = to[q + 1] - to[q];
+            p += (c < r ? c : r) + ((uint32_t)q < sid && c > r ? 1u : 0u);
+        }
+        tinfo[p] = sid | (r << 8);
     }
 }
 
-// ------------------------------------------------------------------ enclosure
+// Window of every (tile, depth): P[u * 32 + d] = (last position of level
+// (s, d) with start <= the tile's first time, last position with start <= its
+// last time), relative to the level's start, -1 for none.  Lane d of a warp
+// takes depth d of one tile.
+__global__ void k_stream_windows(const int64_t *__restrict__ ls, const uint32_t *__restrict__ lvl_off,
+                                 const uint8_t *__restrict__ ndep, const uint32_t *__restrict__ toff,
+                                 const uint32_t *__restrict__ koff, const uint32_t *__restrict__ kcnt,
+                                 const uint32_t *__restrict__ psk, const int64_t *__restrict__ k_start, int64_t nt,
+                                 int2 *__restrict__ P) {
+    for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < nt * 32; q += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t u = q >> 5;
+        const int d = (int)(q & 31);
+        int lo = 0, hi = 256;
+        while (hi - lo > 1) {
+            const int m = (lo + hi) >> 1;
+            if (toff[m] <= (uint32_t)u) lo = m; else hi = m;
+        }
+        const int sid = lo;
+        if (d >= ndep[sid]) continue;
+        const int64_t pos0 = (u - toff[sid]) * (int64_t)EN_TILE;
+        const int64_t cnt = (int64_t)kcnt[sid] - pos0 < EN_TILE ? (int64_t)kcnt[sid] - pos0 : EN_TILE;
+        const long long tf = k_start[psk[koff[sid] + pos0]], tl = k_start[psk[koff[sid] + pos0 + cnt - 1]];
+        const int64_t L0 = lvl_off[sid * 32 + d], L1 = lvl_off[sid * 32 + d + 1];
+        int64_t x = L0, y = L1;                    // first position with start > tf
+        while (x < y) {
+            const int64_t m = (x + y) >> 1;
+            if (ls[m] <= tf) x = m + 1; else y = m;
+        }
+        const int64_t a = x;
+        y = L1;                                    // first position with start > tl (at or after a)
+        while (x < y) {
+            const int64_t m = (x + y) >> 1;
+            if (ls[m] <= tl) x = m + 1; else y = m;
+        }
+        P[q] = make_int2((int)(a - L0 - 1), (int)(x - L0 - 1));
+    }
+}
+
 struct EncArgs {
-    const uint8_t *k_stream;
     const int64_t *k_start;
-    const uint32_t *korder;     // NULL = identity
-    int64_t K;
+    const uint32_t *psk, *tinfo, *toff, *koff, *kcnt;
+    const uint8_t *ndep;
     const int64_t *ls, *le;
     const uint32_t *li;
     const uint32_t *lvl_off;    // [LEVELS + 1]
-    const int32_t *P;           // [(nt + 1) * nl]
-    int nl;
-    int64_t nt;
-    const uint16_t *cbase;      // [256] first compact level of a stream
-    const uint16_t *level_of_compact;   // [nl] level key (stream * 32 + depth) of a compact level
-    const uint8_t *ndepth;      // [256] levels of a stream (depths 0 .. n-1)
+    const int2 *P;              // [tiles * 32]
     int32_t *out_range;
     uint8_t *out_nop;
-    const uint32_t *tiles;      // tiles to process (deferred ones), or NULL for 0 .. nt-1
-    const unsigned *ntiles;     // their count (device), with `tiles`
-    uint32_t *deferred;         // compact-layout pass: tiles handed to the wide pass
-    unsigned *ndeferred;
 };
 
-template <int WIN, int ACT>
 struct EncSmem {
-    uint32_t ws[WIN];               // staged start, relative to tile base (+1, clamped)
-    uint32_t we[WIN];               // staged end, same encoding
-    uint32_t wi[WIN];               // staged lvl_info
-    uint16_t act_off[ACT];          // window offset of an active level
-    uint16_t act_cnt[ACT];          // window length
-    int32_t act_gpos[ACT];          // global level position of the window's first entry (-1 none)
-    uint16_t sbase[256];            // first active slot of a present stream
-    uint32_t kt[ENC_TILE];          // the tile's kernel times, relative to the tile base (+1, clamped)
-    uint8_t ks[ENC_TILE];           // the tile's kernel streams
-    uint16_t klist[ENC_TILE];       // tile positions grouped by stream
-    uint16_t wcnt[ENC_THREADS / 32][256];
-    uint16_t soff[257];
-    uint32_t present[8];
-    uint32_t wbuf[33];
-    int slow;
-    int nact, nwin;
+    uint32_t ws[EN_WIN];        // staged start, relative to the tile's first time (+1, clamped)
+    uint32_t we[EN_WIN];        // staged end, same encoding
+    uint32_t wi[EN_WIN];        // staged lvl_info
+    int woff[32], wcnt[32];     // per depth: first staged entry and count
+    int wlev[32];               // per depth: level position of the window's first entry
+    int nwin;
 };
 
 __device__ __forceinline__ uint32_t rel32(long long x, long long base) {
@@ -371,143 +413,119 @@ __device__ __forceinline__ uint32_t rel32(long long x, long long base) {
     return v <= 0 ? 0u : (v >= 0xFFFFFFFFll ? 0xFFFFFFFFu : (uint32_t)v);
 }
 
-// One tile.  DEFER: a tile that outgrows the layout is handed on (its index
-// appended to A.deferred) instead of taking the global-search path.
-template <int WIN, int ACT, bool DEFER>
-__device__ __forceinline__ void enclose_tile(const EncArgs &A, EncSmem<WIN, ACT> &S, const int64_t t) {
-    const int64_t pos0 = t * ENC_TILE;
-    const int64_t cnt = A.K - pos0 < ENC_TILE ? A.K - pos0 : ENC_TILE;
-    if (threadIdx.x < 8) S.present[threadIdx.x] = 0;
-    __syncthreads();
+// Algorithm 2's walk over one depth's representative, outward-in: a
+// structural range resets the collection (everything above it is beyond the
+// cut), an operator becomes the innermost answer and counts, a non-op range
+// is passed over.
+__device__ __forceinline__ void walk_step(uint32_t info, int32_t &ans, int &nop) {
+    const uint32_t kind = info >> 30;
+    if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
+    else if (kind == KIND_OP) { ans = (int32_t)(info & 0x3FFFFFFFu); nop++; }
+}
 
-    const long long tbase = A.k_start[A.korder ? A.korder[pos0] : pos0];
-    {
-        // all loads first, so they are in flight together
-        constexpr int PER = ENC_TILE / ENC_THREADS;
-        unsigned sv[PER];
-        long long tv[PER];
-#pragma unroll
-        for (int u = 0; u < PER; ++u) {
-            const int j = u * ENC_THREADS + threadIdx.x;
-            const int64_t p = pos0 + (j < cnt ? j : 0);
-            const int64_t k = A.korder ? A.korder[p] : p;
-            sv[u] = A.k_stream[k];
-            tv[u] = A.k_start[k];
+// One tile of one stream.  Thread t sweeps the tile's kernels
+// [t * EN_PER, (t + 1) * EN_PER) in time order, keeping per depth (the first
+// EN_RD in registers) the last staged range starting at or before the
+// current kernel: its position, end and info, and the next range's start.  A
+// depth is searched once at the thread's first kernel and afterwards moves
+// only when the next start is passed, so a kernel usually costs one
+// comparison per depth.  The walk over the tracked depths runs for every
+// kernel without branches (threads of a warp stay together; redoing it only
+// when something changed saves less than the divergence costs); deeper
+// levels are searched when the walk reaches them.  A tile whose windows outgrow the
+// staging, or whose kernels span 2^32 ns or more (relative times no longer
+// fit), searches the global level lists instead.
+__global__ void __launch_bounds__(EN_THREADS) k_enclose(EncArgs A) {
+    __shared__ EncSmem S;
+    const uint32_t info = A.tinfo[blockIdx.x];
+    const int sid = (int)(info & 0xFFu);
+    const uint32_t r = info >> 8;
+    const int64_t u = A.toff[sid] + r;
+    const int64_t pos0 = (int64_t)r * EN_TILE;
+    const int cnt = (int)((int64_t)A.kcnt[sid] - pos0 < EN_TILE ? (int64_t)A.kcnt[sid] - pos0 : EN_TILE);
+    const uint32_t *tk = A.psk + A.koff[sid] + pos0;         // the tile's kernels in time order
+    const int nd = A.ndep[sid];
+    const long long tbase = A.k_start[tk[0]], tlast = A.k_start[tk[cnt - 1]];
+    const unsigned lane = lane_id(), warp = threadIdx.x >> 5;
+    if (warp == 0) {
+        const int d = (int)lane;
+        int c = 0, first = 0;
+        if (d < nd) {
+            const int2 w = A.P[u * 32 + d];
+            first = w.x < 0 ? 0 : w.x;
+            c = w.y < 0 ? 0 : w.y - first + 1;
         }
-#pragma unroll
-        for (int u = 0; u < PER; ++u) {
-            const int j = u * ENC_THREADS + threadIdx.x;
-            if (j < cnt) {
-                S.ks[j] = (uint8_t)sv[u];
-                S.kt[j] = rel32(tv[u], tbase);
-                atomicOr(&S.present[sv[u] >> 5], 1u << (sv[u] & 31));
+        const int incl = warp_inclusive_scan(c);
+        S.woff[d] = incl - c;
+        S.wcnt[d] = c;
+        S.wlev[d] = (d < nd ? (int)A.lvl_off[sid * 32 + d] : 0) + first;
+        if (d == 31) S.nwin = incl;
+    }
+    __syncthreads();
+    const bool slow = S.nwin > EN_WIN || (tlast - tbase) >= 0xFFFFFFF0ll;
+    if (slow) {
+        // global searches inside each depth's window
+        for (int j = threadIdx.x; j < cnt; j += EN_THREADS) {
+            const uint32_t k = tk[j];
+            const long long T = A.k_start[k];
+            int32_t ans = -1;
+            int nop = 0;
+            for (int d = 0; d < nd; ++d) {
+                int64_t x = S.wlev[d], y = x + S.wcnt[d];
+                const int64_t o = x;
+                while (x < y) {
+                    const int64_t m = (x + y) >> 1;
+                    if (A.ls[m] <= T) x = m + 1; else y = m;
+                }
+                if (x == o || A.le[x - 1] < T) break;
+                walk_step(A.li[x - 1], ans, nop);
             }
+            A.out_range[k] = ans;
+            if (A.out_nop) A.out_nop[k] = (uint8_t)nop;
+        }
+        return;
+    }
+    // stage the windows: one warp per depth, each depth's entries contiguous
+    for (int d = (int)warp; d < nd; d += EN_THREADS / 32) {
+        const int c = S.wcnt[d], o = S.woff[d];
+        const int64_t g0 = S.wlev[d];
+        for (int e = (int)lane; e < c; e += 32) {
+            S.ws[o + e] = rel32(A.ls[g0 + e], tbase);
+            S.we[o + e] = rel32(A.le[g0 + e], tbase);
+            S.wi[o + e] = A.li[g0 + e];
         }
     }
     __syncthreads();
-
-    // active levels: the levels of every stream present in the tile
-    {
-        const unsigned s = threadIdx.x;        // ENC_THREADS == 256 streams
-        unsigned n = ((S.present[s >> 5] >> (s & 31)) & 1u) ? A.ndepth[s] : 0u;
-        unsigned tot;
-        unsigned off = block_exclusive_scan<unsigned>(n, S.wbuf, &tot);
-        S.sbase[s] = (uint16_t)(off < ACT ? off : ACT);
-        if (threadIdx.x == 0) S.nact = (int)tot;
-        if (tot <= ACT && n) {
-            const unsigned cb = A.cbase[s];
-            for (unsigned d = 0; d < n; ++d) S.act_off[off + d] = (uint16_t)(cb + d);   // compact level, for now
-        }
-        __syncthreads();
-        // window bounds of every active level, one thread per level
-        if (tot <= ACT) {
-            for (unsigned a = threadIdx.x; a < tot; a += ENC_THREADS) {
-                const int l = S.act_off[a];
-                const int32_t lo = A.P[t * A.nl + l], hi = A.P[(t + 1) * A.nl + l];
-                const int32_t first = lo < 0 ? 0 : lo;
-                int32_t c = hi - first + 1;
-                if (hi < 0) c = 0;
-                S.act_cnt[a] = (uint16_t)(c < 0xFFFF ? c : 0xFFFF);
-                S.act_gpos[a] = (int32_t)(A.lvl_off[A.level_of_compact[l]] + first);
-            }
-        }
-    }
-    __syncthreads();
-    // span of the tile: its last kernel (time order) minus its first
-    const long long tlast = A.k_start[A.korder ? A.korder[pos0 + cnt - 1] : pos0 + cnt - 1];
-    int slow = S.nact > ACT || (tlast - tbase) >= 0xFFFFFFF0ll;
-    if (!slow) {
-        // window offsets: exclusive scan of counts over active slots
-        unsigned carry = 0;
-        for (int b = 0; b < S.nact; b += ENC_THREADS) {
-            int a = b + threadIdx.x;
-            unsigned c = a < S.nact ? S.act_cnt[a] : 0u;
-            unsigned tot;
-            unsigned off = block_exclusive_scan<unsigned>(c, S.wbuf, &tot);
-            if (a < S.nact) S.act_off[a] = (uint16_t)((carry + off) < 0xFFFF ? carry + off : 0xFFFF);
-            carry += tot;
-        }
-        if (threadIdx.x == 0) S.nwin = (int)carry;
-        __syncthreads();
-        slow = S.nwin > WIN;
-    }
-    if (!slow) {
-        // stage the windows: one thread per staged entry (its level found by a
-        // search over the window offsets), so all loads of a round are in flight
-        // together
-        const int nact = S.nact, nwin = S.nwin;
-        for (int e = threadIdx.x; e < nwin; e += ENC_THREADS) {
-            int x = 0, y = nact;                   // last active level with offset <= e
-            while (y - x > 1) {
-                const int m = (x + y) >> 1;
-                if (S.act_off[m] <= e) x = m; else y = m;
-            }
-            while (x + 1 < nact && S.act_off[x + 1] <= e && S.act_cnt[x] == 0) ++x;
-            const int64_t g = S.act_gpos[x] + (e - S.act_off[x]);
-            S.ws[e] = rel32(A.ls[g], tbase);
-            S.we[e] = rel32(A.le[g], tbase);
-            S.wi[e] = A.li[g];
-        }
-        // kernels grouped by stream, so a warp's lanes share windows and
-        // loop trip counts
-        block_group_by_key<ENC_THREADS, ENC_TILE / (ENC_THREADS / 32)>(
-            256, [&](int j) -> unsigned { return j < cnt ? (unsigned)S.ks[j] : GROUP_NONE; }, &S.wcnt[0][0], 256,
-            S.soff, S.klist, S.wbuf);
-        // Each thread sweeps ENC_CHUNK consecutive kernels of one stream in
-        // time order, keeping per depth (the first RD depths, in registers)
-        // the last window range starting at or before the current kernel:
-        // its position, end and info, and the start of the next one.  A depth
-        // is searched once when the stream changes and afterwards moves only
-        // when the next range's start is passed (positions only move
-        // forward), so a kernel usually costs one comparison per depth.
-        // The walk over the depths is redone only when a depth moved or a
-        // range it found has ended; otherwise it would visit the same ranges
-        // with the same results.
-        constexpr int RD = 8;                     // depths whose state stays in registers
-        constexpr uint32_t NONE_T = 0xFFFFFFFFu;
-        int cur_s = -1, nd = 0, a0 = 0;
-        int pos[RD];                              // window position of the depth's range, -1 none
-        uint32_t nxt[RD], cend[RD], cinf[RD];     // next start; end and info of the range
+    constexpr uint32_t NONE_T = 0xFFFFFFFFu;
+    const int j0 = (int)threadIdx.x * EN_PER;
+    const int j1 = j0 + EN_PER < cnt ? j0 + EN_PER : cnt;
+    if (j0 >= j1) return;
+    int pos[EN_RD];                               // window position of the depth's range, -1 none
+    uint32_t nxt[EN_RD], cend[EN_RD], cinf[EN_RD]; // next start; end and info of the range
+    constexpr int B = 4;                          // kernels loaded per batch
+    uint32_t kb[B];
+    long long tb[B];
+    auto load_batch = [&](int jb) {
 #pragma unroll
-        for (int d = 0; d < RD; ++d) pos[d] = -1, nxt[d] = NONE_T, cend[d] = 0, cinf[d] = 0;
-        int32_t ans = -1;
-        int nop = 0;
-        bool redo = true;                         // the walk must be redone
-        uint32_t min_end = 0;                     // earliest end among the ranges the walk went through
-        for (int u = 0; u < ENC_CHUNK; ++u) {
-            const int idx = threadIdx.x * ENC_CHUNK + u;
-            if (idx >= cnt) break;
-            const int j = S.klist[idx];
-            const int64_t k = A.korder ? A.korder[pos0 + j] : pos0 + j;
-            const int s = S.ks[j];
-            const uint32_t T = S.kt[j];
-            if (s != cur_s) {
-                cur_s = s;
-                nd = A.ndepth[s];
-                a0 = S.sbase[s];
+        for (int v = 0; v < B; ++v) kb[v] = tk[jb + v < j1 ? jb + v : j0];
 #pragma unroll
-                for (int d = 0; d < RD; ++d) {
-                    const int c = d < nd ? S.act_cnt[a0 + d] : 0, o = d < nd ? S.act_off[a0 + d] : 0;
+        for (int v = 0; v < B; ++v) tb[v] = A.k_start[kb[v]];
+    };
+    load_batch(j0);
+    for (int jb = j0; jb < j1; jb += B) {
+        uint32_t kc[B], tc[B];
+#pragma unroll
+        for (int v = 0; v < B; ++v) { kc[v] = kb[v]; tc[v] = rel32(tb[v], tbase); }
+        if (jb + B < j1) load_batch(jb + B);      // the next batch in flight during this one
+#pragma unroll
+        for (int v = 0; v < B; ++v) {
+            const int j = jb + v;
+            if (j >= j1) break;
+            const uint32_t T = tc[v];
+            if (j == j0) {
+#pragma unroll
+                for (int d = 0; d < EN_RD; ++d) {
+                    const int c = d < nd ? S.wcnt[d] : 0, o = d < nd ? S.woff[d] : 0;
                     int x = o, y = o + c;         // last window position with start <= T
                     while (x < y) {
                         const int m = (x + y) >> 1;
@@ -519,115 +537,47 @@ __device__ __forceinline__ void enclose_tile(const EncArgs &A, EncSmem<WIN, ACT>
                     cend[d] = p >= 0 ? S.we[o + p] : 0u;
                     cinf[d] = p >= 0 ? S.wi[o + p] : 0u;
                 }
-                redo = true;
             } else {
 #pragma unroll
-                for (int d = 0; d < RD; ++d) {
+                for (int d = 0; d < EN_RD; ++d) {
                     if (nxt[d] <= T) {            // a later range of this depth starts by T
-                        const int c = S.act_cnt[a0 + d], o = S.act_off[a0 + d];
+                        const int c = S.wcnt[d], o = S.woff[d];
                         int p = pos[d] + 1;
                         while (p + 1 < c && S.ws[o + p + 1] <= T) ++p;
                         pos[d] = p;
                         nxt[d] = p + 1 < c ? S.ws[o + p + 1] : NONE_T;
                         cend[d] = S.we[o + p];
                         cinf[d] = S.wi[o + p];
-                        redo = true;
                     }
                 }
-                redo = redo || T > min_end;
             }
-            if (redo) {
-                ans = -1;
-                nop = 0;
-                bool alive = true;
-                min_end = NONE_T;
+            // the walk over the tracked depths, every kernel, without branches
+            int32_t ans = -1;
+            int nop = 0;
+            bool alive = true;
 #pragma unroll
-                for (int d = 0; d < RD; ++d) {
-                    if (alive && d < nd) {
-                        if (pos[d] < 0 || cend[d] < T) {
-                            alive = false;
-                        } else {
-                            min_end = min(min_end, cend[d]);
-                            const uint32_t kind = cinf[d] >> 30;
-                            if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
-                            else if (kind == KIND_OP) { ans = (int32_t)(cinf[d] & 0x3FFFFFFFu); nop++; }
-                        }
-                    }
-                }
-                bool deep = false;
-                for (int d = RD; alive && d < nd; ++d) {   // deeper levels: one search each
-                    deep = true;
-                    const int c = S.act_cnt[a0 + d], o = S.act_off[a0 + d];
+            for (int d = 0; d < EN_RD; ++d) {
+                alive = alive && d < nd && pos[d] >= 0 && cend[d] >= T;
+                const uint32_t kind = cinf[d] >> 30;
+                const bool st_d = alive && kind == KIND_STRUCT, op_d = alive && kind == KIND_OP;
+                ans = st_d ? -1 : (op_d ? (int32_t)(cinf[d] & 0x3FFFFFFFu) : ans);
+                nop = st_d ? 0 : nop + (op_d ? 1 : 0);
+            }
+            if (alive && nd > EN_RD) {
+                for (int d = EN_RD; d < nd; ++d) {   // deeper levels: one search each
+                    const int c = S.wcnt[d], o = S.woff[d];
                     int x = o, y = o + c;
                     while (x < y) {
                         const int m = (x + y) >> 1;
                         if (S.ws[m] <= T) x = m + 1; else y = m;
                     }
                     if (x == o || S.we[x - 1] < T) break;
-                    const uint32_t info = S.wi[x - 1];
-                    const uint32_t kind = info >> 30;
-                    if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
-                    else if (kind == KIND_OP) { ans = (int32_t)(info & 0x3FFFFFFFu); nop++; }
+                    walk_step(S.wi[x - 1], ans, nop);
                 }
-                redo = deep;                      // deep levels are not tracked: search again next time
             }
-            A.out_range[k] = ans;
-            if (A.out_nop) A.out_nop[k] = (uint8_t)nop;
+            A.out_range[kc[v]] = ans;
+            if (A.out_nop) A.out_nop[kc[v]] = (uint8_t)nop;
         }
-        return;
-    }
-    if (DEFER) {                           // the wide pass takes this tile
-        if (threadIdx.x == 0) A.deferred[atomicAdd(A.ndeferred, 1u)] = (uint32_t)t;
-        return;
-    }
-    // slow tile: search the global level lists inside the window bounds
-    for (int j = threadIdx.x; j < cnt; j += ENC_THREADS) {
-        const int64_t p = pos0 + j;
-        const int64_t k = A.korder ? A.korder[p] : p;
-        const unsigned s = A.k_stream[k];
-        const long long T = A.k_start[k];
-        const int nd = A.ndepth[s];
-        int32_t ans = -1;
-        int nop = 0;
-        for (int d = 0; d < nd; ++d) {
-            int l = A.cbase[s] + d;
-            int32_t lo = A.P[t * A.nl + l], hi = A.P[(t + 1) * A.nl + l];
-            if (hi < 0) break;
-            int64_t g0 = A.lvl_off[s * 32 + d];
-            int64_t x = g0 + (lo < 0 ? 0 : lo), y = g0 + hi + 1, o = x;
-            while (x < y) {
-                int64_t m = (x + y) >> 1;
-                if (A.ls[m] <= T) x = m + 1; else y = m;
-            }
-            if (x == o || A.le[x - 1] < T) break;
-            uint32_t info = A.li[x - 1];
-            uint32_t kind = info >> 30;
-            if (kind == KIND_STRUCT) { ans = -1; nop = 0; }
-            else if (kind == KIND_OP) { ans = (int32_t)(info & 0x3FFFFFFFu); nop++; }
-        }
-        A.out_range[k] = ans;
-        if (A.out_nop) A.out_nop[k] = (uint8_t)nop;
-    }
-}
-
-using EncSmemSmall = EncSmem<ENC_WIN_SMALL, ENC_ACT_SMALL>;
-using EncSmemWide = EncSmem<ENC_WIN_WIDE, ENC_ACT_WIDE>;
-
-// Compact layout, one tile per block, four blocks per SM; tiles that outgrow
-// it are deferred to k_enclose_wide.
-__global__ void __launch_bounds__(ENC_THREADS, 4) k_enclose(EncArgs A) {
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    enclose_tile<ENC_WIN_SMALL, ENC_ACT_SMALL, true>(A, *reinterpret_cast<EncSmemSmall *>(smem_raw), blockIdx.x);
-}
-
-// Wide layout: every tile (A.tiles NULL) or the deferred ones.
-__global__ void __launch_bounds__(ENC_THREADS) k_enclose_wide(EncArgs A) {
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    EncSmemWide &S = *reinterpret_cast<EncSmemWide *>(smem_raw);
-    const int64_t n = A.tiles ? (int64_t)*A.ntiles : A.nt;
-    for (int64_t i = blockIdx.x; i < n; i += gridDim.x) {
-        enclose_tile<ENC_WIN_WIDE, ENC_ACT_WIDE, false>(A, S, A.tiles ? (int64_t)A.tiles[i] : i);
-        __syncthreads();                   // the next tile reuses the shared memory
     }
 }
 
@@ -655,35 +605,42 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     if (R > 0 && (!rng->stream || !rng->start_ns || !rng->end_ns || !rng->depth || !rng->op_id))
         return OPATTR_E_INVALID_ARG;
 
-    // scratch: range sort (u64 keys x2, values x2), level arrays, tables, kernel order
-    const int64_t nt = (K + ENC_TILE - 1) / ENC_TILE;
+    // scratch: range sort (u64 keys x2, values x2), level arrays, tables,
+    // kernel order, the stream partition of the kernels and its tile tables
+    const int64_t nt_max = (K + EN_TILE - 1) / EN_TILE + 256;
     Need nd;
-    nd.add<uint32_t>(LEVELS + 1).add<uint32_t>(LEVELS + 1);
+    nd.add<uint32_t>(LEVELS + 1 + 256).add<uint32_t>(LEVELS + 1);
     nd.add<uint64_t>(R).add<uint64_t>(R).add<uint32_t>(R).add<uint32_t>(R);
-    const int64_t part_n = std::max<int64_t>(scan_scratch_elems(radix_hist_elems(R)), scan_scratch_elems(LEVELS + 1));
-    nd.add<uint32_t>(radix_hist_elems(R)).add<uint32_t>(part_n);
+    const int64_t hist_n = std::max(radix_hist_elems(R), radix_hist_elems(K));
+    const int64_t part_n = std::max<int64_t>(scan_scratch_elems(hist_n), scan_scratch_elems(LEVELS + 1));
+    nd.add<uint32_t>(hist_n).add<uint32_t>(part_n);
     nd.add<int64_t>(R).add<int64_t>(R).add<uint32_t>(R);
     nd.add<unsigned char>(STAGE_BYTES);
-    nd.add<int32_t>((nt + 1) * (int64_t)LEVELS).add<uint32_t>(nt).add<unsigned>(1);
+    nd.add<uint32_t>(K).add<uint32_t>(nt_max).add<int2>(nt_max * 32);
     size_t need = nd.bytes + kernel_order_scratch(K) + 4096;
     opattr_status st = ensure_arena(c, need);
     if (st) return st;
     Arena a(c);
     if ((st = reset_status(c))) return st;
 
-    uint32_t *level_hist = a.take<uint32_t>(LEVELS + 1);
+    // level histogram [LEVELS] and kernels per stream [256], zeroed together
+    uint32_t *level_hist = a.take<uint32_t>(LEVELS + 1 + 256);
+    uint32_t *kstream = level_hist + LEVELS + 1;
     uint32_t *lvl_off = a.take<uint32_t>(LEVELS + 1);
     uint32_t *part = a.take<uint32_t>(part_n);
     if (!level_hist || !lvl_off || !part) return OPATTR_E_OOM;
-    cudaMemsetAsync(level_hist, 0, sizeof(uint32_t) * (LEVELS + 1), c.stream);
+    cudaMemsetAsync(level_hist, 0, sizeof(uint32_t) * (LEVELS + 1 + 256), c.stream);
     if (R > 0)
         launch(c, "check_ranges", k_check_ranges, dim3(grid_for(R, RCHK_THREADS * RCHK_ITEMS)), dim3(RCHK_THREADS), 0,
                rng->stream, rng->start_ns, rng->end_ns, rng->depth, R, level_hist, c.d_status);
-    check_kernel_order(c, kern->stream, kern->start_ns, K);
-    // the level offsets come back with the status: one synchronisation for both
+    check_kernel_order(c, kern->stream, kern->start_ns, K, kstream);
+    // the level offsets and the stream counts come back with the status: one
+    // synchronisation for all
     scan_exclusive_u32(c, level_hist, lvl_off, LEVELS + 1, part, nullptr);
     if (cudaMemcpyAsync(c.h_levels, lvl_off, sizeof(uint32_t) * (LEVELS + 1), cudaMemcpyDeviceToHost, c.stream) !=
-        cudaSuccess)
+            cudaSuccess ||
+        cudaMemcpyAsync(c.h_levels + LEVELS + 1, kstream, sizeof(uint32_t) * 256, cudaMemcpyDeviceToHost, c.stream) !=
+            cudaSuccess)
         return cuda_status(c, cudaGetLastError());
     if ((st = read_status(c))) return st;
     if ((st = status_from_err(c.h_status->err))) return st;
@@ -701,18 +658,25 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
         return read_status(c);
     }
 
-    // ---- compact level tables (host side, from the level offsets), built in
-    // pinned staging and sent with one copy: level of each compact level
-    // (u16 [LEVELS]), first compact level of a stream (u16 [256]), levels of a
-    // stream (u8 [256]), compact id of a level (u8 [LEVELS], at most 256 levels)
+    // ---- host-built tables, sent with one copy from pinned staging: level of
+    // each compact level (u16 [LEVELS]), first compact level of a stream
+    // (u16 [256]), levels of a stream (u8 [256]), compact id of a level
+    // (u8 [LEVELS], at most 256 levels), and per stream its first place in
+    // the stream partition, its kernels and its first tile (u32 [256],
+    // [256], [257])
     constexpr size_t ST_LOC = 0, ST_CBASE = ST_LOC + 2 * LEVELS, ST_NDEP = ST_CBASE + 2 * 256,
-                     ST_CMAP = ST_NDEP + 256, ST_END = ST_CMAP + LEVELS;
+                     ST_CMAP = ST_NDEP + 256, ST_KOFF = ST_CMAP + LEVELS, ST_KCNT = ST_KOFF + 4 * 256,
+                     ST_TOFF = ST_KCNT + 4 * 256, ST_END = ST_TOFF + 4 * 257;
     static_assert(ST_END <= STAGE_BYTES, "staging too small");
     const uint32_t *off = c.h_levels;
+    const uint32_t *kcnt_h = c.h_levels + LEVELS + 1;
     uint16_t *level_of_compact = reinterpret_cast<uint16_t *>(c.h_stage + ST_LOC);
     uint16_t *cbase = reinterpret_cast<uint16_t *>(c.h_stage + ST_CBASE);
     uint8_t *ndep = c.h_stage + ST_NDEP;
     uint8_t *cmap = c.h_stage + ST_CMAP;
+    uint32_t *koff_h = reinterpret_cast<uint32_t *>(c.h_stage + ST_KOFF);
+    uint32_t *kcnt_s = reinterpret_cast<uint32_t *>(c.h_stage + ST_KCNT);
+    uint32_t *toff_h = reinterpret_cast<uint32_t *>(c.h_stage + ST_TOFF);
     int nl = 0;
     for (int s = 0; s < 256; ++s) {
         cbase[s] = (uint16_t)nl;
@@ -725,29 +689,45 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     }
     memset(cmap, 0, LEVELS);
     for (int l = 0; l < nl && l < 256; ++l) cmap[level_of_compact[l]] = (uint8_t)l;
+    uint32_t kacc = 0, tacc = 0;
+    for (int s = 0; s < 256; ++s) {
+        koff_h[s] = kacc;
+        kcnt_s[s] = kcnt_h[s];
+        toff_h[s] = tacc;
+        kacc += kcnt_h[s];
+        tacc += (kcnt_h[s] + EN_TILE - 1) / EN_TILE;
+    }
+    toff_h[256] = tacc;
+    const int64_t NT = tacc;
 
     uint64_t *rk0 = a.take<uint64_t>(R), *rk1 = a.take<uint64_t>(R);
     uint32_t *rv0 = a.take<uint32_t>(R), *rv1 = a.take<uint32_t>(R);
-    uint32_t *hist = a.take<uint32_t>(radix_hist_elems(R));
+    uint32_t *hist = a.take<uint32_t>(hist_n);
     int64_t *ls = a.take<int64_t>(R), *le = a.take<int64_t>(R);
     uint32_t *li = a.take<uint32_t>(R);
     unsigned char *d_stage = a.take<unsigned char>(ST_END);
-    const uint16_t *d_loc = reinterpret_cast<const uint16_t *>(d_stage + ST_LOC);
-    const uint16_t *d_cbase = reinterpret_cast<const uint16_t *>(d_stage + ST_CBASE);
+    uint32_t *psk = a.take<uint32_t>(K), *tinfo = a.take<uint32_t>(NT);
+    int2 *P = a.take<int2>(NT * 32);
+    if (!rk0 || !rk1 || !rv0 || !rv1 || !hist || !ls || !le || !li || !d_stage || !psk || !tinfo || !P)
+        return OPATTR_E_OOM;
     const uint8_t *d_ndep = d_stage + ST_NDEP;
     const uint8_t *d_cmap = d_stage + ST_CMAP;
-    uint32_t *deferred = a.take<uint32_t>(nt);
-    unsigned *ndeferred = a.take<unsigned>(1);
-    if (!deferred || !ndeferred) return OPATTR_E_OOM;
-    int32_t *P = a.take<int32_t>((nt + 1) * (int64_t)(nl > 0 ? nl : 1));
-    if (!rk0 || !rk1 || !rv0 || !rv1 || !hist || !ls || !le || !li || !d_stage || !P) return OPATTR_E_OOM;
+    const uint32_t *d_koff = reinterpret_cast<const uint32_t *>(d_stage + ST_KOFF);
+    const uint32_t *d_kcnt = reinterpret_cast<const uint32_t *>(d_stage + ST_KCNT);
+    const uint32_t *d_toff = reinterpret_cast<const uint32_t *>(d_stage + ST_TOFF);
     cudaMemcpyAsync(d_stage, c.h_stage, ST_END, cudaMemcpyHostToDevice, c.stream);
 
-    // ---- kernel time order
+    // ---- kernel time order, then the kernels partitioned by stream
     uint32_t *korder = nullptr;
     if (!k_sorted && K > 0) {
         korder = kernel_time_order(c, a, kern->stream, kern->start_ns, K);
         if (!korder) return OPATTR_E_OOM;
+    }
+    if (K > 0 && nl > 0) {
+        const TimeStreamDigit dg{kern->stream, korder};
+        digit_offsets(c, dg, K, hist, part);
+        digit_rank(c, "stream_place", dg, K, hist, PlaceByStream{korder, psk});
+        launch(c, "tile_order", k_tile_order, dim3(grid_for(NT, 256, 4096)), dim3(256), 0, d_toff, NT, tinfo);
     }
 
     // ---- level lists, their validation, the windows and the enclosure, without
@@ -793,62 +773,32 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
             launch(c, "level_gather", k_level_gather, dim3(g), dim3(256), 0, rng->start_ns, rng->end_ns, rng->op_id,
                    (const uint32_t *)lperm, R, ls, le, li);
         }
-        launch(c, "validate_levels", k_validate_levels, dim3(grid_for(R, 256, 65535)), dim3(256), 0, rng->stream,
+        launch(c, "validate_levels", k_validate_levels, dim3(grid_for(R, 256 * VL_PER, 65535)), dim3(256), 0, rng->stream,
                rng->depth, (const int64_t *)ls, (const int64_t *)le, (const uint32_t *)li, (const uint32_t *)lvl_off,
                R, c.d_status);
         if (K > 0 && nl == 0)
             launch(c, "fill_unattributed", k_fill_unattributed, dim3(grid_for(K, 256, 65535)), dim3(256), 0, out_range,
                    out_nop, K);
         if (K > 0 && nl > 0) {
-            // chunks of WT_CHUNK tiles once the table is large (searches for
-            // every entry in parallel would then repeat most of their steps)
-            const int wt_chunk = (nt + 1) * (int64_t)nl >= ((int64_t)1 << 22) ? WT_CHUNK : 1;
-            launch(c, "window_table", k_window_table,
-                   dim3(grid_for((nt + 1 + wt_chunk - 1) / wt_chunk * nl, 256, 65535)), dim3(256), 0,
-                   (const int64_t *)ls, (const uint32_t *)lvl_off, (const uint16_t *)d_loc, nl, kern->start_ns,
-                   (const uint32_t *)korder, K, nt, wt_chunk, P);
+            launch(c, "stream_windows", k_stream_windows, dim3(grid_for(NT * 32, 256, 65535)), dim3(256), 0,
+                   (const int64_t *)ls, (const uint32_t *)lvl_off, d_ndep, d_toff, d_koff, d_kcnt,
+                   (const uint32_t *)psk, kern->start_ns, NT, P);
             EncArgs A;
-            A.k_stream = kern->stream;
             A.k_start = kern->start_ns;
-            A.korder = korder;
-            A.K = K;
+            A.psk = psk;
+            A.tinfo = tinfo;
+            A.toff = d_toff;
+            A.koff = d_koff;
+            A.kcnt = d_kcnt;
+            A.ndep = d_ndep;
             A.ls = ls;
             A.le = le;
             A.li = li;
             A.lvl_off = lvl_off;
             A.P = P;
-            A.nl = nl;
-            A.nt = nt;
-            A.cbase = d_cbase;
-            A.level_of_compact = d_loc;
-            A.ndepth = d_ndep;
             A.out_range = out_range;
             A.out_nop = out_nop;
-            static unsigned attr_done = 0;
-            if (c.device < 32 && !(attr_done & (1u << c.device))) {
-                cudaFuncSetAttribute(k_enclose, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sizeof(EncSmemSmall));
-                cudaFuncSetAttribute(k_enclose_wide, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                     (int)sizeof(EncSmemWide));
-                attr_done |= 1u << c.device;
-            }
-            A.tiles = nullptr;
-            A.ntiles = nullptr;
-            A.deferred = deferred;
-            A.ndeferred = ndeferred;
-            if (nl <= ENC_ACT_SMALL) {
-                // compact layout first; the tiles it defers go through the wide one
-                cudaMemsetAsync(ndeferred, 0, sizeof(unsigned), c.stream);
-                launch(c, "enclose", k_enclose, dim3((unsigned)nt), dim3(ENC_THREADS), sizeof(EncSmemSmall), A);
-                A.tiles = deferred;
-                A.ntiles = ndeferred;
-                int sms = 0;
-                cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
-                launch(c, "enclose_wide", k_enclose_wide, dim3((unsigned)std::min<int64_t>(nt, 3 * std::max(1, sms))),
-                       dim3(ENC_THREADS), sizeof(EncSmemWide), A);
-            } else {
-                launch(c, "enclose_wide", k_enclose_wide, dim3((unsigned)nt), dim3(ENC_THREADS), sizeof(EncSmemWide),
-                       A);
-            }
+            launch(c, "enclose", k_enclose, dim3((unsigned)NT), dim3(EN_THREADS), 0, A);
         }
         if ((st = read_status(c))) return st;
         if (!full_sort && (c.h_status->flags & F_LEVEL_FIXUP)) {

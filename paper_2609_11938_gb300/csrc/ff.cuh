@@ -133,26 +133,51 @@ __device__ __forceinline__ double ff_to_f64(ff v) {
     return __longlong_as_double((long long)bits);
 }
 
-// hi + lo as a double for a normalised pair, with 32-bit integer operations:
-// hi's bits widened to a double, lo added to its 52-bit fraction as a signed
-// integer (exact while lo's bits reach no lower than 2^-52 of hi, else
-// truncated within one unit).  A normalised lo cannot carry the fraction out
-// of its binade; it can borrow out of it only when hi is a power of two, and
-// then one unit of the lower binade is half as large, so lo counts twice.
-// A zero hi gives +0; a subnormal hi takes ff_to_f64.
+// The rare inputs of the conversions below (subnormal, tiny or non-finite),
+// out of line so the common path stays short.
+__device__ __noinline__ double ff_to_f64_rare(float hi, float lo) { return ff_to_f64(ff{hi, lo}); }
+
+// hi + lo as a double for a normalised pair (|lo| <= ulp(hi) / 2), nearest
+// to within half a double ulp.  lo is scaled exactly (by a power of two) into
+// units of the ulp of hi widened to a double, rounded to an integer q
+// (|q| <= 2^28, so it never carries out of hi's binade) and added to hi's
+// widened bit pattern.  Just below a power of two the ulp halves, so a
+// negative q counts twice there.  A zero pair gives a zero of hi's sign;
+// subnormal, tiny (below 2^-74) and non-finite hi take ff_to_f64.
 __device__ __forceinline__ double ff_to_f64_fast(ff v) {
-    const unsigned uh = __float_as_uint(v.hi), ul = __float_as_uint(v.lo);
-    const unsigned exh = (uh >> 23) & 0xFFu, exl = (ul >> 23) & 0xFFu;
-    if (exh == 0) return (uh << 1) == 0 ? 0.0 : ff_to_f64(v);
+    const unsigned uh = __float_as_uint(v.hi);
+    const unsigned exh = (uh >> 23) & 0xFFu;
+    if (exh - 53u > 201u) {                                    // exh < 53 or exh == 255
+        if ((uh << 1) == 0u) return __longlong_as_double((long long)((unsigned long long)(uh >> 31) << 63));
+        return ff_to_f64_rare(v.hi, v.lo);
+    }
+    const float sc = __uint_as_float((306u - exh) << 23);    // 2^(179 - exh): one ulp of double(hi) -> 1
+    int q = __float2int_rn(__fmul_rn(v.lo, sc));
+    if (uh >> 31) q = -q;                                      // relative to hi's magnitude
     const unsigned mh = uh & 0x7FFFFFu;
-    const unsigned ml = (ul & 0x7FFFFFu) | (exl ? 0x800000u : 0u);
-    const int s = (int)(exl ? exl : 1u) - (int)exh + 29;               // lo's unit against 2^-52 of hi
-    const bool relneg = ((uh ^ ul) >> 31) != 0;
-    unsigned d = s >= 0 ? (s < 32 ? ml << s : 0u) : (-s < 32 ? ml >> -s : 0u);
-    if (mh == 0 && relneg) d <<= 1;
-    const unsigned long long pat = ((unsigned long long)(((exh + 896u) << 20) | (mh >> 3)) << 32) | (mh << 29);
-    const unsigned long long r = relneg ? pat - d : pat + d;
-    return __longlong_as_double((long long)(r | ((unsigned long long)(uh >> 31) << 63)));
+    if (mh == 0 && q < 0) q *= 2;
+    const unsigned long long mag =
+        ((unsigned long long)(((exh + 896u) << 20) | (mh >> 3)) << 32) | ((unsigned long long)mh << 29);
+    const unsigned long long bits = (mag + (unsigned long long)(long long)q) | ((unsigned long long)(uh >> 31) << 63);
+    return __longlong_as_double((long long)bits);
+}
+
+// A float as a double (exact): the bits widened for a normal value, zeros
+// directly, the rest (subnormal, infinite, NaN) through ff_to_f64.
+__device__ __forceinline__ double f32_to_f64_fast(float x) {
+    const unsigned u = __float_as_uint(x);
+    const unsigned ex = (u >> 23) & 0xFFu;
+    if (ex - 1u > 253u) {                                      // zero, subnormal, infinite or NaN
+        if ((u << 1) == 0u) return __longlong_as_double((long long)((unsigned long long)(u >> 31) << 63));
+        if (ex == 0xFFu) {
+            const unsigned long long inf_nan = 0x7FF0000000000000ull | ((unsigned long long)(u & 0x7FFFFFu) << 29);
+            return __longlong_as_double((long long)(inf_nan | ((unsigned long long)(u >> 31) << 63)));
+        }
+        return ff_to_f64_rare(x, 0.f);
+    }
+    const unsigned long long bits = ((unsigned long long)(u >> 31) << 63) |
+                                    ((unsigned long long)(ex + 896u) << 52) | ((unsigned long long)(u & 0x7FFFFFu) << 29);
+    return __longlong_as_double((long long)bits);
 }
 
 // 1 / D for an int64 D > 0 as a normalised pair within about 2^-46 relative:

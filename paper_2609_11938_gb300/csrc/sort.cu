@@ -151,7 +151,7 @@ __global__ void __launch_bounds__(RADIX_THREADS) k_radix_upsweep(const K *__rest
 }
 
 // Stable scatter of one tile.  Warp w ranks its 512 keys in order, 32 at a
-// time, with __match_any_sync peer groups; per-(warp, digit) counts give the
+// time, with peer groups from one ballot per digit bit; per-(warp, digit) counts give the
 // tile-local order; keys are staged in shared memory sorted by digit and
 // then written out so equal-digit runs go to consecutive addresses.
 template <typename K>
@@ -178,19 +178,29 @@ __global__ void __launch_bounds__(RADIX_THREADS) k_radix_downsweep(const K *__re
     uint32_t val[RADIX_ITEMS];
     uint32_t rank[RADIX_ITEMS];
     const unsigned lt = lanemask_lt();
+    unsigned peers[RADIX_ITEMS];
 #pragma unroll
-    for (int it = 0; it < RADIX_ITEMS; ++it) {
+    for (int it = 0; it < RADIX_ITEMS; ++it) {        // keys, digits and peer groups first: independent
         int64_t i = base + it * 32 + lane;
         bool ok = i < n;
         key[it] = ok ? kin[i] : K(0);
         val[it] = ok ? (vin ? vin[i] : (uint32_t)i) : 0u;
-        unsigned d = ok ? digit_of(key[it], shift) : RADIX_BINS;    // RADIX_BINS = no key
-        unsigned peers = __match_any_sync(0xffffffffu, d);
+    }
+#pragma unroll
+    for (int it = 0; it < RADIX_ITEMS; ++it) {
+        const bool ok = base + it * 32 + lane < n;
+        const unsigned d = ok ? digit_of(key[it], shift) : RADIX_BINS;    // RADIX_BINS = no key
+        peers[it] = warp_peers8(d, ok);
+    }
+#pragma unroll
+    for (int it = 0; it < RADIX_ITEMS; ++it) {
+        const bool ok = base + it * 32 + lane < n;
+        const unsigned d = ok ? digit_of(key[it], shift) : RADIX_BINS;
         unsigned before = d < RADIX_BINS ? wcnt[w * RADIX_BINS + d] : 0u;
         __syncwarp();
-        if (d < RADIX_BINS && (peers & lt) == 0) wcnt[w * RADIX_BINS + d] = before + __popc(peers);
+        if (d < RADIX_BINS && (peers[it] & lt) == 0) wcnt[w * RADIX_BINS + d] = before + __popc(peers[it]);
         __syncwarp();
-        rank[it] = before + __popc(peers & lt);
+        rank[it] = before + __popc(peers[it] & lt);
     }
     __syncthreads();
     // per digit: exclusive prefix over warps, then over digits

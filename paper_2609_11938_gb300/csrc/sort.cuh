@@ -46,7 +46,7 @@ void radix_sort_pairs(Ctx &c, K *k0, uint32_t *v0, K *k1, uint32_t *v1, int64_t 
 // moving anything itself.  epi returns problem bits; epi.done(bits) runs in every
 // thread at the end (for warp votes).  Same tiles and ranking as the radix
 // sort: warps own consecutive 512-element runs, ranked 32 at a time with
-// __match_any_sync peer groups.
+// peer groups from one ballot per digit bit.
 template <typename DigitFn>
 __global__ void __launch_bounds__(RADIX_THREADS) k_digit_hist(DigitFn digit, int64_t n, uint32_t *__restrict__ hist,
                                                               int64_t ntiles) {
@@ -83,17 +83,22 @@ __global__ void __launch_bounds__(RADIX_THREADS) k_digit_rank(DigitFn digit, int
     unsigned dig[RADIX_ITEMS];
     uint32_t rank[RADIX_ITEMS];
     const unsigned lt = lanemask_lt();
+    unsigned peers[RADIX_ITEMS];
 #pragma unroll
-    for (int it = 0; it < RADIX_ITEMS; ++it) {
+    for (int it = 0; it < RADIX_ITEMS; ++it) {        // digits and peer groups first: independent
         const int64_t i = base + it * 32 + lane;
         const unsigned d = i < n ? digit(i) : (unsigned)RADIX_BINS;
-        const unsigned peers = __match_any_sync(0xffffffffu, d);
+        peers[it] = warp_peers8(d, d < RADIX_BINS);
+        dig[it] = d;
+    }
+#pragma unroll
+    for (int it = 0; it < RADIX_ITEMS; ++it) {
+        const unsigned d = dig[it];
         const unsigned before = d < RADIX_BINS ? wcnt[w * RADIX_BINS + d] : 0u;
         __syncwarp();
-        if (d < RADIX_BINS && (peers & lt) == 0) wcnt[w * RADIX_BINS + d] = before + __popc(peers);
+        if (d < RADIX_BINS && (peers[it] & lt) == 0) wcnt[w * RADIX_BINS + d] = before + __popc(peers[it]);
         __syncwarp();
-        rank[it] = before + __popc(peers & lt);
-        dig[it] = d;
+        rank[it] = before + __popc(peers[it] & lt);
     }
     __syncthreads();
     // RADIX_THREADS == RADIX_BINS: thread d turns digit d's per-warp counts

@@ -13,9 +13,15 @@ constexpr int CHK_THREADS = 256;
 constexpr int CHK_G = 8;
 __global__ void __launch_bounds__(CHK_THREADS) k_check_kernel_order(const uint8_t *__restrict__ stream,
                                                                     const int64_t *__restrict__ start, int64_t n,
-                                                                    int vec, DevStatus *st) {
+                                                                    int vec, DevStatus *st,
+                                                                    uint32_t *__restrict__ stream_hist) {
     __shared__ long long smin[CHK_THREADS / 32], smax[CHK_THREADS / 32];
     __shared__ int sbad[CHK_THREADS / 32];
+    __shared__ uint32_t sh[256];
+    if (stream_hist) {
+        for (int i = threadIdx.x; i < 256; i += CHK_THREADS) sh[i] = 0;
+        __syncthreads();
+    }
     long long mn = LLONG_MAX, mx = LLONG_MIN;
     int unsorted = 0;
     const int64_t ngroups = (n + CHK_G - 1) / CHK_G;
@@ -53,7 +59,13 @@ __global__ void __launch_bounds__(CHK_THREADS) k_check_kernel_order(const uint8_
             mn = t[u] < mn ? t[u] : mn;
             mx = t[u] > mx ? t[u] : mx;
             if (i0 + u + 1 < n) unsorted |= (t[u + 1] < t[u]) || (t[u + 1] == t[u] && s[u + 1] < s[u]);
+            if (stream_hist) atomicAdd(&sh[s[u]], 1u);
         }
+    }
+    if (stream_hist) {
+        __syncthreads();
+        for (int i = threadIdx.x; i < 256; i += CHK_THREADS)
+            if (sh[i]) atomicAdd(&stream_hist[i], sh[i]);
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
@@ -81,11 +93,11 @@ __global__ void __launch_bounds__(CHK_THREADS) k_check_kernel_order(const uint8_
     }
 }
 
-void check_kernel_order(Ctx &c, const uint8_t *stream, const int64_t *start, int64_t n) {
+void check_kernel_order(Ctx &c, const uint8_t *stream, const int64_t *start, int64_t n, uint32_t *stream_hist) {
     if (n <= 0) return;
     const int vec = ((reinterpret_cast<uintptr_t>(start) & 15) == 0) && ((reinterpret_cast<uintptr_t>(stream) & 7) == 0);
     launch(c, "check_kernel_order", k_check_kernel_order, dim3(grid_for(n, CHK_THREADS * 16, REDUCE_GRID)),
-           dim3(CHK_THREADS), 0, stream, start, n, vec, c.d_status);
+           dim3(CHK_THREADS), 0, stream, start, n, vec, c.d_status, stream_hist);
 }
 
 __global__ void k_time_keys(const uint8_t *__restrict__ stream, const int64_t *__restrict__ start, int64_t n,

@@ -6,8 +6,10 @@
 namespace opattr {
 
 // Sets F_K_UNSORTED unless (start_ns, stream) is non-decreasing along the
-// array, and records min / max start in MM_KSTART_MIN / MM_KSTART_MAX.
-void check_kernel_order(Ctx &c, const uint8_t *stream, const int64_t *start, int64_t n);
+// array, and records min / max start in MM_KSTART_MIN / MM_KSTART_MAX.  With
+// stream_hist (256 zeroed counters), also counts the kernels of each stream.
+void check_kernel_order(Ctx &c, const uint8_t *stream, const int64_t *start, int64_t n,
+                        uint32_t *stream_hist = nullptr);
 
 // Scratch (bytes) of kernel_time_order for n kernels.
 size_t kernel_order_scratch(int64_t n);

@@ -187,6 +187,11 @@ def test_error_statuses(opa):
     bad = rk.clone(); bad[0] = t.R
     with pytest.raises(opa.OpattrError):
         ctx.aggregate(tr, bad, idx)
+    att = int(np.nonzero(rk.cpu().numpy() >= 0)[0][0])   # an attributed kernel's row index past the rows
+    bad = idx.clone(); bad[att] = t.M
+    with pytest.raises(opa.OpattrError) as ei:
+        ctx.aggregate(tr, rk, bad)
+    assert ei.value.status == opa.E_INVALID_ARG
     u = tracegen.small_random(11, n_events=80, max_depth=4)
     u.counters = u.counters.copy(); u.counters[:, 4] = np.inf
     res = oracle.run(u)
