@@ -34,28 +34,44 @@ opattr_status cuda_status(Ctx &c, cudaError_t e) {
     return OPATTR_E_CUDA;
 }
 
-// Grows the arena to at least `bytes`.  OPATTR_FAULT=alloc in the environment
-// makes growth fail, to exercise the out-of-memory path without a GPU fault.
+// Grows the arena to at least `bytes` beyond its kept prefix (the first
+// arena_keep bytes, copied into a grown arena).  OPATTR_FAULT=alloc in the
+// environment makes growth fail, to exercise the out-of-memory path without
+// a GPU fault.
 opattr_status ensure_arena(Ctx &c, size_t bytes) {
+    bytes += c.arena_keep;
     if (bytes <= c.arena_cap) return OPATTR_OK;
     if (c.arena_fixed) return OPATTR_E_OOM;
     const char *fault = getenv("OPATTR_FAULT");
     if (fault && strcmp(fault, "alloc") == 0) return OPATTR_E_OOM;
-    if (c.arena) {
+    size_t cap = std::max(bytes, (size_t)1 << 20);
+    cap = (cap + ((size_t)1 << 20) - 1) & ~(((size_t)1 << 20) - 1);
+    if (c.arena && c.arena_keep == 0) {
+        // nothing to keep: free first, so the old and new arenas are never held together
         if (cudaStreamSynchronize(c.stream) != cudaSuccess) return cuda_status(c, cudaGetLastError());
         cudaFree(c.arena);
         c.arena = nullptr;
         c.arena_cap = 0;
     }
-    size_t cap = std::max(bytes, (size_t)1 << 20);
-    cap = (cap + ((size_t)1 << 20) - 1) & ~(((size_t)1 << 20) - 1);
-    cudaError_t e = cudaMalloc(&c.arena, cap);
+    char *fresh = nullptr;
+    cudaError_t e = cudaMalloc(&fresh, cap);
     if (e == cudaErrorMemoryAllocation) {
         cudaGetLastError();          // clear the sticky-free error state
-        c.arena = nullptr;
         return OPATTR_E_OOM;
     }
     if (e != cudaSuccess) return cuda_status(c, e);
+    if (c.arena) {
+        // the kept prefix moves with the arena
+        e = cudaMemcpyAsync(fresh, c.arena, c.arena_keep, cudaMemcpyDeviceToDevice, c.stream);
+        if (e == cudaSuccess) e = cudaStreamSynchronize(c.stream);
+        if (e != cudaSuccess) {
+            cudaFree(fresh);
+            return cuda_status(c, e);
+        }
+        if (c.join_korder) c.join_korder = reinterpret_cast<uint32_t *>(fresh + (reinterpret_cast<char *>(c.join_korder) - c.arena));
+        cudaFree(c.arena);
+    }
+    c.arena = fresh;
     c.arena_cap = cap;
     return OPATTR_OK;
 }
@@ -238,11 +254,25 @@ opattr_status opattr_join(opattr_ctx *ctx, const opattr_kernels *kernels, const 
     DeviceGuard g(c.device);
     if (!g.ok) return OPATTR_E_CUDA;
     c.enclose_k_sorted = -1;
+    // the enclosure's kernel time order is kept for the matching (arena_keep);
+    // every way out of the join drops it
+    struct JoinScope {
+        Ctx &c;
+        explicit JoinScope(Ctx &ctx) : c(ctx) { c.in_join = true; }
+        ~JoinScope() {
+            c.in_join = false;
+            c.order_from_enclose = false;
+            c.join_korder = nullptr;
+            c.arena_keep = 0;
+        }
+    } scope(c);
     opattr_status st = finish(c, do_enclose(c, kernels, ranges, range_of_kernel, n_op_enclosing));
     if (st < 0) return st;
     c.order_from_enclose = true;
     const opattr_status sm = finish(c, do_match(c, kernels, ncu, dedup, ncu_idx_of_kernel, match_kind, host_summary));
     c.order_from_enclose = false;
+    c.join_korder = nullptr;             // the aggregation needs no time order
+    c.arena_keep = 0;
     if (sm < 0) return sm;
     st = finish(c, do_aggregate(c, kernels, ranges, range_of_kernel, ncu, ncu_idx_of_kernel, n_ops, dev_out,
                                 host_totals));

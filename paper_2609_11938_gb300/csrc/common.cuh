@@ -94,6 +94,12 @@ struct Ctx {
     // and whether the matching may take it instead of checking again (join)
     int enclose_k_sorted = -1;
     bool order_from_enclose = false;
+    // within a join: the enclosure's kernel time order (unsorted kernels), kept
+    // for the matching at the start of the arena (arena_keep bytes survive the
+    // per-call resets and any growth of the arena)
+    bool in_join = false;
+    uint32_t *join_korder = nullptr;
+    size_t arena_keep = 0;
     // launch accounting
     int64_t launches = 0;
     bool timing = false;
@@ -107,7 +113,7 @@ struct Ctx {
 // ------------------------------------------------------------------ scratch
 struct Arena {
     Ctx &c;
-    explicit Arena(Ctx &ctx) : c(ctx) { c.arena_used = 0; }
+    explicit Arena(Ctx &ctx) : c(ctx) { c.arena_used = c.arena_keep; }
     template <typename T>
     T *take(int64_t count) {
         size_t bytes = (size_t)(count > 0 ? count : 1) * sizeof(T);

@@ -308,12 +308,14 @@ constexpr int EN_TILE = EN_THREADS * EN_PER;      // kernels of one stream per t
 constexpr int EN_WIN = 3072;                      // staged range entries per tile
 constexpr int EN_RD = 8;                          // depths whose sweep state stays in registers
 
-// The stream of the kernel at time position i, and its place in psk.
+// The stream of the kernel at time position i (as its compact id: streams
+// with kernels numbered in order), and its place in psk.
 struct TimeStreamDigit {
     const uint8_t *stream;
     const uint32_t *korder;     // time order, NULL = array order
+    const uint8_t *scmap;       // [256] compact id of a stream with kernels
     __device__ __forceinline__ unsigned operator()(int64_t i) const {
-        return stream[korder ? korder[i] : (uint32_t)i];
+        return scmap[stream[korder ? korder[i] : (uint32_t)i]];
     }
 };
 struct PlaceByStream {
@@ -617,10 +619,13 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     nd.add<int64_t>(R).add<int64_t>(R).add<uint32_t>(R);
     nd.add<unsigned char>(STAGE_BYTES);
     nd.add<uint32_t>(K).add<uint32_t>(nt_max).add<int2>(nt_max * 32);
+    const bool keep_order = c.in_join && K > 0;       // a join keeps the time order for its matching
+    if (keep_order) nd.add<uint32_t>(K);
     size_t need = nd.bytes + kernel_order_scratch(K) + 4096;
     opattr_status st = ensure_arena(c, need);
     if (st) return st;
     Arena a(c);
+    uint32_t *kept_order = keep_order ? a.take<uint32_t>(K) : nullptr;     // first: the start of the arena
     if ((st = reset_status(c))) return st;
 
     // level histogram [LEVELS] and kernels per stream [256], zeroed together
@@ -666,7 +671,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     // [256], [257])
     constexpr size_t ST_LOC = 0, ST_CBASE = ST_LOC + 2 * LEVELS, ST_NDEP = ST_CBASE + 2 * 256,
                      ST_CMAP = ST_NDEP + 256, ST_KOFF = ST_CMAP + LEVELS, ST_KCNT = ST_KOFF + 4 * 256,
-                     ST_TOFF = ST_KCNT + 4 * 256, ST_END = ST_TOFF + 4 * 257;
+                     ST_TOFF = ST_KCNT + 4 * 256, ST_SCMAP = ST_TOFF + 4 * 257, ST_END = ST_SCMAP + 256;
     static_assert(ST_END <= STAGE_BYTES, "staging too small");
     const uint32_t *off = c.h_levels;
     const uint32_t *kcnt_h = c.h_levels + LEVELS + 1;
@@ -677,6 +682,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     uint32_t *koff_h = reinterpret_cast<uint32_t *>(c.h_stage + ST_KOFF);
     uint32_t *kcnt_s = reinterpret_cast<uint32_t *>(c.h_stage + ST_KCNT);
     uint32_t *toff_h = reinterpret_cast<uint32_t *>(c.h_stage + ST_TOFF);
+    uint8_t *scmap = c.h_stage + ST_SCMAP;
     int nl = 0;
     for (int s = 0; s < 256; ++s) {
         cbase[s] = (uint16_t)nl;
@@ -690,7 +696,10 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     memset(cmap, 0, LEVELS);
     for (int l = 0; l < nl && l < 256; ++l) cmap[level_of_compact[l]] = (uint8_t)l;
     uint32_t kacc = 0, tacc = 0;
+    int nks = 0;                                  // streams with kernels
     for (int s = 0; s < 256; ++s) {
+        scmap[s] = (uint8_t)nks;
+        nks += kcnt_h[s] > 0;
         koff_h[s] = kacc;
         kcnt_s[s] = kcnt_h[s];
         toff_h[s] = tacc;
@@ -715,6 +724,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     const uint32_t *d_koff = reinterpret_cast<const uint32_t *>(d_stage + ST_KOFF);
     const uint32_t *d_kcnt = reinterpret_cast<const uint32_t *>(d_stage + ST_KCNT);
     const uint32_t *d_toff = reinterpret_cast<const uint32_t *>(d_stage + ST_TOFF);
+    const uint8_t *d_scmap = d_stage + ST_SCMAP;
     cudaMemcpyAsync(d_stage, c.h_stage, ST_END, cudaMemcpyHostToDevice, c.stream);
 
     // ---- kernel time order, then the kernels partitioned by stream
@@ -722,10 +732,15 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     if (!k_sorted && K > 0) {
         korder = kernel_time_order(c, a, kern->stream, kern->start_ns, K);
         if (!korder) return OPATTR_E_OOM;
+        if (kept_order) {
+            cudaMemcpyAsync(kept_order, korder, sizeof(uint32_t) * K, cudaMemcpyDeviceToDevice, c.stream);
+            c.join_korder = kept_order;
+            c.arena_keep = (sizeof(uint32_t) * (size_t)K + 255) & ~(size_t)255;
+        }
     }
     if (K > 0 && nl > 0) {
-        const TimeStreamDigit dg{kern->stream, korder};
-        digit_offsets(c, dg, K, hist, part);
+        const TimeStreamDigit dg{kern->stream, korder, d_scmap};
+        digit_offsets(c, dg, K, hist, part, nks);
         digit_rank(c, "stream_place", dg, K, hist, PlaceByStream{korder, psk});
         launch(c, "tile_order", k_tile_order, dim3(grid_for(NT, 256, 4096)), dim3(256), 0, d_toff, NT, tinfo);
     }
@@ -757,7 +772,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
         if (nl <= 256) {
             // stable partition by compact level id, ranges written in place
             const LevelDigit dg{rng->stream, rng->depth, d_cmap, perm};
-            digit_offsets(c, dg, R, hist, part);
+            digit_offsets(c, dg, R, hist, part, nl);
             const int64_t ntiles = (R + RADIX_TILE - 1) / RADIX_TILE;
             launch(c, "level_place", k_level_place, dim3((unsigned)ntiles), dim3(RADIX_THREADS), 0, dg,
                    rng->start_ns, rng->end_ns, rng->op_id, R, (const uint32_t *)hist, ntiles, ls, le, li);

@@ -438,9 +438,11 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     }
 
     const unsigned gK = grid_for(K, 256, REDUCE_GRID);
-    // within a join the enclosure has just verified these records' order
+    // within a join the enclosure has just verified these records' order, and
+    // kept their time order when they were out of it
     const bool known_sorted = c.order_from_enclose && c.enclose_k_sorted == 1;
-    if (!known_sorted) check_kernel_order(c, kern->stream, kern->start_ns, K);
+    const bool known_unsorted = c.order_from_enclose && c.enclose_k_sorted == 0 && c.join_korder;
+    if (!known_sorted && !known_unsorted) check_kernel_order(c, kern->stream, kern->start_ns, K);
     if (dedup_on && K > 0)
         launch(c, "check_layers", k_check_layers, dim3(gK), dim3(256), 0, kern->layer_id, K, dd->n_layers,
                (const int32_t *)d_rep, c.d_status);
@@ -449,8 +451,8 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
                kern->name_id, K, c.d_status);
     // Speculative fast paths, taking the kernel array to be in time order
     // (confirmed or refuted by the order check in the same batch).
-    const bool try_identity = !dedup_on && !per_stream && K == M && K > 0;
-    const bool try_streams = !dedup_on && per_stream && K == M && K > 0;
+    const bool try_identity = !dedup_on && !per_stream && K == M && K > 0 && !known_unsorted;
+    const bool try_streams = !dedup_on && per_stream && K == M && K > 0 && !known_unsorted;
     if (try_identity)
         launch(c, "match_identity", k_match_identity, dim3(grid_for(K, 256 * 16, REDUCE_GRID)), dim3(256), 0,
                kname, nname, K, out_idx, out_kind, identity_vec(kname, nname, out_idx, out_kind), c.d_status);
@@ -459,7 +461,7 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
                      out_kind);
     if ((st = read_status(c))) return st;
     if (c.h_status->err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
-    const bool k_sorted = known_sorted || !(c.h_status->flags & F_K_UNSORTED);
+    const bool k_sorted = known_sorted || (!known_unsorted && !(c.h_status->flags & F_K_UNSORTED));
     opattr_match_summary S{};
     S.kernels = K;
     S.replayed = dedup_on ? (int64_t)c.h_status->cnt[C_REPLAYED] : K;
@@ -476,7 +478,7 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     if (K > 0) launch(c, "fill_match", k_fill_match, dim3(gK), dim3(256), 0, out_idx, out_kind, K);
     uint32_t *korder = nullptr;
     if (!k_sorted && K > 0) {
-        korder = kernel_time_order(c, a, kern->stream, kern->start_ns, K);
+        korder = known_unsorted ? c.join_korder : kernel_time_order(c, a, kern->stream, kern->start_ns, K);
         if (!korder) return OPATTR_E_OOM;
     }
     // rk[j] = kernel index of the j-th replayed kernel in time order
@@ -493,8 +495,10 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
         else launch(c, "iota", k_iota, dim3(gK), dim3(256), 0, rk, K);
     }
     bool direct_done = false;
+    // rows equal to the replayed kernels in time order, tried before the name
+    // sorts: with layer deduplication, or when the kernels were out of time order
     const bool retry_streams = per_stream && (dedup_on || korder) && nrep == M && nrep > 0;
-    if ((dedup_on && !per_stream && nrep == M && nrep > 0) || retry_streams) {
+    if (((dedup_on || korder) && !per_stream && nrep == M && nrep > 0) || retry_streams) {
         if (retry_streams)
             stream_pairs(c, kern, ncu, rk, nrep, reinterpret_cast<uint8_t *>(n2), n0, n1, hist, part, out_idx,
                          out_kind);

@@ -124,13 +124,15 @@ __global__ void __launch_bounds__(RADIX_THREADS) k_digit_rank(DigitFn digit, int
     epi.done(bits);
 }
 
+// nbins: digits used (every digit below it); only those rows of the matrix
+// are scanned.
 template <typename DigitFn>
-void digit_offsets(Ctx &c, DigitFn digit, int64_t n, uint32_t *hist, uint32_t *partials) {
+void digit_offsets(Ctx &c, DigitFn digit, int64_t n, uint32_t *hist, uint32_t *partials, int nbins = RADIX_BINS) {
     if (n <= 0) return;
     const int64_t ntiles = (n + RADIX_TILE - 1) / RADIX_TILE;
     launch(c, "digit_hist", k_digit_hist<DigitFn>, dim3((unsigned)ntiles), dim3(RADIX_THREADS), 0, digit, n, hist,
            ntiles);
-    scan_exclusive_u32(c, hist, hist, ntiles * RADIX_BINS, partials, nullptr);
+    scan_exclusive_u32(c, hist, hist, ntiles * (int64_t)(nbins < 1 ? 1 : nbins), partials, nullptr);
 }
 
 template <typename DigitFn, typename Epi>

@@ -93,8 +93,9 @@ def test_configs(opa, name, shuffle):
     o = oracle.run(t, enclose_mode="brute" if name in ("tiny", "gpt2") else "indexed")
     assert_parity(g, o)
     assert g["match_status"] == opa.OK and g["summary"]["unmatched"] == 0
-    if not shuffle:
-        assert g["summary"]["fast_path"] == 1
+    # rows follow the replayed launches in time order, shuffled kernel arrays
+    # or not: one pass pairs them, through the time order when it is needed
+    assert g["summary"]["fast_path"] == 1
 
 
 @pytest.mark.parametrize("mode", ["skip_name", "prefix", "error"])
