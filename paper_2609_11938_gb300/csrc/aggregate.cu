@@ -36,7 +36,8 @@ struct AggIn {
     const float *counters;
     int64_t M;                  // ncu rows: a row index at or past M is never read (the count pass reports it)
     int64_t n_ops;
-    unsigned *ctr;              // next chunk of the ops pass, zeroed before it
+    unsigned *ctr;              // [0] next chunk of the ops pass, [1] ops listed in dirty; zeroed before it
+    uint32_t *dirty;            // ops whose fast sums saw a null or infinite value
     const unsigned *nonident;   // nonzero unless ncu_idx[k] == k for every kernel (set by the count pass)
     opattr_op_aggregates out;
 };
@@ -584,11 +585,10 @@ __device__ __forceinline__ void cp_async_wait() {
 }
 
 __global__ void __launch_bounds__(AG_THREADS, 5) k_agg_ops(const uint32_t *__restrict__ off, uint32_t *list,
-                                                          AggIn A, DevStatus *st) {
+                                                          AggIn A) {
     extern __shared__ __align__(16) unsigned char ag_smem[];
     OpsWarp &W = reinterpret_cast<OpsWarp *>(ag_smem)[threadIdx.x / 32];
     const unsigned lane = lane_id();
-    int bad = 0;
     const bool ident = *A.nonident == 0;
     const float4 *rows = reinterpret_cast<const float4 *>(A.counters);
     // row index of kernel k, -1 for none (or for an index past the rows)
@@ -713,15 +713,32 @@ __global__ void __launch_bounds__(AG_THREADS, 5) k_agg_ops(const uint32_t *__res
                 }
                 cp_async_wait<0>();
             }
+            // a null or infinite value poisons a sum: the op is listed for
+            // k_agg_careful
             if (acc.clean()) acc.write(A, o, (int)len);
-            else bad |= op_careful(seg, len, A, o);
+            else A.dirty[atomicAdd(A.ctr + 1, 1u)] = (uint32_t)o;
         }
         __syncwarp();
         o0 = o1;
 #pragma unroll
         for (int q = 0; q < PER; ++q) { oa[q] = na[q]; ob[q] = nb[q]; }
     }
-    if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_err(st, ERR_INVALID);
+}
+
+// The ops k_agg_ops listed as dirty: one thread each puts the segment in
+// ascending kernel index (in place) and redoes it with Acc, which leaves
+// nulls out and reports infinite values.  A separate pass keeps that rare,
+// register-hungry path out of the ops pass.
+__global__ void k_agg_careful(const uint32_t *__restrict__ off, uint32_t *list, AggIn A, DevStatus *st) {
+    int bad = 0;
+    const unsigned n = A.ctr[1];
+    for (unsigned e = blockIdx.x * blockDim.x + threadIdx.x; e < n; e += gridDim.x * blockDim.x) {
+        const uint32_t o = A.dirty[e];
+        const uint32_t s0 = off[o], len = off[o + 1] - s0;
+        sort_segment(list + s0, len);
+        bad |= op_careful(list + s0, len, A, o);
+    }
+    if (bad) set_err(st, ERR_INVALID);
 }
 
 // ------------------------------------------------------------------ host
@@ -1002,7 +1019,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
 
     Need nd;
     nd.add<uint32_t>(O + 1).add<uint32_t>(O + 1).add<uint32_t>(K).add<uint32_t>(K);
-    nd.add<uint32_t>(O + 1).add<unsigned>(1).add<unsigned>(1).add<unsigned>(1);
+    nd.add<uint32_t>(O + 1).add<unsigned>(1).add<unsigned>(2).add<unsigned>(1).add<uint32_t>(O + 1);
     nd.add<uint32_t>(O + 1).add<Acc>(K / AG_PIECE + (K / (AG_SHORT_MAX + 1)) + 1);   // pieces per op, partials
     nd.add<uint32_t>(scan_scratch_elems(std::max<int64_t>(O + 1, radix_hist_elems(K))));
     nd.add<uint32_t>(O + 1).add<uint32_t>(radix_hist_elems(K)).add<uint32_t>(8);   // huge-op index, histogram, info
@@ -1016,17 +1033,18 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     // placed, then serves the segment sorts
     uint32_t *list = a.take<uint32_t>(K), *tmp = a.take<uint32_t>(K), *longs = a.take<uint32_t>(O + 1);
     unsigned *nlong = a.take<unsigned>(1);
-    unsigned *ctr = a.take<unsigned>(1);
+    unsigned *ctr = a.take<unsigned>(2);
     unsigned *nonident = a.take<unsigned>(1);
+    uint32_t *dirty = a.take<uint32_t>(O + 1);
     uint32_t *npc = a.take<uint32_t>(O + 1);
     Acc *partials = a.take<Acc>(K / AG_PIECE + (K / (AG_SHORT_MAX + 1)) + 1);
     if (!npc || !partials) return OPATTR_E_OOM;
-    cudaMemsetAsync(ctr, 0, sizeof(unsigned), c.stream);
+    cudaMemsetAsync(ctr, 0, 2 * sizeof(unsigned), c.stream);
     uint32_t *part = a.take<uint32_t>(scan_scratch_elems(std::max<int64_t>(O + 1, radix_hist_elems(K))));
     uint32_t *hidx = a.take<uint32_t>(O + 1), *hhist = a.take<uint32_t>(radix_hist_elems(K));
     uint32_t *info = a.take<uint32_t>(8), *hop = a.take<uint32_t>(O + 1);
     if (!hidx || !hhist || !info || !hop) return OPATTR_E_OOM;
-    if (!cnt || !off || !list || !tmp || !longs || !nlong || !part || !nonident) return OPATTR_E_OOM;
+    if (!cnt || !off || !list || !tmp || !longs || !nlong || !part || !nonident || !dirty) return OPATTR_E_OOM;
     cudaMemsetAsync(cnt, 0, sizeof(uint32_t) * (O + 1), c.stream);
     cudaMemsetAsync(nlong, 0, sizeof(unsigned), c.stream);
     cudaMemsetAsync(nonident, 0, sizeof(unsigned), c.stream);
@@ -1047,6 +1065,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     in.M = M;
     in.n_ops = O;
     in.ctr = ctr;
+    in.dirty = dirty;
     in.nonident = nonident;
     in.out = *out;
     if (O > 0) {
@@ -1074,7 +1093,9 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
             attr_done |= 1u << c.device;
         }
         launch(c, "agg_ops", k_agg_ops, dim3(ops_grid(c, O)), dim3(AG_THREADS), AG_SMEM,
-               (const uint32_t *)off, list, in, c.d_status);
+               (const uint32_t *)off, list, in);
+        launch(c, "agg_careful", k_agg_careful, dim3(std::max(1, sms)), dim3(128), 0, (const uint32_t *)off, list, in,
+               c.d_status);
         if (cudaEventSynchronize(c.ev_aux) != cudaSuccess) return cuda_status(c, cudaGetLastError());
         const uint32_t pieces = c.h_levels[1], longest = c.h_levels[2], n_huge = c.h_levels[4];
         if (pieces > 0) {
@@ -1235,6 +1256,7 @@ opattr_status do_rollup(Ctx &c, const opattr_kernels *kern, const opattr_ranges 
         in.M = M;
         in.n_ops = C;
         in.ctr = nullptr;
+        in.dirty = nullptr;
         in.nonident = nullptr;
         in.out = *out;
         int sms = 0;

@@ -87,6 +87,8 @@ opattr_status read_status(Ctx &c) {
     if (e == cudaSuccess) e = cudaStreamSynchronize(c.stream);
     if (e != cudaSuccess) return cuda_status(c, e);
     if (c.timing) timing_collect(c);
+    // a chained prefix that gave up waiting leaves results that do not count
+    if (c.h_status->err & ERR_TIMEOUT) return OPATTR_E_TIMEOUT;
     return OPATTR_OK;
 }
 

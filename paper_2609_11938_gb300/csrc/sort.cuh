@@ -14,8 +14,9 @@ constexpr int RADIX_TILE = RADIX_THREADS * RADIX_ITEMS;  // 4096 keys per block
 constexpr int RADIX_BITS = 8;
 constexpr int RADIX_BINS = 1 << RADIX_BITS;
 
-// Scratch for a scan of n elements: partial sums of the tiles (+1 for the total).
-inline int64_t scan_scratch_elems(int64_t n) { return (n + SCAN_TILE - 1) / SCAN_TILE + 1; }
+// Scratch for a scan of n elements (u32 units): one 64-bit status word per
+// tile of the single-pass scan and the tile counter.
+inline int64_t scan_scratch_elems(int64_t n) { return 2 * ((n + SCAN_TILE - 1) / SCAN_TILE) + 4; }
 
 // out[i] = in[0] + ... + in[i-1]; *total_dev (device, may be NULL) = sum of all.
 // in and out may alias.  `partials` holds scan_scratch_elems(n) u32.
@@ -35,6 +36,57 @@ inline int64_t radix_hist_elems(int64_t n) {
 template <typename K>
 void radix_sort_pairs(Ctx &c, K *k0, uint32_t *v0, K *k1, uint32_t *v1, int64_t n, int bits, bool iota,
                       uint32_t *hist, uint32_t *partials, K **kout, uint32_t **vout);
+
+// ------------------------------------------------------------------ chained prefixes
+// Prefix sums across tiles in one pass (decoupled look-back): tile t
+// publishes its own total, then the sum over every tile before it, in one
+// 64-bit word (LB_INC: the low 32 bits are that inclusive prefix; LB_AGG:
+// they are only the tile's own total; 0: nothing yet).  One warp of tile t
+// reads the words of the 32 tiles before a point at once, adds the totals up
+// to the nearest tile whose prefix is known, and moves 32 tiles further back
+// only when none of the 32 has one.  Tiles take their index in the order
+// their blocks start (from a counter), so every tile waited on has started,
+// and it publishes its total without waiting on any other tile.  The wait is
+// bounded all the same: after LB_SPIN_LIMIT polls the tile sets ERR_TIMEOUT
+// and goes on with the part of its prefix it has, which is no larger than the
+// true one (so positions derived from it stay in bounds).  Status words and
+// the counter start at zero (one memset per pass).
+constexpr unsigned long long LB_AGG = 1ull << 62, LB_INC = 1ull << 63;
+constexpr int LB_SPIN_LIMIT = 1 << 20;
+
+// Called by all 32 lanes of one warp with the same arguments; returns the
+// sum of `total` over the tiles before t (in every lane).
+__device__ __forceinline__ uint32_t warp_lookback_exclusive(unsigned long long *status, int64_t t, uint32_t total,
+                                                            DevStatus *st) {
+    const unsigned lane = lane_id();
+    volatile unsigned long long *word = status;
+    if (lane == 0) word[t] = (t == 0 ? LB_INC : LB_AGG) | total;
+    if (t == 0) return 0;
+    uint32_t excl = 0;
+    int64_t j = t - 1;                       // lane i reads tile j - i
+    int spins = 0;
+    for (;;) {
+        const int64_t q = j - (int64_t)lane;
+        const unsigned long long v = q >= 0 ? (unsigned long long)word[q] : 0ull + LB_INC;   // before tile 0: an empty known prefix
+        const unsigned inc = __ballot_sync(0xffffffffu, (v & LB_INC) != 0);
+        const unsigned none = __ballot_sync(0xffffffffu, (v & (LB_INC | LB_AGG)) == 0);
+        const int first = inc ? __ffs(inc) - 1 : 32;               // nearest tile with a known prefix
+        const unsigned upto = first == 32 ? 0xffffffffu : (2u << first) - 1u;
+        if (none & upto) {                   // a tile on the way has published nothing yet
+            if (++spins > LB_SPIN_LIMIT) {
+                if (lane == 0) set_err(st, ERR_TIMEOUT);
+                break;
+            }
+            __nanosleep(64);
+            continue;
+        }
+        excl += warp_sum<uint32_t>(((upto >> lane) & 1u) ? (uint32_t)v : 0u);
+        if (first < 32) break;
+        j -= 32;
+    }
+    if (lane == 0) word[t] = LB_INC | (uint32_t)(excl + total);
+    return excl;
+}
 
 // ------------------------------------------------------------------ digit passes
 // One stable counting pass whose 8-bit digit comes from a functor:
