@@ -144,8 +144,12 @@ typedef struct {
     opattr_mismatch_mode mismatch; /* default OPATTR_MISMATCH_SKIP_NAME */
     int32_t dedup;                 /* 1: apply opattr_dedup when given (default 1) */
     int32_t checked;               /* reserved, 0 */
-    int64_t spin_limit;            /* bound on device-side waits (0 = default); the current
-                                      kernels have none, so it is checked (>= 0) and unused */
+    int64_t spin_limit;            /* polls a device-side wait makes before it gives up (0 =
+                                      default, 2^20; must be >= 0).  The only waits are those of
+                                      the single-pass scans (a tile waiting for an earlier tile's
+                                      prefix); one that gives up sums the earlier tiles' input
+                                      itself, so results stay exact, and the call returns
+                                      OPATTR_E_TIMEOUT */
 } opattr_config;
 
 /* Host-side result of opattr_match. */

@@ -323,7 +323,7 @@ __device__ __forceinline__ int32_t range_of_t(const int32_t *rok, const uint32_t
 // kernels (a multiple of 32, up to AF_RUN) 32 at a time in index order, so an
 // op whose kernels all lie in one run gets ascending slots; the ops pass
 // sorts the few segments that do not.
-constexpr int AF_RUN = 2048;
+constexpr int AF_RUN = 4096;
 
 template <bool DIRECT>
 __global__ void __launch_bounds__(256, 5) k_agg_count(const int64_t *__restrict__ dur, const int32_t *__restrict__ rok,
@@ -1051,8 +1051,8 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     int sms = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
     // runs long enough to keep most segments in one warp, short enough that
-    // small traces still spread over the GPU (64 warps per SM)
-    const int64_t warps = (int64_t)std::max(1, sms) * 64;
+    // the grid is one wave of resident warps (five blocks of eight per SM)
+    const int64_t warps = (int64_t)std::max(1, sms) * 40;
     const int64_t run = std::min<int64_t>(AF_RUN, std::max<int64_t>(32, ((K + warps - 1) / warps + 31) / 32 * 32));
     if (K > 0)
         launch(c, "agg_count", rok ? k_agg_count<false> : k_agg_count<true>,

@@ -1,11 +1,23 @@
 // api.cu -- the C ABI of libopattr: context life cycle, scratch arena, status
 // block, launch timing, and the calls of the join.
+#include <nvtx3/nvToolsExt.h>
 #include <stdlib.h>
 
 #include <algorithm>
 #include <new>
 
 #include "common.cuh"
+
+// One NVTX range per call of the C ABI, named after the entry point, so a
+// timeline (Nsight Systems) shows the library's calls around their kernels.
+// Header-only NVTX: without a tool attached a push or pop costs a few
+// nanoseconds.
+struct NvtxCall {
+    explicit NvtxCall(const char *name) { nvtxRangePushA(name); }
+    ~NvtxCall() { nvtxRangePop(); }
+    NvtxCall(const NvtxCall &) = delete;
+    NvtxCall &operator=(const NvtxCall &) = delete;
+};
 
 namespace opattr {
 
@@ -213,6 +225,7 @@ static opattr_status finish(Ctx &c, opattr_status st) {
 
 opattr_status opattr_enclose(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,
                              int32_t *range_of_kernel, uint8_t *n_op_enclosing) {
+    NvtxCall nvtx("opattr_enclose");
     if (!ctx || !kernels || !ranges) return OPATTR_E_INVALID_ARG;
     Ctx &c = ctx->c;
     if (c.broken) return OPATTR_E_STATE;
@@ -224,6 +237,7 @@ opattr_status opattr_enclose(opattr_ctx *ctx, const opattr_kernels *kernels, con
 opattr_status opattr_match(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ncu *ncu,
                            const opattr_dedup *dedup, int32_t *ncu_idx_of_kernel, uint8_t *match_kind,
                            opattr_match_summary *host_summary) {
+    NvtxCall nvtx("opattr_match");
     if (!ctx || !kernels || !ncu) return OPATTR_E_INVALID_ARG;
     Ctx &c = ctx->c;
     if (c.broken) return OPATTR_E_STATE;
@@ -236,6 +250,7 @@ opattr_status opattr_aggregate(opattr_ctx *ctx, const opattr_kernels *kernels, c
                                const int32_t *range_of_kernel, const opattr_ncu *ncu,
                                const int32_t *ncu_idx_of_kernel, uint32_t n_ops,
                                const opattr_op_aggregates *dev_out, opattr_totals *host_totals) {
+    NvtxCall nvtx("opattr_aggregate");
     if (!ctx || !kernels || !ranges || !ncu) return OPATTR_E_INVALID_ARG;
     Ctx &c = ctx->c;
     if (c.broken) return OPATTR_E_STATE;
@@ -250,6 +265,7 @@ opattr_status opattr_join(opattr_ctx *ctx, const opattr_kernels *kernels, const 
                           int32_t *range_of_kernel, uint8_t *n_op_enclosing, int32_t *ncu_idx_of_kernel,
                           uint8_t *match_kind, const opattr_op_aggregates *dev_out,
                           opattr_match_summary *host_summary, opattr_totals *host_totals) {
+    NvtxCall nvtx("opattr_join");
     if (!ctx || !kernels || !ranges || !ncu) return OPATTR_E_INVALID_ARG;
     Ctx &c = ctx->c;
     if (c.broken) return OPATTR_E_STATE;
@@ -286,6 +302,7 @@ opattr_status opattr_attribute(opattr_ctx *ctx, const opattr_kernels *kernels, c
                                const int32_t *range_of_kernel, const uint8_t *n_op_enclosing, const opattr_corr *corr,
                                const opattr_fusion *fusion, uint32_t n_ops, uint32_t *op_of_kernel, uint8_t *tier,
                                uint32_t *fused_with, uint8_t *is_fused, opattr_attr_summary *host_summary) {
+    NvtxCall nvtx("opattr_attribute");
     if (!ctx || !kernels || !ranges) return OPATTR_E_INVALID_ARG;
     Ctx &c = ctx->c;
     if (c.broken) return OPATTR_E_STATE;
@@ -299,6 +316,7 @@ opattr_status opattr_rollup(opattr_ctx *ctx, const opattr_kernels *kernels, cons
                             const int32_t *range_of_kernel, const opattr_ncu *ncu, const int32_t *ncu_idx_of_kernel,
                             uint32_t n_ops, const uint32_t *class_of_op, uint32_t n_classes,
                             const opattr_op_aggregates *dev_out) {
+    NvtxCall nvtx("opattr_rollup");
     if (!ctx || !kernels || !ranges || !ncu) return OPATTR_E_INVALID_ARG;
     Ctx &c = ctx->c;
     if (c.broken) return OPATTR_E_STATE;

@@ -303,7 +303,7 @@ __global__ void k_validate_levels(const uint8_t *__restrict__ stream, const uint
 // and their gathers of start times and scattered result writes share sectors
 // in L2.
 constexpr int EN_THREADS = 128;
-constexpr int EN_PER = 32;                        // consecutive kernels one thread sweeps
+constexpr int EN_PER = 16;                        // consecutive kernels one thread sweeps
 constexpr int EN_TILE = EN_THREADS * EN_PER;      // kernels of one stream per tile
 constexpr int EN_WIN = 3072;                      // staged range entries per tile
 constexpr int EN_RD = 8;                          // depths whose sweep state stays in registers
@@ -740,8 +740,8 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     }
     if (K > 0 && nl > 0) {
         const TimeStreamDigit dg{kern->stream, korder, d_scmap};
-        digit_offsets(c, dg, K, hist, part, nks);
-        digit_rank(c, "stream_place", dg, K, hist, PlaceByStream{korder, psk});
+        const uint32_t *offs = digit_offsets(c, dg, K, hist, part, nks);
+        digit_rank(c, "stream_place", dg, K, offs, PlaceByStream{korder, psk});
         launch(c, "tile_order", k_tile_order, dim3(grid_for(NT, 256, 4096)), dim3(256), 0, d_toff, NT, tinfo);
     }
 
@@ -772,10 +772,10 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
         if (nl <= 256) {
             // stable partition by compact level id, ranges written in place
             const LevelDigit dg{rng->stream, rng->depth, d_cmap, perm};
-            digit_offsets(c, dg, R, hist, part, nl);
+            const uint32_t *offs = digit_offsets(c, dg, R, hist, part, nl);
             const int64_t ntiles = (R + RADIX_TILE - 1) / RADIX_TILE;
             launch(c, "level_place", k_level_place, dim3((unsigned)ntiles), dim3(RADIX_THREADS), 0, dg,
-                   rng->start_ns, rng->end_ns, rng->op_id, R, (const uint32_t *)hist, ntiles, ls, le, li);
+                   rng->start_ns, rng->end_ns, rng->op_id, R, offs, ntiles, ls, le, li);
         } else {
             // stable partition by level key (13 bits)
             uint32_t *lk0 = reinterpret_cast<uint32_t *>(rk0), *lk1 = reinterpret_cast<uint32_t *>(rk1);

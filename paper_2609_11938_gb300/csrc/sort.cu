@@ -1,24 +1,95 @@
 // sort.cu -- device-wide exclusive scan and a stable LSD radix sort with
 // warp-level digit ranking.
 //
-// The scan is one pass: tiles chain their prefixes by decoupled look-back
-// (lookback_exclusive in sort.cuh, a bounded wait on tiles that started
-// earlier).  A radix sort pass is three launches (tile histograms -> scan of
-// the histogram matrix -> scatter).
+// A scan out of place is one pass: tiles chain their prefixes by decoupled
+// look-back (warp_lookback_exclusive in sort.cuh, a bounded wait on tiles
+// that started earlier); a scan in place is three launches with no waits.  A
+// radix sort pass is three launches (tile histograms -> scan of the histogram
+// matrix -> scatter).
+#include <cstdlib>
+#include <cstring>
+
 #include "sort.cuh"
 
 namespace opattr {
+
+// ------------------------------------------------------------------ scan, in place
+// Three launches (tile sums, their scan, the tiles), no block waits on another:
+// the scan of a buffer onto itself, where the single pass below could not
+// fall back on the input.
+// Each warp owns 512 consecutive elements and walks them 32 at a time
+// (coalesced), carrying its running sum.
+__global__ void __launch_bounds__(SCAN_THREADS) k_scan_reduce(const uint32_t *__restrict__ in, int64_t n,
+                                                              uint32_t *__restrict__ partials) {
+    __shared__ uint32_t wbuf[33];
+    const int64_t base = (int64_t)blockIdx.x * SCAN_TILE + (threadIdx.x >> 5) * (SCAN_TILE / 8);
+    uint32_t s = 0;
+#pragma unroll
+    for (int it = 0; it < SCAN_ITEMS; ++it) {
+        int64_t i = base + it * 32 + lane_id();
+        if (i < n) s += in[i];
+    }
+    uint32_t tot = block_sum<uint32_t>(s, wbuf);
+    if (threadIdx.x == 0) partials[blockIdx.x] = tot;
+}
+
+// One block scans the tile sums (exclusive) in place; partials[nt] = total.
+__global__ void __launch_bounds__(1024) k_scan_partials(uint32_t *partials, int64_t nt, uint32_t *total_dev) {
+    __shared__ uint32_t wbuf[33];
+    uint32_t carry = 0;
+    for (int64_t b = 0; b < nt; b += 1024) {
+        int64_t i = b + threadIdx.x;
+        uint32_t v = i < nt ? partials[i] : 0u;
+        uint32_t tot;
+        uint32_t ex = block_exclusive_scan<uint32_t>(v, wbuf, &tot);
+        if (i < nt) partials[i] = carry + ex;
+        carry += tot;
+    }
+    if (threadIdx.x == 0) {
+        partials[nt] = carry;
+        if (total_dev) *total_dev = carry;
+    }
+}
+
+__global__ void __launch_bounds__(SCAN_THREADS) k_scan_down(const uint32_t *in, uint32_t *out, int64_t n,
+                                                            const uint32_t *__restrict__ partials) {
+    __shared__ uint32_t wbuf[33];
+    const unsigned w = threadIdx.x >> 5;
+    const int64_t base = (int64_t)blockIdx.x * SCAN_TILE + w * (SCAN_TILE / 8);
+    uint32_t v[SCAN_ITEMS];
+    uint32_t carry = 0;
+#pragma unroll
+    for (int it = 0; it < SCAN_ITEMS; ++it) {
+        int64_t i = base + it * 32 + lane_id();
+        uint32_t x = i < n ? in[i] : 0u;
+        uint32_t inc = warp_inclusive_scan(x);
+        v[it] = carry + inc - x;
+        carry += __shfl_sync(0xffffffffu, inc, 31);
+    }
+    // carry = this warp's total; block-exclusive prefix over warps
+    uint32_t wtot;
+    uint32_t wpre = block_exclusive_scan<uint32_t>(lane_id() == 0 ? carry : 0u, wbuf, &wtot);
+    wpre = __shfl_sync(0xffffffffu, wpre, 0);
+    const uint32_t off = partials[blockIdx.x] + wpre;
+#pragma unroll
+    for (int it = 0; it < SCAN_ITEMS; ++it) {
+        int64_t i = base + it * 32 + lane_id();
+        if (i < n) out[i] = off + v[it];
+    }
+}
 
 // ------------------------------------------------------------------ scan
 // One pass: a block takes the next tile of SCAN_TILE elements (tiles in the
 // order blocks start), each warp scans 512 consecutive elements 32 at a time
 // (coalesced) carrying its running sum, the warp totals are scanned across
 // the block, and the tile's offset comes from the chained prefix of the tiles
-// before it.  Each element is read and written by the same thread, so the
-// scan may run in place.
-__global__ void __launch_bounds__(SCAN_THREADS) k_scan_onepass(const uint32_t *in, uint32_t *out, int64_t n,
+// before it.  Out of place only: a tile whose wait gives up sums the input of
+// the tiles before it that are still silent.
+__global__ void __launch_bounds__(SCAN_THREADS) k_scan_onepass(const uint32_t *__restrict__ in,
+                                                               uint32_t *__restrict__ out, int64_t n,
                                                                unsigned long long *status, unsigned *tile_ctr,
-                                                               int64_t nt, uint32_t *total_dev, DevStatus *st) {
+                                                               int64_t nt, uint32_t *total_dev, int64_t spin_limit,
+                                                               int fault, DevStatus *st) {
     __shared__ uint32_t wbuf[33];
     __shared__ unsigned tile_s;
     __shared__ uint32_t off_s;
@@ -42,7 +113,7 @@ __global__ void __launch_bounds__(SCAN_THREADS) k_scan_onepass(const uint32_t *i
     uint32_t wpre = block_exclusive_scan<uint32_t>(lane_id() == 0 ? carry : 0u, wbuf, &btot);
     wpre = __shfl_sync(0xffffffffu, wpre, 0);
     if (threadIdx.x < 32) {
-        const uint32_t ex = warp_lookback_exclusive(status, tile, btot, st);
+        const uint32_t ex = warp_lookback_exclusive(status, tile, btot, in, n, SCAN_TILE, spin_limit, fault != 0, st);
         if (threadIdx.x == 0) {
             off_s = ex;
             if (tile == nt - 1 && total_dev) *total_dev = ex + btot;
@@ -102,10 +173,20 @@ void scan_exclusive_u32(Ctx &c, const uint32_t *in, uint32_t *out, int64_t n, ui
         launch(c, "scan_small", k_scan_small, dim3(1), dim3(1024), 0, in, out, n, total_dev);
         return;
     }
+    if (in == out) {
+        launch(c, "scan_reduce", k_scan_reduce, dim3((unsigned)nt), dim3(SCAN_THREADS), 0, in, n, partials);
+        launch(c, "scan_partials", k_scan_partials, dim3(1), dim3(1024), 0, partials, nt, total_dev);
+        launch(c, "scan_down", k_scan_down, dim3((unsigned)nt), dim3(SCAN_THREADS), 0, in, out, n,
+               (const uint32_t *)partials);
+        return;
+    }
     unsigned long long *status = reinterpret_cast<unsigned long long *>(partials);
     cudaMemsetAsync(status, 0, sizeof(unsigned long long) * (nt + 1), c.stream);
+    const char *fault = getenv("OPATTR_FAULT");
+    const int lb_fault = fault && strcmp(fault, "lookback") == 0;
+    const int64_t spin = c.cfg.spin_limit > 0 ? c.cfg.spin_limit : LB_SPIN_DEFAULT;
     launch(c, "scan", k_scan_onepass, dim3((unsigned)nt), dim3(SCAN_THREADS), 0, in, out, n, status,
-           reinterpret_cast<unsigned *>(status + nt), nt, total_dev, c.d_status);
+           reinterpret_cast<unsigned *>(status + nt), nt, total_dev, spin, lb_fault, c.d_status);
 }
 
 // ------------------------------------------------------------------ radix sort

@@ -45,46 +45,63 @@ void radix_sort_pairs(Ctx &c, K *k0, uint32_t *v0, K *k1, uint32_t *v1, int64_t 
 // reads the words of the 32 tiles before a point at once, adds the totals up
 // to the nearest tile whose prefix is known, and moves 32 tiles further back
 // only when none of the 32 has one.  Tiles take their index in the order
-// their blocks start (from a counter), so every tile waited on has started,
-// and it publishes its total without waiting on any other tile.  The wait is
-// bounded all the same: after LB_SPIN_LIMIT polls the tile sets ERR_TIMEOUT
-// and goes on with the part of its prefix it has, which is no larger than the
-// true one (so positions derived from it stay in bounds).  Status words and
-// the counter start at zero (one memset per pass).
+// their blocks start (from a counter), so every tile waited on has started
+// and publishes its total without waiting on any other tile.  The wait is
+// bounded all the same: after `spin_limit` polls the tile sums the input of
+// every tile still silent itself (the scan is out of place, so that input is
+// intact), sets ERR_TIMEOUT and goes on; its result stays exact.  Status
+// words and the counter start at zero (one memset per pass).  With `fault`
+// set every status word reads as silent, which makes the wait give up (the
+// fault-injection test of the bound).
 constexpr unsigned long long LB_AGG = 1ull << 62, LB_INC = 1ull << 63;
-constexpr int LB_SPIN_LIMIT = 1 << 20;
+constexpr int64_t LB_SPIN_DEFAULT = 1 << 20;
 
 // Called by all 32 lanes of one warp with the same arguments; returns the
-// sum of `total` over the tiles before t (in every lane).
+// sum of `total` over the tiles before t (in every lane).  Tile q covers
+// in[q * tile_elems, min((q + 1) * tile_elems, n)).
 __device__ __forceinline__ uint32_t warp_lookback_exclusive(unsigned long long *status, int64_t t, uint32_t total,
-                                                            DevStatus *st) {
+                                                            const uint32_t *in, int64_t n, int64_t tile_elems,
+                                                            int64_t spin_limit, bool fault, DevStatus *st) {
     const unsigned lane = lane_id();
     volatile unsigned long long *word = status;
     if (lane == 0) word[t] = (t == 0 ? LB_INC : LB_AGG) | total;
     if (t == 0) return 0;
     uint32_t excl = 0;
     int64_t j = t - 1;                       // lane i reads tile j - i
-    int spins = 0;
+    int64_t spins = 0;
+    bool gave_up = false;
     for (;;) {
         const int64_t q = j - (int64_t)lane;
-        const unsigned long long v = q >= 0 ? (unsigned long long)word[q] : 0ull + LB_INC;   // before tile 0: an empty known prefix
-        const unsigned inc = __ballot_sync(0xffffffffu, (v & LB_INC) != 0);
-        const unsigned none = __ballot_sync(0xffffffffu, (v & (LB_INC | LB_AGG)) == 0);
-        const int first = inc ? __ffs(inc) - 1 : 32;               // nearest tile with a known prefix
-        const unsigned upto = first == 32 ? 0xffffffffu : (2u << first) - 1u;
+        unsigned long long v = 0ull + LB_INC;                      // before tile 0: an empty known prefix
+        if (q >= 0) v = fault ? 0ull : (unsigned long long)word[q];
+        unsigned none = __ballot_sync(0xffffffffu, (v & (LB_INC | LB_AGG)) == 0);
+        unsigned inc = __ballot_sync(0xffffffffu, (v & LB_INC) != 0);
+        int first = inc ? __ffs(inc) - 1 : 32;                     // nearest tile with a known prefix
+        unsigned upto = first == 32 ? 0xffffffffu : (2u << first) - 1u;
         if (none & upto) {                   // a tile on the way has published nothing yet
-            if (++spins > LB_SPIN_LIMIT) {
-                if (lane == 0) set_err(st, ERR_TIMEOUT);
-                break;
+            if (!gave_up && ++spins <= spin_limit) {
+                __nanosleep(64);
+                continue;
             }
-            __nanosleep(64);
-            continue;
+            gave_up = true;
+            if ((none >> lane) & 1u) {       // its total, from its input
+                const int64_t e = (q + 1) * tile_elems < n ? (q + 1) * tile_elems : n;
+                uint32_t s = 0;
+                for (int64_t i = q * tile_elems; i < e; ++i) s += in[i];
+                v = LB_AGG | s;
+            }
+            inc = __ballot_sync(0xffffffffu, (v & LB_INC) != 0);
+            first = inc ? __ffs(inc) - 1 : 32;
+            upto = first == 32 ? 0xffffffffu : (2u << first) - 1u;
         }
         excl += warp_sum<uint32_t>(((upto >> lane) & 1u) ? (uint32_t)v : 0u);
         if (first < 32) break;
         j -= 32;
     }
-    if (lane == 0) word[t] = LB_INC | (uint32_t)(excl + total);
+    if (lane == 0) {
+        if (gave_up) set_err(st, ERR_TIMEOUT);
+        word[t] = LB_INC | (uint32_t)(excl + total);
+    }
     return excl;
 }
 
@@ -177,14 +194,20 @@ __global__ void __launch_bounds__(RADIX_THREADS) k_digit_rank(DigitFn digit, int
 }
 
 // nbins: digits used (every digit below it); only those rows of the matrix
-// are scanned.
+// are counted on and scanned.  With at most RADIX_BINS / 2 digits the scan
+// goes out of place, into the free upper half of `hist` (one pass); the
+// offsets' address is returned for digit_rank.
 template <typename DigitFn>
-void digit_offsets(Ctx &c, DigitFn digit, int64_t n, uint32_t *hist, uint32_t *partials, int nbins = RADIX_BINS) {
-    if (n <= 0) return;
+uint32_t *digit_offsets(Ctx &c, DigitFn digit, int64_t n, uint32_t *hist, uint32_t *partials,
+                        int nbins = RADIX_BINS) {
+    if (n <= 0) return hist;
     const int64_t ntiles = (n + RADIX_TILE - 1) / RADIX_TILE;
     launch(c, "digit_hist", k_digit_hist<DigitFn>, dim3((unsigned)ntiles), dim3(RADIX_THREADS), 0, digit, n, hist,
            ntiles);
-    scan_exclusive_u32(c, hist, hist, ntiles * (int64_t)(nbins < 1 ? 1 : nbins), partials, nullptr);
+    const int64_t m = ntiles * (int64_t)(nbins < 1 ? 1 : nbins);
+    uint32_t *offs = nbins <= RADIX_BINS / 2 ? hist + m : hist;
+    scan_exclusive_u32(c, hist, offs, m, partials, nullptr);
+    return offs;
 }
 
 template <typename DigitFn, typename Epi>

@@ -221,6 +221,36 @@ def test_oom_injection(opa, monkeypatch):
     ctx.close()
 
 
+def test_lookback_wait_bound(opa, monkeypatch):
+    """Scans out of place chain their tiles' prefixes by decoupled look-back,
+    whose wait is bounded by the context's spin limit.  With every status word
+    reading as silent (OPATTR_FAULT=lookback) each tile gives up after that
+    many polls and sums the silent tiles' input itself: the call returns
+    E_TIMEOUT and its outputs are still exact."""
+    import torch
+    t = tracegen.generate("dedup")
+    assert t.n_ops + 1 > 32 * 1024            # the per-op offsets take the multi-tile scan
+    ctx = opa.Context(0, spin_limit=64)
+    tr = opa.to_device(t)
+    _, rk, _ = ctx.enclose(tr)
+    _, idx, _, _ = ctx.match(tr, dedup=True)
+    _, want, want_tot = ctx.aggregate(tr, rk, idx)
+    got = ctx.alloc_ops(t.n_ops)
+    monkeypatch.setenv("OPATTR_FAULT", "lookback")
+    with pytest.raises(opa.OpattrError) as ei:
+        ctx.aggregate(tr, rk, idx, ops=got)
+    assert ei.value.status == opa.E_TIMEOUT
+    monkeypatch.delenv("OPATTR_FAULT")
+    torch.cuda.synchronize()
+    for key in want:
+        np.testing.assert_array_equal(got[key].cpu().numpy(), want[key].cpu().numpy(), err_msg=key)
+    # the context goes on as before
+    st, again, tot = ctx.aggregate(tr, rk, idx)
+    assert st >= 0 and tot == want_tot
+    np.testing.assert_array_equal(again["agg"].cpu().numpy(), want["agg"].cpu().numpy())
+    ctx.close()
+
+
 def _agg_inputs(seed, K, seg_lens, n_small_ops, nan_frac=0.0, counter_dist="uniform", dur_sigma=1.2,
                 dur_median=8000.0):
     """Aggregation-only inputs: ops 0..len(seg_lens)-1 get seg_lens[i] kernels,
