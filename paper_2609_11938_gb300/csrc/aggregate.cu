@@ -38,6 +38,8 @@ struct AggIn {
     int64_t n_ops;
     unsigned *ctr;              // [0] next chunk of the ops pass, [1] ops listed in dirty; zeroed before it
     uint32_t *dirty;            // ops whose fast sums saw a null or infinite value
+    uint32_t *longs;            // ops the ops pass leaves to the pieces pass (listed there)
+    unsigned *nlong;            //   and their number (zeroed before the ops pass)
     const unsigned *nonident;   // nonzero unless ncu_idx[k] == k for every kernel (set by the count pass)
     opattr_op_aggregates out;
 };
@@ -417,33 +419,18 @@ __global__ void k_agg_place(const int32_t *__restrict__ rok, const uint32_t *__r
 }
 
 // ------------------------------------------------------------------ long segments
-// Segments longer than AG_SHORT_MAX are sorted by kernel index before the ops
-// pass, one block per segment: up to SL_SMEM entries by a bitonic sort in
-// shared memory; longer ones in SL_SMEM runs sorted that way, then merged
-// pairwise through `tmp` (merge path: each thread merges an equal share of
-// the output after a binary search on its diagonal).
+// Segments of the ops longer than AG_HUGE (the pieces pass below) are sorted
+// by kernel index first, one block per segment: up to SL_SMEM entries by a
+// bitonic sort in shared memory; longer ones in SL_SMEM runs sorted that way,
+// then merged pairwise through `tmp` (merge path: each thread merges an equal
+// share of the output after a binary search on its diagonal).
 constexpr int SL_THREADS = 256;
 constexpr int SL_SMEM = 8192;
-constexpr uint32_t AG_SHORT_MAX = 64;           // segments up to this length: sorted by one warp; longer: one block
 
+constexpr uint32_t AG_SHORT_MAX = 64;           // segments up to this length: sorted in place by one lane
 constexpr uint32_t AG_HUGE = 256;               // longer segments: split into pieces over several warps
 constexpr uint32_t AG_PIECE = 1024;              // kernels of a huge op per warp of the pieces pass
 constexpr uint32_t AG_BLOCK_SORT_MAX = 4096;     // longer huge segments: placed by a counting pass, not sorted
-
-// Ops with segments longer than `limit`, listed (in no particular order).
-__global__ void k_agg_long_list(const uint32_t *__restrict__ off, int64_t n_ops, uint32_t limit,
-                                uint32_t *__restrict__ longs, unsigned *__restrict__ nlong) {
-    for (int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o - threadIdx.x < n_ops;
-         o += (int64_t)gridDim.x * blockDim.x) {
-        const bool is_long = o < n_ops && off[o + 1] - off[o] > limit;
-        const unsigned m = __ballot_sync(0xffffffffu, is_long);
-        if (!m) continue;
-        unsigned base = 0;
-        if (lane_id() == 0) base = atomicAdd(nlong, (unsigned)__popc(m));
-        base = __shfl_sync(0xffffffffu, base, 0);
-        if (is_long) longs[base + __popc(m & lanemask_lt())] = (uint32_t)o;
-    }
-}
 
 __device__ void bitonic_smem(uint32_t *a, int n2) {     // n2 a power of two; the block sorts a[0..n2)
     for (int k = 2; k <= n2; k <<= 1)
@@ -526,8 +513,10 @@ __global__ void __launch_bounds__(SL_THREADS) k_agg_sort_long(const uint32_t *__
 // memory by coalesced loads, and each thread checks its segments there and,
 // in the rare case the count pass met an op in two runs, sorts them in place,
 // so segments are walked in ascending kernel index (a larger chunk reads the
-// list in place: short segments checked there, long ones sorted before by
-// k_agg_sort_long).  While a kernel is added, the counter rows and durations
+// list in place: segments up to AG_SHORT_MAX are checked and sorted there).
+// Ops longer than AG_HUGE, and longer than AG_SHORT_MAX in a chunk that does
+// not fit, are listed for the pieces pass instead (sorted there by a block
+// each).  While a kernel is added, the counter rows and durations
 // of the next two arrive in per-thread shared-memory slots by asynchronous
 // copy (cp.async), with their row indices loaded a step earlier still (or
 // taken to be the kernel indices when the count pass found every row to be
@@ -645,9 +634,11 @@ __global__ void __launch_bounds__(AG_THREADS, 5) k_agg_ops(const uint32_t *__res
             if (i < nchunk) W.order[atomicAdd(&W.lcount[bkt[q]], 1u)] = (uint8_t)i;
             // each thread puts the segments of its own ops in ascending order
             const uint32_t len = i < nchunk ? ob[q] - oa[q] : 0u;
-            if (len > 1 && len <= AG_HUGE) {
+            if (len > AG_HUGE || (!staged && len > AG_SHORT_MAX)) {
+                A.longs[atomicAdd(A.nlong, 1u)] = (uint32_t)(o0 + i);   // for the pieces pass
+            } else if (len > 1) {
                 if (staged) sort_segment(W.L + (oa[q] - cbase), len);
-                else if (len <= AG_SHORT_MAX) sort_segment(list + oa[q], len);
+                else sort_segment(list + oa[q], len);
             }
         }
         __syncwarp();
@@ -675,7 +666,7 @@ __global__ void __launch_bounds__(AG_THREADS, 5) k_agg_ops(const uint32_t *__res
             if (i >= nchunk) continue;
             const int64_t o = o0 + il;
             const uint32_t s0 = sa, len = sb - sa;
-            if (len > AG_HUGE) continue;                 // a huge op: k_agg_long_ops writes it
+            if (len > AG_HUGE || (!staged && len > AG_SHORT_MAX)) continue;   // listed: k_agg_long_ops writes it
             const uint32_t *seg = staged ? W.L + (s0 - cbase) : list + s0;
             AccF acc;
             acc.init();
@@ -743,8 +734,9 @@ __global__ void k_agg_careful(const uint32_t *__restrict__ off, uint32_t *list, 
 
 // ------------------------------------------------------------------ host
 // ------------------------------------------------------------------ long ops
-// Ops whose segments are longer than AG_HUGE (listed by k_agg_long_list,
-// sorted by k_agg_sort_long) are split into pieces of AG_PIECE kernels, so an
+// Ops the ops pass lists (longer than AG_HUGE, or longer than AG_SHORT_MAX
+// in a chunk it could not stage; sorted by k_agg_sort_long or placed in order
+// by a counting pass) are split into pieces of AG_PIECE kernels, so an
 // operator with a very long segment (an Inductor fusion-map operator gathers
 // every unattributed launch of its kernel name) is spread over many warps
 // instead of holding one thread for its whole length.  Each lane adds a
@@ -1066,27 +1058,17 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     in.n_ops = O;
     in.ctr = ctr;
     in.dirty = dirty;
+    in.longs = longs;
+    in.nlong = nlong;
     in.nonident = nonident;
     in.out = *out;
+    bool status_fresh = false;        // no launch since the last status read
     if (O > 0) {
         scan_exclusive_u32(c, cnt, off, O + 1, part, nullptr);
         if (K > 0)
             launch(c, "agg_place", rok ? k_agg_place<false> : k_agg_place<true>,
                    dim3(grid_for(K, 256 * 4, REDUCE_GRID)), dim3(256), 0, rok, rng->op_id, K, R, O,
                    (const uint32_t *)off, (const uint32_t *)tmp, list);
-        launch(c, "agg_long_list", k_agg_long_list, dim3(grid_for(O, 256, 4096)), dim3(256), 0,
-               (const uint32_t *)off, O, AG_SHORT_MAX, longs, nlong);
-        launch(c, "agg_piece_offsets", k_agg_piece_offsets, dim3(1), dim3(1024), 0, (const uint32_t *)off,
-               (const uint32_t *)longs, (const unsigned *)nlong, AG_HUGE, npc, info, hop);
-        // long segments the ops pass walks: sorted first
-        launch(c, "agg_sort_long", k_agg_sort_long, dim3(2 * std::max(1, sms)), dim3(SL_THREADS), 0,
-               (const uint32_t *)off, (const uint32_t *)longs, (const unsigned *)nlong, AG_SHORT_MAX + 1, AG_HUGE,
-               list, tmp);
-        // whether huge ops exist is read while the ops pass runs
-        if (!c.ev_aux && cudaEventCreateWithFlags(&c.ev_aux, cudaEventDisableTiming) != cudaSuccess)
-            return cuda_status(c, cudaGetLastError());
-        cudaMemcpyAsync(c.h_levels, info, 5 * sizeof(uint32_t), cudaMemcpyDeviceToHost, c.stream);
-        cudaEventRecord(c.ev_aux, c.stream);
         static unsigned attr_done = 0;
         if (c.device < 32 && !(attr_done & (1u << c.device))) {
             cudaFuncSetAttribute(k_agg_ops, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)AG_SMEM);
@@ -1094,10 +1076,27 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
         }
         launch(c, "agg_ops", k_agg_ops, dim3(ops_grid(c, O)), dim3(AG_THREADS), AG_SMEM,
                (const uint32_t *)off, list, in);
-        launch(c, "agg_careful", k_agg_careful, dim3(std::max(1, sms)), dim3(128), 0, (const uint32_t *)off, list, in,
-               c.d_status);
-        if (cudaEventSynchronize(c.ev_aux) != cudaSuccess) return cuda_status(c, cudaGetLastError());
-        const uint32_t pieces = c.h_levels[1], longest = c.h_levels[2], n_huge = c.h_levels[4];
+        // the ops the pass left: listed with a null or infinite value (redone
+        // by k_agg_careful), long ones (the pieces pass); both
+        // counts come back with the status
+        cudaMemcpyAsync(c.h_levels, ctr + 1, sizeof(uint32_t), cudaMemcpyDeviceToHost, c.stream);
+        cudaMemcpyAsync(c.h_levels + 1, nlong, sizeof(uint32_t), cudaMemcpyDeviceToHost, c.stream);
+        if ((st = read_status(c))) return st;
+        const uint32_t n_dirty = c.h_levels[0], n_long = c.h_levels[1];
+        status_fresh = n_dirty == 0 && n_long == 0;
+        if (n_dirty > 0)
+            launch(c, "agg_careful", k_agg_careful, dim3(std::max(1, sms)), dim3(128), 0, (const uint32_t *)off, list,
+                   in, c.d_status);
+        uint32_t pieces = 0, longest = 0, n_huge = 0;
+        if (n_long > 0) {
+            launch(c, "agg_piece_offsets", k_agg_piece_offsets, dim3(1), dim3(1024), 0, (const uint32_t *)off,
+                   (const uint32_t *)longs, (const unsigned *)nlong, 0u, npc, info, hop);
+            cudaMemcpyAsync(c.h_levels, info, 5 * sizeof(uint32_t), cudaMemcpyDeviceToHost, c.stream);
+            if ((st = read_status(c))) return st;
+            pieces = c.h_levels[1];
+            longest = c.h_levels[2];
+            n_huge = c.h_levels[4];
+        }
         if (pieces > 0) {
             if (n_huge <= (uint32_t)RADIX_BINS && longest > AG_BLOCK_SORT_MAX && K > 0) {
                 // very long segments: placed in kernel order by one counting pass
@@ -1111,7 +1110,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
                            HugePlace{hhist, ntiles, (const uint32_t *)hop, (const uint32_t *)off, list});
             } else {
                 launch(c, "agg_sort_long", k_agg_sort_long, dim3(2 * std::max(1, sms)), dim3(SL_THREADS), 0,
-                       (const uint32_t *)off, (const uint32_t *)longs, (const unsigned *)nlong, AG_HUGE + 1,
+                       (const uint32_t *)off, (const uint32_t *)longs, (const unsigned *)nlong, 2u,
                        0xFFFFFFFFu, list, tmp);
             }
             launch(c, "agg_pieces", k_agg_pieces, dim3(4 * std::max(1, sms)), dim3(256), 0, (const uint32_t *)off,
@@ -1122,7 +1121,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
                    (const Acc *)partials, 0, in, c.d_status);
         }
     }
-    if ((st = read_status(c))) return st;
+    if (!status_fresh && (st = read_status(c))) return st;
     if (c.h_status->err & ERR_INVALID) return OPATTR_E_INVALID_ARG;
     opattr_totals T{};
     T.total_ns = (int64_t)c.h_status->cnt[C_TOTAL_NS];
@@ -1257,6 +1256,8 @@ opattr_status do_rollup(Ctx &c, const opattr_kernels *kern, const opattr_ranges 
         in.n_ops = C;
         in.ctr = nullptr;
         in.dirty = nullptr;
+        in.longs = nullptr;
+        in.nlong = nullptr;
         in.nonident = nullptr;
         in.out = *out;
         int sms = 0;

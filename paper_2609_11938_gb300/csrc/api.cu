@@ -338,7 +338,6 @@ void opattr_destroy(opattr_ctx *ctx) {
         if (c.h_init) cudaFreeHost(c.h_init);
         if (c.h_levels) cudaFreeHost(c.h_levels);
         if (c.h_stage) cudaFreeHost(c.h_stage);
-        if (c.ev_aux) cudaEventDestroy(c.ev_aux);
         for (auto &p : c.pending) {
             cudaEventDestroy(p.second.first);
             cudaEventDestroy(p.second.second);

@@ -88,7 +88,6 @@ struct Ctx {
     uint32_t *h_levels = nullptr;    // pinned host copy of the enclosure's level offsets [N_LEVELS + 1] and
                                      // kernels per stream [256];
                                      // the aggregation reuses it for a few values read mid-call
-    cudaEvent_t ev_aux = nullptr;    // marks a mid-call host read (created on first use)
     unsigned char *h_stage = nullptr; // pinned staging for small host-built tables [STAGE_BYTES]
     // kernel time order as the last enclosure found it (-1 unknown, 0 / 1),
     // and whether the matching may take it instead of checking again (join)

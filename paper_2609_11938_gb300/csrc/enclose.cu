@@ -328,38 +328,18 @@ struct PlaceByStream {
     __device__ __forceinline__ void done(unsigned) const {}
 };
 
-// Launch position of every tile: tile u = toff[s] + r goes to
-//   sum over streams q of min(tiles of q, r)  +  #{q < s : tiles of q > r}.
-// tinfo[position] = s | r << 8.
-__global__ void k_tile_order(const uint32_t *__restrict__ toff, int64_t nt, uint32_t *__restrict__ tinfo) {
-    __shared__ uint32_t to[257];
-    for (int i = threadIdx.x; i < 257; i += blockDim.x) to[i] = toff[i];
-    __syncthreads();
-    for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < nt; u += (int64_t)gridDim.x * blockDim.x) {
-        int lo = 0, hi = 256;                      // the stream of u: last s with to[s] <= u
-        while (hi - lo > 1) {
-            const int m = (lo + hi) >> 1;
-            if (to[m] <= (uint32_t)u) lo = m; else hi = m;
-        }
-        const uint32_t sid = (uint32_t)lo, r = (uint32_t)u - to[lo];
-        uint32_t p = 0;
-        for (int q = 0; q < 256; ++q) {
-            const uint32_t c = to[q + 1] - to[q];
-            p += (c < r ? c : r) + ((uint32_t)q < sid && c > r ? 1u : 0u);
-        }
-        tinfo[p] = sid | (r << 8);
-    }
-}
-
 // Window of every (tile, depth): P[u * 32 + d] = (last position of level
 // (s, d) with start <= the tile's first time, last position with start <= its
 // last time), relative to the level's start, -1 for none.  Lane d of a warp
-// takes depth d of one tile.
+// takes depth d of one tile.  The warp also places the tile in the launch
+// order: tile u = toff[s] + r goes to
+//   sum over streams q of min(tiles of q, r)  +  #{q < s : tiles of q > r},
+// tinfo[position] = s | r << 8.
 __global__ void k_stream_windows(const int64_t *__restrict__ ls, const uint32_t *__restrict__ lvl_off,
                                  const uint8_t *__restrict__ ndep, const uint32_t *__restrict__ toff,
                                  const uint32_t *__restrict__ koff, const uint32_t *__restrict__ kcnt,
                                  const uint32_t *__restrict__ psk, const int64_t *__restrict__ k_start, int64_t nt,
-                                 int2 *__restrict__ P) {
+                                 int2 *__restrict__ P, uint32_t *__restrict__ tinfo) {
     for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < nt * 32; q += (int64_t)gridDim.x * blockDim.x) {
         const int64_t u = q >> 5;
         const int d = (int)(q & 31);
@@ -369,6 +349,17 @@ __global__ void k_stream_windows(const int64_t *__restrict__ ls, const uint32_t 
             if (toff[m] <= (uint32_t)u) lo = m; else hi = m;
         }
         const int sid = lo;
+        {
+            // the tile's launch position: each lane adds the terms of eight streams
+            const uint32_t r = (uint32_t)u - toff[sid];
+            uint32_t p = 0;
+            for (int qs = d; qs < 256; qs += 32) {
+                const uint32_t c = toff[qs + 1] - toff[qs];
+                p += (c < r ? c : r) + (qs < sid && c > r ? 1u : 0u);
+            }
+            p = warp_sum<uint32_t>(p);
+            if (d == 0) tinfo[p] = (uint32_t)sid | (r << 8);
+        }
         if (d >= ndep[sid]) continue;
         const int64_t pos0 = (u - toff[sid]) * (int64_t)EN_TILE;
         const int64_t cnt = (int64_t)kcnt[sid] - pos0 < EN_TILE ? (int64_t)kcnt[sid] - pos0 : EN_TILE;
@@ -742,7 +733,6 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
         const TimeStreamDigit dg{kern->stream, korder, d_scmap};
         const uint32_t *offs = digit_offsets(c, dg, K, hist, part, nks);
         digit_rank(c, "stream_place", dg, K, offs, PlaceByStream{korder, psk});
-        launch(c, "tile_order", k_tile_order, dim3(grid_for(NT, 256, 4096)), dim3(256), 0, d_toff, NT, tinfo);
     }
 
     // ---- level lists, their validation, the windows and the enclosure, without
@@ -797,7 +787,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
         if (K > 0 && nl > 0) {
             launch(c, "stream_windows", k_stream_windows, dim3(grid_for(NT * 32, 256, 65535)), dim3(256), 0,
                    (const int64_t *)ls, (const uint32_t *)lvl_off, d_ndep, d_toff, d_koff, d_kcnt,
-                   (const uint32_t *)psk, kern->start_ns, NT, P);
+                   (const uint32_t *)psk, kern->start_ns, NT, P, tinfo);
             EncArgs A;
             A.k_start = kern->start_ns;
             A.psk = psk;
