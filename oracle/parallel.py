@@ -118,17 +118,23 @@ def _aggregate(ex, t, rk, idx, parts):
 
 
 def run_threads(trace, threads: int | None = None, mode: str = "skip_name"):
-    """The join (enclose, match, aggregate) of a trace without layer
-    deduplication or per-stream rows, in `threads` host threads (default: all
-    cores).  Returns the same dict as ``oracle.run``."""
-    if trace.k_layer is not None and trace.config.get("dedup"):
-        raise ValueError("run_threads: layer deduplication is not split by name")
-    if getattr(trace, "ncu_stream", None) is not None:
-        raise ValueError("run_threads: per-stream rows are not split by name")
+    """The join (enclose, match, aggregate) of a trace in `threads` host
+    threads (default: all cores).  The matching is split by name; with layer
+    deduplication (a duplicate takes a row of another name's run) or per-stream
+    rows it runs whole in one thread, as ``oracle.match``.  Returns the same
+    dict as ``oracle.run``."""
     threads = threads or os.cpu_count() or 1
+    whole_match = (trace.k_layer is not None and bool(trace.config.get("dedup"))) or \
+        getattr(trace, "ncu_stream", None) is not None
     with cf.ThreadPoolExecutor(max_workers=threads) as ex:
         st_e, rk, nop = _enclose(ex, trace, threads)
-        st_m, idx, kind, summ = _match(ex, trace, threads, mode)
+        if whole_match:
+            st_m, idx, kind, summ = match(trace.k_stream, trace.k_start, trace.k_name, trace.ncu_name,
+                                          trace.k_layer, trace.class_of_layer, trace.rep_of_class, mode=mode,
+                                          dedup=trace.k_layer is not None and bool(trace.config.get("dedup")),
+                                          ncu_stream=getattr(trace, "ncu_stream", None))
+        else:
+            st_m, idx, kind, summ = _match(ex, trace, threads, mode)
         st_a, ops, totals = _aggregate(ex, trace, rk, idx, threads)
     return dict(enclose_status=st_e, range_of_kernel=rk, n_op_enclosing=nop, match_status=st_m, ncu_idx=idx,
                 match_kind=kind, summary=summ, aggregate_status=st_a, ops=ops, totals=totals)

@@ -646,7 +646,8 @@ def test_pins_catch_mutation(tmp_path, golden, label, old, new):
     assert failures, f"no pin caught the planted mistake: {label}"
 
 
-@pytest.mark.parametrize("name,kw", [("tiny", {}), ("gpt2", {}), ("large", dict(n_kernels=150_000)),
+@pytest.mark.parametrize("name,kw", [("tiny", {}), ("gpt2", {}), ("gpt2_dedup", {}), ("dedup", {}),
+                                     ("large", dict(n_kernels=150_000)),
                                      ("adversarial", dict(n_kernels=150_000))])
 def test_threaded_oracle_equals_single_thread(name, kw):
     """The CPU baseline's threaded run (streams, names and op blocks split
