@@ -88,6 +88,26 @@ opattr_status ensure_arena(Ctx &c, size_t bytes) {
     return OPATTR_OK;
 }
 
+opattr_status ensure_side(Ctx &c) {
+    if (c.side) return OPATTR_OK;
+    cudaStream_t s = nullptr;
+    cudaEvent_t e[3] = {nullptr, nullptr, nullptr};
+    bool ok = cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking) == cudaSuccess;
+    for (int i = 0; i < 3 && ok; ++i) ok = cudaEventCreateWithFlags(&e[i], cudaEventDisableTiming) == cudaSuccess;
+    if (!ok) {
+        cudaGetLastError();
+        for (cudaEvent_t x : e)
+            if (x) cudaEventDestroy(x);
+        if (s) cudaStreamDestroy(s);
+        return OPATTR_E_CUDA;
+    }
+    c.side = s;
+    c.ev_fork = e[0];
+    c.ev_join = e[1];
+    c.ev_join2 = e[2];
+    return OPATTR_OK;
+}
+
 opattr_status reset_status(Ctx &c) {
     cudaError_t e = cudaMemcpyAsync(c.d_status, c.h_init, sizeof(DevStatus), cudaMemcpyHostToDevice, c.stream);
     return e == cudaSuccess ? OPATTR_OK : cuda_status(c, e);
@@ -343,6 +363,13 @@ void opattr_destroy(opattr_ctx *ctx) {
             cudaEventDestroy(p.second.second);
         }
         for (cudaEvent_t e : c.event_pool) cudaEventDestroy(e);
+        if (c.side) {
+            cudaStreamSynchronize(c.side);
+            cudaEventDestroy(c.ev_fork);
+            cudaEventDestroy(c.ev_join);
+            cudaEventDestroy(c.ev_join2);
+            cudaStreamDestroy(c.side);
+        }
         cudaGetLastError();
     }
     delete ctx;

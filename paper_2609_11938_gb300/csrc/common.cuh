@@ -75,6 +75,11 @@ constexpr size_t STAGE_BYTES = 32768;  // pinned staging of host-built tables (o
 struct Ctx {
     int device = 0;
     cudaStream_t stream = nullptr;
+    // a second stream for independent chains of one call (the enclosure's
+    // level lists beside its stream partition), with the events that fork
+    // from and join back into `stream`; created on first use
+    cudaStream_t side = nullptr;
+    cudaEvent_t ev_fork = nullptr, ev_join = nullptr, ev_join2 = nullptr;
     opattr_config cfg{};
     bool broken = false;
     // scratch arena (bump allocation, reset per call)
@@ -133,6 +138,23 @@ struct Need {
 };
 
 opattr_status ensure_arena(Ctx &c, size_t bytes);
+opattr_status ensure_side(Ctx &c);       // the side stream and its events
+
+// Launches and async copies within the scope go to stream s (c.stream is
+// swapped and restored).
+struct OnStream {
+    Ctx &c;
+    cudaStream_t prev;
+    OnStream(Ctx &ctx, cudaStream_t s) : c(ctx), prev(ctx.stream) { c.stream = s; }
+    ~OnStream() { c.stream = prev; }
+    OnStream(const OnStream &) = delete;
+    OnStream &operator=(const OnStream &) = delete;
+};
+// `to` waits for the work issued to `from` so far (through event e).
+inline void stream_after(cudaStream_t to, cudaStream_t from, cudaEvent_t e) {
+    cudaEventRecord(e, from);
+    cudaStreamWaitEvent(to, e, 0);
+}
 opattr_status reset_status(Ctx &c);
 opattr_status read_status(Ctx &c);      // D2H copy + stream synchronize
 opattr_status cuda_status(Ctx &c, cudaError_t e);

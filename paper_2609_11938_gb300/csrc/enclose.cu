@@ -606,7 +606,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     nd.add<uint64_t>(R).add<uint64_t>(R).add<uint32_t>(R).add<uint32_t>(R);
     const int64_t hist_n = std::max(radix_hist_elems(R), radix_hist_elems(K));
     const int64_t part_n = std::max<int64_t>(scan_scratch_elems(hist_n), scan_scratch_elems(LEVELS + 1));
-    nd.add<uint32_t>(hist_n).add<uint32_t>(part_n);
+    nd.add<uint32_t>(hist_n).add<uint32_t>(part_n).add<uint32_t>(hist_n).add<uint32_t>(part_n);
     nd.add<int64_t>(R).add<int64_t>(R).add<uint32_t>(R);
     nd.add<unsigned char>(STAGE_BYTES);
     nd.add<uint32_t>(K).add<uint32_t>(nt_max).add<int2>(nt_max * 32);
@@ -615,6 +615,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     size_t need = nd.bytes + kernel_order_scratch(K) + 4096;
     opattr_status st = ensure_arena(c, need);
     if (st) return st;
+    if ((st = ensure_side(c))) return st;
     Arena a(c);
     uint32_t *kept_order = keep_order ? a.take<uint32_t>(K) : nullptr;     // first: the start of the arena
     if ((st = reset_status(c))) return st;
@@ -623,21 +624,29 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     uint32_t *level_hist = a.take<uint32_t>(LEVELS + 1 + 256);
     uint32_t *kstream = level_hist + LEVELS + 1;
     uint32_t *lvl_off = a.take<uint32_t>(LEVELS + 1);
-    uint32_t *part = a.take<uint32_t>(part_n);
-    if (!level_hist || !lvl_off || !part) return OPATTR_E_OOM;
+    uint32_t *part = a.take<uint32_t>(part_n), *part2 = a.take<uint32_t>(part_n);
+    if (!level_hist || !lvl_off || !part || !part2) return OPATTR_E_OOM;
     cudaMemsetAsync(level_hist, 0, sizeof(uint32_t) * (LEVELS + 1 + 256), c.stream);
-    if (R > 0)
-        launch(c, "check_ranges", k_check_ranges, dim3(grid_for(R, RCHK_THREADS * RCHK_ITEMS)), dim3(RCHK_THREADS), 0,
-               rng->stream, rng->start_ns, rng->end_ns, rng->depth, R, level_hist, c.d_status);
+    // the ranges' checks and level histogram on the side stream, beside the
+    // kernels' order check; the level offsets and the stream counts come back
+    // with the status: one synchronisation for all
+    stream_after(c.side, c.stream, c.ev_fork);
+    {
+        OnStream on(c, c.side);
+        if (R > 0)
+            launch(c, "check_ranges", k_check_ranges, dim3(grid_for(R, RCHK_THREADS * RCHK_ITEMS)),
+                   dim3(RCHK_THREADS), 0, rng->stream, rng->start_ns, rng->end_ns, rng->depth, R, level_hist,
+                   c.d_status);
+        scan_exclusive_u32(c, level_hist, lvl_off, LEVELS + 1, part2, nullptr);
+        if (cudaMemcpyAsync(c.h_levels, lvl_off, sizeof(uint32_t) * (LEVELS + 1), cudaMemcpyDeviceToHost,
+                            c.stream) != cudaSuccess)
+            return cuda_status(c, cudaGetLastError());
+    }
     check_kernel_order(c, kern->stream, kern->start_ns, K, kstream);
-    // the level offsets and the stream counts come back with the status: one
-    // synchronisation for all
-    scan_exclusive_u32(c, level_hist, lvl_off, LEVELS + 1, part, nullptr);
-    if (cudaMemcpyAsync(c.h_levels, lvl_off, sizeof(uint32_t) * (LEVELS + 1), cudaMemcpyDeviceToHost, c.stream) !=
-            cudaSuccess ||
-        cudaMemcpyAsync(c.h_levels + LEVELS + 1, kstream, sizeof(uint32_t) * 256, cudaMemcpyDeviceToHost, c.stream) !=
-            cudaSuccess)
+    if (cudaMemcpyAsync(c.h_levels + LEVELS + 1, kstream, sizeof(uint32_t) * 256, cudaMemcpyDeviceToHost, c.stream) !=
+        cudaSuccess)
         return cuda_status(c, cudaGetLastError());
+    stream_after(c.stream, c.side, c.ev_join);
     if ((st = read_status(c))) return st;
     if ((st = status_from_err(c.h_status->err))) return st;
     const bool k_sorted = !(c.h_status->flags & F_K_UNSORTED);
@@ -702,13 +711,13 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
 
     uint64_t *rk0 = a.take<uint64_t>(R), *rk1 = a.take<uint64_t>(R);
     uint32_t *rv0 = a.take<uint32_t>(R), *rv1 = a.take<uint32_t>(R);
-    uint32_t *hist = a.take<uint32_t>(hist_n);
+    uint32_t *hist = a.take<uint32_t>(hist_n), *hist2 = a.take<uint32_t>(hist_n);
     int64_t *ls = a.take<int64_t>(R), *le = a.take<int64_t>(R);
     uint32_t *li = a.take<uint32_t>(R);
     unsigned char *d_stage = a.take<unsigned char>(ST_END);
     uint32_t *psk = a.take<uint32_t>(K), *tinfo = a.take<uint32_t>(NT);
     int2 *P = a.take<int2>(NT * 32);
-    if (!rk0 || !rk1 || !rv0 || !rv1 || !hist || !ls || !le || !li || !d_stage || !psk || !tinfo || !P)
+    if (!rk0 || !rk1 || !rv0 || !rv1 || !hist || !hist2 || !ls || !le || !li || !d_stage || !psk || !tinfo || !P)
         return OPATTR_E_OOM;
     const uint8_t *d_ndep = d_stage + ST_NDEP;
     const uint8_t *d_cmap = d_stage + ST_CMAP;
@@ -717,6 +726,8 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     const uint32_t *d_toff = reinterpret_cast<const uint32_t *>(d_stage + ST_TOFF);
     const uint8_t *d_scmap = d_stage + ST_SCMAP;
     cudaMemcpyAsync(d_stage, c.h_stage, ST_END, cudaMemcpyHostToDevice, c.stream);
+    // the level lists (below) may start on the side stream from here
+    stream_after(c.side, c.stream, c.ev_fork);
 
     // ---- kernel time order, then the kernels partitioned by stream
     uint32_t *korder = nullptr;
@@ -740,47 +751,57 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     // (the enclosure reads only positions found by searches inside the level
     // lists, so non-laminar ranges give wrong answers but no stray access).
     // If ranges with equal starts were not in (start, end, index) order within
-    // a level, the whole pass runs again on fully sorted ranges.
+    // a level, the whole pass runs again on fully sorted ranges.  The level
+    // lists and their validation run on the side stream, beside the stream
+    // partition (their own scratch: hist2, part2); the windows wait for the
+    // lists, the status read for the validation.
     const unsigned g = grid_for(R, 256, 65535);
     for (int attempt = 0; attempt < 2; ++attempt) {
         const bool full_sort = !r_sorted || attempt > 0;
-        uint32_t *perm = nullptr;         // range indices in the order of the level sort
-        if (full_sort) {
-            // (start, end, index) order: sort by end, then stably by start
-            uint64_t *ko;
-            uint32_t *vo;
-            int bits = bits_for((uint64_t)(rmax - rmin));
-            launch(c, "range_time_key", k_time_key, dim3(g), dim3(256), 0, rng->end_ns, (const uint32_t *)nullptr, R,
-                   rmin, rk0);
-            radix_sort_pairs<uint64_t>(c, rk0, rv0, rk1, rv1, R, bits, true, hist, part, &ko, &vo);
-            uint64_t *kfree = ko == rk0 ? rk1 : rk0;
-            uint32_t *vfree = vo == rv0 ? rv1 : rv0;
-            launch(c, "range_time_key", k_time_key, dim3(g), dim3(256), 0, rng->start_ns, (const uint32_t *)vo, R,
-                   rmin, kfree);
-            radix_sort_pairs<uint64_t>(c, kfree, vo, ko, vfree, R, bits, false, hist, part, &ko, &perm);
+        if (attempt > 0) stream_after(c.side, c.stream, c.ev_fork);
+        {
+            OnStream on(c, c.side);
+            uint32_t *perm = nullptr;     // range indices in the order of the level sort
+            if (full_sort) {
+                // (start, end, index) order: sort by end, then stably by start
+                uint64_t *ko;
+                uint32_t *vo;
+                int bits = bits_for((uint64_t)(rmax - rmin));
+                launch(c, "range_time_key", k_time_key, dim3(g), dim3(256), 0, rng->end_ns, (const uint32_t *)nullptr,
+                       R, rmin, rk0);
+                radix_sort_pairs<uint64_t>(c, rk0, rv0, rk1, rv1, R, bits, true, hist2, part2, &ko, &vo);
+                uint64_t *kfree = ko == rk0 ? rk1 : rk0;
+                uint32_t *vfree = vo == rv0 ? rv1 : rv0;
+                launch(c, "range_time_key", k_time_key, dim3(g), dim3(256), 0, rng->start_ns, (const uint32_t *)vo,
+                       R, rmin, kfree);
+                radix_sort_pairs<uint64_t>(c, kfree, vo, ko, vfree, R, bits, false, hist2, part2, &ko, &perm);
+            }
+            if (nl <= 256) {
+                // stable partition by compact level id, ranges written in place
+                const LevelDigit dg{rng->stream, rng->depth, d_cmap, perm};
+                const uint32_t *offs = digit_offsets(c, dg, R, hist2, part2, nl);
+                const int64_t ntiles = (R + RADIX_TILE - 1) / RADIX_TILE;
+                launch(c, "level_place", k_level_place, dim3((unsigned)ntiles), dim3(RADIX_THREADS), 0, dg,
+                       rng->start_ns, rng->end_ns, rng->op_id, R, offs, ntiles, ls, le, li);
+            } else {
+                // stable partition by level key (13 bits)
+                uint32_t *lk0 = reinterpret_cast<uint32_t *>(rk0), *lk1 = reinterpret_cast<uint32_t *>(rk1);
+                uint32_t *va = perm ? perm : rv0;
+                uint32_t *vb = perm == rv0 ? rv1 : (perm == rv1 ? rv0 : rv1);
+                launch(c, "level_keys", k_level_keys, dim3(g), dim3(256), 0, rng->stream, rng->depth,
+                       (const uint32_t *)perm, R, lk0);
+                uint32_t *ko32, *lperm;
+                radix_sort_pairs<uint32_t>(c, lk0, va, lk1, vb, R, 13, perm == nullptr, hist2, part2, &ko32, &lperm);
+                launch(c, "level_gather", k_level_gather, dim3(g), dim3(256), 0, rng->start_ns, rng->end_ns,
+                       rng->op_id, (const uint32_t *)lperm, R, ls, le, li);
+            }
+            cudaEventRecord(c.ev_join, c.side);           // the level lists are in place
+            launch(c, "validate_levels", k_validate_levels, dim3(grid_for(R, 256 * VL_PER, 65535)), dim3(256), 0,
+                   rng->stream, rng->depth, (const int64_t *)ls, (const int64_t *)le, (const uint32_t *)li,
+                   (const uint32_t *)lvl_off, R, c.d_status);
+            cudaEventRecord(c.ev_join2, c.side);          // and checked
         }
-        if (nl <= 256) {
-            // stable partition by compact level id, ranges written in place
-            const LevelDigit dg{rng->stream, rng->depth, d_cmap, perm};
-            const uint32_t *offs = digit_offsets(c, dg, R, hist, part, nl);
-            const int64_t ntiles = (R + RADIX_TILE - 1) / RADIX_TILE;
-            launch(c, "level_place", k_level_place, dim3((unsigned)ntiles), dim3(RADIX_THREADS), 0, dg,
-                   rng->start_ns, rng->end_ns, rng->op_id, R, offs, ntiles, ls, le, li);
-        } else {
-            // stable partition by level key (13 bits)
-            uint32_t *lk0 = reinterpret_cast<uint32_t *>(rk0), *lk1 = reinterpret_cast<uint32_t *>(rk1);
-            uint32_t *va = perm ? perm : rv0;
-            uint32_t *vb = perm == rv0 ? rv1 : (perm == rv1 ? rv0 : rv1);
-            launch(c, "level_keys", k_level_keys, dim3(g), dim3(256), 0, rng->stream, rng->depth,
-                   (const uint32_t *)perm, R, lk0);
-            uint32_t *ko32, *lperm;
-            radix_sort_pairs<uint32_t>(c, lk0, va, lk1, vb, R, 13, perm == nullptr, hist, part, &ko32, &lperm);
-            launch(c, "level_gather", k_level_gather, dim3(g), dim3(256), 0, rng->start_ns, rng->end_ns, rng->op_id,
-                   (const uint32_t *)lperm, R, ls, le, li);
-        }
-        launch(c, "validate_levels", k_validate_levels, dim3(grid_for(R, 256 * VL_PER, 65535)), dim3(256), 0, rng->stream,
-               rng->depth, (const int64_t *)ls, (const int64_t *)le, (const uint32_t *)li, (const uint32_t *)lvl_off,
-               R, c.d_status);
+        cudaStreamWaitEvent(c.stream, c.ev_join, 0);
         if (K > 0 && nl == 0)
             launch(c, "fill_unattributed", k_fill_unattributed, dim3(grid_for(K, 256, 65535)), dim3(256), 0, out_range,
                    out_nop, K);
@@ -805,6 +826,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
             A.out_nop = out_nop;
             launch(c, "enclose", k_enclose, dim3((unsigned)NT), dim3(EN_THREADS), 0, A);
         }
+        cudaStreamWaitEvent(c.stream, c.ev_join2, 0);
         if ((st = read_status(c))) return st;
         if (!full_sort && (c.h_status->flags & F_LEVEL_FIXUP)) {
             // equal starts out of (start, end) order within a level: the
