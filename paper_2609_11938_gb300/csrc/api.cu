@@ -302,8 +302,20 @@ opattr_status opattr_join(opattr_ctx *ctx, const opattr_kernels *kernels, const 
             c.order_from_enclose = false;
             c.join_korder = nullptr;
             c.arena_keep = 0;
+            c.spec_k = 0;
+            c.spec_ran = false;
         }
     } scope(c);
+    // the matching's identity pairing may run beside the enclosure: rows one
+    // for one with the kernels, no layer deduplication, no per-stream rows
+    if (!dedup && !ncu->stream && kernels->n > 0 && kernels->n == ncu->n && kernels->name_id && ncu->name_id &&
+        ncu_idx_of_kernel) {
+        c.spec_kname = kernels->name_id;
+        c.spec_nname = ncu->name_id;
+        c.spec_idx = ncu_idx_of_kernel;
+        c.spec_kind = match_kind;
+        c.spec_k = kernels->n;
+    }
     opattr_status st = finish(c, do_enclose(c, kernels, ranges, range_of_kernel, n_op_enclosing));
     if (st < 0) return st;
     c.order_from_enclose = true;

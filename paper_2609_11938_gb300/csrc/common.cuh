@@ -105,6 +105,15 @@ struct Ctx {
     uint32_t *join_korder = nullptr;
     size_t arena_keep = 0;
     // launch accounting
+    // within a join: the matching's identity pairing (rows equal to the
+    // kernels in time order), launched beside the enclosure when spec_k > 0;
+    // spec_ran: it ran in the enclosure's last attempt, its verdict in the
+    // status the enclosure read last
+    const uint32_t *spec_kname = nullptr, *spec_nname = nullptr;
+    int32_t *spec_idx = nullptr;
+    uint8_t *spec_kind = nullptr;
+    int64_t spec_k = 0;
+    bool spec_ran = false;
     int64_t launches = 0;
     bool timing = false;
     std::string timing_only;         // with timing on: bracket only this kernel (empty = all)
@@ -139,6 +148,10 @@ struct Need {
 
 opattr_status ensure_arena(Ctx &c, size_t bytes);
 opattr_status ensure_side(Ctx &c);       // the side stream and its events
+// Algorithm 1's identity pairing on c.stream (match.cu): kernel j's row is
+// row j, F_NAMES_DIFFER set where the names disagree
+void launch_identity_match(Ctx &c, const uint32_t *kname, const uint32_t *nname, int64_t K, int32_t *out_idx,
+                           uint8_t *out_kind);
 
 // Launches and async copies within the scope go to stream s (c.stream is
 // swapped and restored).

@@ -613,6 +613,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     const bool keep_order = c.in_join && K > 0;       // a join keeps the time order for its matching
     if (keep_order) nd.add<uint32_t>(K);
     size_t need = nd.bytes + kernel_order_scratch(K) + 4096;
+    c.spec_ran = false;
     opattr_status st = ensure_arena(c, need);
     if (st) return st;
     if ((st = ensure_side(c))) return st;
@@ -799,6 +800,11 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
             launch(c, "validate_levels", k_validate_levels, dim3(grid_for(R, 256 * VL_PER, 65535)), dim3(256), 0,
                    rng->stream, rng->depth, (const int64_t *)ls, (const int64_t *)le, (const uint32_t *)li,
                    (const uint32_t *)lvl_off, R, c.d_status);
+            // within a join: the matching's identity pairing, beside the enclosure
+            if (c.spec_k > 0) {
+                launch_identity_match(c, c.spec_kname, c.spec_nname, c.spec_k, c.spec_idx, c.spec_kind);
+                c.spec_ran = true;
+            }
             cudaEventRecord(c.ev_join2, c.side);          // and checked
         }
         cudaStreamWaitEvent(c.stream, c.ev_join, 0);

@@ -61,6 +61,12 @@ __global__ void k_match_identity(const uint32_t *__restrict__ kname, const uint3
     if (__any_sync(0xffffffffu, bad) && lane_id() == 0) set_flag(st, F_NAMES_DIFFER);
 }
 
+void launch_identity_match(Ctx &c, const uint32_t *kname, const uint32_t *nname, int64_t K, int32_t *out_idx,
+                           uint8_t *out_kind) {
+    launch(c, "match_identity", k_match_identity, dim3(grid_for(K, 256 * 16, REDUCE_GRID)), dim3(256), 0, kname,
+           nname, K, out_idx, out_kind, identity_vec(kname, nname, out_idx, out_kind), c.d_status);
+}
+
 // replayed kernels in time order (list rk) against rows 0..n-1
 __global__ void k_match_identity_list(const uint32_t *__restrict__ rk, const uint32_t *__restrict__ kname,
                                       const uint32_t *__restrict__ nname, int64_t n, int32_t *__restrict__ out_idx,
@@ -401,6 +407,21 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     const int64_t NX = std::max(K, M);
     const bool per_stream = ncu->stream != nullptr;
     if (per_stream && M > 0 && !ncu->name_id) return OPATTR_E_INVALID_ARG;
+    // within a join the identity pairing ran beside the enclosure: with the
+    // kernels in time order (the enclosure's verdict) and every name equal,
+    // its outputs are the match
+    if (c.spec_ran && c.order_from_enclose && c.enclose_k_sorted == 1 && c.spec_kname == kern->name_id &&
+        c.spec_nname == ncu->name_id && c.spec_idx == out_idx &&
+        c.spec_kind == out_kind && c.spec_k == K && K == M && !dedup_on && !per_stream &&
+        !(c.h_status->flags & F_NAMES_DIFFER)) {
+        opattr_match_summary S{};
+        S.kernels = K;
+        S.replayed = K;
+        S.direct = K;
+        S.fast_path = 1;
+        if (sum) *sum = S;
+        return OPATTR_OK;
+    }
     Need nd;
     if (per_stream) nd.add<uint32_t>(K).add<uint32_t>(M);        // (name, stream) keys
     nd.add<int32_t>(NL);

@@ -764,11 +764,24 @@ def _join_cases(name):
         keep = np.setdiff1d(np.arange(t.M), np.random.default_rng(7).choice(t.M, 25, replace=False))
         t.ncu_name, t.counters = t.ncu_name[keep].copy(), t.counters[keep].copy()
         return t
+    if name == "gpt2_rows_swapped":
+        # as many rows as kernels, in time order except two rows of different
+        # names swapped: the identity pairing that runs beside the enclosure
+        # finds names that differ, and the ordinal join decides
+        t = tracegen.generate("gpt2")
+        names = t.ncu_name
+        i = 100
+        j = int(np.nonzero(names[i + 1:] != names[i])[0][0]) + i + 1
+        order = np.arange(t.M)
+        order[[i, j]] = order[[j, i]]
+        t.ncu_name, t.counters = names[order].copy(), t.counters[order].copy()
+        assert t.K == t.M
+        return t
     return tracegen.generate(name)
 
 
 @pytest.mark.parametrize("name", ["large1m", "gpt2_shuffled", "dedup", "dedup_per_stream", "gpt2_count_mismatch",
-                                  "tiny"])
+                                  "gpt2_rows_swapped", "tiny"])
 def test_join_matches_three_calls(opa, name):
     """opattr_join gives the three calls' outputs bit for bit (the order
     verdict shared between enclosure and matching, sorted or not), their
