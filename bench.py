@@ -48,7 +48,6 @@ KERNEL_BYTES = {
     "validate_levels": lambda K, R, M, O: 22 * R,
     "stream_place": lambda K, R, M, O: 5 * K,
     "stream_windows": lambda K, R, M, O: 0,
-    "tile_order": lambda K, R, M, O: 0,
 }
 
 WORKLOADS = {

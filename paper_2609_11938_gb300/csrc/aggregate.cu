@@ -1019,7 +1019,9 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     opattr_status st = ensure_arena(c, nd.bytes + 4096);
     if (st) return st;
     Arena a(c);
-    if ((st = reset_status(c))) return st;
+    // with the enclosure's verdict pending (a join) the status block keeps it:
+    // the enclosure's reset left the aggregation's slots at zero
+    if (!c.enclose_pending && (st = reset_status(c))) return st;
     uint32_t *cnt = a.take<uint32_t>(O + 1), *off = a.take<uint32_t>(O + 1);
     // tmp holds each kernel's slot among its op's kernels until the list is
     // placed, then serves the segment sorts

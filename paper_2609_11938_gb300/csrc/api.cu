@@ -237,6 +237,13 @@ opattr_status opattr_create(opattr_ctx **out, int device, void *cuda_stream, con
     return OPATTR_OK;
 }
 
+// The enclosure's error bits as a status (the order of do_enclose's checks).
+static opattr_status status_from_enclose_err(unsigned err) {
+    if (err & ERR_DEPTH) return OPATTR_E_DEPTH;
+    if (err & ERR_NOT_NESTED) return OPATTR_E_NOT_NESTED;
+    return OPATTR_OK;
+}
+
 static opattr_status finish(Ctx &c, opattr_status st) {
     if (c.last_error != cudaSuccess) return cuda_status(c, c.last_error);
     if (st == OPATTR_E_CUDA) c.broken = true;
@@ -291,43 +298,79 @@ opattr_status opattr_join(opattr_ctx *ctx, const opattr_kernels *kernels, const 
     if (c.broken) return OPATTR_E_STATE;
     DeviceGuard g(c.device);
     if (!g.ok) return OPATTR_E_CUDA;
-    c.enclose_k_sorted = -1;
     // the enclosure's kernel time order is kept for the matching (arena_keep);
     // every way out of the join drops it
     struct JoinScope {
         Ctx &c;
         explicit JoinScope(Ctx &ctx) : c(ctx) { c.in_join = true; }
         ~JoinScope() {
+            if (c.enclose_pending) cudaStreamSynchronize(c.stream);     // an early return: nothing left running
             c.in_join = false;
             c.order_from_enclose = false;
             c.join_korder = nullptr;
             c.arena_keep = 0;
             c.spec_k = 0;
             c.spec_ran = false;
+            c.defer_status = false;
+            c.enclose_pending = false;
         }
     } scope(c);
     // the matching's identity pairing may run beside the enclosure: rows one
-    // for one with the kernels, no layer deduplication, no per-stream rows
-    if (!dedup && !ncu->stream && kernels->n > 0 && kernels->n == ncu->n && kernels->name_id && ncu->name_id &&
-        ncu_idx_of_kernel) {
-        c.spec_kname = kernels->name_id;
-        c.spec_nname = ncu->name_id;
-        c.spec_idx = ncu_idx_of_kernel;
-        c.spec_kind = match_kind;
-        c.spec_k = kernels->n;
+    // for one with the kernels, no layer deduplication, no per-stream rows;
+    // then the enclosure's last status read can wait for the aggregation's
+    const bool spec = !dedup && !ncu->stream && kernels->n > 0 && kernels->n == ncu->n && kernels->name_id &&
+                      ncu->name_id && ncu_idx_of_kernel;
+    for (int pass = 0; pass < 2; ++pass) {
+        c.enclose_k_sorted = -1;
+        c.spec_k = 0;
+        c.spec_ran = false;
+        c.enclose_pending = false;
+        if (spec) {
+            c.spec_kname = kernels->name_id;
+            c.spec_nname = ncu->name_id;
+            c.spec_idx = ncu_idx_of_kernel;
+            c.spec_kind = match_kind;
+            c.spec_k = kernels->n;
+        }
+        c.defer_status = spec && pass == 0;
+        opattr_status st = finish(c, do_enclose(c, kernels, ranges, range_of_kernel, n_op_enclosing));
+        c.defer_status = false;
+        if (st < 0) return st;
+        c.order_from_enclose = true;
+        opattr_status sm =
+            finish(c, do_match(c, kernels, ncu, dedup, ncu_idx_of_kernel, match_kind, host_summary));
+        c.order_from_enclose = false;
+        c.join_korder = nullptr;             // the aggregation needs no time order
+        c.arena_keep = 0;
+        if (sm < 0) return sm;
+        st = finish(c, do_aggregate(c, kernels, ranges, range_of_kernel, ncu, ncu_idx_of_kernel, n_ops, dev_out,
+                                    host_totals));
+        if (c.enclose_pending) {
+            // the enclosure's verdict and the identity pairing's, read with the
+            // aggregation's status (read once more if the aggregation stopped
+            // before reading it)
+            c.enclose_pending = false;
+            if (st < 0) {
+                const opattr_status s2 = read_status(c);
+                if (s2 < 0) return s2;
+            }
+            if (c.h_status->flags & F_LEVEL_FIXUP) continue;          // redone without deferring
+            if (c.h_status->err & (ERR_NOT_NESTED | ERR_DEPTH)) return status_from_enclose_err(c.h_status->err);
+            if (st >= 0 && (c.h_status->flags & F_NAMES_DIFFER)) {
+                // the names disagree: the matching and the aggregation proper
+                c.order_from_enclose = true;
+                c.spec_ran = false;
+                sm = finish(c, do_match(c, kernels, ncu, dedup, ncu_idx_of_kernel, match_kind, host_summary));
+                c.order_from_enclose = false;
+                if (sm < 0) return sm;
+                st = finish(c, do_aggregate(c, kernels, ranges, range_of_kernel, ncu, ncu_idx_of_kernel, n_ops,
+                                            dev_out, host_totals));
+            }
+        }
+        if (st < 0) return st;
+        return sm;
     }
-    opattr_status st = finish(c, do_enclose(c, kernels, ranges, range_of_kernel, n_op_enclosing));
-    if (st < 0) return st;
-    c.order_from_enclose = true;
-    const opattr_status sm = finish(c, do_match(c, kernels, ncu, dedup, ncu_idx_of_kernel, match_kind, host_summary));
-    c.order_from_enclose = false;
-    c.join_korder = nullptr;             // the aggregation needs no time order
-    c.arena_keep = 0;
-    if (sm < 0) return sm;
-    st = finish(c, do_aggregate(c, kernels, ranges, range_of_kernel, ncu, ncu_idx_of_kernel, n_ops, dev_out,
-                                host_totals));
-    if (st < 0) return st;
-    return sm;
+    return OPATTR_E_CUDA;
 }
 
 opattr_status opattr_attribute(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,

@@ -114,6 +114,11 @@ struct Ctx {
     uint8_t *spec_kind = nullptr;
     int64_t spec_k = 0;
     bool spec_ran = false;
+    // within a join whose matching can be skipped: the enclosure's last status
+    // read is left to the aggregation's (defer_status), and the enclosure's
+    // verdict is pending until then (enclose_pending; the aggregation keeps
+    // the status block instead of resetting it)
+    bool defer_status = false, enclose_pending = false;
     int64_t launches = 0;
     bool timing = false;
     std::string timing_only;         // with timing on: bracket only this kernel (empty = all)

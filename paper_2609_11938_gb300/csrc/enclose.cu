@@ -318,6 +318,11 @@ struct TimeStreamDigit {
         return scmap[stream[korder ? korder[i] : (uint32_t)i]];
     }
 };
+// The stream of kernel i in array order (the kernels in time order).
+struct ArrayStreamDigit {
+    const uint8_t *stream;
+    __device__ __forceinline__ unsigned operator()(int64_t i) const { return stream[i]; }
+};
 struct PlaceByStream {
     const uint32_t *korder;
     uint32_t *psk;
@@ -602,7 +607,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     // kernel order, the stream partition of the kernels and its tile tables
     const int64_t nt_max = (K + EN_TILE - 1) / EN_TILE + 256;
     Need nd;
-    nd.add<uint32_t>(LEVELS + 1 + 256).add<uint32_t>(LEVELS + 1);
+    nd.add<uint32_t>(LEVELS + 1 + 256).add<uint32_t>(LEVELS + 1).add<uint32_t>(radix_hist_elems(K));
     nd.add<uint64_t>(R).add<uint64_t>(R).add<uint32_t>(R).add<uint32_t>(R);
     const int64_t hist_n = std::max(radix_hist_elems(R), radix_hist_elems(K));
     const int64_t part_n = std::max<int64_t>(scan_scratch_elems(hist_n), scan_scratch_elems(LEVELS + 1));
@@ -626,7 +631,8 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     uint32_t *kstream = level_hist + LEVELS + 1;
     uint32_t *lvl_off = a.take<uint32_t>(LEVELS + 1);
     uint32_t *part = a.take<uint32_t>(part_n), *part2 = a.take<uint32_t>(part_n);
-    if (!level_hist || !lvl_off || !part || !part2) return OPATTR_E_OOM;
+    uint32_t *ktile = a.take<uint32_t>(radix_hist_elems(K));     // per tile, kernels of each stream
+    if (!level_hist || !lvl_off || !part || !part2 || !ktile) return OPATTR_E_OOM;
     cudaMemsetAsync(level_hist, 0, sizeof(uint32_t) * (LEVELS + 1 + 256), c.stream);
     // the ranges' checks and level histogram on the side stream, beside the
     // kernels' order check; the level offsets and the stream counts come back
@@ -643,7 +649,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
                             c.stream) != cudaSuccess)
             return cuda_status(c, cudaGetLastError());
     }
-    check_kernel_order(c, kern->stream, kern->start_ns, K, kstream);
+    check_kernel_order(c, kern->stream, kern->start_ns, K, kstream, ktile);
     if (cudaMemcpyAsync(c.h_levels + LEVELS + 1, kstream, sizeof(uint32_t) * 256, cudaMemcpyDeviceToHost, c.stream) !=
         cudaSuccess)
         return cuda_status(c, cudaGetLastError());
@@ -741,7 +747,17 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
             c.arena_keep = (sizeof(uint32_t) * (size_t)K + 255) & ~(size_t)255;
         }
     }
-    if (K > 0 && nl > 0) {
+    if (K > 0 && nl > 0 && k_sorted) {
+        // in time order already: the order check's tile counts are the
+        // partition's histogram (stream ids as digits)
+        // (rows past the last stream with kernels hold only zeros: not scanned)
+        const int64_t ntk = (K + RADIX_TILE - 1) / RADIX_TILE;
+        int rows = 0;
+        for (int q = 0; q < 256; ++q)
+            if (kcnt_h[q] > 0) rows = q + 1;
+        scan_exclusive_u32(c, ktile, hist, ntk * rows, part, nullptr);
+        digit_rank(c, "stream_place", ArrayStreamDigit{kern->stream}, K, hist, PlaceByStream{nullptr, psk});
+    } else if (K > 0 && nl > 0) {
         const TimeStreamDigit dg{kern->stream, korder, d_scmap};
         const uint32_t *offs = digit_offsets(c, dg, K, hist, part, nks);
         digit_rank(c, "stream_place", dg, K, offs, PlaceByStream{korder, psk});
@@ -833,6 +849,11 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
             launch(c, "enclose", k_enclose, dim3((unsigned)NT), dim3(EN_THREADS), 0, A);
         }
         cudaStreamWaitEvent(c.stream, c.ev_join2, 0);
+        if (c.defer_status && k_sorted && !full_sort) {
+            // the status is read with the aggregation's, which the join checks
+            c.enclose_pending = true;
+            return OPATTR_OK;
+        }
         if ((st = read_status(c))) return st;
         if (!full_sort && (c.h_status->flags & F_LEVEL_FIXUP)) {
             // equal starts out of (start, end) order within a level: the

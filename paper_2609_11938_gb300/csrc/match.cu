@@ -410,10 +410,12 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
     // within a join the identity pairing ran beside the enclosure: with the
     // kernels in time order (the enclosure's verdict) and every name equal,
     // its outputs are the match
+    // (with the enclosure's status still to be read, the names are taken to
+    // agree; the join checks that verdict with the aggregation's status)
     if (c.spec_ran && c.order_from_enclose && c.enclose_k_sorted == 1 && c.spec_kname == kern->name_id &&
         c.spec_nname == ncu->name_id && c.spec_idx == out_idx &&
         c.spec_kind == out_kind && c.spec_k == K && K == M && !dedup_on && !per_stream &&
-        !(c.h_status->flags & F_NAMES_DIFFER)) {
+        (c.enclose_pending || !(c.h_status->flags & F_NAMES_DIFFER))) {
         opattr_match_summary S{};
         S.kernels = K;
         S.replayed = K;

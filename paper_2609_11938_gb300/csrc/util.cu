@@ -6,64 +6,82 @@ namespace opattr {
 
 constexpr int CHK_THREADS = 256;
 
-// Grid-stride over groups of eight consecutive kernels (16-byte loads when
-// the arrays allow), comparing each (start, stream) with its successor; min /
-// max and the order flag are reduced per block and published with one atomic
-// each.
+// Tiles of CHK_TILE consecutive kernels (the digit passes' tiles), a block
+// at a time, each thread taking two groups of eight consecutive kernels per
+// tile (16-byte loads when the arrays allow) and comparing each (start,
+// stream) with its successor; min / max and the order flag are reduced per
+// block and published with one atomic each.  With stream_hist the block also
+// counts the kernels of each stream (added to the 256 counters once per
+// block), and with tile_hist it writes each tile's counts as column `tile`
+// of a stream-major matrix (tile_hist[s * ntiles + tile]): the digit
+// histogram of a stable partition by stream, in array order.
 constexpr int CHK_G = 8;
+constexpr int CHK_TILE = 2 * CHK_THREADS * CHK_G;
+static_assert(CHK_TILE == RADIX_TILE, "the order check's tiles are the digit passes' tiles");
 __global__ void __launch_bounds__(CHK_THREADS) k_check_kernel_order(const uint8_t *__restrict__ stream,
                                                                     const int64_t *__restrict__ start, int64_t n,
                                                                     int vec, DevStatus *st,
-                                                                    uint32_t *__restrict__ stream_hist) {
+                                                                    uint32_t *__restrict__ stream_hist,
+                                                                    uint32_t *__restrict__ tile_hist) {
     __shared__ long long smin[CHK_THREADS / 32], smax[CHK_THREADS / 32];
     __shared__ int sbad[CHK_THREADS / 32];
-    __shared__ uint32_t sh[256];
-    if (stream_hist) {
-        for (int i = threadIdx.x; i < 256; i += CHK_THREADS) sh[i] = 0;
-        __syncthreads();
-    }
+    __shared__ uint32_t sh[256], th[256];
+    const bool count = stream_hist || tile_hist;
+    for (int i = threadIdx.x; i < 256; i += CHK_THREADS) sh[i] = th[i] = 0;
+    __syncthreads();
     long long mn = LLONG_MAX, mx = LLONG_MIN;
     int unsorted = 0;
-    const int64_t ngroups = (n + CHK_G - 1) / CHK_G;
-    for (int64_t g = (int64_t)blockIdx.x * CHK_THREADS + threadIdx.x; g < ngroups;
-         g += (int64_t)gridDim.x * CHK_THREADS) {
-        const int64_t i0 = g * CHK_G;
-        long long t[CHK_G + 1];
-        unsigned s[CHK_G + 1];
-        if (vec && i0 + CHK_G <= n) {
-            const longlong2 *p = reinterpret_cast<const longlong2 *>(start + i0);
+    const int64_t ntiles = (n + CHK_TILE - 1) / CHK_TILE;
+    for (int64_t tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+        for (int r = 0; r < 2; ++r) {
+            const int64_t i0 = (tile * (CHK_TILE / CHK_G) + r * CHK_THREADS + threadIdx.x) * CHK_G;
+            if (i0 >= n) continue;
+            long long t[CHK_G + 1];
+            unsigned s[CHK_G + 1];
+            if (vec && i0 + CHK_G <= n) {
+                const longlong2 *p = reinterpret_cast<const longlong2 *>(start + i0);
 #pragma unroll
-            for (int q = 0; q < CHK_G / 2; ++q) {
-                const longlong2 x = p[q];
-                t[2 * q] = x.x;
-                t[2 * q + 1] = x.y;
-            }
-            const uint2 w = *reinterpret_cast<const uint2 *>(stream + i0);
+                for (int q = 0; q < CHK_G / 2; ++q) {
+                    const longlong2 x = p[q];
+                    t[2 * q] = x.x;
+                    t[2 * q + 1] = x.y;
+                }
+                const uint2 w = *reinterpret_cast<const uint2 *>(stream + i0);
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                s[u] = (w.x >> (8 * u)) & 0xFFu;
-                s[4 + u] = (w.y >> (8 * u)) & 0xFFu;
+                for (int u = 0; u < 4; ++u) {
+                    s[u] = (w.x >> (8 * u)) & 0xFFu;
+                    s[4 + u] = (w.y >> (8 * u)) & 0xFFu;
+                }
+            } else {
+#pragma unroll
+                for (int u = 0; u < CHK_G; ++u) {
+                    t[u] = i0 + u < n ? start[i0 + u] : LLONG_MAX;
+                    s[u] = i0 + u < n ? stream[i0 + u] : 255u;
+                }
             }
-        } else {
+            t[CHK_G] = i0 + CHK_G < n ? start[i0 + CHK_G] : LLONG_MAX;
+            s[CHK_G] = i0 + CHK_G < n ? stream[i0 + CHK_G] : 255u;
 #pragma unroll
             for (int u = 0; u < CHK_G; ++u) {
-                t[u] = i0 + u < n ? start[i0 + u] : LLONG_MAX;
-                s[u] = i0 + u < n ? stream[i0 + u] : 255u;
+                if (i0 + u >= n) break;
+                mn = t[u] < mn ? t[u] : mn;
+                mx = t[u] > mx ? t[u] : mx;
+                if (i0 + u + 1 < n) unsorted |= (t[u + 1] < t[u]) || (t[u + 1] == t[u] && s[u + 1] < s[u]);
+                if (count) atomicAdd(&th[s[u]], 1u);
             }
         }
-        t[CHK_G] = i0 + CHK_G < n ? start[i0 + CHK_G] : LLONG_MAX;
-        s[CHK_G] = i0 + CHK_G < n ? stream[i0 + CHK_G] : 255u;
-#pragma unroll
-        for (int u = 0; u < CHK_G; ++u) {
-            if (i0 + u >= n) break;
-            mn = t[u] < mn ? t[u] : mn;
-            mx = t[u] > mx ? t[u] : mx;
-            if (i0 + u + 1 < n) unsorted |= (t[u + 1] < t[u]) || (t[u + 1] == t[u] && s[u + 1] < s[u]);
-            if (stream_hist) atomicAdd(&sh[s[u]], 1u);
+        if (count) {
+            __syncthreads();
+            for (int i = threadIdx.x; i < 256; i += CHK_THREADS) {
+                const uint32_t x = th[i];
+                if (tile_hist) tile_hist[(int64_t)i * ntiles + tile] = x;
+                sh[i] += x;
+                th[i] = 0;
+            }
+            __syncthreads();
         }
     }
     if (stream_hist) {
-        __syncthreads();
         for (int i = threadIdx.x; i < 256; i += CHK_THREADS)
             if (sh[i]) atomicAdd(&stream_hist[i], sh[i]);
     }
@@ -93,11 +111,12 @@ __global__ void __launch_bounds__(CHK_THREADS) k_check_kernel_order(const uint8_
     }
 }
 
-void check_kernel_order(Ctx &c, const uint8_t *stream, const int64_t *start, int64_t n, uint32_t *stream_hist) {
+void check_kernel_order(Ctx &c, const uint8_t *stream, const int64_t *start, int64_t n, uint32_t *stream_hist,
+                        uint32_t *tile_hist) {
     if (n <= 0) return;
     const int vec = ((reinterpret_cast<uintptr_t>(start) & 15) == 0) && ((reinterpret_cast<uintptr_t>(stream) & 7) == 0);
-    launch(c, "check_kernel_order", k_check_kernel_order, dim3(grid_for(n, CHK_THREADS * 16, REDUCE_GRID)),
-           dim3(CHK_THREADS), 0, stream, start, n, vec, c.d_status, stream_hist);
+    launch(c, "check_kernel_order", k_check_kernel_order, dim3(grid_for(n, CHK_TILE, REDUCE_GRID)),
+           dim3(CHK_THREADS), 0, stream, start, n, vec, c.d_status, stream_hist, tile_hist);
 }
 
 __global__ void k_time_keys(const uint8_t *__restrict__ stream, const int64_t *__restrict__ start, int64_t n,

@@ -2,14 +2,17 @@
 // time-order permutation.
 #pragma once
 #include "common.cuh"
+#include "sort.cuh"
 
 namespace opattr {
 
 // Sets F_K_UNSORTED unless (start_ns, stream) is non-decreasing along the
 // array, and records min / max start in MM_KSTART_MIN / MM_KSTART_MAX.  With
-// stream_hist (256 zeroed counters), also counts the kernels of each stream.
+// stream_hist (256 zeroed counters), also counts the kernels of each stream;
+// with tile_hist (radix_hist_elems(n) counters), writes the stream counts of
+// every RADIX_TILE tile of the array as a stream-major matrix.
 void check_kernel_order(Ctx &c, const uint8_t *stream, const int64_t *start, int64_t n,
-                        uint32_t *stream_hist = nullptr);
+                        uint32_t *stream_hist = nullptr, uint32_t *tile_hist = nullptr);
 
 // Scratch (bytes) of kernel_time_order for n kernels.
 size_t kernel_order_scratch(int64_t n);
