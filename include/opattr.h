@@ -21,7 +21,11 @@
  *    tables, the summaries and totals) live in HOST memory.
  *  - Work is ordered on the context's CUDA stream.  A call returns once its
  *    small host-side results have been copied back; the device outputs are
- *    then complete on that stream.
+ *    then complete on that stream.  Inside a call, independent steps may run
+ *    on a second stream the context owns, forked from and joined back into
+ *    the caller's stream before the call returns.
+ *  - Each call of the library is one NVTX range named after its entry point
+ *    (visible on an Nsight Systems timeline).
  *  - n == 0 is valid everywhere and yields empty results.
  *  - Return value: negative = error (outputs undefined; the context stays
  *    usable except after OPATTR_E_CUDA, after which it must be destroyed),
@@ -329,10 +333,17 @@ opattr_status opattr_aggregate(opattr_ctx *ctx, const opattr_kernels *kernels, c
  * arguments and outputs as the three calls (range_of_kernel is written by the
  * enclosure and read by the aggregation, ncu_idx_of_kernel likewise from the
  * matching).  The kernel records' time order is verified once for both the
- * enclosure and the matching.
+ * enclosure and the matching.  With as many ncu rows as kernels (no
+ * deduplication, no per-stream rows), the identity pairing of the matching
+ * runs beside the enclosure and, when the kernels are in time order, the
+ * enclosure's verdict is read with the aggregation's status: the outputs are
+ * those of the three calls all the same (a disagreeing name redoes the
+ * matching and the aggregation; ranges that need the enclosure's fully
+ * sorted pass run the join again).
  *   n_op_enclosing, match_kind, host_summary, host_totals  may be NULL
- * Returns the first error of the three steps (later steps are not run), else
- * the matching's warning if it gave one, else OPATTR_OK. */
+ * Returns the first error of the three steps in step order (an error of the
+ * enclosure is returned even when the aggregation already ran), else the
+ * matching's warning if it gave one, else OPATTR_OK. */
 opattr_status opattr_join(opattr_ctx *ctx, const opattr_kernels *kernels, const opattr_ranges *ranges,
                           const opattr_ncu *ncu, const opattr_dedup *dedup, uint32_t n_ops,
                           int32_t *range_of_kernel, uint8_t *n_op_enclosing, int32_t *ncu_idx_of_kernel,

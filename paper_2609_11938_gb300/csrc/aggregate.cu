@@ -317,7 +317,9 @@ __device__ __forceinline__ int32_t range_of_t(const int32_t *rok, const uint32_t
 // an operator below n_ops, row index in [-1, M).  Totals: all / attributed
 // time, attributed and matched kernel counts.  Whether every kernel's row is
 // its own index (the match of a trace whose ncu rows follow the kernels one
-// for one) is noted, so the ops pass can skip the row-index gather.  Each
+// for one) is noted, so the ops pass can skip the row-index gather; with
+// ident_rows (a join whose matching was that identity pairing) the row
+// indices are known to be the kernel indices and are not read.  Each
 // attributed kernel (valid range and op id) also takes its slot among its
 // op's kernels: one atomic per distinct op id of a warp on cnt[op], whose old
 // value plus the kernel's rank among its warp peers is the slot (rank[k]);
@@ -331,7 +333,7 @@ template <bool DIRECT>
 __global__ void __launch_bounds__(256, 5) k_agg_count(const int64_t *__restrict__ dur, const int32_t *__restrict__ rok,
                             const int32_t *__restrict__ nidx, const uint32_t *__restrict__ r_op, int64_t K, int64_t R,
                             int64_t M, int64_t n_ops, uint32_t *__restrict__ cnt, uint32_t *__restrict__ rank,
-                            int64_t run, unsigned *__restrict__ nonident, DevStatus *st) {
+                            int64_t run, int ident_rows, unsigned *__restrict__ nonident, DevStatus *st) {
     const unsigned lane = lane_id(), lt = lanemask_lt();
     const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / 32;
     const int64_t nwarps = (int64_t)gridDim.x * blockDim.x / 32;
@@ -346,7 +348,7 @@ __global__ void __launch_bounds__(256, 5) k_agg_count(const int64_t *__restrict_
         int32_t r_c = k < k1 ? range_of_t<DIRECT>(rok, r_op, k) : -1;
         uint32_t op_c = op_of(r_c);
         long long d_c = k < k1 ? dur[k] : 0;
-        int32_t j_c = k < k1 ? nidx[k] : -1;
+        int32_t j_c = k < k1 ? (ident_rows ? (int32_t)k : nidx[k]) : -1;
         int32_t r_n = k + 32 < k1 ? range_of_t<DIRECT>(rok, r_op, k + 32) : -1;
         for (int64_t kb = k0; kb < k1; kb += 32) {
             k = kb + lane;
@@ -357,7 +359,7 @@ __global__ void __launch_bounds__(256, 5) k_agg_count(const int64_t *__restrict_
             r_c = r_n;
             op_c = op_of(r_n);
             d_c = k + 32 < k1 ? dur[k + 32] : 0;
-            j_c = k + 32 < k1 ? nidx[k + 32] : -1;
+            j_c = k + 32 < k1 ? (ident_rows ? (int32_t)(k + 32) : nidx[k + 32]) : -1;
             r_n = k + 64 < k1 ? range_of_t<DIRECT>(rok, r_op, k + 64) : -1;
             nid |= in && (int64_t)j != k;
             bool valid = in;
@@ -1051,7 +1053,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     if (K > 0)
         launch(c, "agg_count", rok ? k_agg_count<false> : k_agg_count<true>,
                dim3(grid_for(K, 256 / 32 * run, 65535)), dim3(256), 0, kern->dur_ns, rok, nidx, rng->op_id, K, R, M,
-               O, cnt, tmp, run, nonident, c.d_status);
+               O, cnt, tmp, run, (int)(c.in_join && c.rows_identity), nonident, c.d_status);
     AggIn in;
     in.dur = kern->dur_ns;
     in.ncu_idx = nidx;

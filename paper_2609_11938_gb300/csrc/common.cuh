@@ -119,6 +119,9 @@ struct Ctx {
     // verdict is pending until then (enclose_pending; the aggregation keeps
     // the status block instead of resetting it)
     bool defer_status = false, enclose_pending = false;
+    // within a join: the matching was the identity pairing (row k for kernel
+    // k), so the aggregation need not read the row indices
+    bool rows_identity = false;
     int64_t launches = 0;
     bool timing = false;
     std::string timing_only;         // with timing on: bracket only this kernel (empty = all)

@@ -384,6 +384,7 @@ static void stream_pairs(Ctx &c, const opattr_kernels *kern, const opattr_ncu *n
 opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu, const opattr_dedup *dd,
                        int32_t *out_idx, uint8_t *out_kind, opattr_match_summary *sum) {
     const int64_t K = kern->n, M = ncu->n;
+    c.rows_identity = false;
     if (K < 0 || M < 0 || K >= (1ll << 31) || M >= (1ll << 31)) return OPATTR_E_INVALID_ARG;
     if (K > 0 && (!kern->stream || !kern->start_ns || !kern->name_id || !out_idx)) return OPATTR_E_INVALID_ARG;
     if (M > 0 && !ncu->name_id) return OPATTR_E_INVALID_ARG;
@@ -422,6 +423,7 @@ opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu
         S.direct = K;
         S.fast_path = 1;
         if (sum) *sum = S;
+        c.rows_identity = true;
         return OPATTR_OK;
     }
     Need nd;

@@ -827,6 +827,31 @@ def test_join_stops_at_the_first_error(opa):
         ctx.close()
 
 
+def test_join_nesting_error_with_deferred_status(opa):
+    """A join whose matching is the identity pairing run beside the
+    enclosure (kernels in (start, stream) order, one row per kernel with the
+    same name) reads the enclosure's status with the aggregation's; a
+    nesting error found there is still the join's status, and the context
+    goes on."""
+    u = _nesting_trace("orphan")
+    order = np.lexsort((u.k_stream, u.k_start))          # strict time order: the deferred path
+    u.k_stream, u.k_start = u.k_stream[order].copy(), u.k_start[order].copy()
+    assert u.K == u.M
+    ctx = opa.Context(0)
+    try:
+        with pytest.raises(opa.OpattrError) as ei:
+            ctx.join(opa.to_device(u))
+        assert ei.value.status == opa.E_NOT_NESTED
+        t = tracegen.generate("tiny")
+        st, out, ops, summ, tot = ctx.join(opa.to_device(t))
+        o = oracle.run(t, enclose_mode="brute")
+        np.testing.assert_array_equal(out["range_of_kernel"].cpu().numpy(), o["range_of_kernel"])
+        np.testing.assert_array_equal(out["ncu_idx"].cpu().numpy(), o["ncu_idx"])
+        assert summ["fast_path"] == 1
+    finally:
+        ctx.close()
+
+
 def _equal_starts_trace():
     """Ranges sorted by start whose equal-start pairs at one depth are not in
     (start, end) order -- a long range listed before a zero-length one at the
