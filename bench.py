@@ -429,9 +429,13 @@ def main():
     for _ in range(args.warmup):
         step()
     sync()
-    # rows matched one for one (the ops pass then skips the row-index gather)
+    # rows matched one for one (the ops pass then skips the row-index gather;
+    # in a join whose matching was that identity pairing, the count pass too)
     if K > 0 and bool((idx == torch.arange(K, dtype=torch.int32, device=idx.device)).all()):
         KERNEL_BYTES["agg_ops"] = lambda K, R, M, O: 92 * K + 188 * O
+        if (tq is tr and tiers_out is None and not use_dedup and not args.per_stream_ncu and M == K
+                and not args.shuffle):
+            KERNEL_BYTES["agg_count"] = lambda K, R, M, O: 20 * K + 4 * O
     # per-kernel breakdown: a few steps with every launch bracketed by events
     n_brk = max(1, min(args.steps, 10))
     ctx.set_timing(True)
