@@ -278,7 +278,9 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", default="large", choices=sorted(WORKLOADS))
     ap.add_argument("--shuffle", action="store_true", help="permute kernel and range arrays (general paths)")
-    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--e2e-steps", type=int, default=8)
+    ap.add_argument("--e2e-copy-streams", type=int, default=2,
+                    help="copy streams per direction in the end-to-end run")
     ap.add_argument("--no-oracle-single", dest="oracle_single", action="store_false",
                     help="skip the single-thread oracle run of the CPU baseline (it takes about 15 s on large)")
     ap.add_argument("--per-stream-ncu", action="store_true",
@@ -390,24 +392,30 @@ def main():
 
     join_out = dict(range_of_kernel=rk, n_op_enclosing=nop, ncu_idx=idx, match_kind=kind)
 
-    def join():
-        if tq is tr and tiers_out is None:
-            # the whole join in one call (one kernel-order check for both steps)
-            ctx.join(tr, dedup=use_dedup, out=join_out, ops=ops)
+    def make_join(tr, tq, join_out, ops, tiers_out, rollup_out):
+        rk, nop, idx, kind = (join_out[k] for k in ("range_of_kernel", "n_op_enclosing", "ncu_idx", "match_kind"))
+
+        def join():
+            if tq is tr and tiers_out is None:
+                # the whole join in one call (one kernel-order check for both steps)
+                ctx.join(tr, dedup=use_dedup, out=join_out, ops=ops)
+                if rollup_out is not None:
+                    ctx.rollup(tr, rk, idx, class_of_op, args.rollup, out=rollup_out)
+                return
+            ctx.enclose(tq, rk, nop)
+            if tiers_out is not None:
+                ctx.attribute(tr, rk, nop, out=tiers_out)
+            ctx.match(tr, dedup=use_dedup, out_idx=idx, out_kind=kind)
+            if tiers_out is not None:
+                ctx.aggregate(tr, None, idx, ops, op_of_kernel=tiers_out["op"])
+            else:
+                ctx.aggregate(tr, rk, idx, ops)
             if rollup_out is not None:
-                ctx.rollup(tr, rk, idx, class_of_op, args.rollup, out=rollup_out)
-            return
-        ctx.enclose(tq, rk, nop)
-        if tiers_out is not None:
-            ctx.attribute(tr, rk, nop, out=tiers_out)
-        ctx.match(tr, dedup=use_dedup, out_idx=idx, out_kind=kind)
-        if tiers_out is not None:
-            ctx.aggregate(tr, None, idx, ops, op_of_kernel=tiers_out["op"])
-        else:
-            ctx.aggregate(tr, rk, idx, ops)
-        if rollup_out is not None:
-            ctx.rollup(tr, rk, idx, class_of_op, args.rollup, out=rollup_out,
-                       op_of_kernel=tiers_out["op"] if tiers_out is not None else None)
+                ctx.rollup(tr, rk, idx, class_of_op, args.rollup, out=rollup_out,
+                           op_of_kernel=tiers_out["op"] if tiers_out is not None else None)
+        return join
+
+    join = make_join(tr, tq, join_out, ops, tiers_out, rollup_out)
     in_bytes = sum(x.numel() * x.element_size() for x in (tr.k_stream, tr.k_start, tr.k_dur, tr.k_name,
                                                            tr.r_stream, tr.r_start, tr.r_end, tr.r_depth, tr.r_op,
                                                            tr.ncu_name, tr.counters))
@@ -473,40 +481,110 @@ def main():
     clocks.stop()
     t_max, units = combine_ranks(max(elapsed, 1e-9), K * args.steps, world, rmax, rsum)
 
-    # ---- end to end through the C ABI with host buffers (pinned), per step:
-    # H2D of every input array, the join, D2H of every output
-    host = {name: torch.from_numpy(getattr(trace, name)).pin_memory()
-            for name in ("k_stream", "k_start", "k_dur", "k_name", "r_stream", "r_start", "r_end", "r_depth",
-                         "r_op", "ncu_name", "counters") + (("corr_name", "corr_inv", "corr_op", "fusion_op",
-                                                             "fusion_len") if args.tiers else ())}
+    # ---- end to end through the C ABI with host buffers (pinned): every step
+    # copies each input array host->device, runs the join and copies each
+    # output device->host.  Steps overlap the way a caller streaming traces
+    # would run them: step i+1's inputs go over on copy streams while step i's
+    # join runs (two device buffer sets, used in turn), and step i's outputs
+    # come back on other copy streams while step i+1 runs.
+    in_names = ("k_stream", "k_start", "k_dur", "k_name", "r_stream", "r_start", "r_end", "r_depth", "r_op",
+                "ncu_name", "counters")
+    if args.tiers:
+        in_names += ("corr_name", "corr_inv", "corr_op", "fusion_op", "fusion_len")
     if trace.k_layer is not None:
-        host["k_layer"] = torch.from_numpy(trace.k_layer).pin_memory()
-    if tq is not tr:
-        launch_host = tq.k_start.cpu().pin_memory()
+        in_names += ("k_layer",)
+    if getattr(trace, "ncu_stream", None) is not None:
+        in_names += ("ncu_stream",)
+    host = {name: torch.from_numpy(getattr(trace, name)).pin_memory() for name in in_names}
+    launch_host = tq.k_start.cpu().pin_memory() if tq is not tr else None
+
+    def device_copy(t):
+        return dataclasses.replace(t, **{f.name: getattr(t, f.name).clone() for f in dataclasses.fields(t)
+                                         if torch.is_tensor(getattr(t, f.name))})
+
+    def buffer_set(tr_b, tq_b, join_out_b, ops_b, tiers_b, rollup_b):
+        return dict(tr=tr_b, tq=tq_b, rk=join_out_b["range_of_kernel"], idx=join_out_b["ncu_idx"], ops=ops_b,
+                    join=make_join(tr_b, tq_b, join_out_b, ops_b, tiers_b, rollup_b))
+
+    tr2 = device_copy(tr)
+    tq2 = tr2 if tq is tr else dataclasses.replace(tr2, k_start=tq.k_start.clone())
+    join_out2 = {k: torch.empty_like(v) for k, v in join_out.items()}
+    ops2 = ctx.alloc_ops(O)
+    tiers2 = {k: torch.empty_like(v) for k, v in tiers_out.items()} if tiers_out is not None else None
+    rollup2 = ctx.alloc_ops(args.rollup) if rollup_out is not None else None
+    sets = [buffer_set(tr, tq, join_out, ops, tiers_out, rollup_out),
+            buffer_set(tr2, tq2, join_out2, ops2, tiers2, rollup2)]
     out_host = {"rk": torch.empty(K, dtype=torch.int32).pin_memory(),
                 "idx": torch.empty(K, dtype=torch.int32).pin_memory()}
     out_host.update({k: torch.empty_like(v, device="cpu").pin_memory() for k, v in ops.items()})
     h2d = sum(v.numel() * v.element_size() for v in host.values())
-    if tq is not tr:
+    if launch_host is not None:
         h2d += launch_host.numel() * launch_host.element_size()
     d2h = sum(v.numel() * v.element_size() for v in out_host.values())
+    n_cs = max(1, args.e2e_copy_streams)
+    copy_in = [torch.cuda.Stream(dev) for _ in range(n_cs)]
+    copy_out = [torch.cuda.Stream(dev) for _ in range(n_cs)]
+    in_ev = [[torch.cuda.Event() for _ in range(n_cs)] for _ in range(2)]
+    out_ev = [[torch.cuda.Event() for _ in range(n_cs)] for _ in range(2)]
 
-    def e2e_step():
-        with torch.cuda.stream(stream):
-            for name, v in host.items():
-                getattr(tr, name).copy_(v, non_blocking=True)
-            if tq is not tr:
-                tq.k_start.copy_(launch_host, non_blocking=True)
-        join()
-        with torch.cuda.stream(stream):
-            out_host["rk"].copy_(rk, non_blocking=True)
-            out_host["idx"].copy_(idx, non_blocking=True)
-            for k, v in ops.items():
-                out_host[k].copy_(v, non_blocking=True)
+    def spread(pairs, streams):
+        """Copies dst <- src, arrays of 64 MB or more cut into one piece per stream."""
+        j = 0
+        for dst, src in pairs:
+            n = dst.shape[0]
+            parts = len(streams) if src.numel() * src.element_size() >= (64 << 20) else 1
+            for p in range(parts):
+                lo, hi = n * p // parts, n * (p + 1) // parts
+                with torch.cuda.stream(streams[j % len(streams)]):
+                    dst[lo:hi].copy_(src[lo:hi], non_blocking=True)
+                j += 1
+
+    def send(b):
+        s = sets[b]
+        pairs = [(getattr(s["tr"], name), v) for name, v in host.items()]
+        if launch_host is not None:
+            pairs.append((s["tq"].k_start, launch_host))
+        spread(pairs, copy_in)
+        for q in range(n_cs):
+            in_ev[b][q].record(copy_in[q])
+
+    def receive(b):
+        s = sets[b]
+        for q in range(n_cs):
+            copy_out[q].wait_stream(stream)
+        pairs = [(out_host["rk"], s["rk"]), (out_host["idx"], s["idx"])]
+        pairs += [(out_host[k], v) for k, v in s["ops"].items()]
+        spread(pairs, copy_out)
+        for q in range(n_cs):
+            out_ev[b][q].record(copy_out[q])
+
+    def e2e_run(n):
+        send(0)
+        for i in range(n):
+            b = i & 1
+            if i + 1 < n:
+                send(1 - b)         # set 1 - b was last read by join i - 1, which has returned
+            for q in range(n_cs):
+                stream.wait_event(in_ev[b][q])
+                stream.wait_event(out_ev[b][q])     # step i - 2's outputs are off the device
+            sets[b]["join"]()
+            receive(b)
+
+    def sync_all():
+        for cs in copy_in + copy_out:
+            cs.synchronize()
         stream.synchronize()
 
-    e2e_step()
-    e2e_s = run_timed(e2e_step, args.e2e_steps, 1, sync, barrier)
+    e2e_run(2)
+    sync_all()
+    barrier()
+    sync_all()
+    t0 = time.perf_counter()
+    e2e_run(args.e2e_steps)
+    sync_all()
+    barrier()
+    sync_all()
+    e2e_s = time.perf_counter() - t0
     e2e_t, e2e_units = combine_ranks(e2e_s, K * args.e2e_steps, world, rmax, rsum)
 
     if rank != 0:

@@ -1013,7 +1013,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
 
     Need nd;
     nd.add<uint32_t>(O + 1).add<uint32_t>(O + 1).add<uint32_t>(K).add<uint32_t>(K);
-    nd.add<uint32_t>(O + 1).add<unsigned>(1).add<unsigned>(2).add<unsigned>(1).add<uint32_t>(O + 1);
+    nd.add<uint32_t>(O + 1).add<unsigned>(3).add<unsigned>(1).add<uint32_t>(O + 1);
     nd.add<uint32_t>(O + 1).add<Acc>(K / AG_PIECE + (K / (AG_SHORT_MAX + 1)) + 1);   // pieces per op, partials
     nd.add<uint32_t>(scan_scratch_elems(std::max<int64_t>(O + 1, radix_hist_elems(K))));
     nd.add<uint32_t>(O + 1).add<uint32_t>(radix_hist_elems(K)).add<uint32_t>(8);   // huge-op index, histogram, info
@@ -1028,21 +1028,22 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
     // tmp holds each kernel's slot among its op's kernels until the list is
     // placed, then serves the segment sorts
     uint32_t *list = a.take<uint32_t>(K), *tmp = a.take<uint32_t>(K), *longs = a.take<uint32_t>(O + 1);
-    unsigned *nlong = a.take<unsigned>(1);
-    unsigned *ctr = a.take<unsigned>(2);
+    // ctr[0] next chunk, ctr[1] ops listed dirty, ctr[2] (nlong) ops listed long:
+    // the two counts come back together
+    unsigned *ctr = a.take<unsigned>(3);
+    unsigned *nlong = ctr ? ctr + 2 : nullptr;
     unsigned *nonident = a.take<unsigned>(1);
     uint32_t *dirty = a.take<uint32_t>(O + 1);
     uint32_t *npc = a.take<uint32_t>(O + 1);
     Acc *partials = a.take<Acc>(K / AG_PIECE + (K / (AG_SHORT_MAX + 1)) + 1);
     if (!npc || !partials) return OPATTR_E_OOM;
-    cudaMemsetAsync(ctr, 0, 2 * sizeof(unsigned), c.stream);
+    cudaMemsetAsync(ctr, 0, 3 * sizeof(unsigned), c.stream);
     uint32_t *part = a.take<uint32_t>(scan_scratch_elems(std::max<int64_t>(O + 1, radix_hist_elems(K))));
     uint32_t *hidx = a.take<uint32_t>(O + 1), *hhist = a.take<uint32_t>(radix_hist_elems(K));
     uint32_t *info = a.take<uint32_t>(8), *hop = a.take<uint32_t>(O + 1);
     if (!hidx || !hhist || !info || !hop) return OPATTR_E_OOM;
     if (!cnt || !off || !list || !tmp || !longs || !nlong || !part || !nonident || !dirty) return OPATTR_E_OOM;
     cudaMemsetAsync(cnt, 0, sizeof(uint32_t) * (O + 1), c.stream);
-    cudaMemsetAsync(nlong, 0, sizeof(unsigned), c.stream);
     cudaMemsetAsync(nonident, 0, sizeof(unsigned), c.stream);
     int sms = 0;
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, c.device);
@@ -1083,8 +1084,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
         // the ops the pass left: listed with a null or infinite value (redone
         // by k_agg_careful), long ones (the pieces pass); both
         // counts come back with the status
-        cudaMemcpyAsync(c.h_levels, ctr + 1, sizeof(uint32_t), cudaMemcpyDeviceToHost, c.stream);
-        cudaMemcpyAsync(c.h_levels + 1, nlong, sizeof(uint32_t), cudaMemcpyDeviceToHost, c.stream);
+        if ((st = copy_small(c, c.h_levels, ctr + 1, 2 * sizeof(uint32_t), cudaMemcpyDeviceToHost))) return st;
         if ((st = read_status(c))) return st;
         const uint32_t n_dirty = c.h_levels[0], n_long = c.h_levels[1];
         status_fresh = n_dirty == 0 && n_long == 0;
@@ -1095,7 +1095,7 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
         if (n_long > 0) {
             launch(c, "agg_piece_offsets", k_agg_piece_offsets, dim3(1), dim3(1024), 0, (const uint32_t *)off,
                    (const uint32_t *)longs, (const unsigned *)nlong, 0u, npc, info, hop);
-            cudaMemcpyAsync(c.h_levels, info, 5 * sizeof(uint32_t), cudaMemcpyDeviceToHost, c.stream);
+            if ((st = copy_small(c, c.h_levels, info, 5 * sizeof(uint32_t), cudaMemcpyDeviceToHost))) return st;
             if ((st = read_status(c))) return st;
             pieces = c.h_levels[1];
             longest = c.h_levels[2];

@@ -108,15 +108,39 @@ opattr_status ensure_side(Ctx &c) {
     return OPATTR_OK;
 }
 
+// Bytes from src to dst, one of them in mapped pinned host memory: words
+// when both ends and the size are 4-byte aligned (every caller's case).
+__global__ void k_copy_small(const unsigned char *__restrict__ src, unsigned char *__restrict__ dst, size_t n) {
+    const size_t t0 = (size_t)blockIdx.x * blockDim.x + threadIdx.x, step = (size_t)gridDim.x * blockDim.x;
+    if (((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst) | n) & 3u) == 0) {
+        const uint32_t *s = reinterpret_cast<const uint32_t *>(src);
+        uint32_t *d = reinterpret_cast<uint32_t *>(dst);
+        for (size_t i = t0; i < n / 4; i += step) d[i] = s[i];
+    } else {
+        for (size_t i = t0; i < n; i += step) dst[i] = src[i];
+    }
+}
+
+opattr_status copy_small(Ctx &c, void *dst, const void *src, size_t bytes, cudaMemcpyKind kind) {
+    if (bytes == 0) return OPATTR_OK;
+    if (!c.host_mapped) {
+        const cudaError_t e = cudaMemcpyAsync(dst, src, bytes, kind, c.stream);
+        return e == cudaSuccess ? OPATTR_OK : cuda_status(c, e);
+    }
+    launch(c, "small_copy", k_copy_small, dim3(grid_for((int64_t)bytes, 256 * 16, 8)), dim3(256), 0,
+           static_cast<const unsigned char *>(src), static_cast<unsigned char *>(dst), bytes);
+    return c.last_error == cudaSuccess ? OPATTR_OK : cuda_status(c, c.last_error);
+}
+
 opattr_status reset_status(Ctx &c) {
-    cudaError_t e = cudaMemcpyAsync(c.d_status, c.h_init, sizeof(DevStatus), cudaMemcpyHostToDevice, c.stream);
-    return e == cudaSuccess ? OPATTR_OK : cuda_status(c, e);
+    return copy_small(c, c.d_status, c.h_init, sizeof(DevStatus), cudaMemcpyHostToDevice);
 }
 
 opattr_status read_status(Ctx &c) {
     if (c.last_error != cudaSuccess) return cuda_status(c, c.last_error);
-    cudaError_t e = cudaMemcpyAsync(c.h_status, c.d_status, sizeof(DevStatus), cudaMemcpyDeviceToHost, c.stream);
-    if (e == cudaSuccess) e = cudaStreamSynchronize(c.stream);
+    opattr_status st = copy_small(c, c.h_status, c.d_status, sizeof(DevStatus), cudaMemcpyDeviceToHost);
+    if (st) return st;
+    cudaError_t e = cudaStreamSynchronize(c.stream);
     if (e != cudaSuccess) return cuda_status(c, e);
     if (c.timing) timing_collect(c);
     // a chained prefix that gave up waiting leaves results that do not count
@@ -227,6 +251,15 @@ opattr_status opattr_create(opattr_ctx **out, int device, void *cuda_stream, con
         delete x;
         return OPATTR_E_OOM;
     }
+    // the pinned buffers are moved by small kernels when the device sees them
+    // at their host addresses (unified addressing), by cudaMemcpyAsync if not
+    bool mapped = true;
+    for (void *h : {(void *)c.h_status, (void *)c.h_init, (void *)c.h_levels, (void *)c.h_stage}) {
+        void *dp = nullptr;
+        mapped = mapped && cudaHostGetDevicePointer(&dp, h, 0) == cudaSuccess && dp == h;
+    }
+    cudaGetLastError();
+    c.host_mapped = mapped;
     memset(c.h_init, 0, sizeof(DevStatus));
     c.h_init->mm[MM_KSTART_MIN] = LLONG_MAX;
     c.h_init->mm[MM_KSTART_MAX] = LLONG_MIN;

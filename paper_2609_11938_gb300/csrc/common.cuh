@@ -94,6 +94,7 @@ struct Ctx {
                                      // kernels per stream [256];
                                      // the aggregation reuses it for a few values read mid-call
     unsigned char *h_stage = nullptr; // pinned staging for small host-built tables [STAGE_BYTES]
+    bool host_mapped = false;        // the four pinned buffers above are addressable from the device as they are
     // kernel time order as the last enclosure found it (-1 unknown, 0 / 1),
     // and whether the matching may take it instead of checking again (join)
     int enclose_k_sorted = -1;
@@ -176,6 +177,13 @@ inline void stream_after(cudaStream_t to, cudaStream_t from, cudaEvent_t e) {
     cudaEventRecord(e, from);
     cudaStreamWaitEvent(to, e, 0);
 }
+// A small transfer between the context's pinned host buffers and device
+// memory, on c.stream.  When those buffers are mapped into the device's
+// address space (opattr_create checks), a small kernel moves the bytes through
+// the mapping instead of a copy engine, so a call's status reads and table
+// uploads never queue behind bulk copies that the caller has on the engines;
+// otherwise (host mirrors in plain host memory) cudaMemcpyAsync.
+opattr_status copy_small(Ctx &c, void *dst, const void *src, size_t bytes, cudaMemcpyKind kind);
 opattr_status reset_status(Ctx &c);
 opattr_status read_status(Ctx &c);      // D2H copy + stream synchronize
 opattr_status cuda_status(Ctx &c, cudaError_t e);

@@ -645,14 +645,12 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
                    dim3(RCHK_THREADS), 0, rng->stream, rng->start_ns, rng->end_ns, rng->depth, R, level_hist,
                    c.d_status);
         scan_exclusive_u32(c, level_hist, lvl_off, LEVELS + 1, part2, nullptr);
-        if (cudaMemcpyAsync(c.h_levels, lvl_off, sizeof(uint32_t) * (LEVELS + 1), cudaMemcpyDeviceToHost,
-                            c.stream) != cudaSuccess)
-            return cuda_status(c, cudaGetLastError());
+        if ((st = copy_small(c, c.h_levels, lvl_off, sizeof(uint32_t) * (LEVELS + 1), cudaMemcpyDeviceToHost)))
+            return st;
     }
     check_kernel_order(c, kern->stream, kern->start_ns, K, kstream, ktile);
-    if (cudaMemcpyAsync(c.h_levels + LEVELS + 1, kstream, sizeof(uint32_t) * 256, cudaMemcpyDeviceToHost, c.stream) !=
-        cudaSuccess)
-        return cuda_status(c, cudaGetLastError());
+    if ((st = copy_small(c, c.h_levels + LEVELS + 1, kstream, sizeof(uint32_t) * 256, cudaMemcpyDeviceToHost)))
+        return st;
     stream_after(c.stream, c.side, c.ev_join);
     if ((st = read_status(c))) return st;
     if ((st = status_from_err(c.h_status->err))) return st;
@@ -732,7 +730,7 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     const uint32_t *d_kcnt = reinterpret_cast<const uint32_t *>(d_stage + ST_KCNT);
     const uint32_t *d_toff = reinterpret_cast<const uint32_t *>(d_stage + ST_TOFF);
     const uint8_t *d_scmap = d_stage + ST_SCMAP;
-    cudaMemcpyAsync(d_stage, c.h_stage, ST_END, cudaMemcpyHostToDevice, c.stream);
+    if ((st = copy_small(c, d_stage, c.h_stage, ST_END, cudaMemcpyHostToDevice))) return st;
     // the level lists (below) may start on the side stream from here
     stream_after(c.side, c.stream, c.ev_fork);
 
