@@ -1108,10 +1108,10 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
                 launch(c, "huge_index", k_huge_index, dim3(grid_for(n_huge, 256, 4096)), dim3(256), 0,
                        (const uint32_t *)hop, (int64_t)n_huge, hidx);
                 const HugeDigit dg{rok, rng->op_id, R, O, hidx};
-                digit_offsets(c, dg, K, hhist, part);
+                const uint32_t *hoffs = digit_offsets(c, dg, K, hhist, part);
                 const int64_t ntiles = (K + RADIX_TILE - 1) / RADIX_TILE;
-                digit_rank(c, "huge_place", dg, K, hhist,
-                           HugePlace{hhist, ntiles, (const uint32_t *)hop, (const uint32_t *)off, list});
+                digit_rank(c, "huge_place", dg, K, hoffs,
+                           HugePlace{hoffs, ntiles, (const uint32_t *)hop, (const uint32_t *)off, list});
             } else {
                 launch(c, "agg_sort_long", k_agg_sort_long, dim3(2 * std::max(1, sms)), dim3(SL_THREADS), 0,
                        (const uint32_t *)off, (const uint32_t *)longs, (const unsigned *)nlong, 2u,

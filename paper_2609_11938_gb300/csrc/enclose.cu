@@ -737,7 +737,8 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
     // ---- kernel time order, then the kernels partitioned by stream
     uint32_t *korder = nullptr;
     if (!k_sorted && K > 0) {
-        korder = kernel_time_order(c, a, kern->stream, kern->start_ns, K);
+        // keyed by the compact ids of the streams with kernels
+        korder = kernel_time_order(c, a, kern->stream, kern->start_ns, K, d_scmap, bits_for((uint64_t)(nks - 1)));
         if (!korder) return OPATTR_E_OOM;
         if (kept_order) {
             cudaMemcpyAsync(kept_order, korder, sizeof(uint32_t) * K, cudaMemcpyDeviceToDevice, c.stream);

@@ -375,10 +375,10 @@ static void stream_pairs(Ctx &c, const opattr_kernels *kern, const opattr_ncu *n
     radix_sort_pairs<uint8_t>(c, const_cast<uint8_t *>(ncu->stream), nv0, nb, nv1, n, 8, true, hist, part, &ko, &pn);
     // kernels: ranked by stream, each paired in the same pass
     const StreamDigit dg{rk, kern->stream};
-    digit_offsets(c, dg, n, hist, part);
+    const uint32_t *offs = digit_offsets(c, dg, n, hist, part);
     const StreamPairs ep{rk, pn, kern->name_id, ncu->name_id, kern->stream, ncu->stream, out_idx, out_kind,
                          c.d_status};
-    digit_rank(c, "match_stream_pairs", dg, n, hist, ep);
+    digit_rank(c, "match_stream_pairs", dg, n, offs, ep);
 }
 
 opattr_status do_match(Ctx &c, const opattr_kernels *kern, const opattr_ncu *ncu, const opattr_dedup *dd,

@@ -4,8 +4,8 @@
 // A scan out of place is one pass: tiles chain their prefixes by decoupled
 // look-back (warp_lookback_exclusive in sort.cuh, a bounded wait on tiles
 // that started earlier); a scan in place is three launches with no waits.  A
-// radix sort pass is three launches (tile histograms -> scan of the histogram
-// matrix -> scatter).
+// radix sort pass is three launches (tile histograms -> single-pass scan of
+// the histogram matrix, out of place -> scatter).
 #include <cstdlib>
 #include <cstring>
 
@@ -328,15 +328,17 @@ void radix_sort_pairs(Ctx &c, K *k0, uint32_t *v0, K *k1, uint32_t *v1, int64_t 
     K *ka = k0, *kb = k1;
     uint32_t *va = v0, *vb = v1;
     const int64_t ntiles = (n + RADIX_TILE - 1) / RADIX_TILE;
+    // the tiles' digit counts, then their scan (out of place, one pass)
+    uint32_t *hcount = hist, *hoff = hist + ntiles * RADIX_BINS;
     if (iota && bits <= 0) bits = 1;   // equal keys: one pass still writes the indices
     for (int shift = 0; shift < bits && n > 0; shift += RADIX_BITS) {
         const bool first = shift == 0;
         launch(c, "radix_upsweep", k_radix_upsweep<K>, dim3((unsigned)ntiles), dim3(RADIX_THREADS), 0,
-               (const K *)ka, n, shift, hist, ntiles);
-        scan_exclusive_u32(c, hist, hist, ntiles * RADIX_BINS, partials, nullptr);
+               (const K *)ka, n, shift, hcount, ntiles);
+        scan_exclusive_u32(c, hcount, hoff, ntiles * RADIX_BINS, partials, nullptr);
         launch(c, "radix_downsweep", k_radix_downsweep<K>, dim3((unsigned)ntiles), dim3(RADIX_THREADS),
                downsweep_smem<K>(), (const K *)ka, (const uint32_t *)((first && iota) ? nullptr : va), kb, vb, n,
-               shift, (const uint32_t *)hist, ntiles);
+               shift, (const uint32_t *)hoff, ntiles);
         K *tk = ka; ka = kb; kb = tk;
         uint32_t *tv = va; va = vb; vb = tv;
     }

@@ -23,16 +23,19 @@ inline int64_t scan_scratch_elems(int64_t n) { return 2 * ((n + SCAN_TILE - 1) /
 void scan_exclusive_u32(Ctx &c, const uint32_t *in, uint32_t *out, int64_t n, uint32_t *partials,
                         uint32_t *total_dev);
 
-// Scratch for a radix sort of n keys: histogram matrix + its scan partials.
+// Scratch for a radix sort or a digit pass over n keys: the tiles' digit
+// counts (a tiles x RADIX_BINS matrix) and, after them, room for their scan
+// out of place (one pass instead of three launches in place).
 inline int64_t radix_hist_elems(int64_t n) {
     int64_t tiles = (n + RADIX_TILE - 1) / RADIX_TILE;
-    return tiles * RADIX_BINS;
+    return 2 * tiles * RADIX_BINS;
 }
 
 // Stable LSD sort of (key, value) pairs on key bits [0, bits), 8 bits per
 // pass.  Ping-pongs between (k0, v0) and (k1, v1), all four n-element device
 // buffers; *kout / *vout receive the buffers that hold the result.  With
-// `iota` the incoming values are ignored and taken to be 0..n-1.
+// `iota` the incoming values are ignored and taken to be 0..n-1.  `hist`
+// holds radix_hist_elems(n) entries, `partials` scan_scratch_elems of that.
 template <typename K>
 void radix_sort_pairs(Ctx &c, K *k0, uint32_t *v0, K *k1, uint32_t *v1, int64_t n, int bits, bool iota,
                       uint32_t *hist, uint32_t *partials, K **kout, uint32_t **vout);
@@ -194,9 +197,9 @@ __global__ void __launch_bounds__(RADIX_THREADS) k_digit_rank(DigitFn digit, int
 }
 
 // nbins: digits used (every digit below it); only those rows of the matrix
-// are counted on and scanned.  With at most RADIX_BINS / 2 digits the scan
-// goes out of place, into the free upper half of `hist` (one pass); the
-// offsets' address is returned for digit_rank.
+// are counted on and scanned.  The scan goes out of place, into the second
+// half of `hist` (radix_hist_elems(n) entries: one pass); the offsets'
+// address is returned for digit_rank.
 template <typename DigitFn>
 uint32_t *digit_offsets(Ctx &c, DigitFn digit, int64_t n, uint32_t *hist, uint32_t *partials,
                         int nbins = RADIX_BINS) {
@@ -205,7 +208,7 @@ uint32_t *digit_offsets(Ctx &c, DigitFn digit, int64_t n, uint32_t *hist, uint32
     launch(c, "digit_hist", k_digit_hist<DigitFn>, dim3((unsigned)ntiles), dim3(RADIX_THREADS), 0, digit, n, hist,
            ntiles);
     const int64_t m = ntiles * (int64_t)(nbins < 1 ? 1 : nbins);
-    uint32_t *offs = nbins <= RADIX_BINS / 2 ? hist + m : hist;
+    uint32_t *offs = hist + ntiles * RADIX_BINS;
     scan_exclusive_u32(c, hist, offs, m, partials, nullptr);
     return offs;
 }

@@ -120,9 +120,12 @@ void check_kernel_order(Ctx &c, const uint8_t *stream, const int64_t *start, int
 }
 
 __global__ void k_time_keys(const uint8_t *__restrict__ stream, const int64_t *__restrict__ start, int64_t n,
-                            long long tmin, uint64_t *__restrict__ keys) {
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
-        keys[i] = ((uint64_t)(start[i] - tmin) << 8) | stream[i];
+                            long long tmin, const uint8_t *__restrict__ scmap, int sbits,
+                            uint64_t *__restrict__ keys) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const unsigned s = scmap ? scmap[stream[i]] : stream[i];
+        keys[i] = ((uint64_t)(start[i] - tmin) << sbits) | s;
+    }
 }
 
 size_t kernel_order_scratch(int64_t n) {
@@ -132,18 +135,21 @@ size_t kernel_order_scratch(int64_t n) {
     return nd.bytes;
 }
 
-uint32_t *kernel_time_order(Ctx &c, Arena &a, const uint8_t *stream, const int64_t *start, int64_t n) {
+uint32_t *kernel_time_order(Ctx &c, Arena &a, const uint8_t *stream, const int64_t *start, int64_t n,
+                            const uint8_t *scmap, int stream_bits) {
     uint64_t *k0 = a.take<uint64_t>(n), *k1 = a.take<uint64_t>(n);
     uint32_t *v0 = a.take<uint32_t>(n), *v1 = a.take<uint32_t>(n);
     uint32_t *hist = a.take<uint32_t>(radix_hist_elems(n));
     uint32_t *part = a.take<uint32_t>(scan_scratch_elems(radix_hist_elems(n)));
     if (!k0 || !k1 || !v0 || !v1 || !hist || !part) return nullptr;
     long long tmin = c.h_status->mm[MM_KSTART_MIN], tmax = c.h_status->mm[MM_KSTART_MAX];
-    launch(c, "time_keys", k_time_keys, dim3(grid_for(n, 256, 65535)), dim3(256), 0, stream, start, n, tmin, k0);
+    const int sbits = scmap ? stream_bits : 8;
+    launch(c, "time_keys", k_time_keys, dim3(grid_for(n, 256, 65535)), dim3(256), 0, stream, start, n, tmin, scmap,
+           sbits, k0);
     uint64_t *ko;
     uint32_t *vo;
-    radix_sort_pairs<uint64_t>(c, k0, v0, k1, v1, n, bits_for((uint64_t)(tmax - tmin)) + 8, true, hist, part, &ko,
-                               &vo);
+    radix_sort_pairs<uint64_t>(c, k0, v0, k1, v1, n, bits_for((uint64_t)(tmax - tmin)) + sbits, true, hist, part,
+                               &ko, &vo);
     return vo;
 }
 

@@ -18,9 +18,13 @@ void check_kernel_order(Ctx &c, const uint8_t *stream, const int64_t *start, int
 size_t kernel_order_scratch(int64_t n);
 
 // Permutation of kernel indices into time order (start, stream, index) by a
-// stable radix sort of ((start - min_start) << 8 | stream).  Needs the
-// min / max from check_kernel_order in c.h_status.  Returns a device array of
-// n indices carved from `a`, or NULL on arena exhaustion.
-uint32_t *kernel_time_order(Ctx &c, struct Arena &a, const uint8_t *stream, const int64_t *start, int64_t n);
+// stable radix sort of ((start - min_start) << sbits | stream).  Needs the
+// min / max from check_kernel_order in c.h_status.  With scmap (device,
+// [256]: increasing compact ids of the streams that have kernels) the key
+// holds the compact id in stream_bits bits instead of the id in 8, which
+// saves a pass when the span and the stream count allow.  Returns a device
+// array of n indices carved from `a`, or NULL on arena exhaustion.
+uint32_t *kernel_time_order(Ctx &c, struct Arena &a, const uint8_t *stream, const int64_t *start, int64_t n,
+                            const uint8_t *scmap = nullptr, int stream_bits = 8);
 
 }  // namespace opattr
