@@ -99,12 +99,17 @@ __global__ void k_level_keys(const uint8_t *__restrict__ stream, const uint8_t *
         keys[i] = (uint32_t)stream[r] * 32u + depth[r];
     }
 }
-__global__ void k_time_key(const int64_t *__restrict__ t, const uint32_t *__restrict__ perm, int64_t n,
-                           long long tmin, uint64_t *__restrict__ keys) {
-    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-        int64_t r = perm ? perm[i] : i;
-        keys[i] = (uint64_t)(t[r] - tmin);
-    }
+// The level lists' order key of range i: its start, then 0 for a
+// zero-length range and 1 for a longer one.  Within a level of laminar
+// ranges two ranges share a start only if all but the last of them have
+// zero length, so a stable sort on this key puts every level in (start,
+// end, index) order -- the order of Algorithm 2's one representative per
+// depth -- in one sort; two longer ranges sharing a start in one level are
+// out of that order only when they overlap, which the validation reports.
+__global__ void k_range_start_key(const int64_t *__restrict__ start, const int64_t *__restrict__ end, int64_t n,
+                                  long long tmin, uint64_t *__restrict__ keys) {
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+        keys[i] = ((uint64_t)(start[i] - tmin) << 1) | (end[i] > start[i] ? 1u : 0u);
 }
 __global__ void k_level_gather(const int64_t *__restrict__ start, const int64_t *__restrict__ end,
                                const uint32_t *__restrict__ op, const uint32_t *__restrict__ perm, int64_t n,
@@ -779,18 +784,13 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
             OnStream on(c, c.side);
             uint32_t *perm = nullptr;     // range indices in the order of the level sort
             if (full_sort) {
-                // (start, end, index) order: sort by end, then stably by start
+                // (start, end, index) order within every level of laminar
+                // ranges: one stable sort on (start, longer than zero)
                 uint64_t *ko;
-                uint32_t *vo;
-                int bits = bits_for((uint64_t)(rmax - rmin));
-                launch(c, "range_time_key", k_time_key, dim3(g), dim3(256), 0, rng->end_ns, (const uint32_t *)nullptr,
-                       R, rmin, rk0);
-                radix_sort_pairs<uint64_t>(c, rk0, rv0, rk1, rv1, R, bits, true, hist2, part2, &ko, &vo);
-                uint64_t *kfree = ko == rk0 ? rk1 : rk0;
-                uint32_t *vfree = vo == rv0 ? rv1 : rv0;
-                launch(c, "range_time_key", k_time_key, dim3(g), dim3(256), 0, rng->start_ns, (const uint32_t *)vo,
-                       R, rmin, kfree);
-                radix_sort_pairs<uint64_t>(c, kfree, vo, ko, vfree, R, bits, false, hist2, part2, &ko, &perm);
+                const int bits = bits_for((uint64_t)(rmax - rmin)) + 1;
+                launch(c, "range_time_key", k_range_start_key, dim3(g), dim3(256), 0, rng->start_ns, rng->end_ns, R,
+                       rmin, rk0);
+                radix_sort_pairs<uint64_t>(c, rk0, rv0, rk1, rv1, R, bits, true, hist2, part2, &ko, &perm);
             }
             if (nl <= 256) {
                 // stable partition by compact level id, ranges written in place
@@ -864,7 +864,9 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
             continue;
         }
         if ((st = status_from_err(c.h_status->err))) return st;
-        if (c.h_status->flags & F_LEVEL_FIXUP) return OPATTR_E_CUDA;   // a full sort leaves no such disorder
+        // after the sort, equal starts out of (start, end) order in a level
+        // are two longer ranges with one start: overlapping, not laminar
+        if (c.h_status->flags & F_LEVEL_FIXUP) return OPATTR_E_NOT_NESTED;
         return OPATTR_OK;
     }
     return OPATTR_E_CUDA;
