@@ -899,6 +899,62 @@ def test_equal_starts_out_of_order(opa):
         ctx.close()
 
 
+def _shared_start_trace(longer_ranges: bool, longer_first: bool, shuffle: bool):
+    """A small trace plus two ranges of one level (stream 0, depth 0) that
+    start at the same instant T, after everything else: [T, T] and
+    [T, T + 10] (laminar: the zero-length range touches the longer one), or
+    [T, T + 10] and [T, T + 20] (overlapping); kernels at T and T + 5.  Ranges
+    in array order or permuted (the level lists then come from the sort)."""
+    import dataclasses
+    u = tracegen.small_random(11, n_events=80, max_depth=4, shuffle=False)
+    T = int(max(u.r_end.max(), u.k_start.max())) + 100
+    ends = [T + 10, T + 20] if longer_ranges else [T, T + 10]
+    if longer_first:
+        ends = ends[::-1]
+    r_start = np.append(u.r_start, [T, T]).astype(np.int64)
+    r_end = np.append(u.r_end, ends).astype(np.int64)
+    r_stream = np.append(u.r_stream, [0, 0]).astype(np.uint8)
+    r_depth = np.append(u.r_depth, [0, 0]).astype(np.uint8)
+    r_op = np.append(u.r_op, [0, 1]).astype(np.uint32)
+    if shuffle:
+        p = np.random.default_rng(5).permutation(len(r_start))
+        r_start, r_end, r_stream, r_depth, r_op = (x[p] for x in (r_start, r_end, r_stream, r_depth, r_op))
+    k_start = np.append(u.k_start, [T, T + 5]).astype(np.int64)
+    return dataclasses.replace(u, k_stream=np.append(u.k_stream, [0, 0]).astype(np.uint8), k_start=k_start,
+                               k_dur=np.append(u.k_dur, [3, 3]).astype(np.int64),
+                               k_name=np.append(u.k_name, [0, 0]).astype(np.uint32),
+                               r_stream=r_stream, r_start=r_start, r_end=r_end, r_depth=r_depth, r_op=r_op)
+
+
+@pytest.mark.parametrize("longer_ranges", [False, True])
+@pytest.mark.parametrize("longer_first", [False, True])
+@pytest.mark.parametrize("shuffle", [False, True])
+def test_shared_start_in_one_level(opa, longer_ranges, longer_first, shuffle):
+    """Two ranges of one level sharing a start: beside a zero-length range the
+    longer one is the level's representative at that instant (Algorithm 2's
+    closed interval, one range per depth); two longer ones overlap and are
+    not nested.  The oracle's status and enclosure, whatever the array order."""
+    t = _shared_start_trace(longer_ranges, longer_first, shuffle)
+    ost, ork, onop = oracle.enclose(t.k_stream, t.k_start, t.r_stream, t.r_start, t.r_end, t.r_depth, t.r_op,
+                                    mode="brute")
+    assert (ost == oracle.E_NOT_NESTED) == longer_ranges
+    ctx = opa.Context(0)
+    try:
+        if longer_ranges:
+            with pytest.raises(opa.OpattrError) as ei:
+                ctx.enclose(opa.to_device(t))
+            assert ei.value.status == opa.E_NOT_NESTED
+        else:
+            st, rk, nop = ctx.enclose(opa.to_device(t))
+            assert st == ost == 0
+            np.testing.assert_array_equal(rk.cpu().numpy(), ork)
+            np.testing.assert_array_equal(nop.cpu().numpy(), onop)
+            longer = int(np.nonzero((t.r_start == t.r_start.max()) & (t.r_end > t.r_start))[0][0])
+            assert (ork[-2:] == longer).all()
+    finally:
+        ctx.close()
+
+
 def _with_gap(t, cut, gap):
     """Every timestamp at or after `cut` moved later by `gap` ns: an idle gap
     in the trace.  The map is monotone, so order, nesting, ties and
