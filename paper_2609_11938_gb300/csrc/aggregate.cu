@@ -334,6 +334,7 @@ __global__ void __launch_bounds__(256, 5) k_agg_count(const int64_t *__restrict_
                             const int32_t *__restrict__ nidx, const uint32_t *__restrict__ r_op, int64_t K, int64_t R,
                             int64_t M, int64_t n_ops, uint32_t *__restrict__ cnt, uint32_t *__restrict__ rank,
                             int64_t run, int ident_rows, unsigned *__restrict__ nonident, DevStatus *st) {
+    pdl_wait();
     const unsigned lane = lane_id(), lt = lanemask_lt();
     const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) / 32;
     const int64_t nwarps = (int64_t)gridDim.x * blockDim.x / 32;
@@ -400,6 +401,7 @@ template <bool DIRECT>
 __global__ void k_agg_place(const int32_t *__restrict__ rok, const uint32_t *__restrict__ r_op, int64_t K, int64_t R,
                             int64_t n_ops, const uint32_t *__restrict__ off, const uint32_t *__restrict__ rank,
                             uint32_t *__restrict__ list) {
+    pdl_wait();
     constexpr int U = 4;                    // kernels per thread per round, loads issued together
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t k0 = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k0 < K; k0 += stride * U) {
@@ -452,6 +454,7 @@ __global__ void __launch_bounds__(SL_THREADS) k_agg_sort_long(const uint32_t *__
                                                               const uint32_t *__restrict__ longs,
                                                               const unsigned *__restrict__ nlong, uint32_t min_len,
                                                               uint32_t max_len, uint32_t *list, uint32_t *tmp) {
+    pdl_wait();
     __shared__ uint32_t a[SL_SMEM];
     const unsigned n_long = *nlong;
     for (unsigned li = blockIdx.x; li < n_long; li += gridDim.x) {
@@ -577,6 +580,7 @@ __device__ __forceinline__ void cp_async_wait() {
 
 __global__ void __launch_bounds__(AG_THREADS, 5) k_agg_ops(const uint32_t *__restrict__ off, uint32_t *list,
                                                           AggIn A) {
+    pdl_wait();
     extern __shared__ __align__(16) unsigned char ag_smem[];
     OpsWarp &W = reinterpret_cast<OpsWarp *>(ag_smem)[threadIdx.x / 32];
     const unsigned lane = lane_id();
@@ -723,6 +727,7 @@ __global__ void __launch_bounds__(AG_THREADS, 5) k_agg_ops(const uint32_t *__res
 // nulls out and reports infinite values.  A separate pass keeps that rare,
 // register-hungry path out of the ops pass.
 __global__ void k_agg_careful(const uint32_t *__restrict__ off, uint32_t *list, AggIn A, DevStatus *st) {
+    pdl_wait();
     int bad = 0;
     const unsigned n = A.ctr[1];
     for (unsigned e = blockIdx.x * blockDim.x + threadIdx.x; e < n; e += gridDim.x * blockDim.x) {
@@ -807,6 +812,7 @@ __global__ void __launch_bounds__(1024) k_agg_piece_offsets(const uint32_t *__re
                                                             const unsigned *__restrict__ nlong, uint32_t huge,
                                                             uint32_t *__restrict__ poff, uint32_t *__restrict__ info,
                                                             uint32_t *__restrict__ hop) {
+    pdl_wait();
     __shared__ uint32_t wbuf[33];
     const int64_t n = *nlong;
     uint32_t carry = 0, longest = 0, kern = 0, hcarry = 0;
@@ -881,6 +887,7 @@ struct HugePlace {
     __device__ __forceinline__ void done(unsigned) const {}
 };
 __global__ void k_huge_index(const uint32_t *__restrict__ hop, int64_t n_huge, uint32_t *__restrict__ hidx) {
+    pdl_wait();
     for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < n_huge; c += (int64_t)gridDim.x * blockDim.x)
         hidx[hop[c]] = (uint32_t)c;
 }
@@ -924,6 +931,7 @@ __device__ __forceinline__ bool piece_fast(const AggIn &A, const uint32_t *seg, 
 __global__ void k_agg_pieces(const uint32_t *__restrict__ off, const uint32_t *__restrict__ list,
                              const uint32_t *__restrict__ longs, const unsigned *__restrict__ nlong,
                              const uint32_t *__restrict__ poff, AggIn A, Acc *__restrict__ part) {
+    pdl_wait();
     const int64_t n = *nlong;
     const int64_t P = poff[n];
     const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
@@ -961,6 +969,7 @@ __global__ void __launch_bounds__(FIN_THREADS) k_agg_long_ops(const uint32_t *__
                                                               const uint32_t *__restrict__ poff,
                                                               const Acc *__restrict__ part, int write_empty, AggIn A,
                                                               DevStatus *st) {
+    pdl_wait();
     __shared__ Acc wpart[FIN_THREADS / 32];
     const int64_t n = *nlong;
     const unsigned lane = lane_id(), w = threadIdx.x >> 5;
@@ -1154,6 +1163,7 @@ namespace opattr {
 // and every class is accumulated by pieces.
 __global__ void k_class_check(const uint32_t *__restrict__ class_of_op, int64_t n_ops, uint32_t n_classes,
                               DevStatus *st) {
+    pdl_wait();
     int bad = 0;
     for (int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; o < n_ops; o += (int64_t)gridDim.x * blockDim.x) {
         const uint32_t c = class_of_op[o];
@@ -1169,6 +1179,7 @@ constexpr int CK_SMEM = 4096;
 __global__ void k_class_keys(const int32_t *__restrict__ rok, const uint32_t *__restrict__ r_op, int64_t K, int64_t R,
                              int64_t n_ops, const uint32_t *__restrict__ class_of_op, uint32_t n_classes,
                              uint32_t *__restrict__ key, uint32_t *__restrict__ cnt) {
+    pdl_wait();
     __shared__ uint32_t h[CK_SMEM];
     const bool local = n_classes <= (uint32_t)CK_SMEM;
     if (local)
@@ -1199,6 +1210,7 @@ __global__ void k_class_keys(const int32_t *__restrict__ rok, const uint32_t *__
     }
 }
 __global__ void k_iota_u32(uint32_t *dst, int64_t n, unsigned *count) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         dst[i] = (uint32_t)i;
     if (blockIdx.x == 0 && threadIdx.x == 0) *count = (unsigned)n;

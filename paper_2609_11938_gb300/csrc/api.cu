@@ -111,6 +111,7 @@ opattr_status ensure_side(Ctx &c) {
 // Bytes from src to dst, one of them in mapped pinned host memory: words
 // when both ends and the size are 4-byte aligned (every caller's case).
 __global__ void k_copy_small(const unsigned char *__restrict__ src, unsigned char *__restrict__ dst, size_t n) {
+    pdl_wait();
     const size_t t0 = (size_t)blockIdx.x * blockDim.x + threadIdx.x, step = (size_t)gridDim.x * blockDim.x;
     if (((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst) | n) & 3u) == 0) {
         const uint32_t *s = reinterpret_cast<const uint32_t *>(src);

@@ -29,6 +29,7 @@ namespace opattr {
 __global__ void k_attr_check_kernels(const int32_t *__restrict__ rok, const uint32_t *__restrict__ r_op, int64_t R,
                                      const uint32_t *__restrict__ name, int64_t K, uint32_t n_ops,
                                      unsigned long long *max_name, DevStatus *st) {
+    pdl_wait();
     int bad = 0;
     uint32_t mx = 0;
     for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < K; k += (int64_t)gridDim.x * blockDim.x) {
@@ -50,6 +51,7 @@ __global__ void k_attr_check_kernels(const int32_t *__restrict__ rok, const uint
 // Every operator of a table below n_ops (OPATTR_OP_NONE allowed where `none_ok`).
 __global__ void k_attr_check_ops(const uint32_t *__restrict__ op, int64_t n, uint32_t n_ops, int none_ok,
                                  DevStatus *st) {
+    pdl_wait();
     int bad = 0;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         const uint32_t x = op[i];
@@ -61,17 +63,20 @@ __global__ void k_attr_check_ops(const uint32_t *__restrict__ op, int64_t n, uin
 // ------------------------------------------------------------------ HIGH tier
 __global__ void k_gather_names(const uint32_t *__restrict__ name, const uint32_t *__restrict__ korder, int64_t n,
                                uint32_t *__restrict__ dst) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         dst[i] = name[korder ? korder[i] : i];
 }
 __device__ __forceinline__ bool run_head_u32(const uint32_t *a, int64_t i) { return i == 0 || a[i - 1] != a[i]; }
 
 __global__ void k_attr_heads(const uint32_t *__restrict__ skn, int64_t n, uint32_t *__restrict__ flag) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         flag[i] = run_head_u32(skn, i);
 }
 __global__ void k_attr_starts(const uint32_t *__restrict__ skn, const uint32_t *__restrict__ pos, int64_t n,
                               uint32_t *__restrict__ start) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         if (run_head_u32(skn, i)) start[pos[i]] = (uint32_t)i;
 }
@@ -83,6 +88,7 @@ __global__ void k_corr_scatter(const uint32_t *__restrict__ c_name, const uint32
                                const uint32_t *__restrict__ c_op, int64_t nc, const uint32_t *__restrict__ skn,
                                const uint32_t *__restrict__ ustart, const uint32_t *__restrict__ n_urun, int64_t K,
                                uint32_t *__restrict__ table, DevStatus *st) {
+    pdl_wait();
     const int64_t U = *n_urun;
     unsigned long long used = 0;
     int dup = 0;
@@ -109,6 +115,7 @@ __global__ void k_corr_scatter(const uint32_t *__restrict__ c_name, const uint32
 // The HIGH operator of each kernel: the table at its sorted position.
 __global__ void k_corr_gather(const uint32_t *__restrict__ table, const uint32_t *__restrict__ skj,
                               const uint32_t *__restrict__ korder, int64_t K, uint32_t *__restrict__ hi_op) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < K; i += (int64_t)gridDim.x * blockDim.x) {
         const uint32_t j = skj[i];
         hi_op[korder ? korder[j] : j] = table[i];
@@ -133,6 +140,7 @@ struct TierIn {
 };
 
 __global__ void k_tiers(TierIn A, DevStatus *st) {
+    pdl_wait();
     constexpr int U = 4;                      // kernels per thread per round, loads issued together
     unsigned long long n_high = 0, n_nvtx = 0, n_ind = 0, n_fused = 0;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;

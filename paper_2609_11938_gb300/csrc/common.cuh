@@ -192,7 +192,12 @@ void timing_begin(Ctx &c, int slot, cudaEvent_t *e0, cudaEvent_t *e1);
 void timing_end(Ctx &c, int slot, cudaEvent_t e0, cudaEvent_t e1);
 void timing_collect(Ctx &c);             // after a stream synchronize
 
-// Launch a kernel on the context stream, counting it and (optionally) timing it.
+// Launch a kernel on the context stream, counting it and (optionally) timing
+// it.  Kernels go out as programmatic dependent launches: the next kernel of
+// the stream is set up and its blocks scheduled while this one's last blocks
+// finish, instead of after its completion; every kernel of the library calls
+// pdl_wait() before its first memory access, which holds it until the
+// kernel before it has completed and its writes are visible.
 template <typename... KArgs, typename... Args>
 inline void launch(Ctx &c, const char *name, void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
                    Args... args) {
@@ -204,7 +209,17 @@ inline void launch(Ctx &c, const char *name, void (*kern)(KArgs...), dim3 grid, 
         slot = timing_slot(c, name);
         timing_begin(c, slot, &e0, &e1);
     }
-    kern<<<grid, block, smem, c.stream>>>(args...);
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = c.stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaLaunchKernelEx(&cfg, kern, args...);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess && c.last_error == cudaSuccess) c.last_error = e;
     c.launches++;
@@ -218,6 +233,13 @@ inline unsigned grid_for(int64_t n, int per_block, unsigned cap = 1u << 30) {
 }
 
 // ------------------------------------------------------------------ device helpers
+// The first statement of every kernel: waits, under a programmatic dependent
+// launch, until the kernel before it in the stream has completed and its
+// memory is visible (returns at once otherwise).  No kernel signals early
+// completion, so a kernel's blocks never hold resources that the blocks of
+// the kernel before it still need.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 __device__ __forceinline__ unsigned lane_id() { return threadIdx.x & 31u; }
 __device__ __forceinline__ unsigned lanemask_lt() {
     unsigned m;

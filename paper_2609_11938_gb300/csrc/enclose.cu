@@ -41,6 +41,7 @@ __global__ void __launch_bounds__(RCHK_THREADS) k_check_ranges(const uint8_t *__
                                                                const int64_t *__restrict__ end,
                                                                const uint8_t *__restrict__ depth, int64_t n,
                                                                uint32_t *__restrict__ level_hist, DevStatus *st) {
+    pdl_wait();
     __shared__ uint32_t h[LEVELS];
     __shared__ int flags;
     __shared__ long long smin, smax;
@@ -94,6 +95,7 @@ __global__ void __launch_bounds__(RCHK_THREADS) k_check_ranges(const uint8_t *__
 // ------------------------------------------------------------------ level lists
 __global__ void k_level_keys(const uint8_t *__restrict__ stream, const uint8_t *__restrict__ depth,
                              const uint32_t *__restrict__ perm, int64_t n, uint32_t *__restrict__ keys) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         int64_t r = perm ? perm[i] : i;
         keys[i] = (uint32_t)stream[r] * 32u + depth[r];
@@ -108,12 +110,14 @@ __global__ void k_level_keys(const uint8_t *__restrict__ stream, const uint8_t *
 // out of that order only when they overlap, which the validation reports.
 __global__ void k_range_start_key(const int64_t *__restrict__ start, const int64_t *__restrict__ end, int64_t n,
                                   long long tmin, uint64_t *__restrict__ keys) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         keys[i] = ((uint64_t)(start[i] - tmin) << 1) | (end[i] > start[i] ? 1u : 0u);
 }
 __global__ void k_level_gather(const int64_t *__restrict__ start, const int64_t *__restrict__ end,
                                const uint32_t *__restrict__ op, const uint32_t *__restrict__ perm, int64_t n,
                                int64_t *__restrict__ ls, int64_t *__restrict__ le, uint32_t *__restrict__ li) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         uint32_t r = perm[i];
         ls[i] = start[r];
@@ -156,6 +160,7 @@ __global__ void __launch_bounds__(RADIX_THREADS) k_level_place(LevelDigit digit,
                                                                const uint32_t *__restrict__ offs, int64_t ntiles,
                                                                int64_t *__restrict__ ls, int64_t *__restrict__ le,
                                                                uint32_t *__restrict__ li) {
+    pdl_wait();
     __shared__ PlaceSmem S;
     const unsigned w = threadIdx.x >> 5, lane = lane_id();
     for (int i = threadIdx.x; i < (RADIX_THREADS / 32) * RADIX_BINS; i += RADIX_THREADS) S.wcnt[i] = 0;
@@ -252,6 +257,7 @@ __global__ void k_validate_levels(const uint8_t *__restrict__ stream, const uint
                                   const int64_t *__restrict__ ls, const int64_t *__restrict__ le,
                                   const uint32_t *__restrict__ li, const uint32_t *__restrict__ lvl_off, int64_t n,
                                   DevStatus *st) {
+    pdl_wait();
     bool err = false, fix = false;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x * VL_PER;
     for (int64_t i0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * VL_PER; i0 < n; i0 += stride) {
@@ -350,6 +356,7 @@ __global__ void k_stream_windows(const int64_t *__restrict__ ls, const uint32_t 
                                  const uint32_t *__restrict__ koff, const uint32_t *__restrict__ kcnt,
                                  const uint32_t *__restrict__ psk, const int64_t *__restrict__ k_start, int64_t nt,
                                  int2 *__restrict__ P, uint32_t *__restrict__ tinfo) {
+    pdl_wait();
     for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < nt * 32; q += (int64_t)gridDim.x * blockDim.x) {
         const int64_t u = q >> 5;
         const int d = (int)(q & 31);
@@ -439,6 +446,7 @@ __device__ __forceinline__ void walk_step(uint32_t info, int32_t &ans, int &nop)
 // staging, or whose kernels span 2^32 ns or more (relative times no longer
 // fit), searches the global level lists instead.
 __global__ void __launch_bounds__(EN_THREADS) k_enclose(EncArgs A) {
+    pdl_wait();
     __shared__ EncSmem S;
     const uint32_t info = A.tinfo[blockIdx.x];
     const int sid = (int)(info & 0xFFu);
@@ -585,6 +593,7 @@ __global__ void __launch_bounds__(EN_THREADS) k_enclose(EncArgs A) {
 }
 
 __global__ void k_fill_unattributed(int32_t *out_range, uint8_t *out_nop, int64_t n) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         out_range[i] = -1;
         if (out_nop) out_nop[i] = 0;

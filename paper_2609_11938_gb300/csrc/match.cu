@@ -31,6 +31,7 @@ static int identity_vec(const void *kname, const void *nname, const void *out_id
 __global__ void k_match_identity(const uint32_t *__restrict__ kname, const uint32_t *__restrict__ nname, int64_t n,
                                  int32_t *__restrict__ out_idx, uint8_t *__restrict__ out_kind, int vec,
                                  DevStatus *st) {
+    pdl_wait();
     constexpr int U = 4;                    // elements per thread per round, loads issued together
     int bad = 0;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x * U;
@@ -71,6 +72,7 @@ void launch_identity_match(Ctx &c, const uint32_t *kname, const uint32_t *nname,
 __global__ void k_match_identity_list(const uint32_t *__restrict__ rk, const uint32_t *__restrict__ kname,
                                       const uint32_t *__restrict__ nname, int64_t n, int32_t *__restrict__ out_idx,
                                       uint8_t *__restrict__ out_kind, DevStatus *st) {
+    pdl_wait();
     int bad = 0;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         uint32_t k = rk[i];
@@ -114,6 +116,7 @@ struct StreamPairs {
 // Name ids of every kernel below 2^24 (per-stream rows with layer classes,
 // where the pairing above sees the replayed kernels only).
 __global__ void k_check_names24(const uint32_t *__restrict__ name, int64_t n, DevStatus *st) {
+    pdl_wait();
     uint32_t acc = 0;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         acc |= name[i];
@@ -121,6 +124,7 @@ __global__ void k_check_names24(const uint32_t *__restrict__ name, int64_t n, De
 }
 
 __global__ void k_fill_match(int32_t *out_idx, uint8_t *out_kind, int64_t n) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         out_idx[i] = -1;
         if (out_kind) out_kind[i] = 0;
@@ -133,6 +137,7 @@ __global__ void k_fill_match(int32_t *out_idx, uint8_t *out_kind, int64_t n) {
 //   what = 1: layer-tagged (layer >= 0)
 __global__ void k_flags(const uint32_t *__restrict__ korder, const int32_t *__restrict__ layer,
                         const int32_t *__restrict__ rep_layer, int64_t n, int what, uint32_t *__restrict__ flag) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         int64_t k = korder ? korder[i] : i;
         int32_t l = layer ? layer[k] : -1;
@@ -143,20 +148,24 @@ __global__ void k_flags(const uint32_t *__restrict__ korder, const int32_t *__re
 // Compact: list[pos[i]] = korder[i] where flag[i]
 __global__ void k_compact(const uint32_t *__restrict__ korder, const uint32_t *__restrict__ flag,
                           const uint32_t *__restrict__ pos, int64_t n, uint32_t *__restrict__ list) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         if (flag[i]) list[pos[i]] = korder ? korder[i] : (uint32_t)i;
 }
 __global__ void k_gather_u32(const uint32_t *__restrict__ src, const uint32_t *__restrict__ idx, int64_t n,
                              uint32_t *__restrict__ dst) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         dst[i] = idx ? src[idx[i]] : src[i];
 }
 __global__ void k_gather_i32_as_u32(const int32_t *__restrict__ src, const uint32_t *__restrict__ idx, int64_t n,
                                     uint32_t *__restrict__ dst) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         dst[i] = (uint32_t)src[idx[i]];
 }
 __global__ void k_max_u32(const uint32_t *__restrict__ a, int64_t n, unsigned long long *out) {
+    pdl_wait();
     uint32_t m = 0;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         m = a[i] > m ? a[i] : m;
@@ -175,6 +184,7 @@ __global__ void k_max_u32(const uint32_t *__restrict__ a, int64_t n, unsigned lo
 }
 __global__ void k_check_layers(const int32_t *__restrict__ layer, int64_t n, int32_t n_layers,
                                const int32_t *__restrict__ rep_layer, DevStatus *st) {
+    pdl_wait();
     unsigned long long rep = 0;
     int bad = 0;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
@@ -211,11 +221,13 @@ __device__ __forceinline__ int64_t upper_bound_u32(const uint32_t *a, int64_t n,
 __device__ __forceinline__ bool run_head(const uint32_t *a, int64_t i) { return i == 0 || a[i - 1] != a[i]; }
 
 __global__ void k_run_heads(const uint32_t *__restrict__ a, int64_t n, uint32_t *__restrict__ flag) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         flag[i] = run_head(a, i);
 }
 __global__ void k_run_starts(const uint32_t *__restrict__ a, const uint32_t *__restrict__ pos, int64_t n,
                              uint32_t *__restrict__ start) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         if (run_head(a, i)) start[pos[i]] = (uint32_t)i;
 }
@@ -238,6 +250,7 @@ __global__ void k_run_pair(const uint32_t *__restrict__ skn, const uint32_t *__r
                            const uint32_t *__restrict__ n_urun, int64_t nrep, const uint32_t *__restrict__ snn,
                            const uint32_t *__restrict__ vstart, const uint32_t *__restrict__ n_vrun, int64_t M,
                            int mode, uint32_t *__restrict__ b_of, uint32_t *__restrict__ cq_of, DevStatus *st) {
+    pdl_wait();
     const int64_t U = *n_urun, V = *n_vrun;
     unsigned long long names_bad = 0;
     for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < U; u += (int64_t)gridDim.x * blockDim.x) {
@@ -263,6 +276,7 @@ __global__ void k_ncu_only_names(const uint32_t *__restrict__ snn, const uint32_
                                  const uint32_t *__restrict__ n_vrun, const uint32_t *__restrict__ skn,
                                  const uint32_t *__restrict__ ustart, const uint32_t *__restrict__ n_urun, int mode,
                                  DevStatus *st) {
+    pdl_wait();
     const int64_t U = *n_urun, V = *n_vrun;
     unsigned long long bad = 0;
     for (int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < V; v += (int64_t)gridDim.x * blockDim.x) {
@@ -287,6 +301,7 @@ __global__ void k_ordinal_join(const uint32_t *__restrict__ skn, const uint32_t 
                                const uint32_t *__restrict__ cq_of, const uint32_t *__restrict__ rk, int64_t nrep,
                                const uint32_t *__restrict__ snj, int mode, int32_t *__restrict__ out_idx,
                                uint8_t *__restrict__ out_kind, DevStatus *st) {
+    pdl_wait();
     const int64_t U = *n_urun;
     unsigned long long direct = 0, unmatched = 0;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nrep; i += (int64_t)gridDim.x * blockDim.x) {
@@ -312,6 +327,7 @@ __global__ void k_dedup_broadcast(const uint32_t *__restrict__ sll, const uint32
                                   const uint32_t *__restrict__ lk, int64_t nl, const int32_t *__restrict__ rep_layer,
                                   const uint32_t *__restrict__ kname, int32_t *__restrict__ out_idx,
                                   uint8_t *__restrict__ out_kind, DevStatus *st) {
+    pdl_wait();
     unsigned long long bc = 0, miss = 0;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < nl; i += (int64_t)gridDim.x * blockDim.x) {
         uint32_t L = sll[i];
@@ -342,6 +358,7 @@ __global__ void k_dedup_broadcast(const uint32_t *__restrict__ sll, const uint32
 // name id of 2^24 or more cannot be packed and is an invalid argument.
 __global__ void k_stream_keys(const uint32_t *__restrict__ name, const uint8_t *__restrict__ stream, int64_t n,
                               uint32_t *__restrict__ key, DevStatus *st) {
+    pdl_wait();
     int bad = 0;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         const uint32_t x = name[i];
@@ -352,6 +369,7 @@ __global__ void k_stream_keys(const uint32_t *__restrict__ name, const uint8_t *
 }
 
 __global__ void k_iota(uint32_t *dst, int64_t n) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
         dst[i] = (uint32_t)i;
 }

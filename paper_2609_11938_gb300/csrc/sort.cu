@@ -21,6 +21,7 @@ namespace opattr {
 // (coalesced), carrying its running sum.
 __global__ void __launch_bounds__(SCAN_THREADS) k_scan_reduce(const uint32_t *__restrict__ in, int64_t n,
                                                               uint32_t *__restrict__ partials) {
+    pdl_wait();
     __shared__ uint32_t wbuf[33];
     const int64_t base = (int64_t)blockIdx.x * SCAN_TILE + (threadIdx.x >> 5) * (SCAN_TILE / 8);
     uint32_t s = 0;
@@ -35,6 +36,7 @@ __global__ void __launch_bounds__(SCAN_THREADS) k_scan_reduce(const uint32_t *__
 
 // One block scans the tile sums (exclusive) in place; partials[nt] = total.
 __global__ void __launch_bounds__(1024) k_scan_partials(uint32_t *partials, int64_t nt, uint32_t *total_dev) {
+    pdl_wait();
     __shared__ uint32_t wbuf[33];
     uint32_t carry = 0;
     for (int64_t b = 0; b < nt; b += 1024) {
@@ -53,6 +55,7 @@ __global__ void __launch_bounds__(1024) k_scan_partials(uint32_t *partials, int6
 
 __global__ void __launch_bounds__(SCAN_THREADS) k_scan_down(const uint32_t *in, uint32_t *out, int64_t n,
                                                             const uint32_t *__restrict__ partials) {
+    pdl_wait();
     __shared__ uint32_t wbuf[33];
     const unsigned w = threadIdx.x >> 5;
     const int64_t base = (int64_t)blockIdx.x * SCAN_TILE + w * (SCAN_TILE / 8);
@@ -90,6 +93,7 @@ __global__ void __launch_bounds__(SCAN_THREADS) k_scan_onepass(const uint32_t *_
                                                                unsigned long long *status, unsigned *tile_ctr,
                                                                int64_t nt, uint32_t *total_dev, int64_t spin_limit,
                                                                int fault, DevStatus *st) {
+    pdl_wait();
     __shared__ uint32_t wbuf[33];
     __shared__ unsigned tile_s;
     __shared__ uint32_t off_s;
@@ -136,6 +140,7 @@ __global__ void __launch_bounds__(SCAN_THREADS) k_scan_onepass(const uint32_t *_
 constexpr int64_t SCAN_ONE_BLOCK = 32 * 1024;
 __global__ void __launch_bounds__(1024) k_scan_small(const uint32_t *in, uint32_t *out, int64_t n,
                                                      uint32_t *total_dev) {
+    pdl_wait();
     __shared__ uint32_t wsum[32];
     const unsigned w = threadIdx.x >> 5, lane = lane_id();
     const int64_t b = (int64_t)w * 1024 + lane;
@@ -199,6 +204,7 @@ __device__ __forceinline__ unsigned digit_of(K key, int shift) {
 template <typename K>
 __global__ void __launch_bounds__(RADIX_THREADS) k_radix_upsweep(const K *__restrict__ keys, int64_t n, int shift,
                                                                  uint32_t *__restrict__ hist, int64_t ntiles) {
+    pdl_wait();
     __shared__ uint32_t h[RADIX_THREADS / 32][RADIX_BINS];
     const unsigned w = threadIdx.x >> 5;
     for (int i = threadIdx.x; i < (RADIX_THREADS / 32) * RADIX_BINS; i += RADIX_THREADS) (&h[0][0])[i] = 0;
@@ -229,6 +235,7 @@ __global__ void __launch_bounds__(RADIX_THREADS) k_radix_downsweep(const K *__re
                                                                    int64_t n, int shift,
                                                                    const uint32_t *__restrict__ offs,
                                                                    int64_t ntiles) {
+    pdl_wait();
     extern __shared__ __align__(16) unsigned char smem_raw[];
     K *ks = reinterpret_cast<K *>(smem_raw);
     uint32_t *vs = reinterpret_cast<uint32_t *>(ks + RADIX_TILE);

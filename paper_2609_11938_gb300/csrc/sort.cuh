@@ -122,6 +122,7 @@ __device__ __forceinline__ uint32_t warp_lookback_exclusive(unsigned long long *
 template <typename DigitFn>
 __global__ void __launch_bounds__(RADIX_THREADS) k_digit_hist(DigitFn digit, int64_t n, uint32_t *__restrict__ hist,
                                                               int64_t ntiles) {
+    pdl_wait();
     __shared__ uint32_t h[RADIX_THREADS / 32][RADIX_BINS];
     const unsigned w = threadIdx.x >> 5;
     for (int i = threadIdx.x; i < (RADIX_THREADS / 32) * RADIX_BINS; i += RADIX_THREADS) (&h[0][0])[i] = 0;
@@ -146,6 +147,7 @@ template <typename DigitFn, typename Epi>
 __global__ void __launch_bounds__(RADIX_THREADS) k_digit_rank(DigitFn digit, int64_t n,
                                                               const uint32_t *__restrict__ offs, int64_t ntiles,
                                                               Epi epi) {
+    pdl_wait();
     __shared__ uint32_t wcnt[(RADIX_THREADS / 32) * RADIX_BINS];
     __shared__ uint32_t gbase[RADIX_BINS];
     const unsigned w = threadIdx.x >> 5, lane = lane_id();

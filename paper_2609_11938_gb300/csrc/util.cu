@@ -23,6 +23,7 @@ __global__ void __launch_bounds__(CHK_THREADS) k_check_kernel_order(const uint8_
                                                                     int vec, DevStatus *st,
                                                                     uint32_t *__restrict__ stream_hist,
                                                                     uint32_t *__restrict__ tile_hist) {
+    pdl_wait();
     __shared__ long long smin[CHK_THREADS / 32], smax[CHK_THREADS / 32];
     __shared__ int sbad[CHK_THREADS / 32];
     __shared__ uint32_t sh[256], th[256];
@@ -122,6 +123,7 @@ void check_kernel_order(Ctx &c, const uint8_t *stream, const int64_t *start, int
 __global__ void k_time_keys(const uint8_t *__restrict__ stream, const int64_t *__restrict__ start, int64_t n,
                             long long tmin, const uint8_t *__restrict__ scmap, int sbits,
                             uint64_t *__restrict__ keys) {
+    pdl_wait();
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
         const unsigned s = scmap ? scmap[stream[i]] : stream[i];
         keys[i] = ((uint64_t)(start[i] - tmin) << sbits) | s;
