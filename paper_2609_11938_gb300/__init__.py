@@ -295,17 +295,20 @@ def opattr_destroy(handle) -> None:
 
 # ---------------------------------------------------------------- torch convenience layer
 def _ptr(t, dtype, name, device):
-    import torch
     if t is None:
         return None
-    ok = (t.dtype == dtype) or (dtype == torch.uint32 and t.dtype == torch.int32)
-    if not ok:
+    if t.dtype is not dtype and not (dtype is _torch().uint32 and t.dtype is _torch().int32):
         raise TypeError(f"{name}: expected {dtype}, got {t.dtype}")
-    if not t.is_cuda or t.device.index != device:
+    if t.get_device() != device:                 # -1 for a host tensor
         raise ValueError(f"{name}: must live on cuda:{device}")
     if not t.is_contiguous():
         raise ValueError(f"{name}: must be contiguous")
     return t.data_ptr() if t.numel() else None
+
+
+def _torch():
+    import torch
+    return torch
 
 
 @dataclass

@@ -1093,8 +1093,8 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
         // the ops the pass left: listed with a null or infinite value (redone
         // by k_agg_careful), long ones (the pieces pass); both
         // counts come back with the status
-        if ((st = copy_small(c, c.h_levels, ctr + 1, 2 * sizeof(uint32_t), cudaMemcpyDeviceToHost))) return st;
-        if ((st = read_status(c))) return st;
+        const SmallCopy counts{c.h_levels, ctr + 1, 2 * sizeof(uint32_t)};
+        if ((st = read_status(c, 1, &counts))) return st;
         const uint32_t n_dirty = c.h_levels[0], n_long = c.h_levels[1];
         status_fresh = n_dirty == 0 && n_long == 0;
         if (n_dirty > 0)
@@ -1104,8 +1104,8 @@ opattr_status do_aggregate(Ctx &c, const opattr_kernels *kern, const opattr_rang
         if (n_long > 0) {
             launch(c, "agg_piece_offsets", k_agg_piece_offsets, dim3(1), dim3(1024), 0, (const uint32_t *)off,
                    (const uint32_t *)longs, (const unsigned *)nlong, 0u, npc, info, hop);
-            if ((st = copy_small(c, c.h_levels, info, 5 * sizeof(uint32_t), cudaMemcpyDeviceToHost))) return st;
-            if ((st = read_status(c))) return st;
+            const SmallCopy pinfo{c.h_levels, info, 5 * sizeof(uint32_t)};
+            if ((st = read_status(c, 1, &pinfo))) return st;
             pieces = c.h_levels[1];
             longest = c.h_levels[2];
             n_huge = c.h_levels[4];

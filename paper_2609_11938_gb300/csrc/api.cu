@@ -108,38 +108,77 @@ opattr_status ensure_side(Ctx &c) {
     return OPATTR_OK;
 }
 
-// Bytes from src to dst, one of them in mapped pinned host memory: words
-// when both ends and the size are 4-byte aligned (every caller's case).
-__global__ void k_copy_small(const unsigned char *__restrict__ src, unsigned char *__restrict__ dst, size_t n) {
+// Up to SMALL_COPIES transfers in one launch, each between mapped pinned host
+// memory and device memory: words when both ends and the size are 4-byte
+// aligned (every caller's case), bytes otherwise.
+constexpr int SMALL_COPIES = 4;
+struct SmallCopies {
+    const unsigned char *src[SMALL_COPIES];
+    unsigned char *dst[SMALL_COPIES];
+    unsigned long long n[SMALL_COPIES];
+    int count;
+};
+__global__ void k_copy_small(SmallCopies cp) {
     pdl_wait();
     const size_t t0 = (size_t)blockIdx.x * blockDim.x + threadIdx.x, step = (size_t)gridDim.x * blockDim.x;
-    if (((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst) | n) & 3u) == 0) {
-        const uint32_t *s = reinterpret_cast<const uint32_t *>(src);
-        uint32_t *d = reinterpret_cast<uint32_t *>(dst);
-        for (size_t i = t0; i < n / 4; i += step) d[i] = s[i];
-    } else {
-        for (size_t i = t0; i < n; i += step) dst[i] = src[i];
+    for (int q = 0; q < cp.count; ++q) {
+        const unsigned char *src = cp.src[q];
+        unsigned char *dst = cp.dst[q];
+        const size_t n = cp.n[q];
+        if (((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst) | n) & 3u) == 0) {
+            const uint32_t *s = reinterpret_cast<const uint32_t *>(src);
+            uint32_t *d = reinterpret_cast<uint32_t *>(dst);
+            for (size_t i = t0; i < n / 4; i += step) d[i] = s[i];
+        } else {
+            for (size_t i = t0; i < n; i += step) dst[i] = src[i];
+        }
     }
+}
+
+opattr_status copy_small_n(Ctx &c, int count, const SmallCopy *cp, cudaMemcpyKind kind) {
+    if (count <= 0) return OPATTR_OK;
+    if (!c.host_mapped) {
+        for (int q = 0; q < count; ++q) {
+            if (cp[q].bytes == 0) continue;
+            const cudaError_t e = cudaMemcpyAsync(cp[q].dst, cp[q].src, cp[q].bytes, kind, c.stream);
+            if (e != cudaSuccess) return cuda_status(c, e);
+        }
+        return OPATTR_OK;
+    }
+    for (int q0 = 0; q0 < count; q0 += SMALL_COPIES) {
+        SmallCopies a{};
+        size_t most = 0;
+        for (int q = q0; q < count && q < q0 + SMALL_COPIES; ++q) {
+            a.src[a.count] = static_cast<const unsigned char *>(cp[q].src);
+            a.dst[a.count] = static_cast<unsigned char *>(cp[q].dst);
+            a.n[a.count] = cp[q].bytes;
+            most = std::max(most, cp[q].bytes);
+            a.count++;
+        }
+        launch(c, "small_copy", k_copy_small, dim3(grid_for((int64_t)std::max<size_t>(most, 1), 256 * 16, 8)),
+               dim3(256), 0, a);
+    }
+    return c.last_error == cudaSuccess ? OPATTR_OK : cuda_status(c, c.last_error);
 }
 
 opattr_status copy_small(Ctx &c, void *dst, const void *src, size_t bytes, cudaMemcpyKind kind) {
     if (bytes == 0) return OPATTR_OK;
-    if (!c.host_mapped) {
-        const cudaError_t e = cudaMemcpyAsync(dst, src, bytes, kind, c.stream);
-        return e == cudaSuccess ? OPATTR_OK : cuda_status(c, e);
-    }
-    launch(c, "small_copy", k_copy_small, dim3(grid_for((int64_t)bytes, 256 * 16, 8)), dim3(256), 0,
-           static_cast<const unsigned char *>(src), static_cast<unsigned char *>(dst), bytes);
-    return c.last_error == cudaSuccess ? OPATTR_OK : cuda_status(c, c.last_error);
+    const SmallCopy cp{dst, src, bytes};
+    return copy_small_n(c, 1, &cp, kind);
 }
 
 opattr_status reset_status(Ctx &c) {
     return copy_small(c, c.d_status, c.h_init, sizeof(DevStatus), cudaMemcpyHostToDevice);
 }
 
-opattr_status read_status(Ctx &c) {
+opattr_status read_status(Ctx &c, int n_extra, const SmallCopy *extra) {
     if (c.last_error != cudaSuccess) return cuda_status(c, c.last_error);
-    opattr_status st = copy_small(c, c.h_status, c.d_status, sizeof(DevStatus), cudaMemcpyDeviceToHost);
+    if (n_extra < 0 || n_extra > SMALL_COPIES - 1) return OPATTR_E_INVALID_ARG;
+    SmallCopy cp[SMALL_COPIES];
+    int n = 0;
+    cp[n++] = SmallCopy{c.h_status, c.d_status, sizeof(DevStatus)};
+    for (int q = 0; q < n_extra; ++q) cp[n++] = extra[q];
+    opattr_status st = copy_small_n(c, n, cp, cudaMemcpyDeviceToHost);
     if (st) return st;
     cudaError_t e = cudaStreamSynchronize(c.stream);
     if (e != cudaSuccess) return cuda_status(c, e);

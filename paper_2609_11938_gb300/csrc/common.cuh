@@ -184,8 +184,17 @@ inline void stream_after(cudaStream_t to, cudaStream_t from, cudaEvent_t e) {
 // uploads never queue behind bulk copies that the caller has on the engines;
 // otherwise (host mirrors in plain host memory) cudaMemcpyAsync.
 opattr_status copy_small(Ctx &c, void *dst, const void *src, size_t bytes, cudaMemcpyKind kind);
+struct SmallCopy {
+    void *dst;
+    const void *src;
+    size_t bytes;
+};
+// Several such transfers of one direction, four to a launch.
+opattr_status copy_small_n(Ctx &c, int count, const SmallCopy *cp, cudaMemcpyKind kind);
 opattr_status reset_status(Ctx &c);
-opattr_status read_status(Ctx &c);      // D2H copy + stream synchronize
+// The status block back to the host (with up to three more device->host
+// transfers in the same launch), then a stream synchronize.
+opattr_status read_status(Ctx &c, int n_extra = 0, const SmallCopy *extra = nullptr);
 opattr_status cuda_status(Ctx &c, cudaError_t e);
 int timing_slot(Ctx &c, const char *name);
 void timing_begin(Ctx &c, int slot, cudaEvent_t *e0, cudaEvent_t *e1);

@@ -659,14 +659,15 @@ opattr_status do_enclose(Ctx &c, const opattr_kernels *kern, const opattr_ranges
                    dim3(RCHK_THREADS), 0, rng->stream, rng->start_ns, rng->end_ns, rng->depth, R, level_hist,
                    c.d_status);
         scan_exclusive_u32(c, level_hist, lvl_off, LEVELS + 1, part2, nullptr);
-        if ((st = copy_small(c, c.h_levels, lvl_off, sizeof(uint32_t) * (LEVELS + 1), cudaMemcpyDeviceToHost)))
-            return st;
     }
     check_kernel_order(c, kern->stream, kern->start_ns, K, kstream, ktile);
-    if ((st = copy_small(c, c.h_levels + LEVELS + 1, kstream, sizeof(uint32_t) * 256, cudaMemcpyDeviceToHost)))
-        return st;
     stream_after(c.stream, c.side, c.ev_join);
-    if ((st = read_status(c))) return st;
+    {
+        // the level offsets and the stream counts come back with the status
+        const SmallCopy back[2] = {{c.h_levels, lvl_off, sizeof(uint32_t) * (LEVELS + 1)},
+                                   {c.h_levels + LEVELS + 1, kstream, sizeof(uint32_t) * 256}};
+        if ((st = read_status(c, 2, back))) return st;
+    }
     if ((st = status_from_err(c.h_status->err))) return st;
     const bool k_sorted = !(c.h_status->flags & F_K_UNSORTED);
     const bool r_sorted = !(c.h_status->flags & F_R_UNSORTED);
