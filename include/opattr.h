@@ -24,6 +24,15 @@
  *    then complete on that stream.  Inside a call, independent steps may run
  *    on a second stream the context owns, forked from and joined back into
  *    the caller's stream before the call returns.
+ *  - Those small transfers (status block, level offsets, host-built tables)
+ *    go through the device mapping of the context's pinned host buffers,
+ *    moved by a small kernel of the library, not through the copy engines:
+ *    a call does not wait behind bulk copies the caller has in flight on
+ *    other streams (where the device cannot map them, cudaMemcpyAsync).
+ *  - The library's kernels are programmatic dependent launches: each is
+ *    scheduled as the kernel before it in the stream finishes, and waits,
+ *    before touching memory, until that kernel has completed.  Work the
+ *    caller queues on the stream before or after a call keeps its order.
  *  - Each call of the library is one NVTX range named after its entry point
  *    (visible on an Nsight Systems timeline).
  *  - n == 0 is valid everywhere and yields empty results.
