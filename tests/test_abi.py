@@ -77,3 +77,24 @@ def test_calls_without_a_context_are_rejected():
     assert lib.opattr_join(None, by(k), by(r), by(n), None, 0, None, None, None, None, by(agg), by(summ),
                            by(tot)) == opa.E_INVALID_ARG
     assert lib.opattr_rollup(None, by(k), by(r), None, by(n), None, 0, None, 0, by(agg)) == opa.E_INVALID_ARG
+
+
+def test_binding_checks_each_array():
+    """The binding refuses an array of the wrong type, one on the host or on
+    another device, and a strided view, before any call; it passes the data
+    pointer of a valid array and NULL for an absent or empty one."""
+    import torch
+
+    import paper_2609_11938_gb300 as opa
+    host = torch.zeros(8, dtype=torch.int64)
+    with pytest.raises(TypeError):
+        opa._ptr(host, torch.int32, "k_start", 0)
+    with pytest.raises(ValueError):
+        opa._ptr(host, torch.int64, "k_start", 0)            # on the host, not on cuda:0
+    assert opa._ptr(host, torch.int64, "k_start", -1) == host.data_ptr()   # the host "device" -1 matches
+    with pytest.raises(ValueError):
+        opa._ptr(host[::2], torch.int64, "k_start", -1)      # not contiguous
+    names = torch.zeros(4, dtype=torch.int32)
+    assert opa._ptr(names, torch.uint32, "k_name", -1) == names.data_ptr()    # int32 stands in for uint32
+    assert opa._ptr(None, torch.int64, "k_layer", 0) is None
+    assert opa._ptr(torch.zeros(0, dtype=torch.int64), torch.int64, "k_start", -1) is None
